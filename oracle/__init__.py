@@ -1,0 +1,264 @@
+"""fp64 CPU oracle of the verify step (test infrastructure).
+
+This package is test infrastructure: only ``tests/``, ``__graft_entry__.smoke()`` and
+the CPU-baseline leg of ``bench.py`` may import it.  The product path (the CUDA
+library and its binding) never loads it, and it imports nothing from the product.
+
+It wraps ``oracle.cpp`` (a plain fp64 statement of the verify step of lossless
+Psi-Spec decoding: Sec. 4.2 and Appendix B.3, Algorithm "Lossless Psi-Spec decoding
+(Linear Sampler)") with ``ctypes``.  Arrays go in and out as numpy arrays; bf16
+tensors travel as their uint16 bit patterns.
+
+Every function of ``oracle.cpp`` is pinned by ``tests/test_oracle_*.py`` against
+facts the paper and the mathematics fix (exact losslessness by enumeration, the
+closed-form acceptance rate, chi-square, special cases, dense-attention brute force).
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "oracle.cpp")
+_LIB_PATH = os.path.join(_HERE, "liboracle.so")
+_lock = threading.Lock()
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    """Compile ``oracle.cpp`` into ``liboracle.so`` (plain g++, -O2, no fast-math)."""
+    if (not force and os.path.exists(_LIB_PATH)
+            and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(_SRC)):
+        return _LIB_PATH
+    tmp = _LIB_PATH + f".tmp{os.getpid()}"
+    cmd = ["g++", "-std=c++17", "-O2", "-fno-fast-math", "-ffp-contract=off", "-fPIC",
+           "-shared", "-pthread", _SRC, "-o", tmp]
+    subprocess.run(cmd, check=True)
+    os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is None:
+            lib = ctypes.CDLL(build())
+            P = ctypes.c_void_p
+            i32, i64, f64 = ctypes.c_int32, ctypes.c_int64, ctypes.c_double
+            lib.oracle_hardware_threads.restype = ctypes.c_int
+            lib.oracle_softmax.argtypes = [P, i64, f64, P]
+            lib.oracle_softmax.restype = ctypes.c_int
+            lib.oracle_argmax.argtypes = [P, i64]
+            lib.oracle_argmax.restype = i64
+            lib.oracle_inverse_cdf.argtypes = [P, i64, f64, P]
+            lib.oracle_inverse_cdf.restype = i64
+            lib.oracle_accept_probs.argtypes = [i32, i64, P, P, P, P, i32, P, P, P, P, P, P, P]
+            lib.oracle_accept_probs.restype = ctypes.c_int
+            lib.oracle_accept_probs_many.argtypes = [i64, i32, i64, P, P, P, P, i32, P, P, P,
+                                                     i32]
+            lib.oracle_accept_probs_many.restype = ctypes.c_int
+            lib.oracle_accept_block.argtypes = [i32, i32, i64, i32, P, P, P, P, P, P, P, P,
+                                                P, P, P, P, i32]
+            lib.oracle_accept_block.restype = ctypes.c_int
+            lib.oracle_verify_attention.argtypes = [i32, i32, i32, i32, i32, i32, i32, i32, f64,
+                                                    P, P, P, P, P, P, P, P, i64, P, i32]
+            lib.oracle_verify_attention.restype = ctypes.c_int
+            _lib = lib
+    return _lib
+
+
+def _ptr(a):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _c(a, dtype):
+    return np.ascontiguousarray(a, dtype=dtype)
+
+
+def hardware_threads() -> int:
+    return int(_load().oracle_hardware_threads())
+
+
+def softmax(logits, temperature: float):
+    """softmax(logits / T) of one row in fp64; raises on an undefined row."""
+    lib = _load()
+    l = _c(logits, np.float64)
+    p = np.empty_like(l)
+    rc = lib.oracle_softmax(_ptr(l), l.size, float(temperature), _ptr(p))
+    if rc:
+        raise ValueError("softmax undefined for this row")
+    return p
+
+
+def argmax(row) -> int:
+    r = _c(row, np.float64)
+    return int(_load().oracle_argmax(_ptr(r), r.size))
+
+
+def inverse_cdf(weights, u: float):
+    """(token, margin) of the inverse-CDF draw from unnormalised weights."""
+    w = _c(weights, np.float64)
+    m = np.zeros(1, np.float64)
+    x = _load().oracle_inverse_cdf(_ptr(w), w.size, float(u), _ptr(m))
+    return int(x), float(m[0])
+
+
+def accept_probs(p_rows, q_rows, tokens, uniforms, greedy: bool = False):
+    """The verify decision of one sequence on fp64 probability rows.
+
+    Returns a dict with n, out_tokens, num_emitted, p_tok, q_tok, accept_margin,
+    sample_margin (see ``oracle_accept_probs`` in oracle.cpp).
+    """
+    lib = _load()
+    p = _c(p_rows, np.float64)
+    gamma, vocab = p.shape
+    q = None if greedy and q_rows is None else _c(q_rows, np.float64)
+    t = _c(tokens, np.int32)
+    u = _c(uniforms, np.float64)
+    n = np.zeros(1, np.int32)
+    ne = np.zeros(1, np.int32)
+    out = np.empty(gamma + 1, np.int32)
+    ptok = np.empty(gamma, np.float64)
+    qtok = np.empty(gamma, np.float64)
+    am = np.empty(gamma, np.float64)
+    sm = np.empty(1, np.float64)
+    rc = lib.oracle_accept_probs(gamma, vocab, _ptr(p), _ptr(q), _ptr(t), _ptr(u),
+                                 1 if greedy else 0, _ptr(n), _ptr(out), _ptr(ne),
+                                 _ptr(ptok), _ptr(qtok), _ptr(am), _ptr(sm))
+    if rc:
+        raise ValueError("token id out of range")
+    return dict(n=int(n[0]), out_tokens=out, num_emitted=int(ne[0]), p_tok=ptok, q_tok=qtok,
+                accept_margin=am, sample_margin=float(sm[0]))
+
+
+def accept_probs_many(p_rows, q_rows, tokens, uniforms, greedy: bool = False,
+                      nthreads: int = 0, lib=None):
+    """accept_probs for many (tokens, uniforms) cases sharing the same rows.
+
+    tokens: int [count][gamma]; uniforms: float [count][gamma].
+    Returns (n [count], out_tokens [count][gamma+1], num_emitted [count]).
+    ``lib`` optionally substitutes another build of oracle.cpp (mutation tests).
+    """
+    lib = lib or _load()
+    p = _c(p_rows, np.float64)
+    gamma, vocab = p.shape
+    q = _c(q_rows, np.float64) if q_rows is not None else None
+    t = _c(tokens, np.int32).reshape(-1, gamma)
+    u = _c(uniforms, np.float64).reshape(-1, gamma)
+    count = t.shape[0]
+    n = np.empty(count, np.int32)
+    ne = np.empty(count, np.int32)
+    out = np.empty((count, gamma + 1), np.int32)
+    rc = lib.oracle_accept_probs_many(count, gamma, vocab, _ptr(p), _ptr(q), _ptr(t), _ptr(u),
+                                      1 if greedy else 0, _ptr(n), _ptr(out), _ptr(ne),
+                                      int(nthreads))
+    if rc:
+        raise ValueError("token id out of range")
+    return n, out, ne
+
+
+def load_variant(src_text: str, tag: str):
+    """Compile a modified copy of oracle.cpp (tests plant mistakes this way) and load it."""
+    import tempfile
+    d = tempfile.mkdtemp(prefix=f"oracle_{tag}_")
+    src = os.path.join(d, "oracle.cpp")
+    so = os.path.join(d, "liboracle.so")
+    with open(src, "w") as f:
+        f.write(src_text)
+    subprocess.run(["g++", "-std=c++17", "-O1", "-fPIC", "-shared", "-pthread", src, "-o", so],
+                   check=True)
+    lib = ctypes.CDLL(so)
+    P = ctypes.c_void_p
+    i32, i64 = ctypes.c_int32, ctypes.c_int64
+    lib.oracle_accept_probs_many.argtypes = [i64, i32, i64, P, P, P, P, i32, P, P, P, i32]
+    lib.oracle_accept_probs_many.restype = ctypes.c_int
+    return lib
+
+
+def source_text() -> str:
+    with open(_SRC) as f:
+        return f.read()
+
+
+def accept_block(target_logits, drafter_logits, block_tokens, temperature, uniforms,
+                 nthreads: int = 0):
+    """The acceptance half of the verify step over a batch, from logits.
+
+    target_logits / drafter_logits: [batch][gamma][vocab] float32, or uint16 bf16 bits.
+    Returns a dict of numpy arrays: num_accepted, out_tokens, num_emitted, diag,
+    accept_margin, sample_margin, status.
+    """
+    lib = _load()
+    tl = np.ascontiguousarray(target_logits)
+    dl = np.ascontiguousarray(drafter_logits)
+    if tl.dtype == np.float32:
+        dtype = 0
+    elif tl.dtype == np.uint16:
+        dtype = 1
+    else:
+        raise TypeError("logits must be float32 or uint16 (bf16 bits)")
+    if dl.dtype != tl.dtype or dl.shape != tl.shape:
+        raise TypeError("target and drafter logits must match in dtype and shape")
+    batch, gamma, vocab = tl.shape
+    bt = _c(block_tokens, np.int32)
+    T = _c(temperature, np.float32)
+    u = _c(uniforms, np.float32)
+    na = np.empty(batch, np.int32)
+    ne = np.empty(batch, np.int32)
+    ot = np.empty((batch, gamma + 1), np.int32)
+    diag = np.empty((batch, gamma, 2), np.float64)
+    am = np.empty((batch, gamma), np.float64)
+    sm = np.empty(batch, np.float64)
+    st = np.empty(batch, np.int32)
+    rc = lib.oracle_accept_block(batch, gamma, vocab, dtype, _ptr(tl), _ptr(dl), _ptr(bt),
+                                 _ptr(T), _ptr(u), _ptr(na), _ptr(ot), _ptr(ne), _ptr(diag),
+                                 _ptr(am), _ptr(sm), _ptr(st), int(nthreads))
+    if rc:
+        raise ValueError("invalid arguments to oracle_accept_block")
+    return dict(num_accepted=na, out_tokens=ot, num_emitted=ne, diag=diag,
+                accept_margin=am, sample_margin=sm, status=st)
+
+
+def verify_attention(q, k_cache, v_cache, page_table, kv_len, gamma: int, softmax_scale=None,
+                     rows=None, nthreads: int = 0):
+    """fp64 block-causal paged GQA attention.
+
+    q: uint16 bf16 bits [batch][gamma][Hq][D]; k_cache, v_cache: uint16
+    [num_pages][Hkv][page_size][D]; page_table: int32 [batch][max_pages];
+    kv_len: int32 [batch].  rows: optional int array [n][3] of (b, j, h) to compute.
+    Returns (out fp64 [batch][gamma][Hq][D], lse fp64 [batch][gamma][Hq], status).
+    Rows not listed in ``rows`` are left NaN.
+    """
+    lib = _load()
+    qa = _c(q, np.uint16)
+    ka = _c(k_cache, np.uint16)
+    va = _c(v_cache, np.uint16)
+    pt = _c(page_table, np.int32)
+    kl = _c(kv_len, np.int32)
+    batch, g, Hq, D = qa.shape
+    if g != gamma:
+        raise ValueError("q's second dimension must equal gamma")
+    num_pages, Hkv, page_size, D2 = ka.shape
+    if D2 != D or va.shape != ka.shape:
+        raise ValueError("cache shapes disagree with q")
+    scale = 1.0 / np.sqrt(D) if softmax_scale is None else float(softmax_scale)
+    out = np.full((batch, gamma, Hq, D), np.nan, np.float64)
+    lse = np.full((batch, gamma, Hq), np.nan, np.float64)
+    st = np.empty(batch, np.int32)
+    r = None
+    nrows = 0
+    if rows is not None:
+        r = _c(rows, np.int32).reshape(-1, 3)
+        nrows = r.shape[0]
+    rc = lib.oracle_verify_attention(batch, gamma, Hq, Hkv, D, page_size, pt.shape[1], num_pages,
+                                     scale, _ptr(qa), _ptr(ka), _ptr(va), _ptr(pt), _ptr(kl),
+                                     _ptr(out), _ptr(lse), _ptr(r), nrows, _ptr(st),
+                                     int(nthreads))
+    if rc:
+        raise ValueError("invalid arguments to oracle_verify_attention")
+    return out, lse, st
