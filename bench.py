@@ -1,0 +1,381 @@
+#!/usr/bin/env python3
+"""Verify-step benchmark: block-causal paged verify attention + lossless acceptance on
+one GB300 (or N independent replicas under torchrun), through the C ABI.
+
+One step = one spec_verify_step call over one batch of synthetic input (attention of
+the gamma block queries over the paged KV cache for one layer, plus the vocabulary-wide
+softmax and acceptance over target and drafter logits). Inputs are resident in HBM;
+L2 is flushed (a 256 MiB write) before every timed step, outside the timed events.
+
+Prints ONE JSON line (rank 0). ``--impl reference`` times the fp64 CPU oracle on the
+host cores instead (the reference arm: there is no runnable reference implementation
+of this path).
+"""
+
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "verify-step tokens/s on 1 GB300; achieved HBM GB/s as fraction of ~8 TB/s"
+UNIT = "tokens/s"
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+L2_FLUSH_BYTES = 256 << 20
+
+
+def parse_args():
+    ap = argparse.ArgumentParser(description=__doc__)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="llama8b",
+                    help="tiny | llama8b | serve64 | long70b | sweep_g<G>_b<B>_s<S>_t<T>")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=10.0,
+                    help="CPU time budget of the oracle baseline sample")
+    return ap.parse_args()
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+# ----------------------------------------------------------------------------------
+# clocks during the timed region
+# ----------------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100", "-i", str(self.gpu)], stdout=subprocess.PIPE,
+                stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append((time.time(), line.strip()))
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.thread.join(timeout=2)
+        sms, maxes, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for _, line in self.lines:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sms.append(float(parts[1]))
+                maxes.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sms:
+            return None
+        return {"sm_mhz": statistics.median(sms), "sm_max_mhz": max(maxes),
+                "samples": len(sms), "reasons": sorted(reasons)}
+
+
+# ----------------------------------------------------------------------------------
+# workload bytes (the roofline's algorithmic traffic)
+# ----------------------------------------------------------------------------------
+def traffic_model(ai, ci):
+    esz = 2 if ci.is_bf16 else 4
+    from paper_2609_04010_gb300 import workloads as W
+    kv = ai.kv_bytes()
+    logits = W.logits_bytes_baseline(ci.batch, ci.gamma, ci.vocab, esz)
+    strict_logits = W.logits_bytes_strict(ci.temperature, ci.gamma, ci.vocab, esz)
+    q_out = 2 * ai.q.size * 2
+    return dict(kv=kv, logits=logits, baseline=kv + logits,
+                strict=kv + strict_logits + q_out + ai.page_table.nbytes)
+
+
+# ----------------------------------------------------------------------------------
+# the oracle on host cores (cpu_baseline and the reference arm)
+# ----------------------------------------------------------------------------------
+class OracleStep:
+    """One verify step of the oracle over the first ``nseq`` sequences of the workload."""
+
+    def __init__(self, ai, ci):
+        import oracle
+        self.oracle = oracle
+        self.ai, self.ci = ai, ci
+
+    def run(self, nseq: int):
+        ai, ci, o = self.ai, self.ci, self.oracle
+        o.verify_attention(ai.q[:nseq], ai.k_cache, ai.v_cache, ai.page_table[:nseq],
+                           ai.kv_len[:nseq], ai.gamma)
+        o.accept_block(ci.target_logits[:nseq], ci.drafter_logits[:nseq],
+                       ci.block_tokens[:nseq], ci.temperature[:nseq], ci.uniforms[:nseq])
+
+    def calibrate(self, budget_s: float):
+        """Sequences per step so that one step takes at most about budget_s."""
+        t0 = time.perf_counter()
+        self.run(1)
+        t1 = max(time.perf_counter() - t0, 1e-6)
+        return int(max(1, min(self.ci.batch, budget_s // t1))), t1
+
+
+def cpu_baseline(ai, ci, seconds: float):
+    import oracle
+    st = OracleStep(ai, ci)
+    nseq, _ = st.calibrate(max(0.5, seconds / 4))
+    tokens, elapsed, steps = 0, 0.0, 0
+    while elapsed < seconds or steps == 0:
+        t0 = time.perf_counter()
+        st.run(nseq)
+        elapsed += time.perf_counter() - t0
+        tokens += nseq * ci.gamma
+        steps += 1
+    return {"value": tokens / elapsed, "unit": UNIT, "cores": oracle.hardware_threads(),
+            "kind": "oracle",
+            "sample": f"{steps} oracle verify steps over the first {nseq} of {ci.batch} "
+                      f"sequences of the workload (attention of every head and block position "
+                      f"+ acceptance), {elapsed:.1f} s, fp64, all host threads"}
+
+
+def reference_arm(args, wl, ai, ci):
+    import oracle
+    st = OracleStep(ai, ci)
+    nseq, _ = st.calibrate(1.0)
+    for _ in range(args.warmup):
+        st.run(nseq)
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        st.run(nseq)
+        times.append(time.perf_counter() - t0)
+    ms = 1000.0 * statistics.mean(times)
+    value = nseq * ci.gamma / (ms / 1000.0)
+    cores = oracle.hardware_threads()
+    sample = (f"each step: the oracle over the first {nseq} of {ci.batch} sequences "
+              f"(attention of every head and block position + acceptance), fp64")
+    return {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": dict(wl.describe(), sample_sequences=nseq),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+
+
+# ----------------------------------------------------------------------------------
+# our arm
+# ----------------------------------------------------------------------------------
+def run_ours(args, wl, ai, ci, rank, world, local_rank):
+    import torch
+    from paper_2609_04010_gb300 import binding, build
+
+    build.build()
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+
+    def bf16(a):
+        return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16)
+
+    def t(a):
+        return torch.from_numpy(np.ascontiguousarray(a))
+
+    host_in = dict(q=bf16(ai.q), k=bf16(ai.k_cache), v=bf16(ai.v_cache), pt=t(ai.page_table),
+                   kvl=t(ai.kv_len),
+                   tl=bf16(ci.target_logits) if ci.is_bf16 else t(ci.target_logits),
+                   dl=bf16(ci.drafter_logits) if ci.is_bf16 else t(ci.drafter_logits),
+                   tok=t(ci.block_tokens), temp=t(ci.temperature), u=t(ci.uniforms))
+    d = {k: v.to(dev) for k, v in host_in.items()}
+    B, G = ci.batch, ci.gamma
+    out = torch.empty_like(d["q"])
+    lse = torch.empty(d["q"].shape[:3], dtype=torch.float32, device=dev)
+    na = torch.empty(B, dtype=torch.int32, device=dev)
+    ot = torch.empty(B, G + 1, dtype=torch.int32, device=dev)
+    ne = torch.empty(B, dtype=torch.int32, device=dev)
+    a = binding.attn_args(d["q"], d["k"], d["v"], d["pt"], d["kvl"], out, lse)
+    c = binding.accept_args(d["tl"], d["dl"], d["tok"], d["temp"], d["u"], na, ot, ne, None)
+    ws = binding.new_workspace(binding.workspace_size(a, c), dev)
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    stream = torch.cuda.current_stream()
+
+    def timed_loop(fn, n):
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(n)]
+        for i in range(n):
+            flush.zero_()
+            evs[i][0].record(stream)
+            fn()
+            evs[i][1].record(stream)
+        torch.cuda.synchronize()
+        return [s.elapsed_time(e) for s, e in evs]
+
+    step = lambda: binding.verify_step_args(a, c, ws)
+    attn_only = lambda: binding.verify_step_args(a, None, ws)
+    acc_only = lambda: binding.verify_step_args(None, c, ws)
+
+    clocks = ClockSampler(local_rank if "CUDA_VISIBLE_DEVICES" not in os.environ else
+                          int(os.environ["CUDA_VISIBLE_DEVICES"].split(",")[local_rank]))
+    clocks.start()
+    time.sleep(0.3)
+    for _ in range(max(3, args.warmup)):
+        flush.zero_()
+        step()
+    torch.cuda.synchronize()
+    code, flags = binding.read_device_status(ws)
+    if code != 0:
+        raise RuntimeError(f"device status after warm-up: {code} flags {flags}")
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    step_ms = timed_loop(step, args.steps)
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    ms = statistics.mean(step_ms)
+    if world > 1:
+        x = torch.tensor([ms], dtype=torch.float64, device=dev)
+        torch.distributed.all_reduce(x, op=torch.distributed.ReduceOp.MAX)
+        ms = float(x.item())
+    parts_n = max(20, min(args.steps, 500))
+    attn_ms = statistics.mean(timed_loop(attn_only, parts_n))
+    acc_ms = statistics.mean(timed_loop(acc_only, parts_n))
+
+    e2e = None
+    if not args.no_e2e:
+        pin = {k: v.pin_memory() for k, v in host_in.items()}
+        outs_h = [torch.empty(x.shape, dtype=x.dtype).pin_memory() for x in (out, lse, na, ot, ne)]
+        h2d = sum(v.numel() * v.element_size() for v in pin.values())
+        d2h = sum(v.numel() * v.element_size() for v in outs_h)
+
+        def e2e_step():
+            for k in d:
+                d[k].copy_(pin[k], non_blocking=True)
+            step()
+            for hst, src in zip(outs_h, (out, lse, na, ot, ne)):
+                hst.copy_(src, non_blocking=True)
+
+        for _ in range(3):
+            e2e_step()
+        n_e2e = max(10, min(args.steps, 200))
+        e2e_ms = statistics.mean(timed_loop(e2e_step, n_e2e))
+        if world > 1:
+            x = torch.tensor([e2e_ms], dtype=torch.float64, device=dev)
+            torch.distributed.all_reduce(x, op=torch.distributed.ReduceOp.MAX)
+            e2e_ms = float(x.item())
+        e2e = {"value": world * B * G / (e2e_ms / 1000.0), "unit": UNIT,
+               "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+               "ms_per_step": e2e_ms}
+
+    tm = traffic_model(ai, ci)
+    peak, peak_src = measured_peaks()
+    attn_gbs = tm["kv"] / (attn_ms / 1000.0) / 1e9
+    step_gbs = tm["baseline"] / (ms / 1000.0) / 1e9
+    dominant = "attention" if attn_ms >= acc_ms else "accept"
+    dom_bytes = tm["kv"] if dominant == "attention" else tm["logits"]
+    dom_ms = attn_ms if dominant == "attention" else acc_ms
+    dom_gbs = dom_bytes / (dom_ms / 1000.0) / 1e9
+    launches_per_step = 3
+    result = {
+        "metric": METRIC, "value": world * B * G / (ms / 1000.0), "unit": UNIT,
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded; no weights or datasets)",
+        "config": dict(wl.describe(), parallelism=f"replicas x{world}",
+                       l2="flushed before every timed step (256 MiB write, outside events)",
+                       attention_path="tensor cores" if binding.tensor_core_min_rows() <=
+                       (ai.num_q_heads // ai.num_kv_heads) * ai.gamma else "CUDA cores"),
+        "roofline": {"bound": "hbm", "kernel": dominant, "achieved": round(dom_gbs, 1),
+                     "peak": peak, "unit": "GB/s", "frac": round(dom_gbs / peak, 4),
+                     "peak_source": peak_src, "traffic": None,
+                     "algorithmic_bytes_per_launch": int(dom_bytes), "launch_ms": dom_ms},
+        "step_roofline": {"bytes": int(tm["baseline"]), "strict_bytes": int(tm["strict"]),
+                          "achieved_gbs": round(step_gbs, 1),
+                          "frac_of_measured": round(step_gbs / peak, 4),
+                          "frac_of_8tbs": round(step_gbs / NOMINAL_HBM_GBS, 4)},
+        "parts_ms": {"attention": attn_ms, "accept": acc_ms,
+                     "attention_gbs": round(attn_gbs, 1)},
+        "gpu_launches": launches_per_step * args.steps,
+        "emitted_tokens_per_step": int(ne.sum().item()) * world,
+        "clocks": clk,
+    }
+    if e2e:
+        result["e2e"] = e2e
+    return result
+
+
+def main():
+    args = parse_args()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference" and rank != 0:
+        return 0
+    from paper_2609_04010_gb300 import workloads as W
+    wl = W.workload(args.workload)
+    seed = rank
+    ai, ci = wl.attn_inputs(seed=seed), wl.accept_inputs(seed=seed)
+    if args.impl == "reference":
+        import oracle
+        oracle.build()
+        print(json.dumps(reference_arm(args, wl, ai, ci)), flush=True)
+        return 0
+    if world > 1:
+        import torch
+        torch.cuda.set_device(local_rank)
+        torch.distributed.init_process_group("nccl")
+    res = run_ours(args, wl, ai, ci, rank, world, local_rank)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
+        oracle.build()
+        res["cpu_baseline"] = cpu_baseline(ai, ci, args.cpu_seconds)
+    if rank == 0:
+        print(json.dumps(res), flush=True)
+    if world > 1:
+        import torch
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

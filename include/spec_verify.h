@@ -1,0 +1,193 @@
+/*
+ * spec_verify.h -- C ABI of the GB300 (sm_103a) verify step of lossless
+ * diffusion-drafted decoding ("Unlocking Lossless Speedups in LLMs via Discrete
+ * Diffusion": Psi-Spec, Sec. 4 and Appendix B.3).
+ *
+ * In one decode step, the drafter proposes a block of gamma tokens
+ * [x^{L+1}, x~^1 .. x~^{gamma-1}] (gamma is the paper's block size B), and the
+ * autoregressive verifier scores the whole block in one forward pass. This library
+ * implements the two data-parallel parts of that verify step:
+ *   (a) block-causal attention of the gamma block queries against a paged bf16 KV
+ *       cache with grouped-query heads (spec_verify_attention);
+ *   (b) the vocabulary-wide softmax of target and drafter logits and the lossless
+ *       acceptance rule: accept draft i with probability min(1, p_i/q_i), on the
+ *       first rejection n draw from Norm([p_n - q_n]_+), otherwise draw the bonus
+ *       token from p_B; at temperature 0, greedy argmax matching
+ *       (spec_accept_block).
+ * spec_verify_step runs both on one stream.
+ *
+ * Conventions shared by every entry point
+ *   - Every tensor argument is a DEVICE pointer owned by the caller, row-major and
+ *     densely packed in the layout stated beside it. The library allocates no
+ *     memory, keeps no state between calls, and never synchronizes the stream
+ *     (except spec_read_device_status). Calls are asynchronous on `stream`.
+ *   - `ws` is a caller-owned device workspace of at least spec_workspace_size()
+ *     bytes, 256-byte aligned. A new workspace must be zero-filled once (e.g.
+ *     spec_workspace_init); every call leaves its internal counters at zero again.
+ *     Concurrent calls need distinct workspaces.
+ *   - Host-side argument checks happen before any launch and return
+ *     SPEC_ERR_INVALID_ARGUMENT / SPEC_ERR_UNSUPPORTED / SPEC_ERR_WORKSPACE_TOO_SMALL
+ *     without touching the device. Launch failures return SPEC_ERR_CUDA.
+ *   - Bad device-resident data (a token id outside [0, vocab), a page id outside
+ *     [0, num_pages), kv_len outside [gamma, max_pages_per_seq * page_size], NaN or
+ *     +inf logits) never traps: the kernels set a bit in the workspace status word
+ *     (SPEC_FLAG_*), write the documented sentinel outputs for the affected
+ *     sequence, and carry on. spec_read_device_status reads and clears the word.
+ *   - Kernels never wait on other thread blocks; every internal wait on an
+ *     asynchronous copy or tensor-core operation is bounded, and a timeout sets
+ *     SPEC_FLAG_TIMEOUT instead of hanging.
+ */
+#ifndef SPEC_VERIFY_H
+#define SPEC_VERIFY_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* A cudaStream_t (the runtime's stream handle); NULL is the legacy default stream. */
+typedef struct CUstream_st* spec_stream_t;
+
+typedef enum {
+  SPEC_OK = 0,
+  SPEC_ERR_INVALID_ARGUMENT = 1,  /* null pointer, non-positive size, inconsistent shape   */
+  SPEC_ERR_UNSUPPORTED = 2,       /* a shape outside the supported limits below            */
+  SPEC_ERR_WORKSPACE_TOO_SMALL = 3,
+  SPEC_ERR_CUDA = 4,              /* a CUDA runtime/driver call or a launch failed          */
+  SPEC_ERR_DEVICE_INPUT = 5,      /* spec_read_device_status found SPEC_FLAG_BAD_* bits    */
+  SPEC_ERR_TIMEOUT = 6            /* spec_read_device_status found SPEC_FLAG_TIMEOUT       */
+} spec_status_t;
+
+typedef enum { SPEC_F32 = 0, SPEC_BF16 = 1 } spec_dtype_t;
+
+/* Attention kernel selection (spec_attn_args_t.path). */
+typedef enum {
+  SPEC_ATTN_AUTO = 0,          /* tensor cores when (Hq/Hkv)*gamma >= the crossover, else CUDA cores */
+  SPEC_ATTN_CUDA_CORES = 1,    /* fp32 CUDA-core kernel                                  */
+  SPEC_ATTN_TENSOR_CORES = 2   /* tcgen05 (TMEM accumulators, TMA-staged KV pages)       */
+} spec_attn_path_t;
+
+/* Device status word bits. */
+#define SPEC_FLAG_BAD_TOKEN 0x1u   /* a block token outside [0, vocab)                      */
+#define SPEC_FLAG_BAD_LOGITS 0x2u  /* a used logits row with NaN, +inf, or no finite entry */
+#define SPEC_FLAG_BAD_PAGE 0x4u    /* a page id of a visible key outside [0, num_pages)      */
+#define SPEC_FLAG_BAD_KV_LEN 0x8u  /* kv_len outside [gamma, max_pages_per_seq * page_size] */
+#define SPEC_FLAG_TIMEOUT 0x10u    /* a bounded internal wait ran out                        */
+
+/*
+ * Part (a): block-causal verify attention (Sec. 4.1: the block [x^{L+1}, z] is
+ * processed while the prefix stays in the KV cache; Alg. "Lossless Psi-Spec":
+ * p <- x_theta([x^{L+1}, x~]; x) is one causal pass over the block).
+ *
+ * For sequence b, kv_len[b] = ctx_b + gamma keys are in the cache: the prefix at
+ * positions 0 .. ctx_b-1 and the block's own keys at ctx_b .. ctx_b+gamma-1 (already
+ * written). Block query j of head h attends to keys k <= ctx_b + j of KV head
+ * h / (num_q_heads / num_kv_heads):
+ *   out[b][j][h] = sum_k softmax_k(scale * q.k_k) v_k,
+ *   lse[b][j][h] = log sum_k exp(scale * q.k_k)       (natural log).
+ * Logical key k lives in physical page page_table[b][k / page_size], slot
+ * k % page_size. Accumulation is fp32; out is rounded to bf16.
+ * A sequence flagged BAD_PAGE or BAD_KV_LEN gets out = 0 and lse = -inf.
+ */
+typedef struct {
+  int32_t batch;              /* >= 1                                                       */
+  int32_t gamma;              /* block size, 1 .. 64                                        */
+  int32_t num_q_heads;        /* Hq, a multiple of num_kv_heads                             */
+  int32_t num_kv_heads;       /* Hkv                                                        */
+  int32_t head_dim;           /* D: 64 or 128                                               */
+  int32_t page_size;          /* 16, 32 or 64 tokens                                        */
+  int32_t max_pages_per_seq;  /* page_table row length                                      */
+  int32_t num_pages;          /* physical pages in k_cache / v_cache                        */
+  float softmax_scale;        /* 0 => 1/sqrt(head_dim)                                      */
+  int32_t path;               /* spec_attn_path_t                                           */
+  const void* q;              /* bf16 [batch][gamma][Hq][D]                                 */
+  const void* k_cache;        /* bf16 [num_pages][Hkv][page_size][D], 16-byte aligned       */
+  const void* v_cache;        /* bf16 [num_pages][Hkv][page_size][D], 16-byte aligned       */
+  const int32_t* page_table;  /* [batch][max_pages_per_seq]; entries past the sequence unread */
+  const int32_t* kv_len;      /* [batch]                                                    */
+  void* out;                  /* bf16 [batch][gamma][Hq][D]                                 */
+  float* lse;                 /* fp32 [batch][gamma][Hq], or NULL                           */
+} spec_attn_args_t;
+
+/*
+ * Part (b): lossless acceptance (Alg. "Lossless Psi-Spec decoding (Linear
+ * Sampler)", the steps after the verifier pass; Sec. 4.2).
+ *
+ * Row conventions (gamma = B): target row j is the verifier's distribution of block
+ * token j+1, so the algorithm's p_i is target row i-1 and the bonus row p_B is row
+ * gamma-1; drafter row j is the distribution block token j was drawn from, so q_i is
+ * drafter row i (drafter row 0 is never read). With T = temperature[b] > 0,
+ * p = softmax(target / T), q = softmax(drafter / T), and
+ *   n = min({i in 1..gamma-1 : uniforms[b][i-1] > min(1, p_i(t_i) / q_i(t_i))} U {gamma});
+ * the final token is the smallest x with C(x) >= uniforms[b][gamma-1] * C(vocab-1),
+ * C the ascending-token cumulative sum of p_B (n = gamma) or of [p_n - q_n]_+.
+ * With T = 0 (greedy): n = the first i whose token is not the lowest-index argmax of
+ * target row i-1, and the final token is that argmax of target row n-1.
+ * Outputs: out_tokens[b] = [t_0, t_1 .. t_{n-1}, final, -1 ...] (gamma+1 entries),
+ * num_accepted[b] = n - 1 in [0, gamma-1], num_emitted[b] = n + 1 in [2, gamma+1].
+ * A sequence flagged BAD_TOKEN or BAD_LOGITS gets num_accepted = -1,
+ * num_emitted = 0 and out_tokens = -1.
+ */
+typedef struct {
+  int32_t batch;               /* >= 1                                                      */
+  int32_t gamma;               /* 1 .. 64                                                   */
+  int32_t vocab;               /* >= 1                                                      */
+  int32_t logits_dtype;        /* spec_dtype_t                                              */
+  const void* target_logits;   /* [batch][gamma][vocab]                                     */
+  const void* drafter_logits;  /* [batch][gamma][vocab]; row 0 of each sequence unread      */
+  const int32_t* block_tokens; /* [batch][gamma]: t_0 = x^{L+1}, t_1.. = drafts            */
+  const float* temperature;    /* [batch]; 0 => greedy                                      */
+  const float* uniforms;       /* [batch][gamma] in (0, 1]; [i-1] tests draft i, [gamma-1] draws the final token */
+  int32_t* num_accepted;       /* [batch]                                                   */
+  int32_t* out_tokens;         /* [batch][gamma+1]                                          */
+  int32_t* num_emitted;        /* [batch]                                                   */
+  float* diag;                 /* [batch][gamma][2] = (p_i(t_i), q_i(t_i)) for the decisions
+                                  taken (entry 0 and untaken = NaN; greedy: (match, 1)), or NULL */
+} spec_accept_args_t;
+
+/* Bytes of workspace the calls below need for these arguments (either may be NULL). */
+size_t spec_workspace_size(const spec_attn_args_t* attn, const spec_accept_args_t* accept);
+
+/* Zero-fills a workspace (cudaMemsetAsync on `stream`). */
+spec_status_t spec_workspace_init(void* ws, size_t ws_bytes, spec_stream_t stream);
+
+/* Part (a) alone. */
+spec_status_t spec_verify_attention(const spec_attn_args_t* attn, void* ws, size_t ws_bytes,
+                                    spec_stream_t stream);
+
+/* Part (b) alone. */
+spec_status_t spec_accept_block(const spec_accept_args_t* accept, void* ws, size_t ws_bytes,
+                                spec_stream_t stream);
+
+/* The whole verify step: parts (a) and (b) on one stream (they share no data: the
+ * logits are inputs). Either argument may be NULL to run only the other part. */
+spec_status_t spec_verify_step(const spec_attn_args_t* attn, const spec_accept_args_t* accept,
+                               void* ws, size_t ws_bytes, spec_stream_t stream);
+
+/*
+ * Seeded uniforms for the acceptance rule (Alg. "Lossless Psi-Spec": r ~ U[0,1]).
+ * out_dev[i] = ((x >> 8) + 1) * 2^-24 in (0, 1], x = word (offset+i) & 3 of
+ * Philox4x32-10 (Salmon et al., SC'11) with key (seed low, seed high) and counter
+ * ((offset+i) >> 2 low, high, 0, 0). n >= 0; out_dev is fp32 device memory.
+ */
+spec_status_t spec_philox_uniforms(uint64_t seed, uint64_t offset, int64_t n, float* out_dev,
+                                   spec_stream_t stream);
+
+/* Synchronizes `stream`, reads the workspace status word into *flags_out and clears
+ * it. Returns SPEC_ERR_TIMEOUT if SPEC_FLAG_TIMEOUT is set, SPEC_ERR_DEVICE_INPUT if
+ * another flag is set, else SPEC_OK. */
+spec_status_t spec_read_device_status(void* ws, spec_stream_t stream, uint32_t* flags_out);
+
+/* A static, human-readable name of a status code. */
+const char* spec_status_string(spec_status_t status);
+
+/* The (Hq/Hkv)*gamma at and above which SPEC_ATTN_AUTO picks the tensor-core kernel. */
+int32_t spec_attn_tensor_core_min_rows(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SPEC_VERIFY_H */

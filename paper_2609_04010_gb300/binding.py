@@ -1,0 +1,242 @@
+"""ctypes binding of libspecverify (include/spec_verify.h).
+
+Argument marshalling only: torch tensors (device memory) are checked for dtype, shape
+and contiguity, and their pointers go into the C structs; every step of the verify
+step runs in the library's CUDA kernels on the current torch stream. The library must
+exist (``python -m paper_2609_04010_gb300.build``); there is no fallback.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+import re
+import threading
+from typing import Dict, Optional
+
+import torch
+
+from . import build as _build
+
+_lock = threading.Lock()
+_lib = None
+
+SPEC_OK = 0
+STATUS_NAMES = {0: "SPEC_OK", 1: "SPEC_ERR_INVALID_ARGUMENT", 2: "SPEC_ERR_UNSUPPORTED",
+                3: "SPEC_ERR_WORKSPACE_TOO_SMALL", 4: "SPEC_ERR_CUDA", 5: "SPEC_ERR_DEVICE_INPUT",
+                6: "SPEC_ERR_TIMEOUT"}
+SPEC_F32, SPEC_BF16 = 0, 1
+ATTN_AUTO, ATTN_CUDA_CORES, ATTN_TENSOR_CORES = 0, 1, 2
+FLAG_BAD_TOKEN, FLAG_BAD_LOGITS, FLAG_BAD_PAGE, FLAG_BAD_KV_LEN, FLAG_TIMEOUT = 1, 2, 4, 8, 16
+
+
+class SpecError(RuntimeError):
+    def __init__(self, code: int, what: str):
+        super().__init__(f"{what}: {STATUS_NAMES.get(code, code)}")
+        self.code = code
+
+
+class AttnArgs(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int32), ("gamma", ctypes.c_int32),
+                ("num_q_heads", ctypes.c_int32), ("num_kv_heads", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32), ("page_size", ctypes.c_int32),
+                ("max_pages_per_seq", ctypes.c_int32), ("num_pages", ctypes.c_int32),
+                ("softmax_scale", ctypes.c_float), ("path", ctypes.c_int32),
+                ("q", ctypes.c_void_p), ("k_cache", ctypes.c_void_p),
+                ("v_cache", ctypes.c_void_p), ("page_table", ctypes.c_void_p),
+                ("kv_len", ctypes.c_void_p), ("out", ctypes.c_void_p), ("lse", ctypes.c_void_p)]
+
+
+class AcceptArgs(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int32), ("gamma", ctypes.c_int32), ("vocab", ctypes.c_int32),
+                ("logits_dtype", ctypes.c_int32), ("target_logits", ctypes.c_void_p),
+                ("drafter_logits", ctypes.c_void_p), ("block_tokens", ctypes.c_void_p),
+                ("temperature", ctypes.c_void_p), ("uniforms", ctypes.c_void_p),
+                ("num_accepted", ctypes.c_void_p), ("out_tokens", ctypes.c_void_p),
+                ("num_emitted", ctypes.c_void_p), ("diag", ctypes.c_void_p)]
+
+
+HEADER = os.path.join(_build.ROOT, "include", "spec_verify.h")
+
+
+def declared_functions():
+    """Names of the functions include/spec_verify.h declares."""
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(spec_[a-z0-9_]+)\s*\(", text)))
+
+
+def lib(build_if_missing: bool = True):
+    """The loaded library (built first if it is missing and the toolkit is present)."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(_build.LIB):
+                if not build_if_missing:
+                    raise RuntimeError("libspecverify.so is not built")
+                _build.build()
+            L = ctypes.CDLL(_build.LIB)
+            P, i32, i64, u64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_uint64
+            L.spec_workspace_size.argtypes = [P, P]
+            L.spec_workspace_size.restype = ctypes.c_size_t
+            L.spec_workspace_init.argtypes = [P, ctypes.c_size_t, P]
+            for f in ("spec_verify_attention", "spec_accept_block"):
+                getattr(L, f).argtypes = [P, P, ctypes.c_size_t, P]
+            L.spec_verify_step.argtypes = [P, P, P, ctypes.c_size_t, P]
+            L.spec_philox_uniforms.argtypes = [u64, u64, i64, P, P]
+            L.spec_read_device_status.argtypes = [P, P, ctypes.POINTER(ctypes.c_uint32)]
+            L.spec_status_string.argtypes = [ctypes.c_int]
+            L.spec_status_string.restype = ctypes.c_char_p
+            L.spec_attn_tensor_core_min_rows.restype = i32
+            for f in ("spec_workspace_init", "spec_verify_attention", "spec_accept_block",
+                      "spec_verify_step", "spec_philox_uniforms", "spec_read_device_status"):
+                getattr(L, f).restype = ctypes.c_int
+            _lib = L
+    return _lib
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream=None):
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _check(t: torch.Tensor, name: str, dtype, shape=None):
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch.Tensor")
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_cuda or not t.is_contiguous():
+        raise ValueError(f"{name} must be a contiguous CUDA tensor")
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} must have shape {tuple(shape)}, got {tuple(t.shape)}")
+
+
+def _raise(code: int, what: str):
+    if code != SPEC_OK:
+        raise SpecError(code, what)
+
+
+def attn_args(q, k_cache, v_cache, page_table, kv_len, out, lse=None, softmax_scale=0.0,
+              path=ATTN_AUTO) -> AttnArgs:
+    B, G, Hq, D = q.shape
+    num_pages, Hkv, P, D2 = k_cache.shape
+    _check(q, "q", torch.bfloat16)
+    _check(k_cache, "k_cache", torch.bfloat16)
+    _check(v_cache, "v_cache", torch.bfloat16, k_cache.shape)
+    _check(page_table, "page_table", torch.int32)
+    _check(kv_len, "kv_len", torch.int32, (B,))
+    _check(out, "out", torch.bfloat16, q.shape)
+    if lse is not None:
+        _check(lse, "lse", torch.float32, (B, G, Hq))
+    if D2 != D or page_table.dim() != 2 or page_table.shape[0] != B:
+        raise ValueError("inconsistent attention shapes")
+    return AttnArgs(B, G, Hq, Hkv, D, P, page_table.shape[1], num_pages, float(softmax_scale),
+                    int(path), q.data_ptr(), k_cache.data_ptr(), v_cache.data_ptr(),
+                    page_table.data_ptr(), kv_len.data_ptr(), out.data_ptr(),
+                    None if lse is None else lse.data_ptr())
+
+
+def accept_args(target_logits, drafter_logits, block_tokens, temperature, uniforms, num_accepted,
+                out_tokens, num_emitted, diag=None) -> AcceptArgs:
+    B, G, V = target_logits.shape
+    if target_logits.dtype == torch.bfloat16:
+        dt = SPEC_BF16
+    elif target_logits.dtype == torch.float32:
+        dt = SPEC_F32
+    else:
+        raise TypeError("logits must be bfloat16 or float32")
+    _check(target_logits, "target_logits", target_logits.dtype)
+    _check(drafter_logits, "drafter_logits", target_logits.dtype, target_logits.shape)
+    _check(block_tokens, "block_tokens", torch.int32, (B, G))
+    _check(temperature, "temperature", torch.float32, (B,))
+    _check(uniforms, "uniforms", torch.float32, (B, G))
+    _check(num_accepted, "num_accepted", torch.int32, (B,))
+    _check(out_tokens, "out_tokens", torch.int32, (B, G + 1))
+    _check(num_emitted, "num_emitted", torch.int32, (B,))
+    if diag is not None:
+        _check(diag, "diag", torch.float32, (B, G, 2))
+    return AcceptArgs(B, G, V, dt, target_logits.data_ptr(), drafter_logits.data_ptr(),
+                      block_tokens.data_ptr(), temperature.data_ptr(), uniforms.data_ptr(),
+                      num_accepted.data_ptr(), out_tokens.data_ptr(), num_emitted.data_ptr(),
+                      None if diag is None else diag.data_ptr())
+
+
+def workspace_size(attn: Optional[AttnArgs] = None, accept: Optional[AcceptArgs] = None) -> int:
+    n = lib().spec_workspace_size(None if attn is None else ctypes.byref(attn),
+                                  None if accept is None else ctypes.byref(accept))
+    if n == 0:
+        raise SpecError(1, "spec_workspace_size")
+    return int(n)
+
+
+def new_workspace(nbytes: int, device=None) -> torch.Tensor:
+    """A zero-filled workspace tensor (torch's allocator is 512-byte aligned)."""
+    return torch.zeros(int(nbytes), dtype=torch.uint8, device=device or "cuda")
+
+
+def verify_attention_args(attn: AttnArgs, ws: torch.Tensor, stream=None):
+    _raise(lib().spec_verify_attention(ctypes.byref(attn), _ptr(ws), ws.numel(), _stream(stream)),
+           "spec_verify_attention")
+
+
+def accept_block_args(acc: AcceptArgs, ws: torch.Tensor, stream=None):
+    _raise(lib().spec_accept_block(ctypes.byref(acc), _ptr(ws), ws.numel(), _stream(stream)),
+           "spec_accept_block")
+
+
+def verify_step_args(attn: Optional[AttnArgs], acc: Optional[AcceptArgs], ws: torch.Tensor,
+                     stream=None):
+    _raise(lib().spec_verify_step(None if attn is None else ctypes.byref(attn),
+                                  None if acc is None else ctypes.byref(acc), _ptr(ws),
+                                  ws.numel(), _stream(stream)), "spec_verify_step")
+
+
+def verify_attention(q, k_cache, v_cache, page_table, kv_len, softmax_scale=0.0, path=ATTN_AUTO,
+                     want_lse=True, ws=None, stream=None):
+    """Block-causal paged GQA verify attention. Returns (out bf16, lse fp32 or None)."""
+    out = torch.empty_like(q)
+    lse = torch.empty(q.shape[:3], dtype=torch.float32, device=q.device) if want_lse else None
+    a = attn_args(q, k_cache, v_cache, page_table, kv_len, out, lse, softmax_scale, path)
+    if ws is None:
+        ws = new_workspace(workspace_size(attn=a), q.device)
+    verify_attention_args(a, ws, stream)
+    return out, lse
+
+
+def accept_block(target_logits, drafter_logits, block_tokens, temperature, uniforms,
+                 want_diag=True, ws=None, stream=None) -> Dict[str, torch.Tensor]:
+    """Lossless acceptance over a batch. Returns num_accepted, out_tokens, num_emitted, diag."""
+    B, G, _ = target_logits.shape
+    dev = target_logits.device
+    res = dict(num_accepted=torch.empty(B, dtype=torch.int32, device=dev),
+               out_tokens=torch.empty(B, G + 1, dtype=torch.int32, device=dev),
+               num_emitted=torch.empty(B, dtype=torch.int32, device=dev),
+               diag=torch.empty(B, G, 2, dtype=torch.float32, device=dev) if want_diag else None)
+    a = accept_args(target_logits, drafter_logits, block_tokens, temperature, uniforms,
+                    res["num_accepted"], res["out_tokens"], res["num_emitted"], res["diag"])
+    if ws is None:
+        ws = new_workspace(workspace_size(accept=a), dev)
+    accept_block_args(a, ws, stream)
+    return res
+
+
+def philox_uniforms(seed: int, n: int, offset: int = 0, device=None, stream=None) -> torch.Tensor:
+    out = torch.empty(n, dtype=torch.float32, device=device or "cuda")
+    _raise(lib().spec_philox_uniforms(ctypes.c_uint64(seed), ctypes.c_uint64(offset), n,
+                                      _ptr(out), _stream(stream)), "spec_philox_uniforms")
+    return out
+
+
+def read_device_status(ws: torch.Tensor, stream=None):
+    """(status code, flags) of the workspace status word; reading clears it."""
+    flags = ctypes.c_uint32(0)
+    code = lib().spec_read_device_status(_ptr(ws), _stream(stream), ctypes.byref(flags))
+    return int(code), int(flags.value)
+
+
+def tensor_core_min_rows() -> int:
+    return int(lib().spec_attn_tensor_core_min_rows())

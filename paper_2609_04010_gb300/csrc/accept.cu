@@ -1,0 +1,615 @@
+// Part (b) of the verify step: vocabulary-wide softmax statistics of the target and
+// drafter rows and the lossless acceptance rule of Alg. "Lossless Psi-Spec decoding
+// (Linear Sampler)" (Appendix B.3; Sec. 4.2).
+//
+// Two launches, no inter-block waiting:
+//   1. row_stats_kernel: one block per (sequence, row, 8192-entry vocab chunk) reads
+//      the chunk once with 16-byte loads and writes its max, its sum of
+//      exp((l - max)/T) and (greedy rows) its lowest-index argmax.
+//   2. decide_sample_kernel: grid (vocab slice, sequence). Every block merges the row
+//      statistics of its sequence and evaluates the gamma-1 decisions
+//      r_i > min(1, p_i(t_i)/q_i(t_i)) (fp64 on the few gathered logits), which fixes
+//      n. Each block then sums the final draw's weights ([p_n - q_n]_+, or p_B for the
+//      bonus) over its slice; the last block of the sequence to finish (atomic ticket)
+//      finds the slice where the ascending cumulative sum crosses u * S and rescans
+//      that slice with a block-wide scan to pick the token.
+#include <cfloat>
+#include <climits>
+#include <cmath>
+
+#include "common.cuh"
+
+namespace specv {
+
+AcceptLayout accept_layout(const spec_accept_args_t& a, size_t base) {
+  AcceptLayout L;
+  L.nchunk = (a.vocab + kStatsChunk - 1) / kStatsChunk;
+  L.nslice = (a.vocab + kSampleSlice - 1) / kSampleSlice;
+  const size_t nrows = 2 * static_cast<size_t>(a.gamma) - 1;
+  L.tickets = base;
+  L.partials = ws_round(L.tickets + sizeof(uint32_t) * a.batch);
+  L.slice_sums = ws_round(L.partials + sizeof(RowPartial) * a.batch * nrows * L.nchunk);
+  L.end = ws_round(L.slice_sums + sizeof(float4) * a.batch * L.nslice);
+  return L;
+}
+
+namespace {
+
+struct SliceSum {  // per (sequence, vocab slice) sums of the final draw's weights
+  float w;         // sum of [p_n - q_n]_+ (residual)
+  float e;         // sum of exp((l_p - M_p)/T) (bonus, and the empty-residual fallback)
+  int32_t wlast;   // last index with positive residual weight, -1 if none
+  int32_t elast;   // last index with positive bonus weight, -1 if none
+};
+
+struct AcceptParams {
+  int batch, gamma, vocab, nchunk, nslice;
+  const void* target;
+  const void* drafter;
+  const int32_t* tokens;
+  const float* temperature;
+  const float* uniforms;
+  int32_t* num_accepted;
+  int32_t* out_tokens;
+  int32_t* num_emitted;
+  float* diag;
+  uint32_t* status;
+  uint32_t* tickets;
+  RowPartial* partials;
+  SliceSum* slices;
+};
+
+template <bool BF16>
+__device__ __forceinline__ float load_elem(const void* base, int64_t i) {
+  if (BF16) return bf16_bits_to_f32(static_cast<const uint16_t*>(base)[i]);
+  return static_cast<const float*>(base)[i];
+}
+
+// Loads kPer consecutive-or-strided values of a row into registers.
+// VEC: element groups of 16 bytes, group g of thread t at g*threads + t (coalesced).
+template <bool BF16, bool VEC, int kPer, int kThreads>
+__device__ __forceinline__ void load_strided(const void* row, int start, int len, float* v,
+                                             int* idx) {
+  const int t = threadIdx.x;
+  if (VEC) {
+    constexpr int kEpv = BF16 ? 8 : 4;
+    constexpr int kVecs = kPer / kEpv;
+    uint4 raw[kVecs];
+#pragma unroll
+    for (int k = 0; k < kVecs; ++k) {
+      const int e = (k * kThreads + t) * kEpv;
+      if (e < len) {
+        const char* p = static_cast<const char*>(row) + static_cast<int64_t>(start + e) * (BF16 ? 2 : 4);
+        raw[k] = __ldg(reinterpret_cast<const uint4*>(p));
+      } else {
+        raw[k] = make_uint4(0xff800000u, 0xff800000u, 0xff800000u, 0xff800000u);
+      }
+    }
+#pragma unroll
+    for (int k = 0; k < kVecs; ++k) {
+      const int e = (k * kThreads + t) * kEpv;
+      const uint32_t w[4] = {raw[k].x, raw[k].y, raw[k].z, raw[k].w};
+#pragma unroll
+      for (int q = 0; q < kEpv; ++q) {
+        float x;
+        if (BF16) {
+          const uint32_t h = (q & 1) ? (w[q >> 1] >> 16) : (w[q >> 1] & 0xffffu);
+          x = bf16_bits_to_f32(h);
+        } else {
+          x = __uint_as_float(w[q]);
+        }
+        const bool ok = e + q < len;
+        v[k * kEpv + q] = ok ? x : -INFINITY;
+        idx[k * kEpv + q] = ok ? start + e + q : INT_MAX;
+      }
+    }
+  } else {
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) {
+      const int e = k * kThreads + t;
+      const bool ok = e < len;
+      v[k] = ok ? load_elem<BF16>(row, start + e) : -INFINITY;
+      idx[k] = ok ? start + e : INT_MAX;
+    }
+  }
+}
+
+// (m, s) pairs of an online softmax sum in base 2 with scale c: value = s * 2^{c*m}.
+__device__ __forceinline__ void merge_ms(float& m, float& s, float m2, float s2, float c) {
+  const float mn = fmaxf(m, m2);
+  float r = 0.f;
+  if (m != -INFINITY) r += s * ex2((m - mn) * c);
+  if (m2 != -INFINITY) r += s2 * ex2((m2 - mn) * c);
+  m = mn;
+  s = r;
+}
+
+__device__ __forceinline__ void merge_arg(float& m, int& a, float m2, int a2) {
+  if (m2 > m || (m2 == m && a2 < a)) {
+    m = m2;
+    a = a2;
+  }
+}
+
+template <bool BF16, bool VEC>
+__global__ void __launch_bounds__(kStatsThreads) row_stats_kernel(AcceptParams p) {
+  constexpr int kPer = kStatsChunk / kStatsThreads;  // 32 values per thread
+  __shared__ float sh_m[kStatsThreads / 32];
+  __shared__ float sh_s[kStatsThreads / 32];
+  __shared__ int sh_a[kStatsThreads / 32];
+  __shared__ uint32_t sh_bad[kStatsThreads / 32];
+
+  const int nrows = 2 * p.gamma - 1;
+  const int64_t item = blockIdx.x;
+  const int c = static_cast<int>(item % p.nchunk);
+  const int r = static_cast<int>((item / p.nchunk) % nrows);
+  const int b = static_cast<int>(item / (static_cast<int64_t>(p.nchunk) * nrows));
+  const float T = p.temperature[b];
+  const bool greedy = !(T > 0.f);
+  if (greedy && r >= p.gamma) return;  // greedy sequences never read drafter rows
+  const int64_t row = static_cast<int64_t>(b) * p.gamma + (r < p.gamma ? r : r - p.gamma + 1);
+  const void* base = r < p.gamma ? p.target : p.drafter;
+  const void* rowp = static_cast<const char*>(base) + row * p.vocab * (BF16 ? 2 : 4);
+  const int start = c * kStatsChunk;
+  const int len = min(kStatsChunk, p.vocab - start);
+
+  float v[kPer];
+  int idx[kPer];
+  load_strided<BF16, VEC, kPer, kStatsThreads>(rowp, start, len, v, idx);
+
+  uint32_t bad = 0;
+  float m = -INFINITY;
+  int a = idx[0];
+#pragma unroll
+  for (int k = 0; k < kPer; ++k) {
+    bad |= !(v[k] <= FLT_MAX) && idx[k] != INT_MAX;  // NaN or +inf inside the row
+    if (greedy) {
+      if (v[k] > m) { m = v[k]; a = idx[k]; }
+    } else {
+      m = fmaxf(m, v[k]);
+    }
+  }
+  const float cs = greedy ? 0.f : kLog2e / T;
+  float s = 0.f;
+  if (!greedy && m != -INFINITY) {
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) s += ex2((v[k] - m) * cs);
+  }
+  // warp then block reduction
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
+    const float s2 = __shfl_xor_sync(0xffffffffu, s, o);
+    const int a2 = __shfl_xor_sync(0xffffffffu, a, o);
+    bad |= __shfl_xor_sync(0xffffffffu, bad, o);
+    if (greedy) merge_arg(m, a, m2, a2);
+    else merge_ms(m, s, m2, s2, cs);
+  }
+  const int w = threadIdx.x >> 5;
+  if ((threadIdx.x & 31) == 0) {
+    sh_m[w] = m; sh_s[w] = s; sh_a[w] = a; sh_bad[w] = bad;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    for (int k = 1; k < kStatsThreads / 32; ++k) {
+      if (greedy) merge_arg(m, a, sh_m[k], sh_a[k]);
+      else merge_ms(m, s, sh_m[k], sh_s[k], cs);
+      bad |= sh_bad[k];
+    }
+    RowPartial out;
+    out.m = m;
+    out.s = s;
+    out.arg = a;
+    out.bad = bad;
+    p.partials[(static_cast<int64_t>(b) * nrows + r) * p.nchunk + c] = out;
+  }
+}
+
+// Block-wide exclusive and inclusive scan of one float per thread, in thread order.
+template <int kThreads>
+__device__ __forceinline__ void block_scan(float x, float& excl, float& incl, float* sh) {
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  float in = x;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const float y = __shfl_up_sync(0xffffffffu, in, o);
+    if (lane >= o) in += y;
+  }
+  float ex = __shfl_up_sync(0xffffffffu, in, 1);
+  if (lane == 0) ex = 0.f;
+  if (lane == 31) sh[w] = in;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float run = 0.f;
+    for (int k = 0; k < kThreads / 32; ++k) {
+      const float t = sh[k];
+      sh[k] = run;
+      run += t;
+    }
+    sh[kThreads / 32] = run;
+  }
+  __syncthreads();
+  excl = sh[w] + ex;
+  incl = sh[w] + in;
+}
+
+// The weights of the final draw on this thread's contiguous run of one slice.
+template <bool BF16, bool VEC>
+__device__ __forceinline__ void final_weights(const AcceptParams& p, const void* prow,
+                                              const void* qrow, bool bonus, int start, float c,
+                                              float Mp, float invSp, float Mq, float invSq,
+                                              float* w, float* e, int& first) {
+  constexpr int kPer = kSamplePerThread;
+  first = start + threadIdx.x * kPer;
+  float lp[kPer], lq[kPer];
+  const int n = min(kPer, p.vocab - first);
+  if (VEC && n == kPer) {
+    constexpr int kEpv = BF16 ? 8 : 4;
+#pragma unroll
+    for (int k = 0; k < kPer / kEpv; ++k) {
+      const int64_t off = static_cast<int64_t>(first + k * kEpv) * (BF16 ? 2 : 4);
+      const uint4 rp = __ldg(reinterpret_cast<const uint4*>(static_cast<const char*>(prow) + off));
+      uint4 rq = make_uint4(0, 0, 0, 0);
+      if (!bonus) rq = __ldg(reinterpret_cast<const uint4*>(static_cast<const char*>(qrow) + off));
+      const uint32_t wp[4] = {rp.x, rp.y, rp.z, rp.w};
+      const uint32_t wq[4] = {rq.x, rq.y, rq.z, rq.w};
+#pragma unroll
+      for (int q = 0; q < kEpv; ++q) {
+        if (BF16) {
+          lp[k * kEpv + q] = bf16_bits_to_f32((q & 1) ? (wp[q >> 1] >> 16) : (wp[q >> 1] & 0xffffu));
+          lq[k * kEpv + q] = bf16_bits_to_f32((q & 1) ? (wq[q >> 1] >> 16) : (wq[q >> 1] & 0xffffu));
+        } else {
+          lp[k * kEpv + q] = __uint_as_float(wp[q]);
+          lq[k * kEpv + q] = __uint_as_float(wq[q]);
+        }
+      }
+    }
+  } else {
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) {
+      lp[k] = k < n ? load_elem<BF16>(prow, first + k) : -INFINITY;
+      lq[k] = (k < n && !bonus) ? load_elem<BF16>(qrow, first + k) : -INFINITY;
+    }
+  }
+#pragma unroll
+  for (int k = 0; k < kPer; ++k) {
+    const float ep = ex2((lp[k] - Mp) * c);
+    e[k] = ep;
+    w[k] = bonus ? 0.f : fmaxf(0.f, ep * invSp - ex2((lq[k] - Mq) * c) * invSq);
+  }
+}
+
+template <bool BF16, bool VEC>
+__global__ void __launch_bounds__(kSampleThreads) decide_sample_kernel(AcceptParams p) {
+  constexpr int kMaxGamma = 64;
+  constexpr int kPer = kSamplePerThread;
+  __shared__ float rM[2 * kMaxGamma], rS[2 * kMaxGamma];
+  __shared__ int rA[2 * kMaxGamma];
+  __shared__ int s_tok[kMaxGamma];
+  __shared__ float s_ptok[kMaxGamma], s_qtok[kMaxGamma];
+  __shared__ int s_bad, s_n, s_last, s_star, s_use_res, s_owner, s_token;
+  __shared__ float s_base, s_target;
+  __shared__ float sh_scan[kSampleThreads / 32 + 1];
+
+  const int b = blockIdx.y, sl = blockIdx.x, tid = threadIdx.x;
+  const int gamma = p.gamma, V = p.vocab, nrows = 2 * gamma - 1;
+  const float T = p.temperature[b];
+  const bool greedy = !(T > 0.f);
+  const float c = greedy ? 0.f : kLog2e / T;
+  if (tid == 0) {
+    s_bad = 0;
+    s_n = gamma;
+    s_owner = INT_MAX;
+    s_token = -1;
+  }
+  __syncthreads();
+
+  // 1. merge the chunk statistics of every row this sequence uses
+  const int rows_needed = greedy ? gamma : nrows;
+  for (int r = tid; r < rows_needed; r += kSampleThreads) {
+    const RowPartial* rp = p.partials + (static_cast<int64_t>(b) * nrows + r) * p.nchunk;
+    float M = -INFINITY;
+    int A = INT_MAX;
+    uint32_t bad = 0;
+    for (int k = 0; k < p.nchunk; ++k) {
+      const RowPartial q = rp[k];
+      bad |= q.bad;
+      if (A == INT_MAX || q.m > M) { M = q.m; A = q.arg; }
+    }
+    float S = 0.f;
+    if (!greedy) {
+      for (int k = 0; k < p.nchunk; ++k) {
+        const RowPartial q = rp[k];
+        if (q.m != -INFINITY) S += q.s * ex2((q.m - M) * c);
+      }
+      if (M == -INFINITY || !(S > 0.f) || !(S <= FLT_MAX)) bad = 1;
+    }
+    rM[r] = M;
+    rS[r] = S;
+    rA[r] = A;
+    if (bad) atomicOr(&s_bad, 1);
+  }
+  if (tid < gamma) {
+    const int t = p.tokens[static_cast<int64_t>(b) * gamma + tid];
+    s_tok[tid] = t;
+    if (t < 0 || t >= V) atomicOr(&s_bad, 2);
+  }
+  __syncthreads();
+
+  const int64_t orow = static_cast<int64_t>(b) * (gamma + 1);
+  if (s_bad) {
+    if (sl == 0) {
+      for (int k = tid; k <= gamma; k += kSampleThreads) p.out_tokens[orow + k] = -1;
+      if (p.diag)
+        for (int k = tid; k < 2 * gamma; k += kSampleThreads)
+          p.diag[static_cast<int64_t>(b) * gamma * 2 + k] = NAN;
+      if (tid == 0) {
+        p.num_accepted[b] = -1;
+        p.num_emitted[b] = 0;
+        set_status(p.status, (s_bad & 2) ? SPEC_FLAG_BAD_TOKEN : SPEC_FLAG_BAD_LOGITS);
+        if ((s_bad & 3) == 3) set_status(p.status, SPEC_FLAG_BAD_LOGITS);
+      }
+    }
+    return;
+  }
+
+  // 2. the gamma-1 acceptance decisions, one per thread
+  if (tid >= 1 && tid < gamma) {
+    const int i = tid, t = s_tok[i];
+    bool reject;
+    float pt, qt;
+    if (greedy) {
+      reject = t != rA[i - 1];
+      pt = reject ? 0.f : 1.f;
+      qt = 1.f;
+    } else {
+      const int64_t prow = static_cast<int64_t>(b) * gamma + (i - 1);
+      const int64_t qrow = static_cast<int64_t>(b) * gamma + i;
+      const double lp = load_elem<BF16>(p.target, prow * V + t);
+      const double lq = load_elem<BF16>(p.drafter, qrow * V + t);
+      const double Td = static_cast<double>(T);
+      const double pd = exp((lp - static_cast<double>(rM[i - 1])) / Td) / static_cast<double>(rS[i - 1]);
+      const double qd = exp((lq - static_cast<double>(rM[gamma + i - 1])) / Td) /
+                        static_cast<double>(rS[gamma + i - 1]);
+      const double ratio = qd > 0.0 ? pd / qd : INFINITY;
+      const double u = static_cast<double>(p.uniforms[static_cast<int64_t>(b) * gamma + i - 1]);
+      reject = u > fmin(1.0, ratio);
+      pt = static_cast<float>(pd);
+      qt = static_cast<float>(qd);
+    }
+    s_ptok[i] = pt;
+    s_qtok[i] = qt;
+    if (reject) atomicMin(&s_n, i);
+  }
+  __syncthreads();
+  const int n = s_n;
+
+  auto write_outputs = [&](int final_token) {
+    for (int k = tid; k <= gamma; k += kSampleThreads)
+      p.out_tokens[orow + k] = k < n ? s_tok[k] : (k == n ? final_token : -1);
+    if (p.diag) {
+      for (int i = tid; i < gamma; i += kSampleThreads) {
+        const int64_t d = (static_cast<int64_t>(b) * gamma + i) * 2;
+        const bool taken = i >= 1 && i <= n && i < gamma;
+        p.diag[d] = i == 0 ? 0.f : (taken ? s_ptok[i] : NAN);
+        p.diag[d + 1] = i == 0 ? 0.f : (taken ? s_qtok[i] : NAN);
+      }
+    }
+    if (tid == 0) {
+      p.num_accepted[b] = n - 1;
+      p.num_emitted[b] = n + 1;
+    }
+  };
+
+  if (greedy) {
+    if (sl == 0) write_outputs(rA[n - 1]);
+    return;
+  }
+
+  // 3. sums of the final draw's weights over this block's slice
+  const bool bonus = n == gamma;
+  const void* prow = static_cast<const char*>(p.target) +
+                     (static_cast<int64_t>(b) * gamma + n - 1) * V * (BF16 ? 2 : 4);
+  const void* qrow = bonus ? prow
+                           : static_cast<const char*>(p.drafter) +
+                                 (static_cast<int64_t>(b) * gamma + n) * V * (BF16 ? 2 : 4);
+  const float Mp = rM[n - 1], invSp = 1.f / rS[n - 1];
+  const float Mq = bonus ? 0.f : rM[gamma + n - 1];
+  const float invSq = bonus ? 0.f : 1.f / rS[gamma + n - 1];
+
+  float w[kPer], e[kPer];
+  int first;
+  final_weights<BF16, VEC>(p, prow, qrow, bonus, sl * kSampleSlice, c, Mp, invSp, Mq, invSq, w,
+                           e, first);
+  float lw = 0.f, le = 0.f;
+  int wlast = -1, elast = -1;
+#pragma unroll
+  for (int k = 0; k < kPer; ++k) {
+    lw += w[k];
+    le += e[k];
+    if (w[k] > 0.f) wlast = first + k;
+    if (e[k] > 0.f) elast = first + k;
+  }
+  float ex, inw, ine;
+  block_scan<kSampleThreads>(lw, ex, inw, sh_scan);
+  const float tot_w = sh_scan[kSampleThreads / 32];
+  __syncthreads();
+  block_scan<kSampleThreads>(le, ex, ine, sh_scan);
+  const float tot_e = sh_scan[kSampleThreads / 32];
+  // last positive indices of the slice
+  int wl = wlast, el = elast;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    wl = max(wl, __shfl_xor_sync(0xffffffffu, wl, o));
+    el = max(el, __shfl_xor_sync(0xffffffffu, el, o));
+  }
+  __shared__ int sh_wl[kSampleThreads / 32], sh_el[kSampleThreads / 32];
+  if ((tid & 31) == 0) {
+    sh_wl[tid >> 5] = wl;
+    sh_el[tid >> 5] = el;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    SliceSum ss;
+    ss.w = tot_w;
+    ss.e = tot_e;
+    ss.wlast = -1;
+    ss.elast = -1;
+    for (int k = 0; k < kSampleThreads / 32; ++k) {
+      ss.wlast = max(ss.wlast, sh_wl[k]);
+      ss.elast = max(ss.elast, sh_el[k]);
+    }
+    p.slices[static_cast<int64_t>(b) * p.nslice + sl] = ss;
+    __threadfence();
+    const uint32_t prev = atomicAdd(&p.tickets[b], 1u);
+    s_last = prev == static_cast<uint32_t>(p.nslice - 1);
+    if (s_last) p.tickets[b] = 0;  // leave the counter at zero for the next call
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+
+  // 4. the last block: locate the crossing slice, then the crossing token
+  const float u = p.uniforms[static_cast<int64_t>(b) * gamma + gamma - 1];
+  if (tid == 0) {
+    const SliceSum* ss = p.slices + static_cast<int64_t>(b) * p.nslice;
+    int use_res = bonus ? 0 : 1;
+    float total = 0.f;
+    for (int k = 0; k < p.nslice; ++k) total += use_res ? __ldcg(&ss[k].w) : __ldcg(&ss[k].e);
+    if (use_res && !(total > 0.f)) {  // residual without mass: draw from p_n itself
+      use_res = 0;
+      total = 0.f;
+      for (int k = 0; k < p.nslice; ++k) total += __ldcg(&ss[k].e);
+    }
+    const float target = u * total;
+    float cum = 0.f;
+    int star = -1;
+    for (int k = 0; k < p.nslice; ++k) {
+      const float x = use_res ? __ldcg(&ss[k].w) : __ldcg(&ss[k].e);
+      if (x > 0.f && cum + x >= target) { star = k; break; }
+      cum += x;
+    }
+    if (star < 0) {  // rounding left u*S above every sum: last positive-weight token
+      for (int k = p.nslice - 1; k >= 0 && s_token < 0; --k)
+        s_token = use_res ? __ldcg(&ss[k].wlast) : __ldcg(&ss[k].elast);
+    }
+    s_star = star;
+    s_use_res = use_res;
+    s_base = cum;
+    s_target = target;
+  }
+  __syncthreads();
+  if (s_star >= 0) {
+    final_weights<BF16, VEC>(p, prow, qrow, bonus, s_star * kSampleSlice, c, Mp, invSp, Mq,
+                             invSq, w, e, first);
+    const bool use_res = s_use_res != 0;
+    float loc = 0.f;
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) loc += use_res ? w[k] : e[k];
+    float excl, incl;
+    block_scan<kSampleThreads>(loc, excl, incl, sh_scan);
+    const float base = s_base, target = s_target;
+    if (base + incl >= target) atomicMin(&s_owner, tid);
+    __syncthreads();
+    if (tid == s_owner) {
+      float run = 0.f;
+      int tok = -1, lastpos = -1;
+#pragma unroll
+      for (int k = 0; k < kPer; ++k) {
+        const float x = use_res ? w[k] : e[k];
+        run += x;
+        if (x > 0.f) {
+          lastpos = first + k;
+          if (tok < 0 && base + excl + run >= target) tok = first + k;
+        }
+      }
+      s_token = tok >= 0 ? tok : lastpos;
+    }
+    __syncthreads();
+    if (s_token < 0 && tid == 0) {  // no owner: fall back to the slice's last positive weight
+      const SliceSum* ss = p.slices + static_cast<int64_t>(b) * p.nslice + s_star;
+      s_token = use_res ? __ldcg(&ss->wlast) : __ldcg(&ss->elast);
+    }
+  }
+  __syncthreads();
+  write_outputs(s_token);
+}
+
+__global__ void philox_uniforms_kernel(uint64_t seed, uint64_t offset, int64_t n, float* out) {
+  // Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11): 10 rounds of two 32x32->64
+  // multiplies by the Philox constants, with the key advanced by the Weyl constants.
+  const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  const uint64_t g = offset + static_cast<uint64_t>(i);
+  const uint64_t blk = g >> 2;
+  uint32_t c0 = static_cast<uint32_t>(blk), c1 = static_cast<uint32_t>(blk >> 32), c2 = 0, c3 = 0;
+  uint32_t k0 = static_cast<uint32_t>(seed), k1 = static_cast<uint32_t>(seed >> 32);
+#pragma unroll
+  for (int r = 0; r < 10; ++r) {
+    if (r) {
+      k0 += 0x9E3779B9u;
+      k1 += 0xBB67AE85u;
+    }
+    const uint32_t hi0 = __umulhi(0xD2511F53u, c0), lo0 = 0xD2511F53u * c0;
+    const uint32_t hi1 = __umulhi(0xCD9E8D57u, c2), lo1 = 0xCD9E8D57u * c2;
+    const uint32_t n0 = hi1 ^ c1 ^ k0, n2 = hi0 ^ c3 ^ k1;
+    c0 = n0;
+    c1 = lo1;
+    c2 = n2;
+    c3 = lo0;
+  }
+  const uint32_t words[4] = {c0, c1, c2, c3};
+  const uint32_t x = words[g & 3];
+  out[i] = static_cast<float>((x >> 8) + 1u) * 5.9604644775390625e-8f;  // * 2^-24
+}
+
+template <bool BF16, bool VEC>
+cudaError_t launch_typed(const AcceptParams& p, cudaStream_t stream) {
+  const int64_t items = static_cast<int64_t>(p.batch) * (2 * p.gamma - 1) * p.nchunk;
+  row_stats_kernel<BF16, VEC><<<static_cast<unsigned>(items), kStatsThreads, 0, stream>>>(p);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  decide_sample_kernel<BF16, VEC><<<dim3(p.nslice, p.batch), kSampleThreads, 0, stream>>>(p);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_accept(const spec_accept_args_t& a, const AcceptLayout& L, char* ws, int,
+                          cudaStream_t stream) {
+  AcceptParams p;
+  p.batch = a.batch;
+  p.gamma = a.gamma;
+  p.vocab = a.vocab;
+  p.nchunk = L.nchunk;
+  p.nslice = L.nslice;
+  p.target = a.target_logits;
+  p.drafter = a.drafter_logits;
+  p.tokens = a.block_tokens;
+  p.temperature = a.temperature;
+  p.uniforms = a.uniforms;
+  p.num_accepted = a.num_accepted;
+  p.out_tokens = a.out_tokens;
+  p.num_emitted = a.num_emitted;
+  p.diag = a.diag;
+  p.status = reinterpret_cast<uint32_t*>(ws);
+  p.tickets = reinterpret_cast<uint32_t*>(ws + L.tickets);
+  p.partials = reinterpret_cast<RowPartial*>(ws + L.partials);
+  p.slices = reinterpret_cast<SliceSum*>(ws + L.slice_sums);
+  const bool bf16 = a.logits_dtype == SPEC_BF16;
+  const size_t esz = bf16 ? 2 : 4;
+  const bool vec = (static_cast<size_t>(a.vocab) * esz) % 16 == 0 &&
+                   reinterpret_cast<uintptr_t>(a.target_logits) % 16 == 0 &&
+                   reinterpret_cast<uintptr_t>(a.drafter_logits) % 16 == 0;
+  if (bf16) return vec ? launch_typed<true, true>(p, stream) : launch_typed<true, false>(p, stream);
+  return vec ? launch_typed<false, true>(p, stream) : launch_typed<false, false>(p, stream);
+}
+
+cudaError_t launch_philox(uint64_t seed, uint64_t offset, int64_t n, float* out, cudaStream_t s) {
+  if (n == 0) return cudaSuccess;
+  const int64_t blocks = (n + 255) / 256;
+  philox_uniforms_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(seed, offset, n, out);
+  return cudaGetLastError();
+}
+
+}  // namespace specv

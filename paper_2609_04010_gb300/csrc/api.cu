@@ -1,0 +1,274 @@
+// The C ABI of libspecverify (include/spec_verify.h): host-side argument checks,
+// workspace layout, kernel selection and launches. No entry point allocates device
+// memory; all state lives in the caller's workspace.
+#include <cuda_runtime.h>
+
+#include <atomic>
+#include <climits>
+#include <cstring>
+
+#include "common.cuh"
+
+namespace specv {
+
+// (Hq/Hkv) * gamma at and above which SPEC_ATTN_AUTO picks the tensor-core kernel.
+constexpr int kTcMinRows = 1 << 30;
+int tc_min_rows() { return kTcMinRows; }
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+std::atomic<int> g_sm_count[kMaxDevices];  // cached multiprocessor counts (0 = unknown)
+
+int device_sm_count(int dev) {
+  if (dev < 0 || dev >= kMaxDevices) return 148;
+  int n = g_sm_count[dev].load(std::memory_order_relaxed);
+  if (n > 0) return n;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
+    n = 148;
+  g_sm_count[dev].store(n, std::memory_order_relaxed);
+  return n;
+}
+
+// Makes the stream's device current for this library's runtime; returns its SM count.
+bool bind_device(cudaStream_t stream, int* sms) {
+  int dev = 0;
+  if (stream != nullptr) {
+    if (cudaStreamGetDevice(stream, &dev) != cudaSuccess) return false;
+  } else if (cudaGetDevice(&dev) != cudaSuccess) {
+    return false;
+  }
+  int cur = -1;
+  if (cudaGetDevice(&cur) != cudaSuccess) return false;
+  if (cur != dev && cudaSetDevice(dev) != cudaSuccess) return false;
+  *sms = device_sm_count(dev);
+  return true;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+spec_status_t check_attn(const spec_attn_args_t* a) {
+  if (!a) return SPEC_ERR_INVALID_ARGUMENT;
+  if (a->batch < 1 || a->gamma < 1 || a->num_q_heads < 1 || a->num_kv_heads < 1 ||
+      a->max_pages_per_seq < 1 || a->num_pages < 1 || a->page_size < 1 || a->head_dim < 1)
+    return SPEC_ERR_INVALID_ARGUMENT;
+  if (a->num_q_heads % a->num_kv_heads != 0) return SPEC_ERR_INVALID_ARGUMENT;
+  if (!a->q || !a->k_cache || !a->v_cache || !a->page_table || !a->kv_len || !a->out)
+    return SPEC_ERR_INVALID_ARGUMENT;
+  if (!aligned16(a->q) || !aligned16(a->k_cache) || !aligned16(a->v_cache) || !aligned16(a->out))
+    return SPEC_ERR_INVALID_ARGUMENT;
+  if (!(a->softmax_scale == 0.f || (a->softmax_scale > 0.f && a->softmax_scale < 1e30f)))
+    return SPEC_ERR_INVALID_ARGUMENT;
+  if (a->path < SPEC_ATTN_AUTO || a->path > SPEC_ATTN_TENSOR_CORES) return SPEC_ERR_INVALID_ARGUMENT;
+  if (a->gamma > 64) return SPEC_ERR_UNSUPPORTED;
+  if (a->head_dim != 64 && a->head_dim != 128) return SPEC_ERR_UNSUPPORTED;
+  if (a->page_size != 16 && a->page_size != 32 && a->page_size != 64) return SPEC_ERR_UNSUPPORTED;
+  const int64_t max_keys = static_cast<int64_t>(a->max_pages_per_seq) * a->page_size;
+  if (max_keys > (1 << 30)) return SPEC_ERR_UNSUPPORTED;
+  const int64_t rows = static_cast<int64_t>(a->num_q_heads / a->num_kv_heads) * a->gamma;
+  const int64_t z = static_cast<int64_t>(a->batch) * ((rows + kSimtRowTile - 1) / kSimtRowTile);
+  if (z > 65535 || a->num_kv_heads > 65535) return SPEC_ERR_UNSUPPORTED;
+  if (static_cast<int64_t>(a->num_pages) * a->num_kv_heads * a->page_size > INT32_MAX)
+    return SPEC_ERR_UNSUPPORTED;
+  return SPEC_OK;
+}
+
+spec_status_t check_accept(const spec_accept_args_t* a) {
+  if (!a) return SPEC_ERR_INVALID_ARGUMENT;
+  if (a->batch < 1 || a->gamma < 1 || a->vocab < 1) return SPEC_ERR_INVALID_ARGUMENT;
+  if (a->logits_dtype != SPEC_F32 && a->logits_dtype != SPEC_BF16) return SPEC_ERR_INVALID_ARGUMENT;
+  if (!a->target_logits || !a->drafter_logits || !a->block_tokens || !a->temperature ||
+      !a->uniforms || !a->num_accepted || !a->out_tokens || !a->num_emitted)
+    return SPEC_ERR_INVALID_ARGUMENT;
+  if (a->gamma > 64 || a->batch > 65535) return SPEC_ERR_UNSUPPORTED;
+  const int64_t nchunk = (static_cast<int64_t>(a->vocab) + kStatsChunk - 1) / kStatsChunk;
+  if (static_cast<int64_t>(a->batch) * (2 * a->gamma - 1) * nchunk > INT32_MAX)
+    return SPEC_ERR_UNSUPPORTED;
+  const int64_t nslice = (static_cast<int64_t>(a->vocab) + kSampleSlice - 1) / kSampleSlice;
+  if (nslice > 65535) return SPEC_ERR_UNSUPPORTED;
+  return SPEC_OK;
+}
+
+int attn_ctas_per_sm(int path, int rows_per_cta) {
+  if (path == SPEC_ATTN_CUDA_CORES) return 2;
+  return rows_per_cta > 128 ? 1 : 2;
+}
+
+}  // namespace
+
+AttnPlan attn_plan(const spec_attn_args_t& a, size_t base, int num_sms, int path_override) {
+  AttnPlan P;
+  P.rows = (a.num_q_heads / a.num_kv_heads) * a.gamma;
+  int path = path_override;
+  if (path == SPEC_ATTN_AUTO)
+    path = P.rows >= tc_min_rows() ? SPEC_ATTN_TENSOR_CORES : SPEC_ATTN_CUDA_CORES;
+  P.path = path;
+  if (path == SPEC_ATTN_CUDA_CORES) {
+    P.rows_per_cta = kSimtRowTile;
+    P.key_tile = kSimtKeyTile;
+  } else {
+    P.rows_per_cta = P.rows <= 128 ? 128 : kTcMaxRows;
+    P.key_tile = kTcKeyTile;
+  }
+  P.row_tiles = (P.rows + P.rows_per_cta - 1) / P.rows_per_cta;
+  P.max_keys = a.max_pages_per_seq * a.page_size;
+  const int max_tiles = (P.max_keys + P.key_tile - 1) / P.key_tile;
+  const int64_t units = static_cast<int64_t>(a.batch) * a.num_kv_heads * P.row_tiles;
+  const int64_t target = static_cast<int64_t>(num_sms) * attn_ctas_per_sm(path, P.rows_per_cta);
+  int64_t nsplit = target / units;
+  if (nsplit < 1) nsplit = 1;
+  if (nsplit > max_tiles) nsplit = max_tiles;
+  P.tiles_per_split = static_cast<int>((max_tiles + nsplit - 1) / nsplit);
+  P.nsplit = (max_tiles + P.tiles_per_split - 1) / P.tiles_per_split;
+  const size_t slots = static_cast<size_t>(units) * P.nsplit * P.rows_per_cta;
+  P.tickets = base;
+  P.partial_o = ws_round(P.tickets + sizeof(uint32_t) * units);
+  const size_t po_bytes = P.nsplit > 1 ? slots * a.head_dim * sizeof(float) : 0;
+  P.partial_ml = ws_round(P.partial_o + po_bytes);
+  P.end = ws_round(P.partial_ml + (P.nsplit > 1 ? slots * sizeof(float2) : 0));
+  return P;
+}
+
+}  // namespace specv
+
+using namespace specv;
+
+namespace {
+
+size_t attn_region(const spec_attn_args_t& a, size_t base, int sms) {
+  size_t end = base;
+  for (int path : {SPEC_ATTN_CUDA_CORES, SPEC_ATTN_TENSOR_CORES}) {
+    const AttnPlan P = attn_plan(a, base, sms, path);
+    if (P.end > end) end = P.end;
+  }
+  return end;
+}
+
+size_t required_bytes(const spec_attn_args_t* attn, const spec_accept_args_t* accept, int sms,
+                      size_t* attn_base) {
+  size_t end = kWsHeader;
+  if (accept) end = accept_layout(*accept, kWsHeader).end;
+  if (attn_base) *attn_base = end;
+  if (attn) end = attn_region(*attn, end, sms);
+  return end;
+}
+
+spec_status_t run(const spec_attn_args_t* attn, const spec_accept_args_t* accept, void* ws,
+                  size_t ws_bytes, spec_stream_t stream_) {
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  if (!attn && !accept) return SPEC_ERR_INVALID_ARGUMENT;
+  if (attn) {
+    const spec_status_t s = check_attn(attn);
+    if (s != SPEC_OK) return s;
+  }
+  if (accept) {
+    const spec_status_t s = check_accept(accept);
+    if (s != SPEC_OK) return s;
+  }
+  if (!ws || (reinterpret_cast<uintptr_t>(ws) % kWsAlign) != 0) return SPEC_ERR_INVALID_ARGUMENT;
+  int sms = 0;
+  if (!bind_device(stream, &sms)) return SPEC_ERR_CUDA;
+  size_t attn_base = 0;
+  if (required_bytes(attn, accept, sms, &attn_base) > ws_bytes) return SPEC_ERR_WORKSPACE_TOO_SMALL;
+  char* w = static_cast<char*>(ws);
+  if (accept) {
+    const AcceptLayout L = accept_layout(*accept, kWsHeader);
+    if (launch_accept(*accept, L, w, sms, stream) != cudaSuccess) return SPEC_ERR_CUDA;
+  }
+  if (attn) {
+    const AttnPlan P = attn_plan(*attn, attn_base, sms, attn->path);
+    const cudaError_t e = P.path == SPEC_ATTN_TENSOR_CORES ? launch_attn_tc(*attn, P, w, stream)
+                                                           : launch_attn_simt(*attn, P, w, stream);
+    if (e != cudaSuccess) return SPEC_ERR_CUDA;
+  }
+  return SPEC_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t spec_workspace_size(const spec_attn_args_t* attn, const spec_accept_args_t* accept) {
+  if (attn && check_attn(attn) != SPEC_OK) return 0;
+  if (accept && check_accept(accept) != SPEC_OK) return 0;
+  // The split count depends on the SM count; size for the larger of the current
+  // device's and a 160-SM part so that a workspace fits every device it may meet.
+  int dev = 0, sms = 160;
+  if (cudaGetDevice(&dev) == cudaSuccess) {
+    const int n = device_sm_count(dev);
+    if (n > sms) sms = n;
+  } else {
+    cudaGetLastError();
+  }
+  size_t need = required_bytes(attn, accept, sms, nullptr);
+  for (int s : {148, 152, sms}) {
+    const size_t x = required_bytes(attn, accept, s, nullptr);
+    if (x > need) need = x;
+  }
+  return need;
+}
+
+spec_status_t spec_workspace_init(void* ws, size_t ws_bytes, spec_stream_t stream) {
+  if (!ws) return SPEC_ERR_INVALID_ARGUMENT;
+  return cudaMemsetAsync(ws, 0, ws_bytes, reinterpret_cast<cudaStream_t>(stream)) == cudaSuccess
+             ? SPEC_OK
+             : SPEC_ERR_CUDA;
+}
+
+spec_status_t spec_verify_attention(const spec_attn_args_t* attn, void* ws, size_t ws_bytes,
+                                    spec_stream_t stream) {
+  if (!attn) return SPEC_ERR_INVALID_ARGUMENT;
+  return run(attn, nullptr, ws, ws_bytes, stream);
+}
+
+spec_status_t spec_accept_block(const spec_accept_args_t* accept, void* ws, size_t ws_bytes,
+                                spec_stream_t stream) {
+  if (!accept) return SPEC_ERR_INVALID_ARGUMENT;
+  return run(nullptr, accept, ws, ws_bytes, stream);
+}
+
+spec_status_t spec_verify_step(const spec_attn_args_t* attn, const spec_accept_args_t* accept,
+                               void* ws, size_t ws_bytes, spec_stream_t stream) {
+  return run(attn, accept, ws, ws_bytes, stream);
+}
+
+spec_status_t spec_philox_uniforms(uint64_t seed, uint64_t offset, int64_t n, float* out_dev,
+                                   spec_stream_t stream) {
+  if (n < 0 || (n > 0 && !out_dev)) return SPEC_ERR_INVALID_ARGUMENT;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  int sms = 0;
+  if (!bind_device(s, &sms)) return SPEC_ERR_CUDA;
+  return launch_philox(seed, offset, n, out_dev, s) == cudaSuccess ? SPEC_OK : SPEC_ERR_CUDA;
+}
+
+spec_status_t spec_read_device_status(void* ws, spec_stream_t stream, uint32_t* flags_out) {
+  if (!ws || !flags_out) return SPEC_ERR_INVALID_ARGUMENT;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  int sms = 0;
+  if (!bind_device(s, &sms)) return SPEC_ERR_CUDA;
+  uint32_t flags = 0;
+  if (cudaMemcpyAsync(&flags, ws, sizeof(flags), cudaMemcpyDeviceToHost, s) != cudaSuccess)
+    return SPEC_ERR_CUDA;
+  if (cudaMemsetAsync(ws, 0, sizeof(flags), s) != cudaSuccess) return SPEC_ERR_CUDA;
+  if (cudaStreamSynchronize(s) != cudaSuccess) return SPEC_ERR_CUDA;
+  *flags_out = flags;
+  if (flags & SPEC_FLAG_TIMEOUT) return SPEC_ERR_TIMEOUT;
+  return flags ? SPEC_ERR_DEVICE_INPUT : SPEC_OK;
+}
+
+const char* spec_status_string(spec_status_t status) {
+  switch (status) {
+    case SPEC_OK: return "SPEC_OK";
+    case SPEC_ERR_INVALID_ARGUMENT: return "SPEC_ERR_INVALID_ARGUMENT";
+    case SPEC_ERR_UNSUPPORTED: return "SPEC_ERR_UNSUPPORTED";
+    case SPEC_ERR_WORKSPACE_TOO_SMALL: return "SPEC_ERR_WORKSPACE_TOO_SMALL";
+    case SPEC_ERR_CUDA: return "SPEC_ERR_CUDA";
+    case SPEC_ERR_DEVICE_INPUT: return "SPEC_ERR_DEVICE_INPUT";
+    case SPEC_ERR_TIMEOUT: return "SPEC_ERR_TIMEOUT";
+  }
+  return "unknown spec_status_t";
+}
+
+int32_t spec_attn_tensor_core_min_rows(void) { return specv::tc_min_rows(); }
+
+}  // extern "C"

@@ -1,0 +1,104 @@
+// Internal declarations shared by the CUDA translation units of libspecverify.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "spec_verify.h"
+
+namespace specv {
+
+// ----------------------------------------------------------------------------------
+// Workspace layout. Every region starts on a 256-byte boundary. The header holds the
+// status word; counters are per-call tickets that the last arriving block resets.
+// ----------------------------------------------------------------------------------
+constexpr size_t kWsAlign = 256;
+constexpr size_t kWsHeader = 256;  // [0] = status word (uint32)
+
+inline size_t ws_round(size_t x) { return (x + kWsAlign - 1) / kWsAlign * kWsAlign; }
+
+// --- acceptance ---
+constexpr int kStatsThreads = 256;
+constexpr int kStatsChunk = 8192;                          // vocab elements per row item
+constexpr int kSampleThreads = 256;
+constexpr int kSampleSlice = 8192;                         // vocab elements per sample block
+constexpr int kSamplePerThread = kSampleSlice / kSampleThreads;  // contiguous per thread
+
+struct RowPartial {  // one (sequence, row, vocab chunk) item of the row statistics
+  float m;           // max raw logit of the chunk (-inf if none finite)
+  float s;           // sum exp((l - m) / T) over the chunk (T > 0 rows)
+  int32_t arg;       // lowest index of the chunk maximum (greedy rows)
+  uint32_t bad;      // NaN / +inf seen
+};
+
+struct AcceptLayout {
+  size_t tickets;      // uint32 [batch]
+  size_t partials;     // RowPartial [batch][2*gamma-1][nchunk]
+  size_t slice_sums;   // float4 [batch][nslice] = (residual sum, p sum, residual last, p last)
+  size_t end;
+  int nchunk, nslice;
+};
+
+AcceptLayout accept_layout(const spec_accept_args_t& a, size_t base);
+
+// --- attention ---
+struct AttnPlan {
+  int path;          // SPEC_ATTN_CUDA_CORES or SPEC_ATTN_TENSOR_CORES
+  int rows;          // (Hq/Hkv) * gamma
+  int rows_per_cta;  // rows one block handles (a row tile)
+  int row_tiles;     // ceil(rows / rows_per_cta)
+  int key_tile;      // keys per pipeline step
+  int max_keys;      // max_pages_per_seq * page_size
+  int nsplit;        // KV splits per (sequence, kv head, row tile)
+  int tiles_per_split;
+  size_t tickets, partial_o, partial_ml, end;
+};
+
+AttnPlan attn_plan(const spec_attn_args_t& a, size_t base, int num_sms, int path_override);
+
+// ----------------------------------------------------------------------------------
+// Launchers (defined in the .cu files); all return cudaGetLastError() of the launch.
+// ----------------------------------------------------------------------------------
+cudaError_t launch_accept(const spec_accept_args_t& a, const AcceptLayout& L, char* ws,
+                          int num_sms, cudaStream_t stream);
+cudaError_t launch_attn_simt(const spec_attn_args_t& a, const AttnPlan& P, char* ws,
+                             cudaStream_t stream);
+cudaError_t launch_attn_tc(const spec_attn_args_t& a, const AttnPlan& P, char* ws,
+                           cudaStream_t stream);
+cudaError_t launch_philox(uint64_t seed, uint64_t offset, int64_t n, float* out, cudaStream_t s);
+
+// Rows of one CUDA-core block and of one tensor-core block.
+constexpr int kSimtRowTile = 16;
+constexpr int kSimtKeyTile = 64;
+constexpr int kSimtThreads = 128;
+constexpr int kTcKeyTile = 64;
+constexpr int kTcMaxRows = 256;  // two M = 128 tiles per block
+
+int tc_min_rows();
+
+}  // namespace specv
+
+// ----------------------------------------------------------------------------------
+// Device helpers
+// ----------------------------------------------------------------------------------
+#ifdef __CUDACC__
+namespace specv {
+
+__device__ __forceinline__ float bf16_bits_to_f32(uint32_t h) { return __uint_as_float(h << 16); }
+
+// 2^x via the PTX approximate base-2 exponential (relative error about 2^-22;
+// results below 2^-126 flush to zero).
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+__device__ __forceinline__ void set_status(uint32_t* status, uint32_t flag) {
+  atomicOr(status, flag);
+}
+
+constexpr float kLog2e = 1.4426950408889634f;
+
+}  // namespace specv
+#endif

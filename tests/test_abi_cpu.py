@@ -1,0 +1,90 @@
+"""The C ABI library on a machine without a GPU: it builds for sm_103a, loads, exports
+every function include/spec_verify.h declares, and rejects bad arguments on the host
+before touching the device."""
+
+import ctypes
+import subprocess
+
+import pytest
+
+from paper_2609_04010_gb300 import binding, build
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return binding.lib()
+
+
+def test_exports_every_declared_function(lib):
+    names = binding.declared_functions()
+    assert len(names) >= 9
+    for n in names:
+        assert hasattr(lib, n), f"{n} declared in spec_verify.h but not exported"
+    out = subprocess.run(["nm", "-D", "--defined-only", build.LIB], capture_output=True,
+                         text=True).stdout
+    exported = {l.split()[-1] for l in out.splitlines() if " T " in l}
+    assert set(names) <= exported
+
+
+def test_library_targets_sm103a(lib):
+    assert build.ARCH == ["-gencode", "arch=compute_103a,code=sm_103a"]
+
+
+def test_status_strings(lib):
+    for code, name in binding.STATUS_NAMES.items():
+        assert lib.spec_status_string(code).decode() == name
+
+
+def test_host_side_argument_checks(lib):
+    # null arguments are rejected before any CUDA call
+    assert lib.spec_verify_attention(None, None, 0, None) == 1
+    assert lib.spec_accept_block(None, None, 0, None) == 1
+    assert lib.spec_verify_step(None, None, None, 0, None) == 1
+    a = binding.AttnArgs(2, 4, 32, 8, 128, 16, 10, 20, 0.0, 0)
+    assert lib.spec_verify_attention(ctypes.byref(a), None, 0, None) == 1  # null tensors
+    acc = binding.AcceptArgs(2, 4, 1000, 1)
+    assert lib.spec_accept_block(ctypes.byref(acc), None, 0, None) == 1
+    assert lib.spec_philox_uniforms(1, 0, -1, None, None) == 1
+    assert lib.spec_read_device_status(None, None, None) == 1
+
+
+def _attn(**kw):
+    base = dict(batch=2, gamma=4, num_q_heads=32, num_kv_heads=8, head_dim=128, page_size=16,
+                max_pages_per_seq=10, num_pages=20, softmax_scale=0.0, path=0)
+    base.update(kw)
+    a = binding.AttnArgs(**base)
+    for f in ("q", "k_cache", "v_cache", "page_table", "kv_len", "out"):
+        setattr(a, f, 4096)  # fake aligned addresses: never dereferenced by the checks
+    return a
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(head_dim=96), 2), (dict(page_size=8), 2), (dict(gamma=65), 2),
+    (dict(num_q_heads=30), 1), (dict(batch=0), 1), (dict(path=7), 1),
+    (dict(softmax_scale=-1.0), 1),
+])
+def test_attention_shape_limits(lib, kw, code):
+    a = _attn(**kw)
+    assert lib.spec_verify_attention(ctypes.byref(a), ctypes.c_void_p(4096), 1 << 30, None) == code
+    assert lib.spec_workspace_size(ctypes.byref(a), None) == 0
+
+
+def test_workspace_size_is_host_only_and_grows_with_work(lib):
+    small = _attn(batch=1, max_pages_per_seq=4)
+    big = _attn(batch=8, max_pages_per_seq=300)
+    s, b = lib.spec_workspace_size(ctypes.byref(small), None), \
+        lib.spec_workspace_size(ctypes.byref(big), None)
+    assert 0 < s <= b
+    acc = binding.AcceptArgs(8, 8, 128256, 1)
+    for f in ("target_logits", "drafter_logits", "block_tokens", "temperature", "uniforms",
+              "num_accepted", "out_tokens", "num_emitted"):
+        setattr(acc, f, 4096)
+    both = lib.spec_workspace_size(ctypes.byref(big), ctypes.byref(acc))
+    assert both > b and both % 256 == 0
+
+
+def test_misaligned_workspace_rejected(lib):
+    a = _attn()
+    assert lib.spec_verify_attention(ctypes.byref(a), ctypes.c_void_p(4096 + 16), 1 << 30,
+                                     None) == 1

@@ -1,0 +1,113 @@
+"""GPU parity of block-causal paged GQA verify attention (spec_verify_attention) with
+the oracle, through the C ABI: within 1e-2 max-abs on outputs (bf16 inputs, fp32
+accumulation, bf16 outputs) and 1e-3 on the log-sum-exp."""
+
+import numpy as np
+import pytest
+import torch
+
+from paper_2609_04010_gb300 import binding
+from paper_2609_04010_gb300 import workloads as W
+
+from helpers import attn_tensors, compare_attention, gpu_attention, sample_rows
+
+pytestmark = pytest.mark.gpu
+
+PATHS = [binding.ATTN_CUDA_CORES]
+
+SMALL = [
+    dict(batch=2, gamma=4, num_q_heads=8, num_kv_heads=8, head_dim=64, page_size=16, ctx=(0, 300)),
+    dict(batch=3, gamma=8, num_q_heads=32, num_kv_heads=8, head_dim=128, page_size=16,
+         ctx=(1, 700)),
+    dict(batch=2, gamma=16, num_q_heads=32, num_kv_heads=8, head_dim=128, page_size=32,
+         ctx=(100, 500)),
+    dict(batch=2, gamma=32, num_q_heads=64, num_kv_heads=8, head_dim=128, page_size=64,
+         ctx=(200, 333)),
+    dict(batch=4, gamma=1, num_q_heads=32, num_kv_heads=8, head_dim=128, page_size=16,
+         ctx=(0, 1000)),
+    dict(batch=1, gamma=3, num_q_heads=6, num_kv_heads=2, head_dim=64, page_size=64, ctx=0),
+    dict(batch=2, gamma=64, num_q_heads=8, num_kv_heads=4, head_dim=64, page_size=16,
+         ctx=(0, 150)),
+]
+
+
+def oracle_attn(oracle_mod, inp, rows=None):
+    return oracle_mod.verify_attention(inp.q, inp.k_cache, inp.v_cache, inp.page_table,
+                                       inp.kv_len, inp.gamma, rows=rows)
+
+
+@pytest.mark.parametrize("path", PATHS)
+@pytest.mark.parametrize("case", range(len(SMALL)))
+def test_small_shapes_full(oracle_mod, case, path):
+    inp = W.make_attn_inputs(seed=case, **SMALL[case])
+    g_out, g_lse = gpu_attention(inp, path)
+    o_out, o_lse, st = oracle_attn(oracle_mod, inp)
+    assert np.all(st == 0)
+    compare_attention(g_out, g_lse, o_out, o_lse)
+
+
+@pytest.mark.parametrize("name", ["tiny", "llama8b", "serve64", "long70b"])
+def test_named_workloads_sampled(oracle_mod, name):
+    """Full-size workloads, in the launch configuration the benchmark times (automatic
+    kernel choice), on sampled (sequence, position, head) rows."""
+    inp = W.workload(name).attn_inputs(seed=0)
+    g_out, g_lse = gpu_attention(inp, binding.ATTN_AUTO)
+    rows = sample_rows(inp, 48)
+    o_out, o_lse, st = oracle_attn(oracle_mod, inp, rows)
+    assert np.all(st == 0)
+    err, lerr = compare_attention(g_out, g_lse, o_out, o_lse, rows)
+    print(f"{name}: max abs err {err:.2e}, lse err {lerr:.2e}")
+
+
+@pytest.mark.parametrize("path", PATHS)
+def test_page_order_invariance_bitwise(path):
+    inp = W.make_attn_inputs(3, 8, 32, 8, 128, 16, (50, 400), permute_pages=False, seed=11)
+    base, base_lse = gpu_attention(inp, path)
+    perm = np.random.default_rng(2).permutation(inp.num_pages)
+    inv = np.argsort(perm)
+    inp.k_cache = inp.k_cache[perm]
+    inp.v_cache = inp.v_cache[perm]
+    inp.page_table = np.where(inp.page_table >= 0, inv[np.maximum(inp.page_table, 0)],
+                              -1).astype(np.int32)
+    out, lse = gpu_attention(inp, path)
+    np.testing.assert_array_equal(out, base)
+    np.testing.assert_array_equal(lse, base_lse)
+
+
+@pytest.mark.parametrize("path", PATHS)
+def test_bad_pages_and_lengths(oracle_mod, path):
+    inp = W.make_attn_inputs(4, 4, 8, 2, 64, 16, (20, 90), seed=12)
+    inp.page_table[1, 2] = inp.num_pages + 5
+    inp.kv_len[2] = 2  # shorter than the block
+    t = attn_tensors(inp)
+    out = torch.empty_like(t[0])
+    lse = torch.empty(t[0].shape[:3], dtype=torch.float32, device="cuda")
+    a = binding.attn_args(*t, out, lse, path=path)
+    ws = binding.new_workspace(binding.workspace_size(attn=a))
+    binding.verify_attention_args(a, ws)
+    code, flags = binding.read_device_status(ws)
+    assert code == 5 and flags == (binding.FLAG_BAD_PAGE | binding.FLAG_BAD_KV_LEN)
+    o_out, o_lse, st = oracle_attn(oracle_mod, inp)
+    assert list(st) == [0, 1, 1, 0]
+    compare_attention(out.float().cpu().numpy(), lse.cpu().numpy(), o_out, o_lse)
+
+
+@pytest.mark.parametrize("path", PATHS)
+def test_garbage_in_unused_slots_is_ignored(oracle_mod, path):
+    inp = W.make_attn_inputs(2, 5, 16, 4, 128, 16, (30, 41), seed=13)
+    for b in range(2):
+        L = int(inp.kv_len[b])
+        last = inp.page_table[b, (L - 1) // 16]
+        inp.k_cache[last, :, L % 16:] = 0x7FC0  # NaN in the unused tail of the last page
+        inp.v_cache[last, :, L % 16:] = 0x7FC0
+    g_out, g_lse = gpu_attention(inp, path)
+    o_out, o_lse, _ = oracle_attn(oracle_mod, inp)
+    compare_attention(g_out, g_lse, o_out, o_lse)
+
+
+def test_deterministic_repeat():
+    inp = W.make_attn_inputs(2, 8, 32, 8, 128, 16, (500, 2000), seed=14)
+    t = attn_tensors(inp)
+    out1, lse1 = binding.verify_attention(*t)
+    out2, lse2 = binding.verify_attention(*t)
+    assert torch.equal(out1, out2) and torch.equal(lse1, lse2)

@@ -1,0 +1,74 @@
+"""GPU tests of the whole verify step and of the support entry points: the fused step
+equals its two parts, device Philox equals the generator bit for bit, and the
+library loaded is the in-tree sm_103a build."""
+
+import os
+
+import numpy as np
+import pytest
+import torch
+
+from paper_2609_04010_gb300 import binding, build
+from paper_2609_04010_gb300 import workloads as W
+
+from helpers import accept_tensors, attn_tensors, compare_accept, compare_attention, sample_rows
+
+pytestmark = pytest.mark.gpu
+
+
+def test_loaded_library_is_in_tree():
+    binding.lib()
+    maps = open("/proc/self/maps").read()
+    assert os.path.realpath(build.LIB) in maps
+
+
+@pytest.mark.parametrize("offset,n", [(0, 1), (0, 1000), (3, 4097), (2 ** 33 + 1, 100)])
+def test_philox_matches_generator(offset, n):
+    seed = 0x1234_5678_9ABC_DEF0
+    dev = binding.philox_uniforms(seed, n, offset).cpu().numpy()
+    host = W.philox_uniforms(seed, n, offset)
+    np.testing.assert_array_equal(dev.view(np.uint32), host.view(np.uint32))
+
+
+@pytest.mark.parametrize("name", ["tiny", "llama8b"])
+def test_step_equals_parts(oracle_mod, name):
+    wl = W.workload(name)
+    ai, ci = wl.attn_inputs(seed=0), wl.accept_inputs(seed=0)
+    at, ct = attn_tensors(ai), accept_tensors(ci)
+    out = torch.empty_like(at[0])
+    lse = torch.empty(at[0].shape[:3], dtype=torch.float32, device="cuda")
+    B, G = ci.batch, ci.gamma
+    res = dict(num_accepted=torch.empty(B, dtype=torch.int32, device="cuda"),
+               out_tokens=torch.empty(B, G + 1, dtype=torch.int32, device="cuda"),
+               num_emitted=torch.empty(B, dtype=torch.int32, device="cuda"),
+               diag=torch.empty(B, G, 2, dtype=torch.float32, device="cuda"))
+    a = binding.attn_args(*at, out, lse)
+    c = binding.accept_args(*ct, res["num_accepted"], res["out_tokens"], res["num_emitted"],
+                            res["diag"])
+    ws = binding.new_workspace(binding.workspace_size(a, c))
+    binding.verify_step_args(a, c, ws)
+    torch.cuda.synchronize()
+    assert binding.read_device_status(ws) == (0, 0)
+    part_out, part_lse = binding.verify_attention(*at)
+    part_acc = binding.accept_block(*ct)
+    assert torch.equal(out, part_out) and torch.equal(lse, part_lse)
+    for k in res:
+        assert torch.equal(res[k].nan_to_num(-7), part_acc[k].nan_to_num(-7)), k
+    o = oracle_mod.accept_block(ci.target_logits, ci.drafter_logits, ci.block_tokens,
+                                ci.temperature, ci.uniforms)
+    compare_accept({k: v.cpu().numpy() for k, v in res.items()}, o, G)
+    rows = sample_rows(ai, 16)
+    o_out, o_lse, _ = oracle_mod.verify_attention(ai.q, ai.k_cache, ai.v_cache, ai.page_table,
+                                                  ai.kv_len, ai.gamma, rows=rows)
+    compare_attention(out.float().cpu().numpy(), lse.cpu().numpy(), o_out, o_lse, rows)
+
+
+def test_workspace_too_small_is_rejected():
+    ci = W.make_accept_inputs(2, 4, 1000, "bf16", seed=1)
+    ct = accept_tensors(ci)
+    r = binding.accept_block(*ct)
+    c = binding.accept_args(*ct, r["num_accepted"], r["out_tokens"], r["num_emitted"], r["diag"])
+    ws = binding.new_workspace(256)
+    with pytest.raises(binding.SpecError) as e:
+        binding.accept_block_args(c, ws)
+    assert e.value.code == 3
