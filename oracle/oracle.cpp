@@ -420,12 +420,13 @@ int oracle_verify_attention(int32_t batch, int32_t gamma, int32_t num_q_heads,
       s[k] = std::exp(s[k] - m);
       l += s[k];
     }
-    for (int32_t d = 0; d < D; ++d) o[d] = 0.0;
+    std::vector<double> acc(D, 0.0);  // local: a row listed twice is computed twice
     for (int32_t k = 0; k < nvis; ++k) {
       const int64_t off = kv_offset(k);
       const double pk = s[k] / l;
-      for (int32_t d = 0; d < D; ++d) o[d] += pk * bf16_bits_to_double(v_cache[off + d]);
+      for (int32_t d = 0; d < D; ++d) acc[d] += pk * bf16_bits_to_double(v_cache[off + d]);
     }
+    for (int32_t d = 0; d < D; ++d) o[d] = acc[d];
     if (lse) lse[orow] = m + std::log(l);
   });
   return 0;

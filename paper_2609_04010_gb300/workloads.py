@@ -160,9 +160,9 @@ def make_accept_inputs(batch: int, gamma: int, vocab: int, logits_dtype: str = "
     whose verifier distribution is target row j-1); drafter row 0 is independent.
     Rows are rounded to bf16 when ``logits_dtype == "bf16"``.  Block token j is drawn
     from drafter row j at the sequence's temperature (argmax at T = 0).
-    ``temperature`` is a scalar or a per-sequence sequence.
+    ``temperature`` is a scalar or a sequence cycled over the batch.
     """
-    temps = np.broadcast_to(np.asarray(temperature, dtype=np.float32), (batch,)).copy()
+    temps = np.resize(np.asarray(temperature, dtype=np.float32).ravel(), batch)
     rng_t = _rng(seed, STREAM_TARGET)
     rng_n = _rng(seed, STREAM_DRAFT_NOISE)
     rng_s = _rng(seed, STREAM_DRAFT_SAMPLE)

@@ -101,7 +101,7 @@ def sample_rows(inp, n, seed=0):
     rows = np.stack([rng.integers(0, B, n), rng.integers(0, G, n), rng.integers(0, Hq, n)], 1)
     # always include the first and last block positions of the first sequence
     extra = np.array([[0, 0, 0], [0, G - 1, Hq - 1], [B - 1, G - 1, 0]])
-    return np.concatenate([rows, extra]).astype(np.int32)
+    return np.unique(np.concatenate([rows, extra]), axis=0).astype(np.int32)
 
 
 def compare_attention(g_out, g_lse, o_out, o_lse, rows=None):
