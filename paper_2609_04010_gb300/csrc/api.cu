@@ -12,7 +12,7 @@
 namespace specv {
 
 // (Hq/Hkv) * gamma at and above which SPEC_ATTN_AUTO picks the tensor-core kernel.
-constexpr int kTcMinRows = 1 << 30;
+constexpr int kTcMinRows = 64;
 int tc_min_rows() { return kTcMinRows; }
 
 namespace {
@@ -60,6 +60,7 @@ spec_status_t check_attn(const spec_attn_args_t* a) {
   if (!(a->softmax_scale == 0.f || (a->softmax_scale > 0.f && a->softmax_scale < 1e30f)))
     return SPEC_ERR_INVALID_ARGUMENT;
   if (a->path < SPEC_ATTN_AUTO || a->path > SPEC_ATTN_TENSOR_CORES) return SPEC_ERR_INVALID_ARGUMENT;
+  if (a->path == SPEC_ATTN_TENSOR_CORES && a->batch > kTcMaxBatch) return SPEC_ERR_UNSUPPORTED;
   if (a->gamma > 64) return SPEC_ERR_UNSUPPORTED;
   if (a->head_dim != 64 && a->head_dim != 128) return SPEC_ERR_UNSUPPORTED;
   if (a->page_size != 16 && a->page_size != 32 && a->page_size != 64) return SPEC_ERR_UNSUPPORTED;
@@ -89,11 +90,6 @@ spec_status_t check_accept(const spec_accept_args_t* a) {
   return SPEC_OK;
 }
 
-int attn_ctas_per_sm(int path, int rows_per_cta) {
-  if (path == SPEC_ATTN_CUDA_CORES) return 2;
-  return rows_per_cta > 128 ? 1 : 2;
-}
-
 }  // namespace
 
 AttnPlan attn_plan(const spec_attn_args_t& a, size_t base, int num_sms, int path_override) {
@@ -101,31 +97,43 @@ AttnPlan attn_plan(const spec_attn_args_t& a, size_t base, int num_sms, int path
   P.rows = (a.num_q_heads / a.num_kv_heads) * a.gamma;
   int path = path_override;
   if (path == SPEC_ATTN_AUTO)
-    path = P.rows >= tc_min_rows() ? SPEC_ATTN_TENSOR_CORES : SPEC_ATTN_CUDA_CORES;
+    path = (P.rows >= tc_min_rows() && a.batch <= kTcMaxBatch) ? SPEC_ATTN_TENSOR_CORES
+                                                               : SPEC_ATTN_CUDA_CORES;
   P.path = path;
+  P.max_keys = a.max_pages_per_seq * a.page_size;
+  int64_t units;
   if (path == SPEC_ATTN_CUDA_CORES) {
+    // static split grid (splits, Hkv, batch * row tiles), two blocks per SM
     P.rows_per_cta = kSimtRowTile;
     P.key_tile = kSimtKeyTile;
+    P.row_tiles = (P.rows + P.rows_per_cta - 1) / P.rows_per_cta;
+    const int max_tiles = (P.max_keys + P.key_tile - 1) / P.key_tile;
+    units = static_cast<int64_t>(a.batch) * a.num_kv_heads * P.row_tiles;
+    int64_t nsplit = static_cast<int64_t>(num_sms) * 2 / units;
+    if (nsplit < 1) nsplit = 1;
+    if (nsplit > max_tiles) nsplit = max_tiles;
+    P.tiles_per_split = static_cast<int>((max_tiles + nsplit - 1) / nsplit);
+    P.nsplit = (max_tiles + P.tiles_per_split - 1) / P.tiles_per_split;
+    P.grid = 0;
+    P.slot_rows = P.rows_per_cta;
+    P.slots = P.nsplit > 1 ? units * P.nsplit : 0;
   } else {
+    // persistent grid; the tile list of all units is cut into equal ranges
     P.rows_per_cta = P.rows <= 128 ? 128 : kTcMaxRows;
     P.key_tile = kTcKeyTile;
+    P.row_tiles = (P.rows + P.rows_per_cta - 1) / P.rows_per_cta;
+    units = static_cast<int64_t>(a.batch) * a.num_kv_heads * P.row_tiles;
+    P.nsplit = 1;
+    P.tiles_per_split = 0;
+    P.grid = num_sms * tc_ctas_per_sm(a.head_dim, P.rows_per_cta, a.batch);
+    P.slot_rows = P.rows < P.rows_per_cta ? P.rows : P.rows_per_cta;
+    P.slots = units + P.grid;
   }
-  P.row_tiles = (P.rows + P.rows_per_cta - 1) / P.rows_per_cta;
-  P.max_keys = a.max_pages_per_seq * a.page_size;
-  const int max_tiles = (P.max_keys + P.key_tile - 1) / P.key_tile;
-  const int64_t units = static_cast<int64_t>(a.batch) * a.num_kv_heads * P.row_tiles;
-  const int64_t target = static_cast<int64_t>(num_sms) * attn_ctas_per_sm(path, P.rows_per_cta);
-  int64_t nsplit = target / units;
-  if (nsplit < 1) nsplit = 1;
-  if (nsplit > max_tiles) nsplit = max_tiles;
-  P.tiles_per_split = static_cast<int>((max_tiles + nsplit - 1) / nsplit);
-  P.nsplit = (max_tiles + P.tiles_per_split - 1) / P.tiles_per_split;
-  const size_t slots = static_cast<size_t>(units) * P.nsplit * P.rows_per_cta;
   P.tickets = base;
   P.partial_o = ws_round(P.tickets + sizeof(uint32_t) * units);
-  const size_t po_bytes = P.nsplit > 1 ? slots * a.head_dim * sizeof(float) : 0;
-  P.partial_ml = ws_round(P.partial_o + po_bytes);
-  P.end = ws_round(P.partial_ml + (P.nsplit > 1 ? slots * sizeof(float2) : 0));
+  P.partial_ml =
+      ws_round(P.partial_o + static_cast<size_t>(P.slots) * P.slot_rows * a.head_dim * 4);
+  P.end = ws_round(P.partial_ml + static_cast<size_t>(P.slots) * P.slot_rows * sizeof(float2));
   return P;
 }
 
@@ -138,6 +146,7 @@ namespace {
 size_t attn_region(const spec_attn_args_t& a, size_t base, int sms) {
   size_t end = base;
   for (int path : {SPEC_ATTN_CUDA_CORES, SPEC_ATTN_TENSOR_CORES}) {
+    if (path == SPEC_ATTN_TENSOR_CORES && a.batch > kTcMaxBatch) continue;
     const AttnPlan P = attn_plan(a, base, sms, path);
     if (P.end > end) end = P.end;
   }

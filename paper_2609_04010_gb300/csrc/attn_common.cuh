@@ -16,6 +16,8 @@ struct AttnParams {
   int batch, gamma, hq, hkv, group, rows, row_tiles, rows_per_cta;
   int page_size, max_pages, num_pages;
   int nsplit, tiles_per_split;
+  int slot_rows;     // rows stored per partial slot
+  int max_keys;      // max_pages * page_size
   float scale_log2;  // softmax_scale * log2(e)
   const void* q;
   const void* k_cache;
@@ -26,8 +28,8 @@ struct AttnParams {
   float* lse;
   uint32_t* status;
   uint32_t* tickets;
-  float* partial_o;    // [unit][split][rows_per_cta][D]
-  float2* partial_ml;  // [unit][split][rows_per_cta] = (m, l); l = -1 marks a bad sequence
+  float* partial_o;    // [slot][slot_rows][D]
+  float2* partial_ml;  // [slot][slot_rows] = (m, l); l = -1 marks a bad sequence
 };
 
 inline AttnParams make_attn_params(const spec_attn_args_t& a, const AttnPlan& P, char* ws) {
@@ -45,6 +47,8 @@ inline AttnParams make_attn_params(const spec_attn_args_t& a, const AttnPlan& P,
   p.num_pages = a.num_pages;
   p.nsplit = P.nsplit;
   p.tiles_per_split = P.tiles_per_split;
+  p.slot_rows = P.slot_rows;
+  p.max_keys = P.max_keys;
   const float scale = a.softmax_scale != 0.f ? a.softmax_scale : 1.f / sqrtf(static_cast<float>(a.head_dim));
   p.scale_log2 = scale * 1.4426950408889634f;
   p.q = a.q;
@@ -86,18 +90,19 @@ __device__ __forceinline__ void write_lse(const AttnParams& p, int b, int g, int
   p.lse[(static_cast<int64_t>(b) * p.gamma + j) * p.hq + h] = v;
 }
 
-// Run by the last block of a unit: combines the nsplit partials of rows
-// [row0, row0 + nrows) and writes the final outputs.
-template <int D, int NT>
+// Run by the last block to finish a unit: combines the partials in slots
+// [slot0, slot0 + nslots) for rows [row0, row0 + nrows) and writes the final
+// outputs. Threads tid .. of nthreads cooperate.
+template <int D>
 __device__ void merge_splits(const AttnParams& p, int b, int g, int row0, int nrows,
-                             int64_t unit) {
+                             int64_t slot0, int nslots, int tid, int nthreads) {
   constexpr int DQ = D / 8;
-  for (int idx = threadIdx.x; idx < nrows * DQ; idx += NT) {
+  for (int idx = tid; idx < nrows * DQ; idx += nthreads) {
     const int r = idx / DQ, dq = idx % DQ;
     float M = -INFINITY;
     bool bad = false;
-    for (int s = 0; s < p.nsplit; ++s) {
-      const float2 ml = __ldcg(&p.partial_ml[(unit * p.nsplit + s) * p.rows_per_cta + r]);
+    for (int s = 0; s < nslots; ++s) {
+      const float2 ml = __ldcg(&p.partial_ml[(slot0 + s) * p.slot_rows + r]);
       if (ml.y < 0.f) bad = true;
       else if (ml.y > 0.f) M = fmaxf(M, ml.x);
     }
@@ -105,8 +110,8 @@ __device__ void merge_splits(const AttnParams& p, int b, int g, int row0, int nr
 #pragma unroll
     for (int e = 0; e < 8; ++e) acc[e] = 0.f;
     if (!bad) {
-      for (int s = 0; s < p.nsplit; ++s) {
-        const int64_t slot = (unit * p.nsplit + s) * p.rows_per_cta + r;
+      for (int s = 0; s < nslots; ++s) {
+        const int64_t slot = (slot0 + s) * p.slot_rows + r;
         const float2 ml = __ldcg(&p.partial_ml[slot]);
         if (!(ml.y > 0.f)) continue;
         const float w = ex2(ml.x - M);

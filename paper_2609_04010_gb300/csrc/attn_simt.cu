@@ -257,11 +257,11 @@ __global__ void __launch_bounds__(NT) attn_simt_kernel(AttnParams p) {
 #pragma unroll
   for (int i = 0; i < RPT; ++i) {
     const int r = rg + i * RG;
-    float4* dst = reinterpret_cast<float4*>(po + (slot * p.rows_per_cta + r) * D + dq * 8);
+    float4* dst = reinterpret_cast<float4*>(po + (slot * p.slot_rows + r) * D + dq * 8);
     dst[0] = make_float4(o[i][0], o[i][1], o[i][2], o[i][3]);
     dst[1] = make_float4(o[i][4], o[i][5], o[i][6], o[i][7]);
   }
-  if (tid < RT) pml[slot * p.rows_per_cta + tid] = make_float2(sm.m[tid], bad ? -1.f : sm.l[tid]);
+  if (tid < RT) pml[slot * p.slot_rows + tid] = make_float2(sm.m[tid], bad ? -1.f : sm.l[tid]);
   if (tid == 0 && bad) set_status(p.status, sm.bad == 2 ? SPEC_FLAG_BAD_KV_LEN : SPEC_FLAG_BAD_PAGE);
   __threadfence();
   __syncthreads();
@@ -273,7 +273,7 @@ __global__ void __launch_bounds__(NT) attn_simt_kernel(AttnParams p) {
   __syncthreads();
   if (!sm.last) return;
   __threadfence();
-  merge_splits<D, NT>(p, b, g, row0, nrows, unit);
+  merge_splits<D>(p, b, g, row0, nrows, unit * p.nsplit, p.nsplit, tid, NT);
 }
 
 }  // namespace

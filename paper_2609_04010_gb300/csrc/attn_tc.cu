@@ -1,10 +1,744 @@
-// Part (a) of the verify step on tcgen05 tensor cores (not built yet in this file).
+// Part (a) of the verify step on tcgen05 tensor cores: block-causal attention of the
+// gamma block queries over a paged bf16 KV cache with grouped-query heads (Sec. 4.1:
+// the prefix stays in the KV cache while the block is processed; Alg. "Lossless
+// Psi-Spec": one causal verifier pass over [x^{L+1}, x~]).
+//
+// One block holds every query row of one KV head (row r = block position j * group +
+// head-in-group), padded to M = 128 rows per tensor-core tile (two tiles when the
+// group has up to 256 rows), so each KV page is read from HBM once.
+//
+// Warp roles (one block per SM, persistent):
+//   warp 0      TMA producer: gathers each 64-key tile of K and V page by page through
+//               the page table with cp.async.bulk.tensor (128-byte swizzle) into a
+//               multi-stage ring; an mbarrier per stage carries the byte count.
+//   warp 1      MMA issuer: S = Q K^T (tcgen05.mma kind::f16, M = 128, N = 64, K = 16
+//               steps over D) into a double-buffered fp32 TMEM accumulator, then
+//               O += P V (N = D) with P from shared memory and V read MN-major.
+//   warps 4..   softmax (one warpgroup per M tile, one thread per query row): load S
+//               from TMEM, scale and mask, online softmax in base 2 with lazy rescale
+//               of O (only when the running max grows by more than 2^8), write P as
+//               bf16 in the swizzled layout the MMA reads, and finally read O from
+//               TMEM and write the output.
+// Work is balanced across blocks "stream-K" style: all 64-key tiles of all (sequence,
+// KV head, row tile) units form one list that is cut into equal contiguous ranges; a
+// unit split between blocks is merged from fp32 partials by the last block to finish
+// it (atomic ticket, no waiting). Every mbarrier wait is bounded: a wait that runs out
+// sets SPEC_FLAG_TIMEOUT, drains the block's own copies and MMAs, frees TMEM and exits.
+#include <cuda.h>  // CUtensorMap and its encoder's signature (resolved at run time)
+
 #include "attn_common.cuh"
 
 namespace specv {
+namespace {
 
-cudaError_t launch_attn_tc(const spec_attn_args_t&, const AttnPlan&, char*, cudaStream_t) {
-  return cudaErrorNotSupported;
+constexpr int TK = kTcKeyTile;               // keys per tile (MMA N of Q K^T)
+constexpr uint64_t kWaitLimitNs = 1000000000ull;  // 1 s per wait
+
+template <int D, int MT>
+struct TcCfg {
+  static constexpr int DH = D / 64;                   // 128-byte column halves of a row
+  static constexpr int STAGES = (D == 128 && MT == 2) ? 3 : 4;
+  static constexpr int THREADS = 128 + 128 * MT;
+  static constexpr uint32_t Q_BYTES = MT * DH * 16384;  // [MT][DH][128 rows x 128 B]
+  static constexpr uint32_t KV_BYTES = DH * 8192;       // one stage of K (or V): [DH][64 x 128 B]
+  static constexpr uint32_t P_BYTES = MT * 16384;       // [MT][128 rows x 128 B]
+  static constexpr uint32_t OFF_Q = 0;
+  static constexpr uint32_t OFF_K = OFF_Q + Q_BYTES;
+  static constexpr uint32_t OFF_V = OFF_K + STAGES * KV_BYTES;
+  static constexpr uint32_t OFF_P = OFF_V + STAGES * KV_BYTES;
+  static constexpr uint32_t OFF_BAR = OFF_P + P_BYTES;
+  // barriers: kv_full[S], kv_empty[S], s_full[MT][2], s_free[MT][2], p_full[MT],
+  // pv_done[MT], seg_ready, grp, drain
+  static constexpr int NBAR = 2 * STAGES + 6 * MT + 3;
+  static constexpr uint32_t OFF_MISC = OFF_BAR + NBAR * 8;  // tmem base, abort, flag
+  static constexpr uint32_t OFF_PB = (OFF_MISC + 16 + 15) / 16 * 16;
+  static constexpr uint32_t TMEM_COLS = (MT * 128 + MT * D) <= 256 ? 256 : 512;
+  static constexpr uint32_t S_COL = 0;           // S[mt][buf] at (mt * 2 + buf) * 64
+  static constexpr uint32_t O_COL = MT * 128;    // O[mt] at O_COL + mt * D
+  static size_t smem_bytes(int batch) { return OFF_PB + 4u * (batch + 1) + 1024; }
+};
+
+// ---------------------------------------------------------------------------------
+// PTX wrappers
+// ---------------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+__device__ __forceinline__ uint64_t globaltimer() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+// Bounded wait on phase `parity` of an mbarrier. On timeout (or when another role has
+// already timed out) it raises the block's abort flag and returns false.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                          uint32_t* status) {
+  if (mbar_try(bar, parity)) return true;
+  const uint64_t t0 = globaltimer();
+  for (uint32_t it = 1;; ++it) {
+    if (mbar_try(bar, parity)) return true;
+    if ((it & 63) == 0) {
+      if (*abort_flag) return false;
+      if (globaltimer() - t0 > kWaitLimitNs) {
+        *abort_flag = 1;
+        atomicOr(status, SPEC_FLAG_TIMEOUT);
+        return false;
+      }
+    }
+  }
+}
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y,
+                                            uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+      : "memory");
+}
+__device__ __forceinline__ void fence_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem),
+               "r"(ncols)
+               : "memory");
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
+                                         uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+__device__ __forceinline__ void mma_commit(uint32_t bar) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+      : "memory");
+}
+
+#define SPECV_R8(i) "=r"(r[i]), "=r"(r[i + 1]), "=r"(r[i + 2]), "=r"(r[i + 3]), \
+                    "=r"(r[i + 4]), "=r"(r[i + 5]), "=r"(r[i + 6]), "=r"(r[i + 7])
+// 32 consecutive fp32 TMEM columns of this thread's lane.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t* r) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11,"
+      " %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29,"
+      " %30, %31}, [%32];"
+      : SPECV_R8(0), SPECV_R8(8), SPECV_R8(16), SPECV_R8(24)
+      : "r"(taddr));
+}
+#undef SPECV_R8
+__device__ __forceinline__ void tmem_wait_ld() {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+#define SPECV_W8(i) "r"(r[i]), "r"(r[i + 1]), "r"(r[i + 2]), "r"(r[i + 3]), "r"(r[i + 4]), \
+                    "r"(r[i + 5]), "r"(r[i + 6]), "r"(r[i + 7])
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t* r) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11,"
+      " %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29,"
+      " %30, %31, %32};" ::"r"(taddr),
+      SPECV_W8(0), SPECV_W8(8), SPECV_W8(16), SPECV_W8(24)
+      : "memory");
+}
+#undef SPECV_W8
+__device__ __forceinline__ void tmem_wait_st() {
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+// Shared-memory matrix descriptor (tcgen05), 128-byte swizzle: start address, leading
+// and stride byte offsets (16-byte units), fixed version bits 46-47 = 1, layout 2.
+__device__ __forceinline__ uint64_t desc_sw128(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  return static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4) |
+         (static_cast<uint64_t>((lbo >> 4) & 0x3FFFu) << 16) |
+         (static_cast<uint64_t>((sbo >> 4) & 0x3FFFu) << 32) | (1ull << 46) | (2ull << 61);
+}
+// Instruction descriptor, kind::f16: fp32 accumulator, bf16 A and B, A K-major,
+// B K-major or MN-major, N >> 3 at bit 17, M >> 4 at bit 24.
+__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, bool b_mn_major) {
+  return (1u << 4) | (1u << 7) | (1u << 10) | ((b_mn_major ? 1u : 0u) << 16) |
+         (static_cast<uint32_t>(N >> 3) << 17) | (static_cast<uint32_t>(M >> 4) << 24);
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
+  const __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
+  return *reinterpret_cast<const uint32_t*>(&v);
+}
+
+// ---------------------------------------------------------------------------------
+// Work list
+// ---------------------------------------------------------------------------------
+__device__ __forceinline__ int unit_tiles(int kv_len, const AttnParams& p) {
+  const bool ok = kv_len >= p.gamma && kv_len <= p.max_keys;
+  return ok ? (kv_len + TK - 1) / TK : 1;  // a malformed sequence keeps one tile to report it
+}
+
+struct Seg {
+  int b, g, rt;      // sequence, KV head, row tile
+  int64_t u;         // unit index (b * Hkv + g) * row_tiles + rt
+  int tile0, ntile;  // first tile within the unit and tile count of this segment
+  int unit_tiles;    // tiles of the whole unit
+  int kv_len;
+  bool len_ok;
+  int64_t unit_start;  // global index of the unit's first tile
+};
+
+__device__ __forceinline__ Seg locate(int64_t t, int64_t t1, const AttnParams& p,
+                                      const int* pb) {
+  int lo = 0, hi = p.batch;  // largest b with pb[b] <= t
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (pb[mid] <= t) lo = mid; else hi = mid;
+  }
+  Seg s;
+  s.b = lo;
+  s.kv_len = p.kv_len[lo];
+  s.len_ok = s.kv_len >= p.gamma && s.kv_len <= p.max_keys;
+  s.unit_tiles = unit_tiles(s.kv_len, p);
+  const int64_t rem = t - pb[lo];
+  const int ub = static_cast<int>(rem / s.unit_tiles);
+  s.tile0 = static_cast<int>(rem % s.unit_tiles);
+  s.g = ub / p.row_tiles;
+  s.rt = ub % p.row_tiles;
+  s.u = static_cast<int64_t>(lo) * p.hkv * p.row_tiles + ub;
+  s.unit_start = t - s.tile0;
+  const int64_t end = s.unit_start + s.unit_tiles;
+  s.ntile = static_cast<int>((end < t1 ? end : t1) - t);
+  return s;
+}
+
+// Block that owns global tile t when `total` tiles are cut into `ctas` ranges
+// [c * total / ctas, (c + 1) * total / ctas).
+__device__ __forceinline__ int owner_of(int64_t t, int64_t total, int ctas) {
+  return static_cast<int>(((t + 1) * ctas - 1) / total);
+}
+
+// A segment is bad when its sequence length is malformed or a page it reads is out
+// of range. The whole warp cooperates; every lane gets the answer.
+__device__ __forceinline__ bool segment_bad(const Seg& s, const AttnParams& p) {
+  if (!s.len_ok) return true;
+  const int k0 = s.tile0 * TK;
+  const int k1 = min(s.kv_len, (s.tile0 + s.ntile) * TK);
+  const int pg0 = k0 / p.page_size, pg1 = (k1 - 1) / p.page_size;
+  bool bad = false;
+  for (int pg = pg0 + (threadIdx.x & 31); pg <= pg1; pg += 32) {
+    const int id = p.page_table[static_cast<int64_t>(s.b) * p.max_pages + pg];
+    bad |= id < 0 || id >= p.num_pages;
+  }
+  return __any_sync(0xffffffffu, bad);
+}
+
+// ---------------------------------------------------------------------------------
+// The kernel
+// ---------------------------------------------------------------------------------
+template <int D, int MT>
+__global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
+    attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
+                   const __grid_constant__ CUtensorMap tmap_v, AttnParams p) {
+  using C = TcCfg<D, MT>;
+  extern __shared__ __align__(1024) unsigned char smem_raw[];
+  unsigned char* smem = reinterpret_cast<unsigned char*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  const uint32_t sbase = smem_u32(smem);
+  const uint32_t bar0 = sbase + C::OFF_BAR;
+  auto kv_full = [&](int s) { return bar0 + 8u * s; };
+  auto kv_empty = [&](int s) { return bar0 + 8u * (C::STAGES + s); };
+  auto s_full = [&](int mt, int bf) { return bar0 + 8u * (2 * C::STAGES + mt * 2 + bf); };
+  auto s_free = [&](int mt, int bf) { return bar0 + 8u * (2 * C::STAGES + 2 * MT + mt * 2 + bf); };
+  auto p_full = [&](int mt) { return bar0 + 8u * (2 * C::STAGES + 4 * MT + mt); };
+  auto pv_done = [&](int mt) { return bar0 + 8u * (2 * C::STAGES + 5 * MT + mt); };
+  const uint32_t seg_ready = bar0 + 8u * (2 * C::STAGES + 6 * MT);
+  const uint32_t grp_bar = seg_ready + 8;
+  const uint32_t drain_bar = seg_ready + 16;
+  uint32_t* misc = reinterpret_cast<uint32_t*>(smem + C::OFF_MISC);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 1);
+  volatile int* merge_flag = reinterpret_cast<volatile int*>(misc + 2);
+  int* pb = reinterpret_cast<int*>(smem + C::OFF_PB);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  // ---- prologue: barriers, TMEM, per-sequence tile prefix sums ----
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::STAGES; ++s) {
+      mbar_init(kv_full(s), 1);
+      mbar_init(kv_empty(s), 1);
+    }
+    for (int mt = 0; mt < MT; ++mt) {
+      for (int bf = 0; bf < 2; ++bf) {
+        mbar_init(s_full(mt, bf), 1);
+        mbar_init(s_free(mt, bf), 4);
+      }
+      mbar_init(p_full(mt), 4);
+      mbar_init(pv_done(mt), 1);
+    }
+    mbar_init(seg_ready, 4 * MT);
+    mbar_init(grp_bar, 4 * MT);
+    mbar_init(drain_bar, 1);
+    *abort_flag = 0;
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 1) tmem_alloc(smem_u32(misc), C::TMEM_COLS);
+  if (warp == 0) {
+    const int per_b = p.hkv * p.row_tiles;
+    int carry = 0;
+    for (int b0 = 0; b0 < p.batch; b0 += 32) {
+      const int b = b0 + lane;
+      int v = b < p.batch ? unit_tiles(p.kv_len[b], p) * per_b : 0;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, v, o);
+        if (lane >= o) v += y;
+      }
+      if (b < p.batch) pb[b + 1] = carry + v;
+      carry += __shfl_sync(0xffffffffu, v, 31);
+    }
+    if (lane == 0) pb[0] = 0;
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = misc[0];
+
+  const int64_t total = pb[p.batch];
+  const int ctas = static_cast<int>(total < gridDim.x ? total : gridDim.x);
+  const int cta = blockIdx.x;
+  const int64_t t0 = cta < ctas ? static_cast<int64_t>(cta) * total / ctas : 0;
+  const int64_t t1 = cta < ctas ? static_cast<int64_t>(cta + 1) * total / ctas : 0;
+
+  if (warp == 0) {
+    // =========================== TMA producer ===========================
+    uint32_t it = 0;
+    bool ok = true;
+    for (int64_t t = t0; t < t1 && ok;) {
+      const Seg s = locate(t, t1, p, pb);
+      const bool bad = segment_bad(s, p);
+      for (int k = 0; k < s.ntile && ok; ++k, ++it) {
+        const int st = it % C::STAGES;
+        if (it >= static_cast<uint32_t>(C::STAGES))
+          ok = mbar_wait(kv_empty(st), ((it / C::STAGES) - 1) & 1, abort_flag, p.status);
+        if (!ok) break;
+        if (lane == 0) {
+          if (bad) {
+            mbar_arrive(kv_full(st));
+          } else {
+            const int key0 = (s.tile0 + k) * TK;
+            const int npg = TK / p.page_size;
+            int nvalid = 0;
+            for (int q = 0; q < npg; ++q) nvalid += (key0 + q * p.page_size) < s.kv_len;
+            mbar_arrive_tx(kv_full(st), static_cast<uint32_t>(nvalid) * p.page_size * D * 2 * 2);
+            for (int q = 0; q < nvalid; ++q) {
+              const int key = key0 + q * p.page_size;
+              const int page = p.page_table[static_cast<int64_t>(s.b) * p.max_pages + key / p.page_size];
+              const int y = (page * p.hkv + s.g) * p.page_size;
+              const uint32_t row_off = static_cast<uint32_t>(q * p.page_size) * 128u;
+#pragma unroll
+              for (int h = 0; h < C::DH; ++h) {
+                tma_load_2d(sbase + C::OFF_K + st * C::KV_BYTES + h * 8192u + row_off, &tmap_k,
+                            h * 64, y, kv_full(st));
+                tma_load_2d(sbase + C::OFF_V + st * C::KV_BYTES + h * 8192u + row_off, &tmap_v,
+                            h * 64, y, kv_full(st));
+              }
+            }
+          }
+        }
+        __syncwarp();
+      }
+      t += s.ntile;
+    }
+    if (!ok) {  // drain this block's copies still in flight (bounded)
+      for (uint32_t x = it > static_cast<uint32_t>(C::STAGES) ? it - C::STAGES : 0; x < it; ++x) {
+        const uint64_t t_0 = globaltimer();
+        while (!mbar_try(kv_full(x % C::STAGES), (x / C::STAGES) & 1) &&
+               globaltimer() - t_0 < kWaitLimitNs) {
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ============================ MMA issuer ============================
+    constexpr uint32_t kIdescQK = idesc_bf16(128, TK, false);
+    constexpr uint32_t kIdescPV = idesc_bf16(128, D, true);
+    uint32_t it = 0, seg_no = 0;
+    bool ok = true;
+    bool issued = false;
+    // S = Q K^T for tile x into S[mt][x & 1]; returns false on timeout.
+    auto issue_qk = [&](uint32_t x, const Seg& s, int k) -> bool {
+      const int st = x % C::STAGES;
+      if (!mbar_wait(kv_full(st), (x / C::STAGES) & 1, abort_flag, p.status)) return false;
+      // keys past the end of the sequence: zero their V rows so that P = 0 meets finite V
+      const int key0 = (s.tile0 + k) * TK;
+      const int nvalid = s.len_ok ? min(TK, max(0, s.kv_len - key0)) : TK;
+      if (nvalid < TK) {
+        for (int h = 0; h < C::DH; ++h) {
+          uint4* vrow = reinterpret_cast<uint4*>(smem + C::OFF_V + st * C::KV_BYTES + h * 8192u +
+                                                 nvalid * 128u);
+          for (int i = lane; i < (TK - nvalid) * 8; i += 32) vrow[i] = make_uint4(0, 0, 0, 0);
+        }
+        fence_async_smem();
+      }
+      __syncwarp();
+      if (x >= 2)
+        for (int mt = 0; mt < MT; ++mt)
+          if (!mbar_wait(s_free(mt, x & 1), ((x >> 1) - 1) & 1, abort_flag, p.status)) return false;
+      tc_fence_after();
+      if (lane == 0) {
+        for (int mt = 0; mt < MT; ++mt) {
+          const uint32_t d_tmem = tmem + C::S_COL + (mt * 2 + (x & 1)) * TK;
+#pragma unroll
+          for (int kk = 0; kk < D / 16; ++kk) {
+            const uint32_t qa = sbase + C::OFF_Q + (mt * C::DH + kk / 4) * 16384u + (kk % 4) * 32u;
+            const uint32_t kb = sbase + C::OFF_K + st * C::KV_BYTES + (kk / 4) * 8192u + (kk % 4) * 32u;
+            mma_bf16(d_tmem, desc_sw128(qa, 16, 1024), desc_sw128(kb, 16, 1024), kIdescQK, kk > 0);
+          }
+          mma_commit(s_full(mt, x & 1));
+        }
+      }
+      __syncwarp();
+      return true;
+    };
+    for (int64_t t = t0; t < t1 && ok;) {
+      const Seg s = locate(t, t1, p, pb);
+      ok = mbar_wait(seg_ready, seg_no & 1, abort_flag, p.status);
+      if (!ok) break;
+      tc_fence_after();
+      for (int k = 0; k < s.ntile && ok; ++k) {
+        const uint32_t x = it + k;
+        if (k == 0) ok = issue_qk(x, s, 0);
+        if (ok && k + 1 < s.ntile) ok = issue_qk(x + 1, s, k + 1);
+        for (int mt = 0; mt < MT && ok; ++mt) ok = mbar_wait(p_full(mt), x & 1, abort_flag, p.status);
+        if (!ok) break;
+        tc_fence_after();
+        if (lane == 0) {
+          const int st = x % C::STAGES;
+          for (int mt = 0; mt < MT; ++mt) {
+            const uint32_t d_tmem = tmem + C::O_COL + mt * D;
+#pragma unroll
+            for (int kk = 0; kk < TK / 16; ++kk) {
+              const uint32_t pa = sbase + C::OFF_P + mt * 16384u + kk * 32u;
+              const uint32_t vb = sbase + C::OFF_V + st * C::KV_BYTES + kk * 2048u;
+              mma_bf16(d_tmem, desc_sw128(pa, 16, 1024), desc_sw128(vb, 8192, 1024), kIdescPV,
+                       (k > 0 || kk > 0) ? 1u : 0u);
+            }
+            mma_commit(pv_done(mt));
+          }
+          mma_commit(kv_empty(st));
+          issued = true;
+        }
+        __syncwarp();
+      }
+      it += s.ntile;
+      t += s.ntile;
+      ++seg_no;
+    }
+    if (!ok && __any_sync(0xffffffffu, issued)) {  // drain this block's MMAs (bounded)
+      if (lane == 0) mma_commit(drain_bar);
+      __syncwarp();
+      const uint64_t t_0 = globaltimer();
+      while (!mbar_try(drain_bar, 0) && globaltimer() - t_0 < kWaitLimitNs) {
+      }
+    }
+  } else if (warp >= 4) {
+    // ============================== softmax ==============================
+    const int sw = warp - 4, mt = sw >> 2, q4 = sw & 3;
+    const int row = q4 * 32 + lane;  // TMEM lane = row of this M tile
+    const uint32_t lane_base = tmem + (static_cast<uint32_t>(q4 * 32) << 16);
+    const int gtid = threadIdx.x - 128, gthreads = 128 * MT;
+    uint32_t it = 0, gphase = 0;
+    bool ok = true;
+    unsigned char* prow = smem + C::OFF_P + mt * 16384u + row * 128u;
+    auto group_sync = [&]() -> bool {
+      __syncwarp();
+      if (lane == 0) mbar_arrive(grp_bar);
+      const bool r = mbar_wait(grp_bar, gphase & 1, abort_flag, p.status);
+      ++gphase;
+      return r;
+    };
+    for (int64_t t = t0; t < t1 && ok;) {
+      const Seg s = locate(t, t1, p, pb);
+      const bool bad = segment_bad(s, p);
+      const int row0 = s.rt * p.rows_per_cta;
+      const int lrow = mt * 128 + row;           // row within the block's row tile
+      const int urow = row0 + lrow;              // row within the unit (j * group + hh)
+      const bool real = urow < p.rows && lrow < p.rows_per_cta;
+      const int j = urow / p.group, h = s.g * p.group + urow % p.group;
+      // queries of this row into the swizzled Q tile (zeros for padding rows)
+      {
+        const uint4* src = reinterpret_cast<const uint4*>(
+            static_cast<const __nv_bfloat16*>(p.q) +
+            ((static_cast<int64_t>(s.b) * p.gamma + (real ? j : 0)) * p.hq + (real ? h : 0)) * D);
+#pragma unroll
+        for (int c = 0; c < D / 8; ++c) {
+          const uint4 v = real ? __ldg(src + c) : make_uint4(0, 0, 0, 0);
+          const int half = c >> 3, ch = c & 7;
+          *reinterpret_cast<uint4*>(smem + C::OFF_Q + (mt * C::DH + half) * 16384u + row * 128u +
+                                    ((ch ^ (row & 7)) << 4)) = v;
+        }
+      }
+      fence_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(seg_ready);
+
+      const int ctx = s.kv_len - p.gamma;
+      float m = -INFINITY, l = 0.f;
+      for (int k = 0; k < s.ntile; ++k) {
+        const uint32_t x = it + k;
+        ok = mbar_wait(s_full(mt, x & 1), (x >> 1) & 1, abort_flag, p.status);
+        if (!ok) break;
+        tc_fence_after();
+        float v[TK];
+        {
+          uint32_t r[32];
+          const uint32_t col = C::S_COL + (mt * 2 + (x & 1)) * TK;
+          tmem_ld32(lane_base + col, r);
+          tmem_wait_ld();
+#pragma unroll
+          for (int c = 0; c < 32; ++c) v[c] = __uint_as_float(r[c]);
+          tmem_ld32(lane_base + col + 32, r);
+          tmem_wait_ld();
+#pragma unroll
+          for (int c = 0; c < 32; ++c) v[32 + c] = __uint_as_float(r[c]);
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(s_free(mt, x & 1));
+        // scale to base 2 and mask keys past ctx + j
+        const int key0 = (s.tile0 + k) * TK;
+        const int lim = ctx + j - key0;  // keys c <= lim are visible
+        float tmax = -INFINITY;
+#pragma unroll
+        for (int c = 0; c < TK; ++c) {
+          v[c] = c <= lim ? v[c] * p.scale_log2 : -INFINITY;
+          tmax = fmaxf(tmax, v[c]);
+        }
+        const float m_new = fmaxf(m, tmax);
+        const bool want = k > 0 && m_new > m + 8.f;
+        const bool rescale = __any_sync(0xffffffffu, want);
+        float alpha = 1.f;
+        if (k == 0) {
+          m = m_new;
+        } else if (rescale) {
+          alpha = m == -INFINITY ? 0.f : ex2(m - m_new);
+          m = m_new;
+        }
+        const float msub = m == -INFINITY ? 0.f : m;
+        uint32_t pk[TK / 2];
+        float sum = 0.f;
+#pragma unroll
+        for (int c = 0; c < TK / 2; ++c) {
+          const float a = ex2(v[2 * c] - msub), b2 = ex2(v[2 * c + 1] - msub);
+          sum += a + b2;
+          pk[c] = pack_bf16(a, b2);
+        }
+        l = l * alpha + sum;
+        if (k > 0) {  // P(x-1) consumed and O(x-1) complete
+          ok = mbar_wait(pv_done(mt), (x - 1) & 1, abort_flag, p.status);
+          if (!ok) break;
+          tc_fence_after();
+          if (rescale) {
+            const uint32_t ocol = lane_base + C::O_COL + mt * D;
+#pragma unroll
+            for (int cc = 0; cc < D / 32; ++cc) {
+              uint32_t r[32];
+              tmem_ld32(ocol + cc * 32, r);
+              tmem_wait_ld();
+#pragma unroll
+              for (int e = 0; e < 32; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
+              tmem_st32(ocol + cc * 32, r);
+            }
+            tmem_wait_st();
+          }
+        }
+#pragma unroll
+        for (int c = 0; c < 8; ++c)
+          *reinterpret_cast<uint4*>(prow + ((c ^ (row & 7)) << 4)) =
+              make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
+        fence_async_smem();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(p_full(mt));
+      }
+      if (!ok) break;
+      // ---- epilogue: O (TMEM) -> output or partial ----
+      const uint32_t xl = it + s.ntile - 1;
+      ok = mbar_wait(pv_done(mt), xl & 1, abort_flag, p.status);
+      if (!ok) break;
+      tc_fence_after();
+      const bool whole = s.tile0 == 0 && s.ntile == s.unit_tiles;
+      const uint32_t ocol = lane_base + C::O_COL + mt * D;
+      const int c_first = owner_of(s.unit_start, total, ctas);
+      const int c_last = owner_of(s.unit_start + s.unit_tiles - 1, total, ctas);
+      const int64_t slot = s.u + cta;
+      if (bad && sw == 0 && lane == 0 && (whole || cta == c_first))
+        set_status(p.status, s.len_ok ? SPEC_FLAG_BAD_PAGE : SPEC_FLAG_BAD_KV_LEN);
+#pragma unroll 1
+      for (int cc = 0; cc < D / 32; ++cc) {
+        uint32_t r[32];
+        tmem_ld32(ocol + cc * 32, r);
+        tmem_wait_ld();
+        if (!real) continue;
+        if (whole) {
+          const float inv = bad ? 0.f : 1.f / l;
+#pragma unroll
+          for (int e = 0; e < 32; e += 8) {
+            float o8[8];
+#pragma unroll
+            for (int f = 0; f < 8; ++f) o8[f] = __uint_as_float(r[e + f]);
+            write_out_row<D>(p, s.b, s.g, urow, cc * 32 + e, o8, inv);
+          }
+        } else {
+          float4* dst = reinterpret_cast<float4*>(p.partial_o + (slot * p.slot_rows + lrow) * D + cc * 32);
+#pragma unroll
+          for (int e = 0; e < 8; ++e)
+            dst[e] = make_float4(__uint_as_float(r[4 * e]), __uint_as_float(r[4 * e + 1]),
+                                 __uint_as_float(r[4 * e + 2]), __uint_as_float(r[4 * e + 3]));
+        }
+      }
+      tc_fence_before();
+      if (real) {
+        if (whole) write_lse(p, s.b, s.g, urow, m, l, bad);
+        else p.partial_ml[slot * p.slot_rows + lrow] = make_float2(m, bad ? -1.f : l);
+      }
+      if (!whole) {
+        __threadfence();
+        ok = group_sync();
+        if (!ok) break;
+        if (gtid == 0) {
+          const uint32_t prev = atomicAdd(&p.tickets[s.u], 1u);
+          const bool last = prev == static_cast<uint32_t>(c_last - c_first);
+          if (last) p.tickets[s.u] = 0;  // leave the counter at zero for the next call
+          *merge_flag = last;
+        }
+        ok = group_sync();
+        if (!ok) break;
+        if (*merge_flag) {
+          __threadfence();
+          const int nrows = min(p.rows_per_cta, p.rows - row0);
+          merge_splits<D>(p, s.b, s.g, row0, nrows, s.u + c_first, c_last - c_first + 1, gtid,
+                          gthreads);
+        }
+        ok = group_sync();  // merge_flag is rewritten by the next segment
+        if (!ok) break;
+      }
+      it += s.ntile;
+      t += s.ntile;
+    }
+    tc_fence_before();
+  }
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, C::TMEM_COLS);
+  }
+}
+
+// ---------------------------------------------------------------------------------
+// Host side
+// ---------------------------------------------------------------------------------
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encoder() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(ptr);
+  }
+  return fn;
+}
+
+// K or V cache viewed as a 2-D tensor [num_pages * Hkv * page_size rows][D] of bf16;
+// one box is one page of one KV head, 64 columns (128 bytes) wide.
+bool encode_cache_map(CUtensorMap* map, const void* base, const spec_attn_args_t& a) {
+  EncodeTiledFn enc = encoder();
+  if (!enc) return false;
+  const cuuint64_t dims[2] = {static_cast<cuuint64_t>(a.head_dim),
+                              static_cast<cuuint64_t>(a.num_pages) * a.num_kv_heads * a.page_size};
+  const cuuint64_t strides[1] = {static_cast<cuuint64_t>(a.head_dim) * 2};
+  const cuuint32_t box[2] = {64, static_cast<cuuint32_t>(a.page_size)};
+  const cuuint32_t estr[2] = {1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int D, int MT>
+cudaError_t launch_typed(const spec_attn_args_t& a, const AttnPlan& P, char* ws,
+                         cudaStream_t stream) {
+  using Cf = TcCfg<D, MT>;
+  CUtensorMap mk, mv;
+  if (!encode_cache_map(&mk, a.k_cache, a) || !encode_cache_map(&mv, a.v_cache, a))
+    return cudaErrorInvalidValue;
+  const AttnParams p = make_attn_params(a, P, ws);
+  const size_t smem = Cf::smem_bytes(a.batch);
+  cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel<D, MT>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  attn_tc_kernel<D, MT><<<P.grid, Cf::THREADS, smem, stream>>>(mk, mv, p);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+size_t tc_smem_bytes(int head_dim, int rows_per_cta, int batch) {
+  const bool two = rows_per_cta > 128;
+  if (head_dim == 128) return two ? TcCfg<128, 2>::smem_bytes(batch) : TcCfg<128, 1>::smem_bytes(batch);
+  return two ? TcCfg<64, 2>::smem_bytes(batch) : TcCfg<64, 1>::smem_bytes(batch);
+}
+
+int tc_ctas_per_sm(int head_dim, int rows_per_cta, int batch) {
+  // Shared memory bounds residency (227 KB usable per SM); TMEM (512 columns) too.
+  const size_t smem = tc_smem_bytes(head_dim, rows_per_cta, batch);
+  int by_smem = static_cast<int>((227u * 1024u) / (smem + 1024));
+  const int cols = rows_per_cta > 128 ? 512 : 256;
+  const int by_tmem = 512 / cols;
+  int n = by_smem < by_tmem ? by_smem : by_tmem;
+  return n < 1 ? 1 : n;
+}
+
+cudaError_t launch_attn_tc(const spec_attn_args_t& a, const AttnPlan& P, char* ws,
+                           cudaStream_t stream) {
+  const bool two = P.rows_per_cta > 128;
+  if (a.head_dim == 128)
+    return two ? launch_typed<128, 2>(a, P, ws, stream) : launch_typed<128, 1>(a, P, ws, stream);
+  return two ? launch_typed<64, 2>(a, P, ws, stream) : launch_typed<64, 1>(a, P, ws, stream);
 }
 
 }  // namespace specv

@@ -49,8 +49,11 @@ struct AttnPlan {
   int row_tiles;     // ceil(rows / rows_per_cta)
   int key_tile;      // keys per pipeline step
   int max_keys;      // max_pages_per_seq * page_size
-  int nsplit;        // KV splits per (sequence, kv head, row tile)
+  int nsplit;        // KV splits per (sequence, kv head, row tile) (CUDA-core path)
   int tiles_per_split;
+  int grid;          // blocks launched
+  int slot_rows;     // rows per partial slot
+  int64_t slots;     // partial slots
   size_t tickets, partial_o, partial_ml, end;
 };
 
@@ -75,6 +78,9 @@ constexpr int kTcKeyTile = 64;
 constexpr int kTcMaxRows = 256;  // two M = 128 tiles per block
 
 int tc_min_rows();
+int tc_ctas_per_sm(int head_dim, int rows_per_cta, int batch);
+size_t tc_smem_bytes(int head_dim, int rows_per_cta, int batch);
+constexpr int kTcMaxBatch = 4096;  // batch prefix sums live in shared memory
 
 }  // namespace specv
 

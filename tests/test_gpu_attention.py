@@ -13,7 +13,7 @@ from helpers import attn_tensors, compare_attention, gpu_attention, sample_rows
 
 pytestmark = pytest.mark.gpu
 
-PATHS = [binding.ATTN_CUDA_CORES]
+PATHS = [binding.ATTN_CUDA_CORES, binding.ATTN_TENSOR_CORES]
 
 SMALL = [
     dict(batch=2, gamma=4, num_q_heads=8, num_kv_heads=8, head_dim=64, page_size=16, ctx=(0, 300)),
