@@ -5,7 +5,9 @@ one GB300 (or N independent replicas under torchrun), through the C ABI.
 One step = one spec_verify_step call over one batch of synthetic input (attention of
 the gamma block queries over the paged KV cache for one layer, plus the vocabulary-wide
 softmax and acceptance over target and drafter logits). Inputs are resident in HBM;
-L2 is flushed (a 256 MiB write) before every timed step, outside the timed events.
+L2 is flushed before every timed step, outside the timed events: a 256 MiB write, then
+a read of a different 256 MiB buffer, so the step neither hits its inputs in L2 nor pays
+to write back the flush's dirty lines.
 
 Prints ONE JSON line (rank 0). ``--impl reference`` times the fp64 CPU oracle on the
 host cores instead (the reference arm: there is no runnable reference implementation
@@ -44,6 +46,8 @@ def parse_args():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="llama8b",
                     help="tiny | llama8b | serve64 | long70b | sweep_g<G>_b<B>_s<S>_t<T>")
+    ap.add_argument("--attn-path", choices=["auto", "cuda-cores", "tensor-cores"], default="auto",
+                    help="attention kernel (auto: tensor cores from the library's row crossover)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=10.0,
@@ -206,6 +210,13 @@ def reference_arm(args, wl, ai, ci):
 # ----------------------------------------------------------------------------------
 # our arm
 # ----------------------------------------------------------------------------------
+def attn_path_name(choice, binding, ai):
+    if choice == "auto":
+        rows = (ai.num_q_heads // ai.num_kv_heads) * ai.gamma
+        return "tensor cores" if rows >= binding.tensor_core_min_rows() else "CUDA cores"
+    return choice.replace("-", " ")
+
+
 def run_ours(args, wl, ai, ci, rank, world, local_rank):
     import torch
     from paper_2609_04010_gb300 import binding, build
@@ -232,17 +243,25 @@ def run_ours(args, wl, ai, ci, rank, world, local_rank):
     na = torch.empty(B, dtype=torch.int32, device=dev)
     ot = torch.empty(B, G + 1, dtype=torch.int32, device=dev)
     ne = torch.empty(B, dtype=torch.int32, device=dev)
-    a = binding.attn_args(d["q"], d["k"], d["v"], d["pt"], d["kvl"], out, lse)
+    path = {"auto": binding.ATTN_AUTO, "cuda-cores": binding.ATTN_CUDA_CORES,
+            "tensor-cores": binding.ATTN_TENSOR_CORES}[args.attn_path]
+    a = binding.attn_args(d["q"], d["k"], d["v"], d["pt"], d["kvl"], out, lse, path=path)
     c = binding.accept_args(d["tl"], d["dl"], d["tok"], d["temp"], d["u"], na, ot, ne, None)
     ws = binding.new_workspace(binding.workspace_size(a, c), dev)
-    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    flush_w = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    flush_r = torch.ones(L2_FLUSH_BYTES // 4, dtype=torch.int32, device=dev)
+    flush_sink = torch.empty(1, dtype=torch.int64, device=dev)
     stream = torch.cuda.current_stream()
+
+    def flush_l2():
+        flush_w.zero_()
+        flush_sink.copy_(flush_r.sum(dtype=torch.int64).reshape(1))
 
     def timed_loop(fn, n):
         evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
                for _ in range(n)]
         for i in range(n):
-            flush.zero_()
+            flush_l2()
             evs[i][0].record(stream)
             fn()
             evs[i][1].record(stream)
@@ -258,7 +277,7 @@ def run_ours(args, wl, ai, ci, rank, world, local_rank):
     clocks.start()
     time.sleep(0.3)
     for _ in range(max(3, args.warmup)):
-        flush.zero_()
+        flush_l2()
         step()
     torch.cuda.synchronize()
     code, flags = binding.read_device_status(ws)
@@ -322,9 +341,8 @@ def run_ours(args, wl, ai, ci, rank, world, local_rank):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded; no weights or datasets)",
         "config": dict(wl.describe(), parallelism=f"replicas x{world}",
-                       l2="flushed before every timed step (256 MiB write, outside events)",
-                       attention_path="tensor cores" if binding.tensor_core_min_rows() <=
-                       (ai.num_q_heads // ai.num_kv_heads) * ai.gamma else "CUDA cores"),
+                       l2="flushed before every timed step (256 MiB write + 256 MiB read, outside events)",
+                       attention_path=attn_path_name(args.attn_path, binding, ai)),
         "roofline": {"bound": "hbm", "kernel": dominant, "achieved": round(dom_gbs, 1),
                      "peak": peak, "unit": "GB/s", "frac": round(dom_gbs / peak, 4),
                      "peak_source": peak_src, "traffic": None,

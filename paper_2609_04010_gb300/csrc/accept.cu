@@ -132,7 +132,7 @@ __device__ __forceinline__ void merge_arg(float& m, int& a, float m2, int a2) {
 }
 
 template <bool BF16, bool VEC>
-__global__ void __launch_bounds__(kStatsThreads) row_stats_kernel(AcceptParams p) {
+__global__ void __launch_bounds__(kStatsThreads, 4) row_stats_kernel(AcceptParams p) {
   constexpr int kPer = kStatsChunk / kStatsThreads;  // 32 values per thread
   __shared__ float sh_m[kStatsThreads / 32];
   __shared__ float sh_s[kStatsThreads / 32];
@@ -153,27 +153,73 @@ __global__ void __launch_bounds__(kStatsThreads) row_stats_kernel(AcceptParams p
   const int start = c * kStatsChunk;
   const int len = min(kStatsChunk, p.vocab - start);
 
-  float v[kPer];
-  int idx[kPer];
-  load_strided<BF16, VEC, kPer, kStatsThreads>(rowp, start, len, v, idx);
-
   uint32_t bad = 0;
   float m = -INFINITY;
-  int a = idx[0];
-#pragma unroll
-  for (int k = 0; k < kPer; ++k) {
-    bad |= !(v[k] <= FLT_MAX) && idx[k] != INT_MAX;  // NaN or +inf inside the row
-    if (greedy) {
-      if (v[k] > m) { m = v[k]; a = idx[k]; }
-    } else {
-      m = fmaxf(m, v[k]);
-    }
-  }
-  const float cs = greedy ? 0.f : kLog2e / T;
+  int a = INT_MAX;
   float s = 0.f;
-  if (!greedy && m != -INFINITY) {
+  const float cs = greedy ? 0.f : kLog2e / T;
+  if (VEC) {
+    // The chunk stays packed in registers (16-byte groups, group g of thread t at
+    // g * threads + t) and is decoded twice: once for the max, once for the sum.
+    constexpr int kEpv = BF16 ? 8 : 4;
+    constexpr int kVecs = kPer / kEpv;
+    const int t = threadIdx.x;
+    uint4 raw[kVecs];
+    const uint32_t ninf = BF16 ? 0xFF80FF80u : 0xFF800000u;  // -inf padding past the row end
 #pragma unroll
-    for (int k = 0; k < kPer; ++k) s += ex2((v[k] - m) * cs);
+    for (int k = 0; k < kVecs; ++k) {
+      const int e = (k * kStatsThreads + t) * kEpv;
+      raw[k] = e < len ? __ldg(reinterpret_cast<const uint4*>(
+                             static_cast<const char*>(rowp) + static_cast<int64_t>(start + e) * (BF16 ? 2 : 4)))
+                       : make_uint4(ninf, ninf, ninf, ninf);
+    }
+    auto elem = [&](int k, int q) -> float {
+      const int wi = BF16 ? (q >> 1) : q;
+      const uint32_t word = wi == 0 ? raw[k].x : wi == 1 ? raw[k].y : wi == 2 ? raw[k].z : raw[k].w;
+      if (BF16) return __uint_as_float((q & 1) ? (word & 0xffff0000u) : (word << 16));
+      return __uint_as_float(word);
+    };
+    // this thread's elements in increasing index order: a strict > keeps the lowest
+    // index of the maximum; all -inf leaves the first index
+    a = start + t * kEpv;
+#pragma unroll
+    for (int k = 0; k < kVecs; ++k) {
+#pragma unroll
+      for (int q = 0; q < kEpv; ++q) {
+        const float x = elem(k, q);
+        bad |= !(x <= FLT_MAX);  // NaN or +inf (the padding is -inf)
+        if (greedy) {
+          if (x > m) { m = x; a = start + (k * kStatsThreads + t) * kEpv + q; }
+        } else {
+          m = fmaxf(m, x);
+        }
+      }
+    }
+    if (a >= start + len) a = INT_MAX;  // a thread past the row end loses every tie
+    if (!greedy && m != -INFINITY) {
+#pragma unroll
+      for (int k = 0; k < kVecs; ++k)
+#pragma unroll
+        for (int q = 0; q < kEpv; ++q) s += ex2((elem(k, q) - m) * cs);
+    }
+  } else {
+    float v[kPer];
+    int idx[kPer];
+    load_strided<BF16, false, kPer, kStatsThreads>(rowp, start, len, v, idx);
+    a = idx[0];
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) {
+      bad |= !(v[k] <= FLT_MAX) && idx[k] != INT_MAX;  // NaN or +inf inside the row
+      if (greedy) {
+        if (v[k] > m) { m = v[k]; a = idx[k]; }
+      } else {
+        m = fmaxf(m, v[k]);
+      }
+    }
+    if (!greedy && m != -INFINITY) {
+#pragma unroll
+      for (int k = 0; k < kPer; ++k) s += ex2((v[k] - m) * cs);
+    }
   }
   // warp then block reduction
 #pragma unroll

@@ -90,42 +90,75 @@ __device__ __forceinline__ void write_lse(const AttnParams& p, int b, int g, int
   p.lse[(static_cast<int64_t>(b) * p.gamma + j) * p.hq + h] = v;
 }
 
-// Run by the last block to finish a unit: combines the partials in slots
-// [slot0, slot0 + nslots) for rows [row0, row0 + nrows) and writes the final
-// outputs. Threads tid .. of nthreads cooperate.
+// Combines the split-KV partials of one unit, held in slots [slot0, slot0 + nslots), for
+// rows [row0, row0 + nrows) and writes the final outputs. All nthreads threads of the
+// block call it together (it synchronizes the block between its two passes); sh_m and
+// sh_l are shared-memory scratch for nrows floats each. Pass 1 takes each row's
+// largest base-2 max M and its total L = sum_s l_s 2^(m_s - M); pass 2 gives every
+// (row, 4-column) item all its slot loads at once, so the merge is not a chain of
+// dependent L2 round trips.
 template <int D>
-__device__ void merge_splits(const AttnParams& p, int b, int g, int row0, int nrows,
-                             int64_t slot0, int nslots, int tid, int nthreads) {
-  constexpr int DQ = D / 8;
-  for (int idx = tid; idx < nrows * DQ; idx += nthreads) {
-    const int r = idx / DQ, dq = idx % DQ;
+__device__ void merge_unit(const AttnParams& p, int b, int g, int row0, int nrows, int64_t slot0,
+                           int nslots, float* sh_m, float* sh_l, int tid, int nthreads) {
+  for (int r = tid; r < nrows; r += nthreads) {
     float M = -INFINITY;
     bool bad = false;
     for (int s = 0; s < nslots; ++s) {
       const float2 ml = __ldcg(&p.partial_ml[(slot0 + s) * p.slot_rows + r]);
-      if (ml.y < 0.f) bad = true;
-      else if (ml.y > 0.f) M = fmaxf(M, ml.x);
+      bad |= ml.y < 0.f;
+      if (ml.y > 0.f) M = fmaxf(M, ml.x);
     }
-    float L = 0.f, acc[8];
-#pragma unroll
-    for (int e = 0; e < 8; ++e) acc[e] = 0.f;
-    if (!bad) {
-      for (int s = 0; s < nslots; ++s) {
-        const int64_t slot = (slot0 + s) * p.slot_rows + r;
-        const float2 ml = __ldcg(&p.partial_ml[slot]);
-        if (!(ml.y > 0.f)) continue;
-        const float w = ex2(ml.x - M);
-        L += ml.y * w;
-        const float4* src = reinterpret_cast<const float4*>(p.partial_o + slot * D + dq * 8);
-        const float4 a = __ldcg(src), c = __ldcg(src + 1);
-        acc[0] += a.x * w; acc[1] += a.y * w; acc[2] += a.z * w; acc[3] += a.w * w;
-        acc[4] += c.x * w; acc[5] += c.y * w; acc[6] += c.z * w; acc[7] += c.w * w;
-      }
+    float L = 0.f;
+    for (int s = 0; s < nslots; ++s) {
+      const float2 ml = __ldcg(&p.partial_ml[(slot0 + s) * p.slot_rows + r]);
+      if (ml.y > 0.f) L += ml.y * ex2(ml.x - M);
     }
     const bool dead = bad || !(L > 0.f);
-    write_out_row<D>(p, b, g, row0 + r, dq * 8, acc, dead ? 0.f : 1.f / L);
-    if (dq == 0) write_lse(p, b, g, row0 + r, M, L, dead);
+    sh_m[r] = M;
+    sh_l[r] = dead ? 0.f : L;
+    write_lse(p, b, g, row0 + r, M, L, dead);
   }
+  __syncthreads();
+  constexpr int C4 = D / 4;
+  for (int idx = tid; idx < nrows * C4; idx += nthreads) {
+    const int r = idx / C4, c4 = idx % C4;
+    const float M = sh_m[r], L = sh_l[r];
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (L > 0.f) {
+      int s = 0;
+      for (; s + 4 <= nslots; s += 4) {
+        float2 ml[4];
+        float4 o[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const int64_t slot = (slot0 + s + e) * p.slot_rows + r;
+          ml[e] = __ldcg(&p.partial_ml[slot]);
+          o[e] = __ldcg(reinterpret_cast<const float4*>(p.partial_o + slot * D) + c4);
+        }
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+          const float w = ml[e].y > 0.f ? ex2(ml[e].x - M) : 0.f;
+          acc.x += o[e].x * w; acc.y += o[e].y * w; acc.z += o[e].z * w; acc.w += o[e].w * w;
+        }
+      }
+      for (; s < nslots; ++s) {
+        const int64_t slot = (slot0 + s) * p.slot_rows + r;
+        const float2 ml = __ldcg(&p.partial_ml[slot]);
+        const float4 o = __ldcg(reinterpret_cast<const float4*>(p.partial_o + slot * D) + c4);
+        const float w = ml.y > 0.f ? ex2(ml.x - M) : 0.f;
+        acc.x += o.x * w; acc.y += o.y * w; acc.z += o.z * w; acc.w += o.w * w;
+      }
+    }
+    const float inv = L > 0.f ? 1.f / L : 0.f;
+    const int row = row0 + r, j = row / p.group, h = g * p.group + row % p.group;
+    __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(p.out) +
+                         ((static_cast<int64_t>(b) * p.gamma + j) * p.hq + h) * D + c4 * 4;
+    const __nv_bfloat162 lo = __floats2bfloat162_rn(acc.x * inv, acc.y * inv);
+    const __nv_bfloat162 hi = __floats2bfloat162_rn(acc.z * inv, acc.w * inv);
+    *reinterpret_cast<uint2*>(dst) = make_uint2(*reinterpret_cast<const uint32_t*>(&lo),
+                                               *reinterpret_cast<const uint32_t*>(&hi));
+  }
+  __syncthreads();
 }
 #endif
 

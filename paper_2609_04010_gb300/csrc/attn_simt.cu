@@ -273,7 +273,7 @@ __global__ void __launch_bounds__(NT) attn_simt_kernel(AttnParams p) {
   __syncthreads();
   if (!sm.last) return;
   __threadfence();
-  merge_splits<D>(p, b, g, row0, nrows, unit * p.nsplit, p.nsplit, tid, NT);
+  merge_unit<D>(p, b, g, row0, nrows, unit * p.nsplit, p.nsplit, &sm.s[0][0], &sm.s[1][0], tid, NT);
 }
 
 }  // namespace

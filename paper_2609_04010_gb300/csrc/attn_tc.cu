@@ -8,12 +8,16 @@
 // group has up to 256 rows), so each KV page is read from HBM once.
 //
 // Warp roles (one block per SM, persistent):
-//   warp 0      TMA producer: gathers each 64-key tile of K and V page by page through
-//               the page table with cp.async.bulk.tensor (128-byte swizzle) into a
-//               multi-stage ring; an mbarrier per stage carries the byte count.
+//   warps 0,2,3 KV producers: gather each 64-key tile of K and V page by page through
+//               the page table, one 5-D cp.async.bulk.tensor box (128-byte swizzle) per
+//               (page, K or V), spread over three issuing warps (one issuer cannot keep
+//               the copy engine busy with page-sized boxes), into a multi-stage ring; an
+//               mbarrier per stage carries the byte count. The box lays a page out in
+//               8-key groups so that the MMAs below can span pages.
 //   warp 1      MMA issuer: S = Q K^T (tcgen05.mma kind::f16, M = 128, N = 64, K = 16
 //               steps over D) into a double-buffered fp32 TMEM accumulator, then
 //               O += P V (N = D) with P from shared memory and V read MN-major.
+//   warps 4..   softmax warps with real rows (one per 32 query rows); the others idle.
 //   warps 4..   softmax (one warpgroup per M tile, one thread per query row): load S
 //               from TMEM, scale and mask, online softmax in base 2 with lazy rescale
 //               of O (only when the running max grows by more than 2^8), write P as
@@ -31,8 +35,8 @@
 namespace specv {
 namespace {
 
-constexpr int TK = kTcKeyTile;               // keys per tile (MMA N of Q K^T)
-constexpr uint64_t kWaitLimitNs = 1000000000ull;  // 1 s per wait
+constexpr int TK = kTcKeyTile;               // keys per tile
+
 
 template <int D, int MT>
 struct TcCfg {
@@ -50,8 +54,9 @@ struct TcCfg {
   // barriers: kv_full[S], kv_empty[S], s_full[MT][2], s_free[MT][2], p_full[MT],
   // pv_done[MT], seg_ready, grp, drain
   static constexpr int NBAR = 2 * STAGES + 6 * MT + 3;
-  static constexpr uint32_t OFF_MISC = OFF_BAR + NBAR * 8;  // tmem base, abort, flag
-  static constexpr uint32_t OFF_PB = (OFF_MISC + 16 + 15) / 16 * 16;
+  static constexpr uint32_t OFF_MISC = OFF_BAR + NBAR * 8;  // tmem base, abort, flag, merges
+  static constexpr uint32_t OFF_MERGE = OFF_MISC + 16;          // 2 deferred merges x 8 ints
+  static constexpr uint32_t OFF_PB = (OFF_MERGE + 64 + 15) / 16 * 16;
   static constexpr uint32_t TMEM_COLS = (MT * 128 + MT * D) <= 256 ? 256 : 512;
   static constexpr uint32_t S_COL = 0;           // S[mt][buf] at (mt * 2 + buf) * 64
   static constexpr uint32_t O_COL = MT * 128;    // O[mt] at O_COL + mt * D
@@ -84,22 +89,23 @@ __device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
-__device__ __forceinline__ uint64_t globaltimer() {
-  uint64_t t;
-  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-  return t;
-}
-// Bounded wait on phase `parity` of an mbarrier. On timeout (or when another role has
-// already timed out) it raises the block's abort flag and returns false.
+// Bounded wait on phase `parity` of an mbarrier. The bound is counted in SM clock
+// cycles (kWaitLimitCycles, about 1 s at the 2.07 GHz maximum clock and longer at lower
+// clocks), read only every 256 tries. On timeout (or when another role has already
+// timed out) it raises the block's abort flag and returns false.
+constexpr long long kWaitLimitCycles = 2000000000ll;
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort_flag,
                                           uint32_t* status) {
   if (mbar_try(bar, parity)) return true;
-  const uint64_t t0 = globaltimer();
+  long long t0 = 0;
   for (uint32_t it = 1;; ++it) {
     if (mbar_try(bar, parity)) return true;
-    if ((it & 63) == 0) {
+    if ((it & 255) == 0) {
       if (*abort_flag) return false;
-      if (globaltimer() - t0 > kWaitLimitNs) {
+      const long long now = clock64();
+      if (t0 == 0) {
+        t0 = now;
+      } else if (now - t0 > kWaitLimitCycles) {
         *abort_flag = 1;
         atomicOr(status, SPEC_FLAG_TIMEOUT);
         return false;
@@ -107,12 +113,15 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatil
     }
   }
 }
-__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y,
-                                            uint32_t bar) {
+// One page of one KV head (box of the 5-D view of the cache, see encode_cache_map),
+// landing as [8-row group][128-byte column half][8 rows][128 B], 128-byte swizzle.
+__device__ __forceinline__ void tma_load_page(uint32_t dst, const CUtensorMap* map, int page_head,
+                                              uint32_t bar) {
   asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
-      " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+      "cp.async.bulk.tensor.5d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4, %5, %6}], [%7];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(0), "r"(0), "r"(0), "r"(0), "r"(page_head),
+      "r"(bar)
       : "memory");
 }
 __device__ __forceinline__ void fence_async_smem() {
@@ -285,28 +294,45 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
   uint32_t* misc = reinterpret_cast<uint32_t*>(smem + C::OFF_MISC);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 1);
   volatile int* merge_flag = reinterpret_cast<volatile int*>(misc + 2);
+  volatile int* merge_count = reinterpret_cast<volatile int*>(misc + 3);
+  int* merges = reinterpret_cast<int*>(smem + C::OFF_MERGE);  // [2][8]
   int* pb = reinterpret_cast<int*>(smem + C::OFF_PB);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
 
+  // ---- roles ----
+  // Softmax warps take part only as far as the row tile has real rows (32 per warp).
+  const int rows_cta = min(p.rows_per_cta, p.rows);
+  int nact[MT];
+  int nact_total = 0;
+#pragma unroll
+  for (int mt = 0; mt < MT; ++mt) {
+    nact[mt] = min(4, max(0, (rows_cta - 128 * mt + 31) / 32));
+    nact_total += nact[mt];
+  }
+  constexpr int nprod = 3;  // KV producer warps 0, 2, 3
+  const int pw = (threadIdx.x >> 5) == 0 ? 0 : ((threadIdx.x >> 5) == 2 || (threadIdx.x >> 5) == 3)
+                                                    ? (threadIdx.x >> 5) - 1 : -1;
+
   // ---- prologue: barriers, TMEM, per-sequence tile prefix sums ----
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::STAGES; ++s) {
-      mbar_init(kv_full(s), 1);
+      mbar_init(kv_full(s), nprod);
       mbar_init(kv_empty(s), 1);
     }
     for (int mt = 0; mt < MT; ++mt) {
       for (int bf = 0; bf < 2; ++bf) {
         mbar_init(s_full(mt, bf), 1);
-        mbar_init(s_free(mt, bf), 4);
+        mbar_init(s_free(mt, bf), nact[mt] > 0 ? nact[mt] : 1);
       }
-      mbar_init(p_full(mt), 4);
+      mbar_init(p_full(mt), nact[mt] > 0 ? nact[mt] : 1);
       mbar_init(pv_done(mt), 1);
     }
-    mbar_init(seg_ready, 4 * MT);
-    mbar_init(grp_bar, 4 * MT);
+    mbar_init(seg_ready, nact_total);
+    mbar_init(grp_bar, nact_total);
     mbar_init(drain_bar, 1);
     *abort_flag = 0;
+    *merge_count = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 1) tmem_alloc(smem_u32(misc), C::TMEM_COLS);
@@ -337,10 +363,25 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
   const int64_t t0 = cta < ctas ? static_cast<int64_t>(cta) * total / ctas : 0;
   const int64_t t1 = cta < ctas ? static_cast<int64_t>(cta + 1) * total / ctas : 0;
 
-  if (warp == 0) {
-    // =========================== TMA producer ===========================
+  if (pw >= 0) {
+    // ============================ KV producers ============================
+    // A tile needs one box per (page, K or V); producer pw issues boxes pw, pw + nprod,
+    // ... (one issuer cannot keep the copy engine busy with page-sized boxes).
     uint32_t it = 0;
     bool ok = true;
+    // Page ids are read 32 at a time (lane i holds page cache_base + i of sequence
+    // cache_b) so that one L2 round trip serves several tiles.
+    int cache_b = -1, cache_base = 0, cache_val = 0;
+    auto page_of = [&](int b, int pi) -> int {  // warp-uniform
+      if (b != cache_b || pi < cache_base || pi >= cache_base + 32) {
+        cache_b = b;
+        cache_base = pi;
+        const int idx = pi + lane;
+        cache_val = idx < p.max_pages ? __ldg(&p.page_table[static_cast<int64_t>(b) * p.max_pages + idx]) : 0;
+      }
+      return __shfl_sync(0xffffffffu, cache_val, pi - cache_base);
+    };
+    const uint32_t box_bytes = static_cast<uint32_t>(p.page_size) * D * 2;  // one page of one head
     for (int64_t t = t0; t < t1 && ok;) {
       const Seg s = locate(t, t1, p, pb);
       const bool bad = segment_bad(s, p);
@@ -349,27 +390,25 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
         if (it >= static_cast<uint32_t>(C::STAGES))
           ok = mbar_wait(kv_empty(st), ((it / C::STAGES) - 1) & 1, abort_flag, p.status);
         if (!ok) break;
-        if (lane == 0) {
-          if (bad) {
-            mbar_arrive(kv_full(st));
-          } else {
-            const int key0 = (s.tile0 + k) * TK;
-            const int npg = TK / p.page_size;
-            int nvalid = 0;
-            for (int q = 0; q < npg; ++q) nvalid += (key0 + q * p.page_size) < s.kv_len;
-            mbar_arrive_tx(kv_full(st), static_cast<uint32_t>(nvalid) * p.page_size * D * 2 * 2);
-            for (int q = 0; q < nvalid; ++q) {
-              const int key = key0 + q * p.page_size;
-              const int page = p.page_table[static_cast<int64_t>(s.b) * p.max_pages + key / p.page_size];
-              const int y = (page * p.hkv + s.g) * p.page_size;
-              const uint32_t row_off = static_cast<uint32_t>(q * p.page_size) * 128u;
-#pragma unroll
-              for (int h = 0; h < C::DH; ++h) {
-                tma_load_2d(sbase + C::OFF_K + st * C::KV_BYTES + h * 8192u + row_off, &tmap_k,
-                            h * 64, y, kv_full(st));
-                tma_load_2d(sbase + C::OFF_V + st * C::KV_BYTES + h * 8192u + row_off, &tmap_v,
-                            h * 64, y, kv_full(st));
-              }
+        if (bad) {
+          if (lane == 0) mbar_arrive(kv_full(st));
+        } else {
+          const int key0 = (s.tile0 + k) * TK;
+          const int npg = TK / p.page_size;
+          int nvalid = 0;
+          for (int q = 0; q < npg; ++q) nvalid += (key0 + q * p.page_size) < s.kv_len;
+          // box bx: page q = bx >> 1, K (even) or V (odd)
+          const int nbox = 2 * nvalid;
+          uint32_t mine = 0;
+          for (int bx = pw; bx < nbox; bx += nprod) mine += box_bytes;
+          if (lane == 0) mbar_arrive_tx(kv_full(st), mine);
+          for (int bx = pw; bx < nbox; bx += nprod) {
+            const int q = bx >> 1, isv = bx & 1;
+            const int page = page_of(s.b, key0 / p.page_size + q);
+            if (lane == 0) {
+              const uint32_t dst = sbase + (isv ? C::OFF_V : C::OFF_K) + st * C::KV_BYTES +
+                                   static_cast<uint32_t>(q) * box_bytes;
+              tma_load_page(dst, isv ? &tmap_v : &tmap_k, page * p.hkv + s.g, kv_full(st));
             }
           }
         }
@@ -379,14 +418,19 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
     }
     if (!ok) {  // drain this block's copies still in flight (bounded)
       for (uint32_t x = it > static_cast<uint32_t>(C::STAGES) ? it - C::STAGES : 0; x < it; ++x) {
-        const uint64_t t_0 = globaltimer();
+        const long long t_0 = clock64();
         while (!mbar_try(kv_full(x % C::STAGES), (x / C::STAGES) & 1) &&
-               globaltimer() - t_0 < kWaitLimitNs) {
+               clock64() - t_0 < kWaitLimitCycles) {
         }
       }
     }
   } else if (warp == 1) {
     // ============================ MMA issuer ============================
+    // K and V stages hold a tile as [8-key group][128-byte column half][8 keys][128 B]:
+    // 8-key groups sit at a uniform stride of DH KB across pages, so Q K^T runs with
+    // N = 64 keys (a tcgen05 MMA costs about the same for N = 16 and N = 64) and P V
+    // reads V MN-major with the column halves 1 KB apart.
+    constexpr uint32_t kGroup = C::DH * 1024u;
     constexpr uint32_t kIdescQK = idesc_bf16(128, TK, false);
     constexpr uint32_t kIdescPV = idesc_bf16(128, D, true);
     uint32_t it = 0, seg_no = 0;
@@ -400,10 +444,11 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
       const int key0 = (s.tile0 + k) * TK;
       const int nvalid = s.len_ok ? min(TK, max(0, s.kv_len - key0)) : TK;
       if (nvalid < TK) {
-        for (int h = 0; h < C::DH; ++h) {
-          uint4* vrow = reinterpret_cast<uint4*>(smem + C::OFF_V + st * C::KV_BYTES + h * 8192u +
-                                                 nvalid * 128u);
-          for (int i = lane; i < (TK - nvalid) * 8; i += 32) vrow[i] = make_uint4(0, 0, 0, 0);
+        unsigned char* vst = smem + C::OFF_V + st * C::KV_BYTES;
+        for (int i = lane; i < (TK - nvalid) * C::DH * 8; i += 32) {
+          const int key = nvalid + i / (C::DH * 8), h = (i / 8) % C::DH, c = i % 8;
+          *reinterpret_cast<uint4*>(vst + (key >> 3) * kGroup + h * 1024u + (key & 7) * 128u +
+                                    c * 16u) = make_uint4(0, 0, 0, 0);
         }
         fence_async_smem();
       }
@@ -418,8 +463,8 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
 #pragma unroll
           for (int kk = 0; kk < D / 16; ++kk) {
             const uint32_t qa = sbase + C::OFF_Q + (mt * C::DH + kk / 4) * 16384u + (kk % 4) * 32u;
-            const uint32_t kb = sbase + C::OFF_K + st * C::KV_BYTES + (kk / 4) * 8192u + (kk % 4) * 32u;
-            mma_bf16(d_tmem, desc_sw128(qa, 16, 1024), desc_sw128(kb, 16, 1024), kIdescQK, kk > 0);
+            const uint32_t kb = sbase + C::OFF_K + st * C::KV_BYTES + (kk / 4) * 1024u + (kk % 4) * 32u;
+            mma_bf16(d_tmem, desc_sw128(qa, 16, 1024), desc_sw128(kb, 16, kGroup), kIdescQK, kk > 0);
           }
           mma_commit(s_full(mt, x & 1));
         }
@@ -446,8 +491,8 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
 #pragma unroll
             for (int kk = 0; kk < TK / 16; ++kk) {
               const uint32_t pa = sbase + C::OFF_P + mt * 16384u + kk * 32u;
-              const uint32_t vb = sbase + C::OFF_V + st * C::KV_BYTES + kk * 2048u;
-              mma_bf16(d_tmem, desc_sw128(pa, 16, 1024), desc_sw128(vb, 8192, 1024), kIdescPV,
+              const uint32_t vb = sbase + C::OFF_V + st * C::KV_BYTES + kk * 2u * kGroup;
+              mma_bf16(d_tmem, desc_sw128(pa, 16, 1024), desc_sw128(vb, 1024, kGroup), kIdescPV,
                        (k > 0 || kk > 0) ? 1u : 0u);
             }
             mma_commit(pv_done(mt));
@@ -464,16 +509,17 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
     if (!ok && __any_sync(0xffffffffu, issued)) {  // drain this block's MMAs (bounded)
       if (lane == 0) mma_commit(drain_bar);
       __syncwarp();
-      const uint64_t t_0 = globaltimer();
-      while (!mbar_try(drain_bar, 0) && globaltimer() - t_0 < kWaitLimitNs) {
+      const long long t_0 = clock64();
+      while (!mbar_try(drain_bar, 0) && clock64() - t_0 < kWaitLimitCycles) {
       }
     }
-  } else if (warp >= 4) {
-    // ============================== softmax ==============================
+  } else if (warp >= 4 && ((warp - 4) & 3) < nact[(warp - 4) >> 2]) {
+    // ====================== softmax (warps with real rows) ======================
     const int sw = warp - 4, mt = sw >> 2, q4 = sw & 3;
     const int row = q4 * 32 + lane;  // TMEM lane = row of this M tile
     const uint32_t lane_base = tmem + (static_cast<uint32_t>(q4 * 32) << 16);
-    const int gtid = threadIdx.x - 128, gthreads = 128 * MT;
+    // active softmax warps are numbered densely: M tile 0's first, then M tile 1's
+    const int gtid = (mt == 0 ? q4 : nact[0] + q4) * 32 + lane, gthreads = 32 * nact_total;
     uint32_t it = 0, gphase = 0;
     bool ok = true;
     unsigned char* prow = smem + C::OFF_P + mt * 16384u + row * 128u;
@@ -641,11 +687,13 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
         }
         ok = group_sync();
         if (!ok) break;
-        if (*merge_flag) {
-          __threadfence();
-          const int nrows = min(p.rows_per_cta, p.rows - row0);
-          merge_splits<D>(p, s.b, s.g, row0, nrows, s.u + c_first, c_last - c_first + 1, gtid,
-                          gthreads);
+        if (*merge_flag && gtid == 0) {
+          // the unit is complete: merge it once every role of this block is done (only a
+          // block's first and last segments can be split, so at most two)
+          int* e = merges + 8 * (*merge_count);
+          e[0] = s.b; e[1] = s.g; e[2] = row0; e[3] = min(p.rows_per_cta, p.rows - row0);
+          e[4] = static_cast<int>(s.u + c_first); e[5] = c_last - c_first + 1;
+          *merge_count = *merge_count + 1;
         }
         ok = group_sync();  // merge_flag is rewritten by the next segment
         if (!ok) break;
@@ -659,6 +707,17 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem, C::TMEM_COLS);
+  }
+  // deferred merges of split units this block completed, by all of its threads
+  if (!*abort_flag) {
+    const int nm = *merge_count;
+    float* sh = reinterpret_cast<float*>(smem + C::OFF_P);  // P tile is free now
+    for (int mi = 0; mi < nm; ++mi) {
+      const int* e = merges + 8 * mi;
+      __threadfence();
+      merge_unit<D>(p, e[0], e[1], e[2], e[3], e[4], e[5], sh, sh + kTcMaxRows, threadIdx.x,
+                    C::THREADS);
+    }
   }
 }
 
@@ -683,17 +742,22 @@ EncodeTiledFn encoder() {
   return fn;
 }
 
-// K or V cache viewed as a 2-D tensor [num_pages * Hkv * page_size rows][D] of bf16;
-// one box is one page of one KV head, 64 columns (128 bytes) wide.
+// K or V cache viewed as a 5-D tensor of bf16 whose box is one page of one KV head:
+// (64 columns; 8 rows at stride D*2 bytes; D/64 column halves at stride 128 bytes;
+// page/8 groups of 8 rows at stride 8*D*2 bytes; page * Hkv + head at stride page*D*2).
+// The box lands in shared memory as [row group][column half][8 rows][128 B], so the
+// 8-row groups of a 64-key tile sit at a uniform stride whatever the page size.
 bool encode_cache_map(CUtensorMap* map, const void* base, const spec_attn_args_t& a) {
   EncodeTiledFn enc = encoder();
   if (!enc) return false;
-  const cuuint64_t dims[2] = {static_cast<cuuint64_t>(a.head_dim),
-                              static_cast<cuuint64_t>(a.num_pages) * a.num_kv_heads * a.page_size};
-  const cuuint64_t strides[1] = {static_cast<cuuint64_t>(a.head_dim) * 2};
-  const cuuint32_t box[2] = {64, static_cast<cuuint32_t>(a.page_size)};
-  const cuuint32_t estr[2] = {1, 1};
-  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+  const cuuint64_t D = static_cast<cuuint64_t>(a.head_dim);
+  const cuuint64_t dims[5] = {64, 8, D / 64, static_cast<cuuint64_t>(a.page_size / 8),
+                              static_cast<cuuint64_t>(a.num_pages) * a.num_kv_heads};
+  const cuuint64_t strides[4] = {D * 2, 128, 8 * D * 2, static_cast<cuuint64_t>(a.page_size) * D * 2};
+  const cuuint32_t box[5] = {64, 8, static_cast<cuuint32_t>(D / 64),
+                             static_cast<cuuint32_t>(a.page_size / 8), 1};
+  const cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void*>(base), dims, strides, box,
              estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
