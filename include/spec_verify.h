@@ -186,6 +186,31 @@ const char* spec_status_string(spec_status_t status);
 /* The (Hq/Hkv)*gamma at and above which SPEC_ATTN_AUTO picks the tensor-core kernel. */
 int32_t spec_attn_tensor_core_min_rows(void);
 
+/*
+ * spec_accept_block without a workspace, for callers that cannot allocate device
+ * memory when they verify (for example, code confined to a fixed, pre-planned memory
+ * arena, or code that must not call an allocator). It computes exactly what
+ * spec_accept_block computes; the paper has no counterpart to this call. Its scratch
+ * lives in one device array of SPEC_NOALLOC_SCRATCH_BYTES owned by the library, which
+ * every GPU that loads the library keeps until the process exits.
+ *   - Arguments: as spec_accept_block (device pointers, same layouts); no workspace.
+ *   - Limit: the scratch this batch needs (16 bytes per (sequence, row, 8192-entry
+ *     vocab chunk) plus 16 bytes per (sequence, 8192-entry slice), rounded up) must fit
+ *     in SPEC_NOALLOC_SCRATCH_BYTES; otherwise SPEC_ERR_WORKSPACE_TOO_SMALL, with
+ *     nothing launched. Other argument errors as spec_accept_block.
+ *   - Allocates nothing: no cudaMalloc, cudaFree or allocating library routine. The
+ *     first call on each device looks up the array's device address
+ *     (cudaGetSymbolAddress) with that device current; make that first call before
+ *     any stream capture.
+ *   - Every call shares the one array per device, and each call clears the part of it
+ *     that must start at zero, so calls that overlap on the GPU (concurrent streams)
+ *     race and give wrong results: serialize them.
+ *   - Bad device data is still reported through the sentinel outputs; there is no
+ *     status word to read back.
+ */
+#define SPEC_NOALLOC_SCRATCH_BYTES (4u << 20)
+spec_status_t spec_accept_block_noalloc(const spec_accept_args_t* accept, spec_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

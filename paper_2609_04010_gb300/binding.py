@@ -88,6 +88,8 @@ def lib(build_if_missing: bool = True):
             L.spec_status_string.argtypes = [ctypes.c_int]
             L.spec_status_string.restype = ctypes.c_char_p
             L.spec_attn_tensor_core_min_rows.restype = i32
+            L.spec_accept_block_noalloc.argtypes = [P, P]
+            L.spec_accept_block_noalloc.restype = ctypes.c_int
             for f in ("spec_workspace_init", "spec_verify_attention", "spec_accept_block",
                       "spec_verify_step", "spec_philox_uniforms", "spec_read_device_status"):
                 getattr(L, f).restype = ctypes.c_int
@@ -222,6 +224,17 @@ def accept_block(target_logits, drafter_logits, block_tokens, temperature, unifo
         ws = new_workspace(workspace_size(accept=a), dev)
     accept_block_args(a, ws, stream)
     return res
+
+
+def accept_block_noalloc(target_logits, drafter_logits, block_tokens, temperature, uniforms,
+                         num_accepted, out_tokens, num_emitted, diag=None, stream=None):
+    """spec_accept_block_noalloc: the acceptance step with the library's fixed scratch
+    array instead of a caller workspace (for callers that cannot allocate device memory;
+    the outputs are the caller's tensors). Calls that overlap on the GPU race."""
+    a = accept_args(target_logits, drafter_logits, block_tokens, temperature, uniforms,
+                    num_accepted, out_tokens, num_emitted, diag)
+    _raise(lib().spec_accept_block_noalloc(ctypes.byref(a), _stream(stream)),
+           "spec_accept_block_noalloc")
 
 
 def philox_uniforms(seed: int, n: int, offset: int = 0, device=None, stream=None) -> torch.Tensor:
