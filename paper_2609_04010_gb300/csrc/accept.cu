@@ -2,7 +2,9 @@
 // drafter rows and the lossless acceptance rule of Alg. "Lossless Psi-Spec decoding
 // (Linear Sampler)" (Appendix B.3; Sec. 4.2).
 //
-// Two launches, no inter-block waiting:
+// Two launches, no inter-block waiting (the second is a programmatic dependent of the
+// first and waits for it on the device; in a verify step the first is a programmatic
+// dependent of the attention kernel and runs beside it):
 //   1. row_stats_kernel: one block per (sequence, row, 8192-entry vocab chunk) reads
 //      the chunk once with 16-byte loads and writes its max, its sum of
 //      exp((l - max)/T) and (greedy rows) its lowest-index argmax.
@@ -13,6 +15,8 @@
 //      bonus) over its slice; the last block of the sequence to finish (atomic ticket)
 //      finds the slice where the ascending cumulative sum crosses u * S and rescans
 //      that slice with a block-wide scan to pick the token.
+#include <cuda_bf16.h>
+
 #include <cfloat>
 #include <climits>
 #include <cmath>
@@ -132,8 +136,9 @@ __device__ __forceinline__ void merge_arg(float& m, int& a, float m2, int a2) {
 }
 
 template <bool BF16, bool VEC>
-__global__ void __launch_bounds__(kStatsThreads, 4) row_stats_kernel(AcceptParams p) {
+__global__ void __launch_bounds__(kStatsThreads, 8) row_stats_kernel(AcceptParams p) {
   constexpr int kPer = kStatsChunk / kStatsThreads;  // 32 values per thread
+  pdl_launch_dependents();
   __shared__ float sh_m[kStatsThreads / 32];
   __shared__ float sh_s[kStatsThreads / 32];
   __shared__ int sh_a[kStatsThreads / 32];
@@ -160,47 +165,61 @@ __global__ void __launch_bounds__(kStatsThreads, 4) row_stats_kernel(AcceptParam
   const float cs = greedy ? 0.f : kLog2e / T;
   if (VEC) {
     // The chunk stays packed in registers (16-byte groups, group g of thread t at
-    // g * threads + t) and is decoded twice: once for the max, once for the sum.
+    // g * threads + t) and is decoded on the fly.
     constexpr int kEpv = BF16 ? 8 : 4;
     constexpr int kVecs = kPer / kEpv;
     const int t = threadIdx.x;
-    uint4 raw[kVecs];
+    uint32_t w[kVecs * 4];
     const uint32_t ninf = BF16 ? 0xFF80FF80u : 0xFF800000u;  // -inf padding past the row end
 #pragma unroll
     for (int k = 0; k < kVecs; ++k) {
       const int e = (k * kStatsThreads + t) * kEpv;
-      raw[k] = e < len ? __ldg(reinterpret_cast<const uint4*>(
-                             static_cast<const char*>(rowp) + static_cast<int64_t>(start + e) * (BF16 ? 2 : 4)))
-                       : make_uint4(ninf, ninf, ninf, ninf);
+      const uint4 r = e < len ? __ldg(reinterpret_cast<const uint4*>(
+                                    static_cast<const char*>(rowp) + static_cast<int64_t>(start + e) * (BF16 ? 2 : 4)))
+                              : make_uint4(ninf, ninf, ninf, ninf);
+      w[4 * k] = r.x; w[4 * k + 1] = r.y; w[4 * k + 2] = r.z; w[4 * k + 3] = r.w;
     }
+    // element q of 16-byte group k
     auto elem = [&](int k, int q) -> float {
-      const int wi = BF16 ? (q >> 1) : q;
-      const uint32_t word = wi == 0 ? raw[k].x : wi == 1 ? raw[k].y : wi == 2 ? raw[k].z : raw[k].w;
-      if (BF16) return __uint_as_float((q & 1) ? (word & 0xffff0000u) : (word << 16));
-      return __uint_as_float(word);
+      if (BF16) {
+        const uint32_t word = w[4 * k + (q >> 1)];
+        return __uint_as_float((q & 1) ? (word & 0xffff0000u) : (word << 16));
+      }
+      return __uint_as_float(w[4 * k + q]);
     };
-    // this thread's elements in increasing index order: a strict > keeps the lowest
-    // index of the maximum; all -inf leaves the first index
-    a = start + t * kEpv;
+    if (greedy) {
+      // this thread's elements in increasing index order: a strict > keeps the lowest
+      // index of the maximum; all -inf leaves the first index
+      a = start + t * kEpv;
 #pragma unroll
-    for (int k = 0; k < kVecs; ++k) {
+      for (int k = 0; k < kVecs; ++k) {
 #pragma unroll
-      for (int q = 0; q < kEpv; ++q) {
-        const float x = elem(k, q);
-        bad |= !(x <= FLT_MAX);  // NaN or +inf (the padding is -inf)
-        if (greedy) {
+        for (int q = 0; q < kEpv; ++q) {
+          const float x = elem(k, q);
+          bad |= x != x;  // NaN (+inf is a legal maximum for a greedy row)
           if (x > m) { m = x; a = start + (k * kStatsThreads + t) * kEpv + q; }
-        } else {
-          m = fmaxf(m, x);
         }
       }
-    }
-    if (a >= start + len) a = INT_MAX;  // a thread past the row end loses every tie
-    if (!greedy && m != -INFINITY) {
+      if (a >= start + len) a = INT_MAX;  // a thread past the row end loses every tie
+    } else {
+      // max (NaN is skipped here and caught by the sum below)
+      if (BF16) {
+        __nv_bfloat162 mx = *reinterpret_cast<const __nv_bfloat162*>(&w[0]);
 #pragma unroll
-      for (int k = 0; k < kVecs; ++k)
+        for (int i = 1; i < kVecs * 4; ++i) mx = __hmax2(mx, *reinterpret_cast<const __nv_bfloat162*>(&w[i]));
+        m = fmaxf(__bfloat162float(mx.x), __bfloat162float(mx.y));
+      } else {
 #pragma unroll
-        for (int q = 0; q < kEpv; ++q) s += ex2((elem(k, q) - m) * cs);
+        for (int i = 0; i < kVecs * 4; ++i) m = fmaxf(m, __uint_as_float(w[i]));
+      }
+      if (m != -INFINITY) {
+#pragma unroll
+        for (int k = 0; k < kVecs; ++k)
+#pragma unroll
+          for (int q = 0; q < kEpv; ++q) s += ex2((elem(k, q) - m) * cs);
+      }
+      // NaN anywhere, or +inf (then +inf - +inf), makes the sum NaN
+      bad |= !(s <= FLT_MAX) || !(m <= FLT_MAX);
     }
   } else {
     float v[kPer];
@@ -209,7 +228,8 @@ __global__ void __launch_bounds__(kStatsThreads, 4) row_stats_kernel(AcceptParam
     a = idx[0];
 #pragma unroll
     for (int k = 0; k < kPer; ++k) {
-      bad |= !(v[k] <= FLT_MAX) && idx[k] != INT_MAX;  // NaN or +inf inside the row
+      // greedy rows: NaN; tempered rows: NaN or +inf (padding past the row end is -inf)
+      bad |= greedy ? (v[k] != v[k]) : !(v[k] <= FLT_MAX);
       if (greedy) {
         if (v[k] > m) { m = v[k]; a = idx[k]; }
       } else {
@@ -326,7 +346,7 @@ __device__ __forceinline__ void final_weights(const AcceptParams& p, const void*
 }
 
 template <bool BF16, bool VEC>
-__global__ void __launch_bounds__(kSampleThreads) decide_sample_kernel(AcceptParams p) {
+__global__ void __launch_bounds__(kSampleThreads, 5) decide_sample_kernel(AcceptParams p) {
   constexpr int kMaxGamma = 64;
   constexpr int kPer = kSamplePerThread;
   __shared__ float rM[2 * kMaxGamma], rS[2 * kMaxGamma];
@@ -348,32 +368,43 @@ __global__ void __launch_bounds__(kSampleThreads) decide_sample_kernel(AcceptPar
     s_owner = INT_MAX;
     s_token = -1;
   }
+  pdl_wait_prior();  // the row statistics kernel has finished and its writes are visible
   __syncthreads();
 
-  // 1. merge the chunk statistics of every row this sequence uses
+  // 1. merge the chunk statistics of every row this sequence uses: one warp per row,
+  // the lanes load the row's chunk partials in parallel and reduce them with shuffles
+  // (chunks are in increasing index order, so ties keep the lowest index)
   const int rows_needed = greedy ? gamma : nrows;
-  for (int r = tid; r < rows_needed; r += kSampleThreads) {
-    const RowPartial* rp = p.partials + (static_cast<int64_t>(b) * nrows + r) * p.nchunk;
-    float M = -INFINITY;
-    int A = INT_MAX;
-    uint32_t bad = 0;
-    for (int k = 0; k < p.nchunk; ++k) {
-      const RowPartial q = rp[k];
-      bad |= q.bad;
-      if (A == INT_MAX || q.m > M) { M = q.m; A = q.arg; }
-    }
-    float S = 0.f;
-    if (!greedy) {
-      for (int k = 0; k < p.nchunk; ++k) {
+  {
+    const int warp = tid >> 5, lane = tid & 31;
+    for (int r = warp; r < rows_needed; r += kSampleThreads / 32) {
+      const RowPartial* rp = p.partials + (static_cast<int64_t>(b) * nrows + r) * p.nchunk;
+      float M = -INFINITY, S = 0.f;
+      int A = INT_MAX;
+      uint32_t bad = 0;
+      for (int k = lane; k < p.nchunk; k += 32) {
         const RowPartial q = rp[k];
-        if (q.m != -INFINITY) S += q.s * ex2((q.m - M) * c);
+        bad |= q.bad;
+        if (greedy) merge_arg(M, A, q.m, q.arg);
+        else merge_ms(M, S, q.m, q.s, c);
       }
-      if (M == -INFINITY || !(S > 0.f) || !(S <= FLT_MAX)) bad = 1;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        const float m2 = __shfl_xor_sync(0xffffffffu, M, o);
+        const float s2 = __shfl_xor_sync(0xffffffffu, S, o);
+        const int a2 = __shfl_xor_sync(0xffffffffu, A, o);
+        bad |= __shfl_xor_sync(0xffffffffu, bad, o);
+        if (greedy) merge_arg(M, A, m2, a2);
+        else merge_ms(M, S, m2, s2, c);
+      }
+      if (!greedy && (M == -INFINITY || !(S > 0.f) || !(S <= FLT_MAX))) bad = 1;
+      if (lane == 0) {
+        rM[r] = M;
+        rS[r] = S;
+        rA[r] = A;
+        if (bad) atomicOr(&s_bad, 1);
+      }
     }
-    rM[r] = M;
-    rS[r] = S;
-    rA[r] = A;
-    if (bad) atomicOr(&s_bad, 1);
   }
   if (tid < gamma) {
     const int t = p.tokens[static_cast<int64_t>(b) * gamma + tid];
@@ -515,34 +546,57 @@ __global__ void __launch_bounds__(kSampleThreads) decide_sample_kernel(AcceptPar
   if (!s_last) return;
   __threadfence();
 
-  // 4. the last block: locate the crossing slice, then the crossing token
+  // 4. the last block: locate the crossing slice (warp 0: the slices' sums in parallel,
+  // a warp scan in slice order, a ballot for the first crossing), then the token
   const float u = p.uniforms[static_cast<int64_t>(b) * gamma + gamma - 1];
-  if (tid == 0) {
+  if (tid < 32) {
+    const int lane = tid;
     const SliceSum* ss = p.slices + static_cast<int64_t>(b) * p.nslice;
-    int use_res = bonus ? 0 : 1;
-    float total = 0.f;
-    for (int k = 0; k < p.nslice; ++k) total += use_res ? __ldcg(&ss[k].w) : __ldcg(&ss[k].e);
-    if (use_res && !(total > 0.f)) {  // residual without mass: draw from p_n itself
-      use_res = 0;
-      total = 0.f;
-      for (int k = 0; k < p.nslice; ++k) total += __ldcg(&ss[k].e);
+    auto scan32 = [&](float v) {
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const float y = __shfl_up_sync(0xffffffffu, v, o);
+        if (lane >= o) v += y;
+      }
+      return v;
+    };
+    // totals, as the end of the inclusive scan in slice order
+    float tw = 0.f, te = 0.f;
+    for (int k0 = 0; k0 < p.nslice; k0 += 32) {
+      const int k = k0 + lane;
+      const float vw = k < p.nslice ? __ldcg(&ss[k].w) : 0.f;
+      const float ve = k < p.nslice ? __ldcg(&ss[k].e) : 0.f;
+      tw += __shfl_sync(0xffffffffu, scan32(vw), 31);
+      te += __shfl_sync(0xffffffffu, scan32(ve), 31);
     }
-    const float target = u * total;
-    float cum = 0.f;
-    int star = -1;
-    for (int k = 0; k < p.nslice; ++k) {
-      const float x = use_res ? __ldcg(&ss[k].w) : __ldcg(&ss[k].e);
-      if (x > 0.f && cum + x >= target) { star = k; break; }
-      cum += x;
+    // residual without mass (only through rounding): draw from p_n itself
+    const int use_res = (!bonus && tw > 0.f) ? 1 : 0;
+    const float target = u * (use_res ? tw : te);
+    float carry = 0.f;
+    int star = -1, lastk = -1;
+    float base = 0.f;
+    for (int k0 = 0; k0 < p.nslice && star < 0; k0 += 32) {
+      const int k = k0 + lane;
+      const float v = k < p.nslice ? (use_res ? __ldcg(&ss[k].w) : __ldcg(&ss[k].e)) : 0.f;
+      const float incl = scan32(v);
+      const unsigned hit = __ballot_sync(0xffffffffu, v > 0.f && carry + incl >= target);
+      const unsigned pos = __ballot_sync(0xffffffffu, v > 0.f);
+      if (pos) lastk = k0 + 31 - __clz(pos);
+      if (hit) {
+        const int f = __ffs(hit) - 1;
+        star = k0 + f;
+        base = carry + __shfl_sync(0xffffffffu, incl - v, f);
+      }
+      carry += __shfl_sync(0xffffffffu, incl, 31);
     }
-    if (star < 0) {  // rounding left u*S above every sum: last positive-weight token
-      for (int k = p.nslice - 1; k >= 0 && s_token < 0; --k)
-        s_token = use_res ? __ldcg(&ss[k].wlast) : __ldcg(&ss[k].elast);
+    if (lane == 0) {
+      if (star < 0 && lastk >= 0)  // rounding left u*S above every sum: last positive weight
+        s_token = use_res ? __ldcg(&ss[lastk].wlast) : __ldcg(&ss[lastk].elast);
+      s_star = star;
+      s_use_res = use_res;
+      s_base = base;
+      s_target = target;
     }
-    s_star = star;
-    s_use_res = use_res;
-    s_base = cum;
-    s_target = target;
   }
   __syncthreads();
   if (s_star >= 0) {
@@ -610,19 +664,34 @@ __global__ void philox_uniforms_kernel(uint64_t seed, uint64_t offset, int64_t n
 }
 
 template <bool BF16, bool VEC>
-cudaError_t launch_typed(const AcceptParams& p, cudaStream_t stream) {
+cudaError_t launch_typed(const AcceptParams& p, cudaStream_t stream, bool overlap_prior) {
   const int64_t items = static_cast<int64_t>(p.batch) * (2 * p.gamma - 1) * p.nchunk;
-  row_stats_kernel<BF16, VEC><<<static_cast<unsigned>(items), kStatsThreads, 0, stream>>>(p);
-  cudaError_t e = cudaGetLastError();
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  // row statistics: a programmatic dependent of the attention kernel in a verify step
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(items));
+  cfg.blockDim = dim3(kStatsThreads);
+  cfg.stream = stream;
+  cfg.attrs = attr;
+  cfg.numAttrs = overlap_prior ? 1 : 0;
+  cudaError_t e = cudaLaunchKernelEx(&cfg, row_stats_kernel<BF16, VEC>, p);
   if (e != cudaSuccess) return e;
-  decide_sample_kernel<BF16, VEC><<<dim3(p.nslice, p.batch), kSampleThreads, 0, stream>>>(p);
+  // decisions and draws: a programmatic dependent of the statistics kernel (it waits
+  // for that kernel's completion before reading the partials)
+  cfg.gridDim = dim3(p.nslice, p.batch);
+  cfg.blockDim = dim3(kSampleThreads);
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, decide_sample_kernel<BF16, VEC>, p);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 
 }  // namespace
 
 cudaError_t launch_accept(const spec_accept_args_t& a, const AcceptLayout& L, char* ws, int,
-                          cudaStream_t stream) {
+                          cudaStream_t stream, bool overlap_prior) {
   AcceptParams p;
   p.batch = a.batch;
   p.gamma = a.gamma;
@@ -647,13 +716,17 @@ cudaError_t launch_accept(const spec_accept_args_t& a, const AcceptLayout& L, ch
   const bool vec = (static_cast<size_t>(a.vocab) * esz) % 16 == 0 &&
                    reinterpret_cast<uintptr_t>(a.target_logits) % 16 == 0 &&
                    reinterpret_cast<uintptr_t>(a.drafter_logits) % 16 == 0;
-  if (bf16) return vec ? launch_typed<true, true>(p, stream) : launch_typed<true, false>(p, stream);
-  return vec ? launch_typed<false, true>(p, stream) : launch_typed<false, false>(p, stream);
+  if (bf16)
+    return vec ? launch_typed<true, true>(p, stream, overlap_prior)
+               : launch_typed<true, false>(p, stream, overlap_prior);
+  return vec ? launch_typed<false, true>(p, stream, overlap_prior)
+             : launch_typed<false, false>(p, stream, overlap_prior);
 }
 
 cudaError_t launch_philox(uint64_t seed, uint64_t offset, int64_t n, float* out, cudaStream_t s) {
   if (n == 0) return cudaSuccess;
   const int64_t blocks = (n + 255) / 256;
+  (void)cudaGetLastError();  // report this launch's error only
   philox_uniforms_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(seed, offset, n, out);
   return cudaGetLastError();
 }

@@ -60,16 +60,13 @@ extern "C" spec_status_t spec_accept_block_noalloc(const spec_accept_args_t* acc
   if (L.end > kScratchBytes) return SPEC_ERR_WORKSPACE_TOO_SMALL;  // beyond the fixed array
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
   int dev = 0;
-  if (stream != nullptr) {
-    if (cudaStreamGetDevice(stream, &dev) != cudaSuccess) return SPEC_ERR_CUDA;
-  } else if (cudaGetDevice(&dev) != cudaSuccess) {
-    return SPEC_ERR_CUDA;
-  }
+  if (stream_device(stream, &dev) != cudaSuccess) return SPEC_ERR_CUDA;
   int cur = -1;
   if (cudaGetDevice(&cur) != cudaSuccess) return SPEC_ERR_CUDA;
   if (cur != dev && cudaSetDevice(dev) != cudaSuccess) return SPEC_ERR_CUDA;
   void* ptr = nullptr;
   if (scratch_address(dev, &ptr) != cudaSuccess) return SPEC_ERR_CUDA;
+  (void)cudaGetLastError();  // a failed call before this one must not fail our launches
   char* ws = static_cast<char*>(ptr);
   // The status word and the tickets must start at zero; the array keeps whatever the
   // previous call (possibly an interrupted one) left, so clear them on the stream.

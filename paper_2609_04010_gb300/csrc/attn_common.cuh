@@ -91,74 +91,61 @@ __device__ __forceinline__ void write_lse(const AttnParams& p, int b, int g, int
 }
 
 // Combines the split-KV partials of one unit, held in slots [slot0, slot0 + nslots), for
-// rows [row0, row0 + nrows) and writes the final outputs. All nthreads threads of the
-// block call it together (it synchronizes the block between its two passes); sh_m and
-// sh_l are shared-memory scratch for nrows floats each. Pass 1 takes each row's
-// largest base-2 max M and its total L = sum_s l_s 2^(m_s - M); pass 2 gives every
-// (row, 4-column) item all its slot loads at once, so the merge is not a chain of
-// dependent L2 round trips.
+// rows [row0, row0 + nrows) and writes the final outputs (nthreads threads from tid
+// cooperate; no block synchronization). Each (row, 8-column) item walks the slots in
+// batches of four, loading a batch's (m, l) pairs and output pieces together and
+// folding them into a running base-2 max, so a unit with up to four slots costs one
+// round trip to L2.
 template <int D>
 __device__ void merge_unit(const AttnParams& p, int b, int g, int row0, int nrows, int64_t slot0,
-                           int nslots, float* sh_m, float* sh_l, int tid, int nthreads) {
-  for (int r = tid; r < nrows; r += nthreads) {
-    float M = -INFINITY;
+                           int nslots, int tid, int nthreads) {
+  constexpr int C8 = D / 8;
+  for (int idx = tid; idx < nrows * C8; idx += nthreads) {
+    const int r = idx / C8, c8 = idx % C8;
+    float M = -INFINITY, L = 0.f, acc[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) acc[e] = 0.f;
     bool bad = false;
-    for (int s = 0; s < nslots; ++s) {
-      const float2 ml = __ldcg(&p.partial_ml[(slot0 + s) * p.slot_rows + r]);
-      bad |= ml.y < 0.f;
-      if (ml.y > 0.f) M = fmaxf(M, ml.x);
-    }
-    float L = 0.f;
-    for (int s = 0; s < nslots; ++s) {
-      const float2 ml = __ldcg(&p.partial_ml[(slot0 + s) * p.slot_rows + r]);
-      if (ml.y > 0.f) L += ml.y * ex2(ml.x - M);
+    for (int s0 = 0; s0 < nslots; s0 += 4) {
+      float2 ml[4];
+      float4 lo[4], hi[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        if (s0 + e < nslots) {
+          const int64_t slot = (slot0 + s0 + e) * p.slot_rows + r;
+          ml[e] = __ldcg(&p.partial_ml[slot]);
+          const float4* src = reinterpret_cast<const float4*>(p.partial_o + slot * D) + 2 * c8;
+          lo[e] = __ldcg(src);
+          hi[e] = __ldcg(src + 1);
+        } else {
+          ml[e] = make_float2(-INFINITY, 0.f);
+        }
+      }
+      float mb = M;
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        bad |= ml[e].y < 0.f;
+        if (ml[e].y > 0.f) mb = fmaxf(mb, ml[e].x);
+      }
+      if (mb == -INFINITY) continue;
+      const float scale = M == -INFINITY ? 0.f : ex2(M - mb);
+      L *= scale;
+#pragma unroll
+      for (int e = 0; e < 8; ++e) acc[e] *= scale;
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        if (!(ml[e].y > 0.f)) continue;
+        const float w = ex2(ml[e].x - mb);
+        L += ml[e].y * w;
+        acc[0] += lo[e].x * w; acc[1] += lo[e].y * w; acc[2] += lo[e].z * w; acc[3] += lo[e].w * w;
+        acc[4] += hi[e].x * w; acc[5] += hi[e].y * w; acc[6] += hi[e].z * w; acc[7] += hi[e].w * w;
+      }
+      M = mb;
     }
     const bool dead = bad || !(L > 0.f);
-    sh_m[r] = M;
-    sh_l[r] = dead ? 0.f : L;
-    write_lse(p, b, g, row0 + r, M, L, dead);
+    write_out_row<D>(p, b, g, row0 + r, c8 * 8, acc, dead ? 0.f : 1.f / L);
+    if (c8 == 0) write_lse(p, b, g, row0 + r, M, L, dead);
   }
-  __syncthreads();
-  constexpr int C4 = D / 4;
-  for (int idx = tid; idx < nrows * C4; idx += nthreads) {
-    const int r = idx / C4, c4 = idx % C4;
-    const float M = sh_m[r], L = sh_l[r];
-    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (L > 0.f) {
-      int s = 0;
-      for (; s + 4 <= nslots; s += 4) {
-        float2 ml[4];
-        float4 o[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const int64_t slot = (slot0 + s + e) * p.slot_rows + r;
-          ml[e] = __ldcg(&p.partial_ml[slot]);
-          o[e] = __ldcg(reinterpret_cast<const float4*>(p.partial_o + slot * D) + c4);
-        }
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float w = ml[e].y > 0.f ? ex2(ml[e].x - M) : 0.f;
-          acc.x += o[e].x * w; acc.y += o[e].y * w; acc.z += o[e].z * w; acc.w += o[e].w * w;
-        }
-      }
-      for (; s < nslots; ++s) {
-        const int64_t slot = (slot0 + s) * p.slot_rows + r;
-        const float2 ml = __ldcg(&p.partial_ml[slot]);
-        const float4 o = __ldcg(reinterpret_cast<const float4*>(p.partial_o + slot * D) + c4);
-        const float w = ml.y > 0.f ? ex2(ml.x - M) : 0.f;
-        acc.x += o.x * w; acc.y += o.y * w; acc.z += o.z * w; acc.w += o.w * w;
-      }
-    }
-    const float inv = L > 0.f ? 1.f / L : 0.f;
-    const int row = row0 + r, j = row / p.group, h = g * p.group + row % p.group;
-    __nv_bfloat16* dst = static_cast<__nv_bfloat16*>(p.out) +
-                         ((static_cast<int64_t>(b) * p.gamma + j) * p.hq + h) * D + c4 * 4;
-    const __nv_bfloat162 lo = __floats2bfloat162_rn(acc.x * inv, acc.y * inv);
-    const __nv_bfloat162 hi = __floats2bfloat162_rn(acc.z * inv, acc.w * inv);
-    *reinterpret_cast<uint2*>(dst) = make_uint2(*reinterpret_cast<const uint32_t*>(&lo),
-                                               *reinterpret_cast<const uint32_t*>(&hi));
-  }
-  __syncthreads();
 }
 #endif
 

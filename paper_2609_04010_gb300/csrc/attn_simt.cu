@@ -74,6 +74,7 @@ template <int D>
 __global__ void __launch_bounds__(NT) attn_simt_kernel(AttnParams p) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   SimtSmem<D>& sm = *reinterpret_cast<SimtSmem<D>*>(smem_raw);
+  pdl_launch_dependents();  // the acceptance kernels of a verify step may start beside us
   const int split = blockIdx.x, g = blockIdx.y;
   const int b = blockIdx.z / p.row_tiles, rt = blockIdx.z % p.row_tiles;
   const int tid = threadIdx.x;
@@ -273,7 +274,7 @@ __global__ void __launch_bounds__(NT) attn_simt_kernel(AttnParams p) {
   __syncthreads();
   if (!sm.last) return;
   __threadfence();
-  merge_unit<D>(p, b, g, row0, nrows, unit * p.nsplit, p.nsplit, &sm.s[0][0], &sm.s[1][0], tid, NT);
+  merge_unit<D>(p, b, g, row0, nrows, unit * p.nsplit, p.nsplit, tid, NT);
 }
 
 }  // namespace

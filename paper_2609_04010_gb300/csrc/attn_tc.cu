@@ -299,6 +299,7 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
   int* pb = reinterpret_cast<int*>(smem + C::OFF_PB);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  pdl_launch_dependents();  // the acceptance kernels of a verify step may start beside us
 
   // ---- roles ----
   // Softmax warps take part only as far as the row tile has real rows (32 per warp).
@@ -711,12 +712,10 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
   // deferred merges of split units this block completed, by all of its threads
   if (!*abort_flag) {
     const int nm = *merge_count;
-    float* sh = reinterpret_cast<float*>(smem + C::OFF_P);  // P tile is free now
+    if (nm > 0) __threadfence();
     for (int mi = 0; mi < nm; ++mi) {
       const int* e = merges + 8 * mi;
-      __threadfence();
-      merge_unit<D>(p, e[0], e[1], e[2], e[3], e[4], e[5], sh, sh + kTcMaxRows, threadIdx.x,
-                    C::THREADS);
+      merge_unit<D>(p, e[0], e[1], e[2], e[3], e[4], e[5], threadIdx.x, C::THREADS);
     }
   }
 }

@@ -18,10 +18,12 @@ constexpr size_t kWsHeader = 256;  // [0] = status word (uint32)
 inline size_t ws_round(size_t x) { return (x + kWsAlign - 1) / kWsAlign * kWsAlign; }
 
 // --- acceptance ---
-constexpr int kStatsThreads = 256;
-constexpr int kStatsChunk = 8192;                          // vocab elements per row item
-constexpr int kSampleThreads = 256;
-constexpr int kSampleSlice = 8192;                         // vocab elements per sample block
+// 128-thread blocks with few registers, so that they fit beside a resident attention
+// block when the verify step overlaps the two parts.
+constexpr int kStatsThreads = 128;
+constexpr int kStatsChunk = 4096;                          // vocab elements per row item
+constexpr int kSampleThreads = 128;
+constexpr int kSampleSlice = 4096;                         // vocab elements per sample block
 constexpr int kSamplePerThread = kSampleSlice / kSampleThreads;  // contiguous per thread
 
 struct RowPartial {  // one (sequence, row, vocab chunk) item of the row statistics
@@ -62,8 +64,11 @@ AttnPlan attn_plan(const spec_attn_args_t& a, size_t base, int num_sms, int path
 // ----------------------------------------------------------------------------------
 // Launchers (defined in the .cu files); all return cudaGetLastError() of the launch.
 // ----------------------------------------------------------------------------------
+// overlap_prior: launch the acceptance kernels as programmatic dependents of the kernel
+// just launched on the stream (the attention kernel of the same verify step, which
+// reads none of their inputs and writes none of their outputs).
 cudaError_t launch_accept(const spec_accept_args_t& a, const AcceptLayout& L, char* ws,
-                          int num_sms, cudaStream_t stream);
+                          int num_sms, cudaStream_t stream, bool overlap_prior = false);
 cudaError_t launch_attn_simt(const spec_attn_args_t& a, const AttnPlan& P, char* ws,
                              cudaStream_t stream);
 cudaError_t launch_attn_tc(const spec_attn_args_t& a, const AttnPlan& P, char* ws,
@@ -78,6 +83,19 @@ constexpr int kTcKeyTile = 64;
 constexpr int kTcMaxRows = 256;  // two M = 128 tiles per block
 
 int tc_min_rows();
+
+// The device a stream belongs to. cudaStreamGetDevice is not allowed on a capturing
+// stream (it invalidates the capture), so a stream under capture is taken to belong
+// to the current device, the one its captured work must run on.
+inline cudaError_t stream_device(cudaStream_t stream, int* dev) {
+  if (stream != nullptr) {
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    const cudaError_t e = cudaStreamIsCapturing(stream, &cs);
+    if (e != cudaSuccess) return e;
+    if (cs == cudaStreamCaptureStatusNone) return cudaStreamGetDevice(stream, dev);
+  }
+  return cudaGetDevice(dev);
+}
 int tc_ctas_per_sm(int head_dim, int rows_per_cta, int batch);
 size_t tc_smem_bytes(int head_dim, int rows_per_cta, int batch);
 constexpr int kTcMaxBatch = 4096;  // batch prefix sums live in shared memory
@@ -99,6 +117,13 @@ __device__ __forceinline__ float ex2(float x) {
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
 }
+
+// Programmatic dependent launch: let the next kernel on the stream start now / wait for
+// the kernel this one depends on (no-ops for kernels launched without the attribute).
+__device__ __forceinline__ void pdl_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait_prior() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 
 __device__ __forceinline__ void set_status(uint32_t* status, uint32_t flag) {
   atomicOr(status, flag);

@@ -72,3 +72,48 @@ def test_workspace_too_small_is_rejected():
     with pytest.raises(binding.SpecError) as e:
         binding.accept_block_args(c, ws)
     assert e.value.code == 3
+
+
+@pytest.mark.parametrize("name,path", [("tiny", binding.ATTN_TENSOR_CORES),
+                                       ("llama8b", binding.ATTN_AUTO),
+                                       ("tiny", binding.ATTN_CUDA_CORES)])
+def test_step_replays_in_a_cuda_graph(name, path):
+    """spec_verify_step captured on a stream replays to the eager call's outputs, bit
+    for bit, replay after replay (the workspace's tickets reset themselves)."""
+    wl = W.workload(name)
+    ai, ci = wl.attn_inputs(seed=3), wl.accept_inputs(seed=3)
+    at, ct = attn_tensors(ai), accept_tensors(ci)
+    B, G = ci.batch, ci.gamma
+
+    def outputs():
+        return dict(out=torch.empty_like(at[0]),
+                    lse=torch.empty(at[0].shape[:3], dtype=torch.float32, device="cuda"),
+                    num_accepted=torch.empty(B, dtype=torch.int32, device="cuda"),
+                    out_tokens=torch.empty(B, G + 1, dtype=torch.int32, device="cuda"),
+                    num_emitted=torch.empty(B, dtype=torch.int32, device="cuda"),
+                    diag=torch.empty(B, G, 2, dtype=torch.float32, device="cuda"))
+
+    def args(r):
+        a = binding.attn_args(*at, r["out"], r["lse"], path=path)
+        c = binding.accept_args(*ct, r["num_accepted"], r["out_tokens"], r["num_emitted"],
+                                r["diag"])
+        return a, c
+
+    eager, graphed = outputs(), outputs()
+    a0, c0 = args(eager)
+    a1, c1 = args(graphed)
+    ws0 = binding.new_workspace(binding.workspace_size(a0, c0))
+    ws1 = binding.new_workspace(binding.workspace_size(a1, c1))
+    binding.verify_step_args(a0, c0, ws0)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        binding.verify_step_args(a1, c1, ws1)
+    for _ in range(3):
+        for v in graphed.values():
+            v.fill_(0)
+        g.replay()
+        torch.cuda.synchronize()
+        assert binding.read_device_status(ws1) == (0, 0)
+        for k in eager:
+            assert torch.equal(eager[k].nan_to_num(-7), graphed[k].nan_to_num(-7)), k
