@@ -144,7 +144,8 @@ typedef struct {
   int32_t* out_tokens;         /* [batch][gamma+1]                                          */
   int32_t* num_emitted;        /* [batch]                                                   */
   float* diag;                 /* [batch][gamma][2] = (p_i(t_i), q_i(t_i)) for the decisions
-                                  taken (entry 0 and untaken = NaN; greedy: (match, 1)), or NULL */
+                                  taken (entry 0 = (0, 0); untaken = NaN; greedy: (match, 1);
+                                  a sequence with bad input: all NaN), or NULL              */
 } spec_accept_args_t;
 
 /* Bytes of workspace the calls below need for these arguments (either may be NULL). */
@@ -194,8 +195,8 @@ int32_t spec_attn_tensor_core_min_rows(void);
  * lives in one device array of SPEC_NOALLOC_SCRATCH_BYTES owned by the library, which
  * every GPU that loads the library keeps until the process exits.
  *   - Arguments: as spec_accept_block (device pointers, same layouts); no workspace.
- *   - Limit: the scratch this batch needs (16 bytes per (sequence, row, 8192-entry
- *     vocab chunk) plus 16 bytes per (sequence, 8192-entry slice), rounded up) must fit
+ *   - Limit: the scratch this batch needs (16 bytes per (sequence, row, 4096-entry
+ *     vocab chunk) plus 16 bytes per (sequence, 4096-entry slice), rounded up) must fit
  *     in SPEC_NOALLOC_SCRATCH_BYTES; otherwise SPEC_ERR_WORKSPACE_TOO_SMALL, with
  *     nothing launched. Other argument errors as spec_accept_block.
  *   - Allocates nothing: no cudaMalloc, cudaFree or allocating library routine. The

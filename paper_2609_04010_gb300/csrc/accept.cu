@@ -5,7 +5,7 @@
 // Two launches, no inter-block waiting (the second is a programmatic dependent of the
 // first and waits for it on the device; in a verify step the first is a programmatic
 // dependent of the attention kernel and runs beside it):
-//   1. row_stats_kernel: one block per (sequence, row, 8192-entry vocab chunk) reads
+//   1. row_stats_kernel: one block per (sequence, row, 4096-entry vocab chunk) reads
 //      the chunk once with 16-byte loads and writes its max, its sum of
 //      exp((l - max)/T) and (greedy rows) its lowest-index argmax.
 //   2. decide_sample_kernel: grid (vocab slice, sequence). Every block merges the row

@@ -19,7 +19,7 @@ from paper_2609_04010_gb300 import workloads as W
 
 def test_oversized_batch_is_rejected_without_launch():
     binding.lib()
-    # 512 sequences x 127 rows x 16 chunks x 16 bytes is far beyond the fixed 4 MiB array;
+    # 512 sequences x 127 rows x 32 chunks x 16 bytes is far beyond the fixed 4 MiB array;
     # the size check happens before any device call (none is available here).
     a = binding.AcceptArgs(512, 64, 128256, binding.SPEC_BF16)
     for f in ("target_logits", "drafter_logits", "block_tokens", "temperature", "uniforms",
