@@ -8,21 +8,23 @@
 // group has up to 256 rows), so each KV page is read from HBM once.
 //
 // Warp roles (one block per SM, persistent):
-//   warps 0,2,3 KV producers: gather each 64-key tile of K and V page by page through
+//   warps 0,2   KV producers: gather each 64-key tile of K and V page by page through
 //               the page table, one 5-D cp.async.bulk.tensor box (128-byte swizzle) per
-//               (page, K or V), spread over three issuing warps (one issuer cannot keep
+//               (page, K or V), spread over two issuing warps (one issuer cannot keep
 //               the copy engine busy with page-sized boxes), into a multi-stage ring; an
 //               mbarrier per stage carries the byte count. The box lays a page out in
 //               8-key groups so that the MMAs below can span pages.
-//   warp 1      MMA issuer: S = Q K^T (tcgen05.mma kind::f16, M = 128, N = 64, K = 16
-//               steps over D) into a double-buffered fp32 TMEM accumulator, then
-//               O += P V (N = D) with P from shared memory and V read MN-major.
-//   warps 4..   softmax warps with real rows (one per 32 query rows); the others idle.
-//   warps 4..   softmax (one warpgroup per M tile, one thread per query row): load S
-//               from TMEM, scale and mask, online softmax in base 2 with lazy rescale
-//               of O (only when the running max grows by more than 2^8), write P as
-//               bf16 in the swizzled layout the MMA reads, and finally read O from
-//               TMEM and write the output.
+//   warp 1      Q K^T issuer: S = Q K^T (tcgen05.mma kind::f16, M = 128, N = 64, K = 16
+//               steps over D) into a double-buffered fp32 TMEM accumulator.
+//   warp 3      P V issuer: O += P V (N = D) with P from shared memory, V read MN-major.
+//   warps 4..11 softmax, one thread per query row; with one M tile two warps share a
+//               32-row quadrant, one per half of each tile's keys, each with its own
+//               online softmax and O (merged at the end of a unit); with two M tiles
+//               one warp per quadrant. Load S from TMEM, scale and mask, online
+//               softmax in base 2 with lazy rescale of O (only when the running max
+//               grows by more than 2^8), write P as bf16 in the swizzled layout the MMA
+//               reads (double-buffered with one M tile), and at the end of a unit read
+//               O from TMEM and write the output. Warps without real rows idle.
 // Work is balanced across blocks "stream-K" style: all 64-key tiles of all (sequence,
 // KV head, row tile) units form one list that is cut into equal contiguous ranges; a
 // unit split between blocks is merged from fp32 partials by the last block to finish
@@ -41,25 +43,33 @@ constexpr int TK = kTcKeyTile;               // keys per tile
 template <int D, int MT>
 struct TcCfg {
   static constexpr int DH = D / 64;                   // 128-byte column halves of a row
-  static constexpr int STAGES = (D == 128 && MT == 2) ? 3 : 4;
-  static constexpr int THREADS = 128 + 128 * MT;
+  // Softmax warps per 32-row quadrant. With one M tile, two warps share each quadrant,
+  // one per half of the tile's keys, each with its own online-softmax state and its own
+  // O accumulator (merged once per unit); with two M tiles one warp per quadrant.
+  static constexpr int SPLIT = MT == 1 ? 2 : 1;
+  static constexpr int KH = TK / SPLIT;               // keys of a tile per softmax warp
+  static constexpr int PB = MT == 1 ? 2 : 1;          // P buffers (double with one M tile)
+  static constexpr int STAGES = (D == 128 && MT == 2) || (D == 64 && MT == 1) ? 3 : 4;
+  static constexpr int THREADS = 128 + 256;           // 4 producer / MMA warps + 8 softmax
   static constexpr uint32_t Q_BYTES = MT * DH * 16384;  // [MT][DH][128 rows x 128 B]
   static constexpr uint32_t KV_BYTES = DH * 8192;       // one stage of K (or V): [DH][64 x 128 B]
-  static constexpr uint32_t P_BYTES = MT * 16384;       // [MT][128 rows x 128 B]
+  static constexpr uint32_t P_BYTES = PB * MT * 16384;  // [PB][MT][128 rows x 128 B]
   static constexpr uint32_t OFF_Q = 0;
   static constexpr uint32_t OFF_K = OFF_Q + Q_BYTES;
   static constexpr uint32_t OFF_V = OFF_K + STAGES * KV_BYTES;
   static constexpr uint32_t OFF_P = OFF_V + STAGES * KV_BYTES;
   static constexpr uint32_t OFF_BAR = OFF_P + P_BYTES;
-  // barriers: kv_full[S], kv_empty[S], s_full[MT][2], s_free[MT][2], p_full[MT],
-  // pv_done[MT], seg_ready, grp, drain
-  static constexpr int NBAR = 2 * STAGES + 6 * MT + 3;
-  static constexpr uint32_t OFF_MISC = OFF_BAR + NBAR * 8;  // tmem base, abort, flag, merges
-  static constexpr uint32_t OFF_MERGE = OFF_MISC + 16;          // 2 deferred merges x 8 ints
-  static constexpr uint32_t OFF_PB = (OFF_MERGE + 64 + 15) / 16 * 16;
-  static constexpr uint32_t TMEM_COLS = (MT * 128 + MT * D) <= 256 ? 256 : 512;
+  // barriers: kv_full[S], kv_empty[S], s_full[MT][2], s_free[MT][2], p_full[MT][PB],
+  // pv_done[MT][PB], seg_ready, drain[2], xch[4]
+  static constexpr int NBAR = 2 * STAGES + 4 * MT + 2 * MT * PB + 3 + 4;
+  static constexpr uint32_t OFF_MISC = OFF_BAR + NBAR * 8;  // tmem base, abort, pending count
+  static constexpr uint32_t OFF_XCH = OFF_MISC + 16;        // [4][2][32] float2 (m, l) per half
+  static constexpr uint32_t OFF_PEND = OFF_XCH + (SPLIT == 2 ? 4 * 2 * 32 * 8 : 0);  // [2][8]
+  static constexpr uint32_t OFF_PB = (OFF_PEND + 64 + 15) / 16 * 16;
+  static constexpr uint32_t TMEM_NEED = MT * 128 + MT * SPLIT * D;
+  static constexpr uint32_t TMEM_COLS = TMEM_NEED <= 256 ? 256 : 512;
   static constexpr uint32_t S_COL = 0;           // S[mt][buf] at (mt * 2 + buf) * 64
-  static constexpr uint32_t O_COL = MT * 128;    // O[mt] at O_COL + mt * D
+  static constexpr uint32_t O_COL = MT * 128;    // O[mt][half] at O_COL + (mt * SPLIT + half) * D
   static size_t smem_bytes(int batch) { return OFF_PB + 4u * (batch + 1) + 1024; }
 };
 
@@ -255,16 +265,21 @@ __device__ __forceinline__ int owner_of(int64_t t, int64_t total, int ctas) {
 }
 
 // A segment is bad when its sequence length is malformed or a page it reads is out
-// of range. The whole warp cooperates; every lane gets the answer.
+// of range. The whole warp cooperates (up to 128 page ids in flight per round trip);
+// every lane gets the answer.
 __device__ __forceinline__ bool segment_bad(const Seg& s, const AttnParams& p) {
   if (!s.len_ok) return true;
   const int k0 = s.tile0 * TK;
   const int k1 = min(s.kv_len, (s.tile0 + s.ntile) * TK);
   const int pg0 = k0 / p.page_size, pg1 = (k1 - 1) / p.page_size;
+  const int* row = p.page_table + static_cast<int64_t>(s.b) * p.max_pages;
   bool bad = false;
-  for (int pg = pg0 + (threadIdx.x & 31); pg <= pg1; pg += 32) {
-    const int id = p.page_table[static_cast<int64_t>(s.b) * p.max_pages + pg];
-    bad |= id < 0 || id >= p.num_pages;
+  for (int base = pg0 + (threadIdx.x & 31); base <= pg1; base += 128) {
+    int id[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) id[u] = base + 32 * u <= pg1 ? __ldg(row + base + 32 * u) : 0;
+#pragma unroll
+    for (int u = 0; u < 4; ++u) bad |= id[u] < 0 || id[u] >= p.num_pages;
   }
   return __any_sync(0xffffffffu, bad);
 }
@@ -277,6 +292,7 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
                    const __grid_constant__ CUtensorMap tmap_v, AttnParams p) {
   using C = TcCfg<D, MT>;
+  constexpr int SPLIT = C::SPLIT, KH = C::KH, PB = C::PB;
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
@@ -286,16 +302,20 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
   auto kv_empty = [&](int s) { return bar0 + 8u * (C::STAGES + s); };
   auto s_full = [&](int mt, int bf) { return bar0 + 8u * (2 * C::STAGES + mt * 2 + bf); };
   auto s_free = [&](int mt, int bf) { return bar0 + 8u * (2 * C::STAGES + 2 * MT + mt * 2 + bf); };
-  auto p_full = [&](int mt) { return bar0 + 8u * (2 * C::STAGES + 4 * MT + mt); };
-  auto pv_done = [&](int mt) { return bar0 + 8u * (2 * C::STAGES + 5 * MT + mt); };
-  const uint32_t seg_ready = bar0 + 8u * (2 * C::STAGES + 6 * MT);
-  const uint32_t grp_bar = seg_ready + 8;
-  const uint32_t drain_bar = seg_ready + 16;
+  // P buffer pb of M tile mt: written by the softmax warps, read by the P V MMAs
+  auto p_full = [&](int mt, int pb) { return bar0 + 8u * (2 * C::STAGES + 4 * MT + mt * PB + pb); };
+  auto pv_done = [&](int mt, int pb) {
+    return bar0 + 8u * (2 * C::STAGES + 4 * MT + MT * PB + mt * PB + pb);
+  };
+  const uint32_t seg_ready = bar0 + 8u * (2 * C::STAGES + 4 * MT + 2 * MT * PB);
+  auto drain_bar = [&](int i) { return seg_ready + 8 + 8u * i; };  // per MMA issuer
+  auto xch_bar = [&](int q) { return seg_ready + 24 + 8u * q; };   // the two halves of quadrant q
   uint32_t* misc = reinterpret_cast<uint32_t*>(smem + C::OFF_MISC);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 1);
-  volatile int* merge_flag = reinterpret_cast<volatile int*>(misc + 2);
-  volatile int* merge_count = reinterpret_cast<volatile int*>(misc + 3);
-  int* merges = reinterpret_cast<int*>(smem + C::OFF_MERGE);  // [2][8]
+  volatile int* pend_count = reinterpret_cast<volatile int*>(misc + 2);
+  // split units this block wrote partials for (only a block's first and last segments
+  // can be split): b, g, row0, nrows, first slot, slots, unit, merge-here flag
+  int* pend = reinterpret_cast<int*>(smem + C::OFF_PEND);
   int* pb = reinterpret_cast<int*>(smem + C::OFF_PB);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -311,9 +331,9 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
     nact[mt] = min(4, max(0, (rows_cta - 128 * mt + 31) / 32));
     nact_total += nact[mt];
   }
-  constexpr int nprod = 3;  // KV producer warps 0, 2, 3
-  const int pw = (threadIdx.x >> 5) == 0 ? 0 : ((threadIdx.x >> 5) == 2 || (threadIdx.x >> 5) == 3)
-                                                    ? (threadIdx.x >> 5) - 1 : -1;
+  const int nsoft = nact_total * SPLIT;  // active softmax warps
+  constexpr int nprod = 2;  // KV producer warps 0 and 2
+  const int pw = warp == 0 ? 0 : (warp == 2 ? 1 : -1);
 
   // ---- prologue: barriers, TMEM, per-sequence tile prefix sums ----
   if (threadIdx.x == 0) {
@@ -322,18 +342,22 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
       mbar_init(kv_empty(s), 1);
     }
     for (int mt = 0; mt < MT; ++mt) {
+      const uint32_t nw = nact[mt] > 0 ? nact[mt] * SPLIT : 1;
       for (int bf = 0; bf < 2; ++bf) {
         mbar_init(s_full(mt, bf), 1);
-        mbar_init(s_free(mt, bf), nact[mt] > 0 ? nact[mt] : 1);
+        mbar_init(s_free(mt, bf), nw);
       }
-      mbar_init(p_full(mt), nact[mt] > 0 ? nact[mt] : 1);
-      mbar_init(pv_done(mt), 1);
+      for (int pb = 0; pb < PB; ++pb) {
+        mbar_init(p_full(mt, pb), nw);
+        mbar_init(pv_done(mt, pb), 1);
+      }
     }
-    mbar_init(seg_ready, nact_total);
-    mbar_init(grp_bar, nact_total);
-    mbar_init(drain_bar, 1);
+    mbar_init(seg_ready, nsoft);
+    mbar_init(drain_bar(0), 1);
+    mbar_init(drain_bar(1), 1);
+    for (int q = 0; q < 4; ++q) mbar_init(xch_bar(q), 2);
     *abort_flag = 0;
-    *merge_count = 0;
+    *pend_count = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 1) tmem_alloc(smem_u32(misc), C::TMEM_COLS);
@@ -379,13 +403,16 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
         cache_base = pi;
         const int idx = pi + lane;
         cache_val = idx < p.max_pages ? __ldg(&p.page_table[static_cast<int64_t>(b) * p.max_pages + idx]) : 0;
+        // an out-of-range id is read as page 0; the softmax side flags the segment
+        // and writes zeros for it
+        if (cache_val < 0 || cache_val >= p.num_pages) cache_val = 0;
       }
       return __shfl_sync(0xffffffffu, cache_val, pi - cache_base);
     };
     const uint32_t box_bytes = static_cast<uint32_t>(p.page_size) * D * 2;  // one page of one head
     for (int64_t t = t0; t < t1 && ok;) {
       const Seg s = locate(t, t1, p, pb);
-      const bool bad = segment_bad(s, p);
+      const bool bad = !s.len_ok;  // nothing to read; page ids are checked on the softmax side
       for (int k = 0; k < s.ntile && ok; ++k, ++it) {
         const int st = it % C::STAGES;
         if (it >= static_cast<uint32_t>(C::STAGES))
@@ -425,137 +452,170 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
         }
       }
     }
-  } else if (warp == 1) {
-    // ============================ MMA issuer ============================
+  } else if (warp == 1 || warp == 3) {
+    // ============================ MMA issuers ============================
+    // Two issuing warps feed the tensor pipe: warp 1 issues S = Q K^T as soon as a
+    // tile's K has landed and its S buffer is free (so it runs up to two tiles ahead),
+    // warp 3 issues O += P V as soon as a tile's P is written. A blocked issue of one
+    // kind never delays the other.
     // K and V stages hold a tile as [8-key group][128-byte column half][8 keys][128 B]:
     // 8-key groups sit at a uniform stride of DH KB across pages, so Q K^T runs with
-    // N = 64 keys (a tcgen05 MMA costs about the same for N = 16 and N = 64) and P V
-    // reads V MN-major with the column halves 1 KB apart.
+    // N = 64 keys and P V reads V MN-major with the column halves 1 KB apart.
     constexpr uint32_t kGroup = C::DH * 1024u;
     constexpr uint32_t kIdescQK = idesc_bf16(128, TK, false);
     constexpr uint32_t kIdescPV = idesc_bf16(128, D, true);
+    const bool qk_role = warp == 1;
     uint32_t it = 0, seg_no = 0;
     bool ok = true;
     bool issued = false;
-    // S = Q K^T for tile x into S[mt][x & 1]; returns false on timeout.
-    auto issue_qk = [&](uint32_t x, const Seg& s, int k) -> bool {
-      const int st = x % C::STAGES;
-      if (!mbar_wait(kv_full(st), (x / C::STAGES) & 1, abort_flag, p.status)) return false;
-      // keys past the end of the sequence: zero their V rows so that P = 0 meets finite V
-      const int key0 = (s.tile0 + k) * TK;
-      const int nvalid = s.len_ok ? min(TK, max(0, s.kv_len - key0)) : TK;
-      if (nvalid < TK) {
-        unsigned char* vst = smem + C::OFF_V + st * C::KV_BYTES;
-        for (int i = lane; i < (TK - nvalid) * C::DH * 8; i += 32) {
-          const int key = nvalid + i / (C::DH * 8), h = (i / 8) % C::DH, c = i % 8;
-          *reinterpret_cast<uint4*>(vst + (key >> 3) * kGroup + h * 1024u + (key & 7) * 128u +
-                                    c * 16u) = make_uint4(0, 0, 0, 0);
-        }
-        fence_async_smem();
-      }
-      __syncwarp();
-      if (x >= 2)
-        for (int mt = 0; mt < MT; ++mt)
-          if (!mbar_wait(s_free(mt, x & 1), ((x >> 1) - 1) & 1, abort_flag, p.status)) return false;
-      tc_fence_after();
-      if (lane == 0) {
-        for (int mt = 0; mt < MT; ++mt) {
-          const uint32_t d_tmem = tmem + C::S_COL + (mt * 2 + (x & 1)) * TK;
-#pragma unroll
-          for (int kk = 0; kk < D / 16; ++kk) {
-            const uint32_t qa = sbase + C::OFF_Q + (mt * C::DH + kk / 4) * 16384u + (kk % 4) * 32u;
-            const uint32_t kb = sbase + C::OFF_K + st * C::KV_BYTES + (kk / 4) * 1024u + (kk % 4) * 32u;
-            mma_bf16(d_tmem, desc_sw128(qa, 16, 1024), desc_sw128(kb, 16, kGroup), kIdescQK, kk > 0);
-          }
-          mma_commit(s_full(mt, x & 1));
-        }
-      }
-      __syncwarp();
-      return true;
-    };
     for (int64_t t = t0; t < t1 && ok;) {
       const Seg s = locate(t, t1, p, pb);
-      ok = mbar_wait(seg_ready, seg_no & 1, abort_flag, p.status);
-      if (!ok) break;
-      tc_fence_after();
-      for (int k = 0; k < s.ntile && ok; ++k) {
-        const uint32_t x = it + k;
-        if (k == 0) ok = issue_qk(x, s, 0);
-        if (ok && k + 1 < s.ntile) ok = issue_qk(x + 1, s, k + 1);
-        for (int mt = 0; mt < MT && ok; ++mt) ok = mbar_wait(p_full(mt), x & 1, abort_flag, p.status);
+      if (qk_role) {
+        ok = mbar_wait(seg_ready, seg_no & 1, abort_flag, p.status);
         if (!ok) break;
         tc_fence_after();
-        if (lane == 0) {
-          const int st = x % C::STAGES;
-          for (int mt = 0; mt < MT; ++mt) {
-            const uint32_t d_tmem = tmem + C::O_COL + mt * D;
-#pragma unroll
-            for (int kk = 0; kk < TK / 16; ++kk) {
-              const uint32_t pa = sbase + C::OFF_P + mt * 16384u + kk * 32u;
-              const uint32_t vb = sbase + C::OFF_V + st * C::KV_BYTES + kk * 2u * kGroup;
-              mma_bf16(d_tmem, desc_sw128(pa, 16, 1024), desc_sw128(vb, 1024, kGroup), kIdescPV,
-                       (k > 0 || kk > 0) ? 1u : 0u);
+      }
+      for (int k = 0; k < s.ntile && ok; ++k) {
+        const uint32_t x = it + k;
+        const int st = x % C::STAGES;
+        if (qk_role) {
+          // S = Q K^T for tile x into S[mt][x & 1]
+          ok = mbar_wait(kv_full(st), (x / C::STAGES) & 1, abort_flag, p.status);
+          if (!ok) break;
+          // keys past the end of the sequence: zero their V rows so that P = 0 meets
+          // finite V
+          const int key0 = (s.tile0 + k) * TK;
+          const int nvalid = s.len_ok ? min(TK, max(0, s.kv_len - key0)) : TK;
+          if (nvalid < TK) {
+            unsigned char* vst = smem + C::OFF_V + st * C::KV_BYTES;
+            for (int i = lane; i < (TK - nvalid) * C::DH * 8; i += 32) {
+              const int key = nvalid + i / (C::DH * 8), h = (i / 8) % C::DH, c = i % 8;
+              *reinterpret_cast<uint4*>(vst + (key >> 3) * kGroup + h * 1024u + (key & 7) * 128u +
+                                        c * 16u) = make_uint4(0, 0, 0, 0);
             }
-            mma_commit(pv_done(mt));
+            fence_async_smem();
           }
-          mma_commit(kv_empty(st));
-          issued = true;
+          __syncwarp();
+          if (x >= 2)
+            for (int mt = 0; mt < MT && ok; ++mt)
+              ok = mbar_wait(s_free(mt, x & 1), ((x >> 1) - 1) & 1, abort_flag, p.status);
+          if (!ok) break;
+          tc_fence_after();
+          if (lane == 0) {
+            for (int mt = 0; mt < MT; ++mt) {
+              const uint32_t d_tmem = tmem + C::S_COL + (mt * 2 + (x & 1)) * TK;
+#pragma unroll
+              for (int kk = 0; kk < D / 16; ++kk) {
+                const uint32_t qa = sbase + C::OFF_Q + (mt * C::DH + kk / 4) * 16384u + (kk % 4) * 32u;
+                const uint32_t kb = sbase + C::OFF_K + st * C::KV_BYTES + (kk / 4) * 1024u + (kk % 4) * 32u;
+                mma_bf16(d_tmem, desc_sw128(qa, 16, 1024), desc_sw128(kb, 16, kGroup), kIdescQK, kk > 0);
+              }
+              mma_commit(s_full(mt, x & 1));
+            }
+            issued = true;
+          }
+          __syncwarp();
+        } else {
+          // O += P V for tile x (its P implies its S, hence its landed stage)
+          const int pbuf = static_cast<int>(x % PB);
+          for (int mt = 0; mt < MT && ok; ++mt)
+            ok = mbar_wait(p_full(mt, pbuf), (x / PB) & 1, abort_flag, p.status);
+          if (!ok) break;
+          tc_fence_after();
+          if (lane == 0) {
+            for (int mt = 0; mt < MT; ++mt) {
+#pragma unroll
+              for (int hf = 0; hf < SPLIT; ++hf) {
+                // each key half accumulates into its own O
+                const uint32_t d_tmem = tmem + C::O_COL + (mt * SPLIT + hf) * D;
+#pragma unroll
+                for (int kk = 0; kk < KH / 16; ++kk) {
+                  const int kg = hf * (KH / 16) + kk;  // 16-key step within the tile
+                  const uint32_t pa = sbase + C::OFF_P + (pbuf * MT + mt) * 16384u + kg * 32u;
+                  const uint32_t vb = sbase + C::OFF_V + st * C::KV_BYTES + kg * 2u * kGroup;
+                  mma_bf16(d_tmem, desc_sw128(pa, 16, 1024), desc_sw128(vb, 1024, kGroup), kIdescPV,
+                           (k > 0 || kk > 0) ? 1u : 0u);
+                }
+              }
+              mma_commit(pv_done(mt, pbuf));
+            }
+            mma_commit(kv_empty(st));
+            issued = true;
+          }
+          __syncwarp();
         }
-        __syncwarp();
       }
       it += s.ntile;
       t += s.ntile;
       ++seg_no;
     }
-    if (!ok && __any_sync(0xffffffffu, issued)) {  // drain this block's MMAs (bounded)
-      if (lane == 0) mma_commit(drain_bar);
+    if (!ok && __any_sync(0xffffffffu, issued)) {  // drain this warp's MMAs (bounded)
+      const uint32_t db = drain_bar(qk_role ? 0 : 1);
+      if (lane == 0) mma_commit(db);
       __syncwarp();
       const long long t_0 = clock64();
-      while (!mbar_try(drain_bar, 0) && clock64() - t_0 < kWaitLimitCycles) {
+      while (!mbar_try(db, 0) && clock64() - t_0 < kWaitLimitCycles) {
       }
     }
-  } else if (warp >= 4 && ((warp - 4) & 3) < nact[(warp - 4) >> 2]) {
+  } else if (warp >= 4 && ((warp - 4) & 3) < nact[((warp - 4) >> 2) / SPLIT]) {
     // ====================== softmax (warps with real rows) ======================
-    const int sw = warp - 4, mt = sw >> 2, q4 = sw & 3;
+    const int sw = warp - 4, q4 = sw & 3, mt = (sw >> 2) / SPLIT, hf = (sw >> 2) % SPLIT;
     const int row = q4 * 32 + lane;  // TMEM lane = row of this M tile
+    const int lrow = mt * 128 + row;  // row within the block's row tile
     const uint32_t lane_base = tmem + (static_cast<uint32_t>(q4 * 32) << 16);
-    // active softmax warps are numbered densely: M tile 0's first, then M tile 1's
-    const int gtid = (mt == 0 ? q4 : nact[0] + q4) * 32 + lane, gthreads = 32 * nact_total;
-    uint32_t it = 0, gphase = 0;
+    const uint32_t ocol = lane_base + C::O_COL + (mt * SPLIT + hf) * D;  // this half's O
+    const uint32_t o0col = lane_base + C::O_COL + mt * SPLIT * D;        // first half's O
+    constexpr int kChunks = D / 8 / SPLIT;  // 16-byte pieces of a query row per warp
+    uint32_t it = 0, xphase = 0;
     bool ok = true;
-    unsigned char* prow = smem + C::OFF_P + mt * 16384u + row * 128u;
-    auto group_sync = [&]() -> bool {
-      __syncwarp();
-      if (lane == 0) mbar_arrive(grp_bar);
-      const bool r = mbar_wait(grp_bar, gphase & 1, abort_flag, p.status);
-      ++gphase;
+    // A row of a segment: the unit row it holds and whether it is a real query row.
+    struct RowOf {
+      int urow, j, h;
+      bool real;
+    };
+    auto row_of = [&](const Seg& sg) {
+      RowOf r;
+      r.urow = sg.rt * p.rows_per_cta + lrow;
+      r.real = r.urow < p.rows && lrow < p.rows_per_cta;
+      r.j = r.urow / p.group;
+      r.h = sg.g * p.group + r.urow % p.group;
       return r;
     };
-    for (int64_t t = t0; t < t1 && ok;) {
-      const Seg s = locate(t, t1, p, pb);
-      const bool bad = segment_bad(s, p);
-      const int row0 = s.rt * p.rows_per_cta;
-      const int lrow = mt * 128 + row;           // row within the block's row tile
-      const int urow = row0 + lrow;              // row within the unit (j * group + hh)
-      const bool real = urow < p.rows && lrow < p.rows_per_cta;
-      const int j = urow / p.group, h = s.g * p.group + urow % p.group;
-      // queries of this row into the swizzled Q tile (zeros for padding rows)
-      {
-        const uint4* src = reinterpret_cast<const uint4*>(
-            static_cast<const __nv_bfloat16*>(p.q) +
-            ((static_cast<int64_t>(s.b) * p.gamma + (real ? j : 0)) * p.hq + (real ? h : 0)) * D);
+    // this warp's share of a query row (zeros for padding rows)
+    auto load_q = [&](const Seg& sg, uint4* qr) {
+      const RowOf r = row_of(sg);
+      const uint4* src = reinterpret_cast<const uint4*>(
+          static_cast<const __nv_bfloat16*>(p.q) +
+          ((static_cast<int64_t>(sg.b) * p.gamma + (r.real ? r.j : 0)) * p.hq + (r.real ? r.h : 0)) * D);
 #pragma unroll
-        for (int c = 0; c < D / 8; ++c) {
-          const uint4 v = real ? __ldg(src + c) : make_uint4(0, 0, 0, 0);
-          const int half = c >> 3, ch = c & 7;
-          *reinterpret_cast<uint4*>(smem + C::OFF_Q + (mt * C::DH + half) * 16384u + row * 128u +
-                                    ((ch ^ (row & 7)) << 4)) = v;
-        }
+      for (int c2 = 0; c2 < kChunks; ++c2)
+        qr[c2] = r.real ? __ldg(src + hf * kChunks + c2) : make_uint4(0, 0, 0, 0);
+    };
+    // ... into the swizzled Q tile, then tell the MMA warp the segment may start
+    auto store_q = [&](const uint4* qr) {
+#pragma unroll
+      for (int c2 = 0; c2 < kChunks; ++c2) {
+        const int c = hf * kChunks + c2, half = c >> 3, ch = c & 7;
+        *reinterpret_cast<uint4*>(smem + C::OFF_Q + (mt * C::DH + half) * 16384u + row * 128u +
+                                  ((ch ^ (row & 7)) << 4)) = qr[c2];
       }
       fence_async_smem();
       __syncwarp();
       if (lane == 0) mbar_arrive(seg_ready);
-
+    };
+    uint4 qr[kChunks];
+    Seg s;
+    bool bad = false;
+    if (t0 < t1) {
+      s = locate(t0, t1, p, pb);
+      load_q(s, qr);
+      store_q(qr);
+      bad = segment_bad(s, p);  // needed only at this segment's epilogue
+    }
+    for (int64_t t = t0; t < t1 && ok;) {
+      const int64_t tn = t + s.ntile;
+      const bool has_next = tn < t1;
+      const RowOf ro = row_of(s);
       const int ctx = s.kv_len - p.gamma;
       float m = -INFINITY, l = 0.f;
       for (int k = 0; k < s.ntile; ++k) {
@@ -563,28 +623,27 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
         ok = mbar_wait(s_full(mt, x & 1), (x >> 1) & 1, abort_flag, p.status);
         if (!ok) break;
         tc_fence_after();
-        float v[TK];
+        float v[KH];
         {
           uint32_t r[32];
-          const uint32_t col = C::S_COL + (mt * 2 + (x & 1)) * TK;
-          tmem_ld32(lane_base + col, r);
-          tmem_wait_ld();
+          const uint32_t col = C::S_COL + (mt * 2 + (x & 1)) * TK + hf * KH;
 #pragma unroll
-          for (int c = 0; c < 32; ++c) v[c] = __uint_as_float(r[c]);
-          tmem_ld32(lane_base + col + 32, r);
-          tmem_wait_ld();
+          for (int q = 0; q < KH / 32; ++q) {
+            tmem_ld32(lane_base + col + q * 32, r);
+            tmem_wait_ld();
 #pragma unroll
-          for (int c = 0; c < 32; ++c) v[32 + c] = __uint_as_float(r[c]);
+            for (int c = 0; c < 32; ++c) v[q * 32 + c] = __uint_as_float(r[c]);
+          }
         }
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(s_free(mt, x & 1));
         // scale to base 2 and mask keys past ctx + j
-        const int key0 = (s.tile0 + k) * TK;
-        const int lim = ctx + j - key0;  // keys c <= lim are visible
+        const int key0 = (s.tile0 + k) * TK + hf * KH;
+        const int lim = ctx + ro.j - key0;  // keys c <= lim are visible
         float tmax = -INFINITY;
 #pragma unroll
-        for (int c = 0; c < TK; ++c) {
+        for (int c = 0; c < KH; ++c) {
           v[c] = c <= lim ? v[c] * p.scale_log2 : -INFINITY;
           tmax = fmaxf(tmax, v[c]);
         }
@@ -599,108 +658,142 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
           m = m_new;
         }
         const float msub = m == -INFINITY ? 0.f : m;
-        uint32_t pk[TK / 2];
+        uint32_t pk[KH / 2];
         float sum = 0.f;
 #pragma unroll
-        for (int c = 0; c < TK / 2; ++c) {
+        for (int c = 0; c < KH / 2; ++c) {
           const float a = ex2(v[2 * c] - msub), b2 = ex2(v[2 * c + 1] - msub);
           sum += a + b2;
           pk[c] = pack_bf16(a, b2);
         }
         l = l * alpha + sum;
-        if (k > 0) {  // P(x-1) consumed and O(x-1) complete
-          ok = mbar_wait(pv_done(mt), (x - 1) & 1, abort_flag, p.status);
+        const int pbuf = static_cast<int>(x % PB);
+        if (k >= PB) {  // the P V that last read this P buffer is complete
+          ok = mbar_wait(pv_done(mt, pbuf), ((x - PB) / PB) & 1, abort_flag, p.status);
           if (!ok) break;
           tc_fence_after();
-          if (rescale) {
-            const uint32_t ocol = lane_base + C::O_COL + mt * D;
-#pragma unroll
-            for (int cc = 0; cc < D / 32; ++cc) {
-              uint32_t r[32];
-              tmem_ld32(ocol + cc * 32, r);
-              tmem_wait_ld();
-#pragma unroll
-              for (int e = 0; e < 32; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
-              tmem_st32(ocol + cc * 32, r);
-            }
-            tmem_wait_st();
-          }
         }
+        if (rescale) {  // k > 0: O must hold every earlier tile before it is scaled
+          if (PB > 1) {
+            ok = mbar_wait(pv_done(mt, (x - 1) % PB), ((x - 1) / PB) & 1, abort_flag, p.status);
+            if (!ok) break;
+            tc_fence_after();
+          }
 #pragma unroll
-        for (int c = 0; c < 8; ++c)
+          for (int cc = 0; cc < D / 32; ++cc) {
+            uint32_t r[32];
+            tmem_ld32(ocol + cc * 32, r);
+            tmem_wait_ld();
+#pragma unroll
+            for (int e = 0; e < 32; ++e) r[e] = __float_as_uint(__uint_as_float(r[e]) * alpha);
+            tmem_st32(ocol + cc * 32, r);
+          }
+          tmem_wait_st();
+        }
+        unsigned char* prow = smem + C::OFF_P + (pbuf * MT + mt) * 16384u + row * 128u;
+#pragma unroll
+        for (int c2 = 0; c2 < KH / 8; ++c2) {
+          const int c = hf * (KH / 8) + c2;
           *reinterpret_cast<uint4*>(prow + ((c ^ (row & 7)) << 4)) =
-              make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
+              make_uint4(pk[4 * c2], pk[4 * c2 + 1], pk[4 * c2 + 2], pk[4 * c2 + 3]);
+        }
         fence_async_smem();
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(p_full(mt));
+        if (lane == 0) mbar_arrive(p_full(mt, pbuf));
       }
       if (!ok) break;
+      // The next segment's scores may start now: every Q K^T of this segment is done
+      // (its last S was read above), so its Q tile can be replaced while this
+      // segment's epilogue runs. Its first P V waits for this epilogue (program order).
+      Seg sn;
+      bool bad_next = false;
+      if (has_next) {
+        sn = locate(tn, t1, p, pb);
+        load_q(sn, qr);
+        store_q(qr);
+        bad_next = segment_bad(sn, p);
+      }
       // ---- epilogue: O (TMEM) -> output or partial ----
       const uint32_t xl = it + s.ntile - 1;
-      ok = mbar_wait(pv_done(mt), xl & 1, abort_flag, p.status);
+      ok = mbar_wait(pv_done(mt, xl % PB), (xl / PB) & 1, abort_flag, p.status);
       if (!ok) break;
       tc_fence_after();
+      // statistics of the whole tile range: the two key halves merged (identically in
+      // both warps of the quadrant)
+      float M = m, L = l, sc0 = 1.f, sc1 = 0.f;
+      if (SPLIT == 2) {
+        float2* xch = reinterpret_cast<float2*>(smem + C::OFF_XCH);
+        xch[(q4 * 2 + hf) * 32 + lane] = make_float2(m, l);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(xch_bar(q4));
+        ok = mbar_wait(xch_bar(q4), xphase & 1, abort_flag, p.status);
+        ++xphase;
+        if (!ok) break;
+        const float2 other = xch[(q4 * 2 + (hf ^ 1)) * 32 + lane];
+        const float m0 = hf == 0 ? m : other.x, l0 = hf == 0 ? l : other.y;
+        const float m1 = hf == 0 ? other.x : m, l1 = hf == 0 ? other.y : l;
+        M = fmaxf(m0, m1);
+        sc0 = m0 == -INFINITY ? 0.f : ex2(m0 - M);
+        sc1 = m1 == -INFINITY ? 0.f : ex2(m1 - M);
+        L = l0 * sc0 + l1 * sc1;
+      }
       const bool whole = s.tile0 == 0 && s.ntile == s.unit_tiles;
-      const uint32_t ocol = lane_base + C::O_COL + mt * D;
       const int c_first = owner_of(s.unit_start, total, ctas);
       const int c_last = owner_of(s.unit_start + s.unit_tiles - 1, total, ctas);
       const int64_t slot = s.u + cta;
       if (bad && sw == 0 && lane == 0 && (whole || cta == c_first))
         set_status(p.status, s.len_ok ? SPEC_FLAG_BAD_PAGE : SPEC_FLAG_BAD_KV_LEN);
+      // this warp writes output columns [hf * D / SPLIT, (hf + 1) * D / SPLIT)
 #pragma unroll 1
-      for (int cc = 0; cc < D / 32; ++cc) {
+      for (int cc = hf * (D / 32 / SPLIT); cc < (hf + 1) * (D / 32 / SPLIT); ++cc) {
         uint32_t r[32];
-        tmem_ld32(ocol + cc * 32, r);
+        float o[32];
+        tmem_ld32(o0col + cc * 32, r);
         tmem_wait_ld();
-        if (!real) continue;
+#pragma unroll
+        for (int e = 0; e < 32; ++e) o[e] = __uint_as_float(r[e]) * sc0;
+        if (SPLIT == 2) {
+          tmem_ld32(o0col + D + cc * 32, r);
+          tmem_wait_ld();
+#pragma unroll
+          for (int e = 0; e < 32; ++e) o[e] = fmaf(__uint_as_float(r[e]), sc1, o[e]);
+        }
+        if (!ro.real) continue;
         if (whole) {
-          const float inv = bad ? 0.f : 1.f / l;
+          // a bad segment's scores came from stale stages: write exact zeros
+          const float inv = bad ? 0.f : 1.f / L;
+          if (bad) {
 #pragma unroll
-          for (int e = 0; e < 32; e += 8) {
-            float o8[8];
-#pragma unroll
-            for (int f = 0; f < 8; ++f) o8[f] = __uint_as_float(r[e + f]);
-            write_out_row<D>(p, s.b, s.g, urow, cc * 32 + e, o8, inv);
+            for (int e = 0; e < 32; ++e) o[e] = 0.f;
           }
+#pragma unroll
+          for (int e = 0; e < 32; e += 8) write_out_row<D>(p, s.b, s.g, ro.urow, cc * 32 + e, o + e, inv);
         } else {
           float4* dst = reinterpret_cast<float4*>(p.partial_o + (slot * p.slot_rows + lrow) * D + cc * 32);
 #pragma unroll
           for (int e = 0; e < 8; ++e)
-            dst[e] = make_float4(__uint_as_float(r[4 * e]), __uint_as_float(r[4 * e + 1]),
-                                 __uint_as_float(r[4 * e + 2]), __uint_as_float(r[4 * e + 3]));
+            dst[e] = make_float4(o[4 * e], o[4 * e + 1], o[4 * e + 2], o[4 * e + 3]);
         }
       }
       tc_fence_before();
-      if (real) {
-        if (whole) write_lse(p, s.b, s.g, urow, m, l, bad);
-        else p.partial_ml[slot * p.slot_rows + lrow] = make_float2(m, bad ? -1.f : l);
+      if (ro.real && hf == 0) {
+        if (whole) write_lse(p, s.b, s.g, ro.urow, M, L, bad);
+        else p.partial_ml[slot * p.slot_rows + lrow] = make_float2(M, bad ? -1.f : L);
       }
-      if (!whole) {
-        __threadfence();
-        ok = group_sync();
-        if (!ok) break;
-        if (gtid == 0) {
-          const uint32_t prev = atomicAdd(&p.tickets[s.u], 1u);
-          const bool last = prev == static_cast<uint32_t>(c_last - c_first);
-          if (last) p.tickets[s.u] = 0;  // leave the counter at zero for the next call
-          *merge_flag = last;
-        }
-        ok = group_sync();
-        if (!ok) break;
-        if (*merge_flag && gtid == 0) {
-          // the unit is complete: merge it once every role of this block is done (only a
-          // block's first and last segments can be split, so at most two)
-          int* e = merges + 8 * (*merge_count);
-          e[0] = s.b; e[1] = s.g; e[2] = row0; e[3] = min(p.rows_per_cta, p.rows - row0);
-          e[4] = static_cast<int>(s.u + c_first); e[5] = c_last - c_first + 1;
-          *merge_count = *merge_count + 1;
-        }
-        ok = group_sync();  // merge_flag is rewritten by the next segment
-        if (!ok) break;
+      if (!whole && sw == 0 && lane == 0) {
+        // the ticket of a split unit is taken at the end of the block, after a fence
+        int* e = pend + 8 * (*pend_count);
+        const int row0 = s.rt * p.rows_per_cta;
+        e[0] = s.b; e[1] = s.g; e[2] = row0; e[3] = min(p.rows_per_cta, p.rows - row0);
+        e[4] = static_cast<int>(s.u + c_first); e[5] = c_last - c_first + 1;
+        e[6] = static_cast<int>(s.u); e[7] = 0;
+        *pend_count = *pend_count + 1;
       }
       it += s.ntile;
-      t += s.ntile;
+      t = tn;
+      s = sn;
+      bad = bad_next;
     }
     tc_fence_before();
   }
@@ -709,13 +802,29 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
     tc_fence_after();
     tmem_dealloc(tmem, C::TMEM_COLS);
   }
-  // deferred merges of split units this block completed, by all of its threads
+  // Split units: every thread makes its partial writes visible, then the block takes
+  // one ticket per unit it wrote; the block that completes a unit merges it.
   if (!*abort_flag) {
-    const int nm = *merge_count;
-    if (nm > 0) __threadfence();
-    for (int mi = 0; mi < nm; ++mi) {
-      const int* e = merges + 8 * mi;
-      merge_unit<D>(p, e[0], e[1], e[2], e[3], e[4], e[5], threadIdx.x, C::THREADS);
+    const int np = *pend_count;  // block-uniform
+    if (np > 0) {
+      __threadfence();
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        for (int i = 0; i < np; ++i) {
+          int* e = pend + 8 * i;
+          const uint32_t prev = atomicAdd(&p.tickets[e[6]], 1u);
+          e[7] = prev == static_cast<uint32_t>(e[5] - 1);
+          if (e[7]) p.tickets[e[6]] = 0;  // leave the counter at zero for the next call
+        }
+      }
+      __syncthreads();
+      bool any = false;
+      for (int i = 0; i < np; ++i) any |= pend[8 * i + 7] != 0;
+      if (any) __threadfence();
+      for (int i = 0; i < np; ++i) {
+        const int* e = pend + 8 * i;
+        if (e[7]) merge_unit<D>(p, e[0], e[1], e[2], e[3], e[4], e[5], threadIdx.x, C::THREADS);
+      }
     }
   }
 }
@@ -790,7 +899,10 @@ int tc_ctas_per_sm(int head_dim, int rows_per_cta, int batch) {
   // Shared memory bounds residency (227 KB usable per SM); TMEM (512 columns) too.
   const size_t smem = tc_smem_bytes(head_dim, rows_per_cta, batch);
   int by_smem = static_cast<int>((227u * 1024u) / (smem + 1024));
-  const int cols = rows_per_cta > 128 ? 512 : 256;
+  const bool two = rows_per_cta > 128;
+  const int cols = static_cast<int>(
+      head_dim == 128 ? (two ? TcCfg<128, 2>::TMEM_COLS : TcCfg<128, 1>::TMEM_COLS)
+                      : (two ? TcCfg<64, 2>::TMEM_COLS : TcCfg<64, 1>::TMEM_COLS));
   const int by_tmem = 512 / cols;
   int n = by_smem < by_tmem ? by_smem : by_tmem;
   return n < 1 ? 1 : n;
