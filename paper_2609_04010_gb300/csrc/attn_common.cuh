@@ -30,6 +30,7 @@ struct AttnParams {
   uint32_t* tickets;
   float* partial_o;    // [slot][slot_rows][D]
   float2* partial_ml;  // [slot][slot_rows] = (m, l); l = -1 marks a bad sequence
+  int q_tma;           // tensor-core kernel: Q tiles arrive by TMA (else softmax warps load them)
 };
 
 inline AttnParams make_attn_params(const spec_attn_args_t& a, const AttnPlan& P, char* ws) {
@@ -62,6 +63,7 @@ inline AttnParams make_attn_params(const spec_attn_args_t& a, const AttnPlan& P,
   p.tickets = reinterpret_cast<uint32_t*>(ws + P.tickets);
   p.partial_o = reinterpret_cast<float*>(ws + P.partial_o);
   p.partial_ml = reinterpret_cast<float2*>(ws + P.partial_ml);
+  p.q_tma = 0;
   return p;
 }
 

@@ -60,12 +60,13 @@ struct TcCfg {
   static constexpr uint32_t OFF_P = OFF_V + STAGES * KV_BYTES;
   static constexpr uint32_t OFF_BAR = OFF_P + P_BYTES;
   // barriers: kv_full[S], kv_empty[S], s_full[MT][2], s_free[MT][2], p_full[MT][PB],
-  // pv_done[MT][PB], seg_ready, drain[2], xch[4]
-  static constexpr int NBAR = 2 * STAGES + 4 * MT + 2 * MT * PB + 3 + 4;
+  // pv_done[MT][PB], seg_ready, drain[2], xch[4], q_full, seg_flag_ready[8]
+  static constexpr int NBAR = 2 * STAGES + 4 * MT + 2 * MT * PB + 3 + 4 + 1 + 8;
   static constexpr uint32_t OFF_MISC = OFF_BAR + NBAR * 8;  // tmem base, abort, pending count
   static constexpr uint32_t OFF_XCH = OFF_MISC + 16;        // [4][2][32] float2 (m, l) per half
   static constexpr uint32_t OFF_PEND = OFF_XCH + (SPLIT == 2 ? 4 * 2 * 32 * 8 : 0);  // [2][8]
-  static constexpr uint32_t OFF_PB = (OFF_PEND + 64 + 15) / 16 * 16;
+  static constexpr uint32_t OFF_FLAG = OFF_PEND + 64;  // [8] bad flags of segments
+  static constexpr uint32_t OFF_PB = (OFF_FLAG + 32 + 15) / 16 * 16;
   static constexpr uint32_t TMEM_NEED = MT * 128 + MT * SPLIT * D;
   static constexpr uint32_t TMEM_COLS = TMEM_NEED <= 256 ? 256 : 512;
   static constexpr uint32_t S_COL = 0;           // S[mt][buf] at (mt * 2 + buf) * 64
@@ -132,6 +133,16 @@ __device__ __forceinline__ void tma_load_page(uint32_t dst, const CUtensorMap* m
       " [%0], [%1, {%2, %3, %4, %5, %6}], [%7];" ::"r"(dst),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(0), "r"(0), "r"(0), "r"(0), "r"(page_head),
       "r"(bar)
+      : "memory");
+}
+// Rows of one M tile of Q: 128 / group block positions of `group` heads, one
+// 128-byte column half (box of the 4-D view of Q, see encode_q_map).
+__device__ __forceinline__ void tma_load_q(uint32_t dst, const CUtensorMap* map, int half, int head0,
+                                           int pos0, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.4d.shared::cluster.global.mbarrier::complete_tx::bytes"
+      " [%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(0), "r"(half), "r"(head0), "r"(pos0), "r"(bar)
       : "memory");
 }
 __device__ __forceinline__ void fence_async_smem() {
@@ -264,33 +275,14 @@ __device__ __forceinline__ int owner_of(int64_t t, int64_t total, int ctas) {
   return static_cast<int>(((t + 1) * ctas - 1) / total);
 }
 
-// A segment is bad when its sequence length is malformed or a page it reads is out
-// of range. The whole warp cooperates (up to 128 page ids in flight per round trip);
-// every lane gets the answer.
-__device__ __forceinline__ bool segment_bad(const Seg& s, const AttnParams& p) {
-  if (!s.len_ok) return true;
-  const int k0 = s.tile0 * TK;
-  const int k1 = min(s.kv_len, (s.tile0 + s.ntile) * TK);
-  const int pg0 = k0 / p.page_size, pg1 = (k1 - 1) / p.page_size;
-  const int* row = p.page_table + static_cast<int64_t>(s.b) * p.max_pages;
-  bool bad = false;
-  for (int base = pg0 + (threadIdx.x & 31); base <= pg1; base += 128) {
-    int id[4];
-#pragma unroll
-    for (int u = 0; u < 4; ++u) id[u] = base + 32 * u <= pg1 ? __ldg(row + base + 32 * u) : 0;
-#pragma unroll
-    for (int u = 0; u < 4; ++u) bad |= id[u] < 0 || id[u] >= p.num_pages;
-  }
-  return __any_sync(0xffffffffu, bad);
-}
-
 // ---------------------------------------------------------------------------------
 // The kernel
 // ---------------------------------------------------------------------------------
 template <int D, int MT>
 __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
-                   const __grid_constant__ CUtensorMap tmap_v, AttnParams p) {
+                   const __grid_constant__ CUtensorMap tmap_v,
+                   const __grid_constant__ CUtensorMap tmap_q, AttnParams p) {
   using C = TcCfg<D, MT>;
   constexpr int SPLIT = C::SPLIT, KH = C::KH, PB = C::PB;
   extern __shared__ __align__(1024) unsigned char smem_raw[];
@@ -310,6 +302,11 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
   const uint32_t seg_ready = bar0 + 8u * (2 * C::STAGES + 4 * MT + 2 * MT * PB);
   auto drain_bar = [&](int i) { return seg_ready + 8 + 8u * i; };  // per MMA issuer
   auto xch_bar = [&](int q) { return seg_ready + 24 + 8u * q; };   // the two halves of quadrant q
+  const uint32_t q_full = seg_ready + 56;  // Q tile of the next segment landed (TMA)
+  // segment flags: the producer publishes whether a segment reads a bad page or has a
+  // malformed length (ring of 8, far more than the producer can run ahead)
+  auto flag_bar = [&](int i) { return seg_ready + 64 + 8u * i; };
+  volatile int* seg_flag = reinterpret_cast<volatile int*>(smem + C::OFF_FLAG);
   uint32_t* misc = reinterpret_cast<uint32_t*>(smem + C::OFF_MISC);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 1);
   volatile int* pend_count = reinterpret_cast<volatile int*>(misc + 2);
@@ -356,6 +353,8 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
     mbar_init(drain_bar(0), 1);
     mbar_init(drain_bar(1), 1);
     for (int q = 0; q < 4; ++q) mbar_init(xch_bar(q), 2);
+    mbar_init(q_full, 1);
+    for (int i = 0; i < 8; ++i) mbar_init(flag_bar(i), 1);
     *abort_flag = 0;
     *pend_count = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -403,16 +402,15 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
         cache_base = pi;
         const int idx = pi + lane;
         cache_val = idx < p.max_pages ? __ldg(&p.page_table[static_cast<int64_t>(b) * p.max_pages + idx]) : 0;
-        // an out-of-range id is read as page 0; the softmax side flags the segment
-        // and writes zeros for it
-        if (cache_val < 0 || cache_val >= p.num_pages) cache_val = 0;
       }
       return __shfl_sync(0xffffffffu, cache_val, pi - cache_base);
     };
     const uint32_t box_bytes = static_cast<uint32_t>(p.page_size) * D * 2;  // one page of one head
-    for (int64_t t = t0; t < t1 && ok;) {
+    uint32_t seg_no = 0;
+    for (int64_t t = t0; t < t1 && ok; ++seg_no) {
       const Seg s = locate(t, t1, p, pb);
-      const bool bad = !s.len_ok;  // nothing to read; page ids are checked on the softmax side
+      const bool bad = !s.len_ok;  // nothing to read
+      bool flag = bad;             // ... or a page id out of range (read as page 0)
       for (int k = 0; k < s.ntile && ok; ++k, ++it) {
         const int st = it % C::STAGES;
         if (it >= static_cast<uint32_t>(C::STAGES))
@@ -432,7 +430,10 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
           if (lane == 0) mbar_arrive_tx(kv_full(st), mine);
           for (int bx = pw; bx < nbox; bx += nprod) {
             const int q = bx >> 1, isv = bx & 1;
-            const int page = page_of(s.b, key0 / p.page_size + q);
+            const int raw = page_of(s.b, key0 / p.page_size + q);
+            const bool in_range = raw >= 0 && raw < p.num_pages;
+            flag |= !in_range;
+            const int page = in_range ? raw : 0;
             if (lane == 0) {
               const uint32_t dst = sbase + (isv ? C::OFF_V : C::OFF_K) + st * C::KV_BYTES +
                                    static_cast<uint32_t>(q) * box_bytes;
@@ -441,6 +442,10 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
           }
         }
         __syncwarp();
+      }
+      if (ok && pw == 0 && lane == 0) {  // both producers see every page; one publishes
+        seg_flag[seg_no & 7] = flag ? 1 : 0;
+        mbar_arrive(flag_bar(seg_no & 7));
       }
       t += s.ntile;
     }
@@ -468,10 +473,23 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
     uint32_t it = 0, seg_no = 0;
     bool ok = true;
     bool issued = false;
+    // Q tiles of a segment (all M tiles, both column halves) by TMA, on q_full
+    auto issue_q = [&](const Seg& sg) {
+      if (lane == 0) {
+        mbar_arrive_tx(q_full, MT * C::DH * 16384u);
+        for (int mt = 0; mt < MT; ++mt)
+          for (int half = 0; half < C::DH; ++half)
+            tma_load_q(sbase + C::OFF_Q + (mt * C::DH + half) * 16384u, &tmap_q, half,
+                       sg.g * p.group,
+                       sg.b * p.gamma + (sg.rt * p.rows_per_cta + mt * 128) / p.group, q_full);
+      }
+      __syncwarp();
+    };
+    if (qk_role && p.q_tma && t0 < t1) issue_q(locate(t0, t1, p, pb));
     for (int64_t t = t0; t < t1 && ok;) {
       const Seg s = locate(t, t1, p, pb);
       if (qk_role) {
-        ok = mbar_wait(seg_ready, seg_no & 1, abort_flag, p.status);
+        ok = mbar_wait(p.q_tma ? q_full : seg_ready, seg_no & 1, abort_flag, p.status);
         if (!ok) break;
         tc_fence_after();
       }
@@ -515,6 +533,13 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
             issued = true;
           }
           __syncwarp();
+          if (p.q_tma && k == s.ntile - 1 && t + s.ntile < t1) {
+            // the segment's last scores are done with its Q tile: fetch the next one
+            for (int mt = 0; mt < MT && ok; ++mt)
+              ok = mbar_wait(s_full(mt, x & 1), (x >> 1) & 1, abort_flag, p.status);
+            if (!ok) break;
+            issue_q(locate(t + s.ntile, t1, p, pb));
+          }
         } else {
           // O += P V for tile x (its P implies its S, hence its landed stage)
           const int pbuf = static_cast<int>(x % PB);
@@ -605,12 +630,13 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
     };
     uint4 qr[kChunks];
     Seg s;
-    bool bad = false;
+    uint32_t seg_no = 0;
     if (t0 < t1) {
       s = locate(t0, t1, p, pb);
-      load_q(s, qr);
-      store_q(qr);
-      bad = segment_bad(s, p);  // needed only at this segment's epilogue
+      if (!p.q_tma) {
+        load_q(s, qr);
+        store_q(qr);
+      }
     }
     for (int64_t t = t0; t < t1 && ok;) {
       const int64_t tn = t + s.ntile;
@@ -707,18 +733,21 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
       // (its last S was read above), so its Q tile can be replaced while this
       // segment's epilogue runs. Its first P V waits for this epilogue (program order).
       Seg sn;
-      bool bad_next = false;
       if (has_next) {
         sn = locate(tn, t1, p, pb);
-        load_q(sn, qr);
-        store_q(qr);
-        bad_next = segment_bad(sn, p);
+        if (!p.q_tma) {
+          load_q(sn, qr);
+          store_q(qr);
+        }
       }
       // ---- epilogue: O (TMEM) -> output or partial ----
       const uint32_t xl = it + s.ntile - 1;
       ok = mbar_wait(pv_done(mt, xl % PB), (xl / PB) & 1, abort_flag, p.status);
       if (!ok) break;
       tc_fence_after();
+      ok = mbar_wait(flag_bar(seg_no & 7), (seg_no >> 3) & 1, abort_flag, p.status);
+      if (!ok) break;
+      const bool bad = seg_flag[seg_no & 7] != 0;
       // statistics of the whole tile range: the two key halves merged (identically in
       // both warps of the quadrant)
       float M = m, L = l, sc0 = 1.f, sc1 = 0.f;
@@ -793,7 +822,7 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
       it += s.ntile;
       t = tn;
       s = sn;
-      bad = bad_next;
+      ++seg_no;
     }
     tc_fence_before();
   }
@@ -870,20 +899,44 @@ bool encode_cache_map(CUtensorMap* map, const void* base, const spec_attn_args_t
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Q [batch][gamma][Hq][D] viewed as a 4-D tensor (64 columns; D/64 column halves at
+// stride 128 bytes; Hq heads at stride D*2; batch*gamma block positions at stride
+// Hq*D*2) whose box is one M tile of one column half: the group's heads at 128/group
+// consecutive block positions, landing as 128 rows of 128 bytes (row = j * group + head)
+// with the 128-byte swizzle. Needs group to divide 128; positions past the end read
+// zeros and only fill padding rows.
+bool encode_q_map(CUtensorMap* map, const spec_attn_args_t& a) {
+  const int group = a.num_q_heads / a.num_kv_heads;
+  if (group < 1 || 128 % group != 0) return false;
+  EncodeTiledFn enc = encoder();
+  if (!enc) return false;
+  const cuuint64_t D = static_cast<cuuint64_t>(a.head_dim);
+  const cuuint64_t dims[4] = {64, D / 64, static_cast<cuuint64_t>(a.num_q_heads),
+                              static_cast<cuuint64_t>(a.batch) * a.gamma};
+  const cuuint64_t strides[3] = {128, D * 2, static_cast<cuuint64_t>(a.num_q_heads) * D * 2};
+  const cuuint32_t box[4] = {64, 1, static_cast<cuuint32_t>(group), static_cast<cuuint32_t>(128 / group)};
+  const cuuint32_t estr[4] = {1, 1, 1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(a.q), dims, strides, box,
+             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 template <int D, int MT>
 cudaError_t launch_typed(const spec_attn_args_t& a, const AttnPlan& P, char* ws,
                          cudaStream_t stream) {
   using Cf = TcCfg<D, MT>;
-  CUtensorMap mk, mv;
+  CUtensorMap mk, mv, mq;
   if (!encode_cache_map(&mk, a.k_cache, a) || !encode_cache_map(&mv, a.v_cache, a))
     return cudaErrorInvalidValue;
-  const AttnParams p = make_attn_params(a, P, ws);
+  AttnParams p = make_attn_params(a, P, ws);
+  p.q_tma = encode_q_map(&mq, a) ? 1 : 0;
+  if (!p.q_tma) mq = mk;  // unused
   const size_t smem = Cf::smem_bytes(a.batch);
   cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel<D, MT>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  attn_tc_kernel<D, MT><<<P.grid, Cf::THREADS, smem, stream>>>(mk, mv, p);
+  attn_tc_kernel<D, MT><<<P.grid, Cf::THREADS, smem, stream>>>(mk, mv, mq, p);
   return cudaGetLastError();
 }
 

@@ -28,6 +28,12 @@ SMALL = [
     dict(batch=1, gamma=3, num_q_heads=6, num_kv_heads=2, head_dim=64, page_size=64, ctx=0),
     dict(batch=2, gamma=64, num_q_heads=8, num_kv_heads=4, head_dim=64, page_size=16,
          ctx=(0, 150)),
+    # 512 rows per kv head: two row tiles of two M tiles each
+    dict(batch=2, gamma=32, num_q_heads=128, num_kv_heads=8, head_dim=128, page_size=16,
+         ctx=(10, 300)),
+    # a group that does not divide 128, with two M tiles
+    dict(batch=2, gamma=64, num_q_heads=6, num_kv_heads=2, head_dim=128, page_size=32,
+         ctx=(5, 200)),
 ]
 
 
