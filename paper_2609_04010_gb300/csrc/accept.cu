@@ -5,7 +5,7 @@
 // Two launches, no inter-block waiting (the second is a programmatic dependent of the
 // first and waits for it on the device; in a verify step the first is a programmatic
 // dependent of the attention kernel and runs beside it):
-//   1. row_stats_kernel: one block per (sequence, row, 4096-entry vocab chunk) reads
+//   1. row_stats_kernel: one warp per (sequence, row, 4096-entry vocab chunk) reads
 //      the chunk once with 16-byte loads and writes its max, its sum of
 //      exp((l - max)/T) and (greedy rows) its lowest-index argmax.
 //   2. decide_sample_kernel: grid (vocab slice, sequence). Every block merges the row
@@ -69,55 +69,6 @@ __device__ __forceinline__ float load_elem(const void* base, int64_t i) {
   return static_cast<const float*>(base)[i];
 }
 
-// Loads kPer consecutive-or-strided values of a row into registers.
-// VEC: element groups of 16 bytes, group g of thread t at g*threads + t (coalesced).
-template <bool BF16, bool VEC, int kPer, int kThreads>
-__device__ __forceinline__ void load_strided(const void* row, int start, int len, float* v,
-                                             int* idx) {
-  const int t = threadIdx.x;
-  if (VEC) {
-    constexpr int kEpv = BF16 ? 8 : 4;
-    constexpr int kVecs = kPer / kEpv;
-    uint4 raw[kVecs];
-#pragma unroll
-    for (int k = 0; k < kVecs; ++k) {
-      const int e = (k * kThreads + t) * kEpv;
-      if (e < len) {
-        const char* p = static_cast<const char*>(row) + static_cast<int64_t>(start + e) * (BF16 ? 2 : 4);
-        raw[k] = __ldg(reinterpret_cast<const uint4*>(p));
-      } else {
-        raw[k] = make_uint4(0xff800000u, 0xff800000u, 0xff800000u, 0xff800000u);
-      }
-    }
-#pragma unroll
-    for (int k = 0; k < kVecs; ++k) {
-      const int e = (k * kThreads + t) * kEpv;
-      const uint32_t w[4] = {raw[k].x, raw[k].y, raw[k].z, raw[k].w};
-#pragma unroll
-      for (int q = 0; q < kEpv; ++q) {
-        float x;
-        if (BF16) {
-          const uint32_t h = (q & 1) ? (w[q >> 1] >> 16) : (w[q >> 1] & 0xffffu);
-          x = bf16_bits_to_f32(h);
-        } else {
-          x = __uint_as_float(w[q]);
-        }
-        const bool ok = e + q < len;
-        v[k * kEpv + q] = ok ? x : -INFINITY;
-        idx[k * kEpv + q] = ok ? start + e + q : INT_MAX;
-      }
-    }
-  } else {
-#pragma unroll
-    for (int k = 0; k < kPer; ++k) {
-      const int e = k * kThreads + t;
-      const bool ok = e < len;
-      v[k] = ok ? load_elem<BF16>(row, start + e) : -INFINITY;
-      idx[k] = ok ? start + e : INT_MAX;
-    }
-  }
-}
-
 // (m, s) pairs of an online softmax sum in base 2 with scale c: value = s * 2^{c*m}.
 __device__ __forceinline__ void merge_ms(float& m, float& s, float m2, float s2, float c) {
   const float mn = fmaxf(m, m2);
@@ -128,6 +79,20 @@ __device__ __forceinline__ void merge_ms(float& m, float& s, float m2, float s2,
   s = r;
 }
 
+// Warp-wide combination of the lanes' (m, s) pairs: the maximum by shuffles, then each
+// lane's sum rescaled once to it and the sums added (a lane with m = -inf adds 0; a NaN
+// or infinite input leaves a NaN sum).
+__device__ __forceinline__ void warp_merge_ms(float& m, float& s, float c) {
+  float mx = m;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+  float sc = m != -INFINITY ? s * ex2((m - mx) * c) : 0.f;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) sc += __shfl_xor_sync(0xffffffffu, sc, o);
+  m = mx;
+  s = sc;
+}
+
 __device__ __forceinline__ void merge_arg(float& m, int& a, float m2, int a2) {
   if (m2 > m || (m2 == m && a2 < a)) {
     m = m2;
@@ -135,133 +100,147 @@ __device__ __forceinline__ void merge_arg(float& m, int& a, float m2, int a2) {
   }
 }
 
-template <bool BF16, bool VEC>
-__global__ void __launch_bounds__(kStatsThreads, 8) row_stats_kernel(AcceptParams p) {
-  constexpr int kPer = kStatsChunk / kStatsThreads;  // 32 values per thread
-  pdl_launch_dependents();
-  __shared__ float sh_m[kStatsThreads / 32];
-  __shared__ float sh_s[kStatsThreads / 32];
-  __shared__ int sh_a[kStatsThreads / 32];
-  __shared__ uint32_t sh_bad[kStatsThreads / 32];
+// Warp-wide lowest-index argmax of the lanes' (m, a) pairs.
+__device__ __forceinline__ void warp_merge_arg(float& m, int& a) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
+    const int a2 = __shfl_xor_sync(0xffffffffu, a, o);
+    merge_arg(m, a, m2, a2);
+  }
+}
 
+// One warp per (sequence, row, kStatsChunk-entry chunk), with no block-wide step: the
+// warp issues all of its chunk's 16-byte loads together (sixteen per lane and round;
+// one round for bf16, two for fp32) and reduces with shuffles. Grid (chunk groups of
+// kStatsThreads / 32, row, sequence).
+template <bool BF16, bool VEC>
+__global__ void __launch_bounds__(kStatsThreads, 5) row_stats_kernel(AcceptParams p) {
+  pdl_launch_dependents();
+  const int lane = threadIdx.x & 31;
+  const int c = blockIdx.x * (kStatsThreads / 32) + (threadIdx.x >> 5);
+  const int r = blockIdx.y, b = blockIdx.z;
+  if (c >= p.nchunk) return;
   const int nrows = 2 * p.gamma - 1;
-  const int64_t item = blockIdx.x;
-  const int c = static_cast<int>(item % p.nchunk);
-  const int r = static_cast<int>((item / p.nchunk) % nrows);
-  const int b = static_cast<int>(item / (static_cast<int64_t>(p.nchunk) * nrows));
   const float T = p.temperature[b];
   const bool greedy = !(T > 0.f);
   if (greedy && r >= p.gamma) return;  // greedy sequences never read drafter rows
   const int64_t row = static_cast<int64_t>(b) * p.gamma + (r < p.gamma ? r : r - p.gamma + 1);
   const void* base = r < p.gamma ? p.target : p.drafter;
-  const void* rowp = static_cast<const char*>(base) + row * p.vocab * (BF16 ? 2 : 4);
+  const char* rowp = static_cast<const char*>(base) + row * p.vocab * (BF16 ? 2 : 4);
   const int start = c * kStatsChunk;
   const int len = min(kStatsChunk, p.vocab - start);
 
   uint32_t bad = 0;
-  float m = -INFINITY;
+  float m = -INFINITY, s = 0.f;
   int a = INT_MAX;
-  float s = 0.f;
   const float cs = greedy ? 0.f : kLog2e / T;
   if (VEC) {
-    // The chunk stays packed in registers (16-byte groups, group g of thread t at
-    // g * threads + t) and is decoded on the fly.
-    constexpr int kEpv = BF16 ? 8 : 4;
-    constexpr int kVecs = kPer / kEpv;
-    const int t = threadIdx.x;
-    uint32_t w[kVecs * 4];
+    constexpr int kEpv = BF16 ? 8 : 4;  // elements per 16-byte group
+    constexpr int kGroups = 16;         // groups per lane and round
+    constexpr int kRounds = kStatsChunk / (32 * kGroups * kEpv);
+    static_assert(kRounds * 32 * kGroups * kEpv == kStatsChunk, "chunk must fill whole rounds");
     const uint32_t ninf = BF16 ? 0xFF80FF80u : 0xFF800000u;  // -inf padding past the row end
+    // greedy: this lane's first element starts the argmax (an all -inf chunk reports
+    // its lowest index); a lane past the row end loses every tie
+    a = lane * kEpv < len ? start + lane * kEpv : INT_MAX;
 #pragma unroll
-    for (int k = 0; k < kVecs; ++k) {
-      const int e = (k * kStatsThreads + t) * kEpv;
-      const uint4 r = e < len ? __ldg(reinterpret_cast<const uint4*>(
-                                    static_cast<const char*>(rowp) + static_cast<int64_t>(start + e) * (BF16 ? 2 : 4)))
-                              : make_uint4(ninf, ninf, ninf, ninf);
-      w[4 * k] = r.x; w[4 * k + 1] = r.y; w[4 * k + 2] = r.z; w[4 * k + 3] = r.w;
-    }
-    // element q of 16-byte group k
-    auto elem = [&](int k, int q) -> float {
-      if (BF16) {
-        const uint32_t word = w[4 * k + (q >> 1)];
-        return __uint_as_float((q & 1) ? (word & 0xffff0000u) : (word << 16));
+    for (int rd = 0; rd < kRounds; ++rd) {
+      uint32_t w[kGroups * 4];
+#pragma unroll
+      for (int k = 0; k < kGroups; ++k) {
+        const int e = ((rd * kGroups + k) * 32 + lane) * kEpv;  // first element of the group
+        const uint4 v = e < len ? __ldg(reinterpret_cast<const uint4*>(rowp + static_cast<int64_t>(start + e) * (BF16 ? 2 : 4)))
+                                : make_uint4(ninf, ninf, ninf, ninf);
+        w[4 * k] = v.x; w[4 * k + 1] = v.y; w[4 * k + 2] = v.z; w[4 * k + 3] = v.w;
       }
-      return __uint_as_float(w[4 * k + q]);
-    };
-    if (greedy) {
-      // this thread's elements in increasing index order: a strict > keeps the lowest
-      // index of the maximum; all -inf leaves the first index
-      a = start + t * kEpv;
+      auto elem = [&](int k, int q) -> float {
+        if (BF16) {
+          const uint32_t word = w[4 * k + (q >> 1)];
+          return __uint_as_float((q & 1) ? (word & 0xffff0000u) : (word << 16));
+        }
+        return __uint_as_float(w[4 * k + q]);
+      };
+      if (greedy) {
+        // elements in increasing index order: a strict > keeps the lowest index
 #pragma unroll
-      for (int k = 0; k < kVecs; ++k) {
+        for (int k = 0; k < kGroups; ++k) {
+          const int e = ((rd * kGroups + k) * 32 + lane) * kEpv;
 #pragma unroll
-        for (int q = 0; q < kEpv; ++q) {
-          const float x = elem(k, q);
-          bad |= x != x;  // NaN (+inf is a legal maximum for a greedy row)
-          if (x > m) { m = x; a = start + (k * kStatsThreads + t) * kEpv + q; }
+          for (int q = 0; q < kEpv; ++q) {
+            const float x = elem(k, q);
+            bad |= x != x;  // NaN (+inf is a legal maximum for a greedy row)
+            if (x > m) { m = x; a = start + e + q; }
+          }
+        }
+      } else {
+        // max (NaN is skipped here and caught by the sum below), then the sum
+        float mr;
+        if (BF16) {
+          __nv_bfloat162 mx = *reinterpret_cast<const __nv_bfloat162*>(&w[0]);
+#pragma unroll
+          for (int i = 1; i < kGroups * 4; ++i) mx = __hmax2(mx, *reinterpret_cast<const __nv_bfloat162*>(&w[i]));
+          mr = fmaxf(__bfloat162float(mx.x), __bfloat162float(mx.y));
+        } else {
+          mr = -INFINITY;
+#pragma unroll
+          for (int i = 0; i < kGroups * 4; ++i) mr = fmaxf(mr, __uint_as_float(w[i]));
+        }
+        float sr = 0.f;
+        if (mr != -INFINITY) {
+#pragma unroll
+          for (int k = 0; k < kGroups; ++k)
+#pragma unroll
+            for (int q = 0; q < kEpv; ++q) sr += ex2((elem(k, q) - mr) * cs);
+        }
+        if (rd == 0) {
+          m = mr;
+          s = sr;
+        } else {
+          merge_ms(m, s, mr, sr, cs);
         }
       }
-      if (a >= start + len) a = INT_MAX;  // a thread past the row end loses every tie
-    } else {
-      // max (NaN is skipped here and caught by the sum below)
-      if (BF16) {
-        __nv_bfloat162 mx = *reinterpret_cast<const __nv_bfloat162*>(&w[0]);
-#pragma unroll
-        for (int i = 1; i < kVecs * 4; ++i) mx = __hmax2(mx, *reinterpret_cast<const __nv_bfloat162*>(&w[i]));
-        m = fmaxf(__bfloat162float(mx.x), __bfloat162float(mx.y));
-      } else {
-#pragma unroll
-        for (int i = 0; i < kVecs * 4; ++i) m = fmaxf(m, __uint_as_float(w[i]));
-      }
-      if (m != -INFINITY) {
-#pragma unroll
-        for (int k = 0; k < kVecs; ++k)
-#pragma unroll
-          for (int q = 0; q < kEpv; ++q) s += ex2((elem(k, q) - m) * cs);
-      }
-      // NaN anywhere, or +inf (then +inf - +inf), makes the sum NaN
-      bad |= !(s <= FLT_MAX) || !(m <= FLT_MAX);
     }
+    // NaN anywhere, or +inf (then +inf - +inf), makes the sum NaN
+    if (!greedy) bad |= !(s <= FLT_MAX) || !(m <= FLT_MAX);
   } else {
-    float v[kPer];
-    int idx[kPer];
-    load_strided<BF16, false, kPer, kStatsThreads>(rowp, start, len, v, idx);
-    a = idx[0];
+    // element loads (rows not 16-byte aligned): element k * 32 + lane, in batches
+    constexpr int kBatch = 16;
+    a = lane < len ? start + lane : INT_MAX;
+    for (int k0 = 0; k0 < kStatsChunk / 32; k0 += kBatch) {
+      float v[kBatch];
 #pragma unroll
-    for (int k = 0; k < kPer; ++k) {
-      // greedy rows: NaN; tempered rows: NaN or +inf (padding past the row end is -inf)
-      bad |= greedy ? (v[k] != v[k]) : !(v[k] <= FLT_MAX);
+      for (int k = 0; k < kBatch; ++k) {
+        const int e = (k0 + k) * 32 + lane;
+        v[k] = e < len ? load_elem<BF16>(rowp, start + e) : -INFINITY;
+      }
       if (greedy) {
-        if (v[k] > m) { m = v[k]; a = idx[k]; }
+#pragma unroll
+        for (int k = 0; k < kBatch; ++k) {
+          bad |= v[k] != v[k];
+          if (v[k] > m) { m = v[k]; a = start + (k0 + k) * 32 + lane; }
+        }
       } else {
-        m = fmaxf(m, v[k]);
+        float mr = -INFINITY;
+#pragma unroll
+        for (int k = 0; k < kBatch; ++k) {
+          bad |= !(v[k] <= FLT_MAX);  // NaN or +inf (padding past the row end is -inf)
+          mr = fmaxf(mr, v[k]);
+        }
+        float sr = 0.f;
+        if (mr != -INFINITY) {
+#pragma unroll
+          for (int k = 0; k < kBatch; ++k) sr += ex2((v[k] - mr) * cs);
+        }
+        merge_ms(m, s, mr, sr, cs);
       }
     }
-    if (!greedy && m != -INFINITY) {
-#pragma unroll
-      for (int k = 0; k < kPer; ++k) s += ex2((v[k] - m) * cs);
-    }
   }
-  // warp then block reduction
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
-    const float s2 = __shfl_xor_sync(0xffffffffu, s, o);
-    const int a2 = __shfl_xor_sync(0xffffffffu, a, o);
-    bad |= __shfl_xor_sync(0xffffffffu, bad, o);
-    if (greedy) merge_arg(m, a, m2, a2);
-    else merge_ms(m, s, m2, s2, cs);
-  }
-  const int w = threadIdx.x >> 5;
-  if ((threadIdx.x & 31) == 0) {
-    sh_m[w] = m; sh_s[w] = s; sh_a[w] = a; sh_bad[w] = bad;
-  }
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    for (int k = 1; k < kStatsThreads / 32; ++k) {
-      if (greedy) merge_arg(m, a, sh_m[k], sh_a[k]);
-      else merge_ms(m, s, sh_m[k], sh_s[k], cs);
-      bad |= sh_bad[k];
-    }
+  // warp reduction
+  bad = __reduce_or_sync(0xffffffffu, bad);
+  if (greedy) warp_merge_arg(m, a);
+  else warp_merge_ms(m, s, cs);
+  if (lane == 0) {
     RowPartial out;
     out.m = m;
     out.s = s;
@@ -361,6 +340,7 @@ __global__ void __launch_bounds__(kSampleThreads, 5) decide_sample_kernel(Accept
   const int gamma = p.gamma, V = p.vocab, nrows = 2 * gamma - 1;
   const float T = p.temperature[b];
   const bool greedy = !(T > 0.f);
+  if (greedy && sl != 0) return;  // a greedy sequence draws nothing: slice 0 decides alone
   const float c = greedy ? 0.f : kLog2e / T;
   if (tid == 0) {
     s_bad = 0;
@@ -368,6 +348,8 @@ __global__ void __launch_bounds__(kSampleThreads, 5) decide_sample_kernel(Accept
     s_owner = INT_MAX;
     s_token = -1;
   }
+  // the block's tokens do not depend on the statistics: their load goes out first
+  const int my_tok = tid < gamma ? p.tokens[static_cast<int64_t>(b) * gamma + tid] : 0;
   pdl_wait_prior();  // the row statistics kernel has finished and its writes are visible
   __syncthreads();
 
@@ -388,15 +370,9 @@ __global__ void __launch_bounds__(kSampleThreads, 5) decide_sample_kernel(Accept
         if (greedy) merge_arg(M, A, q.m, q.arg);
         else merge_ms(M, S, q.m, q.s, c);
       }
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        const float m2 = __shfl_xor_sync(0xffffffffu, M, o);
-        const float s2 = __shfl_xor_sync(0xffffffffu, S, o);
-        const int a2 = __shfl_xor_sync(0xffffffffu, A, o);
-        bad |= __shfl_xor_sync(0xffffffffu, bad, o);
-        if (greedy) merge_arg(M, A, m2, a2);
-        else merge_ms(M, S, m2, s2, c);
-      }
+      bad = __reduce_or_sync(0xffffffffu, bad);
+      if (greedy) warp_merge_arg(M, A);
+      else warp_merge_ms(M, S, c);
       if (!greedy && (M == -INFINITY || !(S > 0.f) || !(S <= FLT_MAX))) bad = 1;
       if (lane == 0) {
         rM[r] = M;
@@ -407,9 +383,8 @@ __global__ void __launch_bounds__(kSampleThreads, 5) decide_sample_kernel(Accept
     }
   }
   if (tid < gamma) {
-    const int t = p.tokens[static_cast<int64_t>(b) * gamma + tid];
-    s_tok[tid] = t;
-    if (t < 0 || t >= V) atomicOr(&s_bad, 2);
+    s_tok[tid] = my_tok;
+    if (my_tok < 0 || my_tok >= V) atomicOr(&s_bad, 2);
   }
   __syncthreads();
 
@@ -665,13 +640,12 @@ __global__ void philox_uniforms_kernel(uint64_t seed, uint64_t offset, int64_t n
 
 template <bool BF16, bool VEC>
 cudaError_t launch_typed(const AcceptParams& p, cudaStream_t stream, bool overlap_prior) {
-  const int64_t items = static_cast<int64_t>(p.batch) * (2 * p.gamma - 1) * p.nchunk;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   // row statistics: a programmatic dependent of the attention kernel in a verify step
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(static_cast<unsigned>(items));
+  cfg.gridDim = dim3((p.nchunk + kStatsThreads / 32 - 1) / (kStatsThreads / 32), 2 * p.gamma - 1, p.batch);
   cfg.blockDim = dim3(kStatsThreads);
   cfg.stream = stream;
   cfg.attrs = attr;
