@@ -2,19 +2,21 @@
 // drafter rows and the lossless acceptance rule of Alg. "Lossless Psi-Spec decoding
 // (Linear Sampler)" (Appendix B.3; Sec. 4.2).
 //
-// Two launches, no inter-block waiting (the second is a programmatic dependent of the
-// first and waits for it on the device; in a verify step the first is a programmatic
+// Three launches, no inter-block waiting (each is a programmatic dependent of the one
+// before and waits for it on the device; in a verify step the first is a programmatic
 // dependent of the attention kernel and runs beside it):
 //   1. row_stats_kernel: one warp per (sequence, row, 4096-entry vocab chunk) reads
 //      the chunk once with 16-byte loads and writes its max, its sum of
 //      exp((l - max)/T) and (greedy rows) its lowest-index argmax.
-//   2. decide_sample_kernel: grid (vocab slice, sequence). Every block merges the row
-//      statistics of its sequence and evaluates the gamma-1 decisions
-//      r_i > min(1, p_i(t_i)/q_i(t_i)) (fp64 on the few gathered logits), which fixes
-//      n. Each block then sums the final draw's weights ([p_n - q_n]_+, or p_B for the
-//      bonus) over its slice; the last block of the sequence to finish (atomic ticket)
-//      finds the slice where the ascending cumulative sum crosses u * S and rescans
-//      that slice with a block-wide scan to pick the token.
+//   2. decide_kernel: one block per sequence merges the row statistics and evaluates
+//      the gamma-1 decisions r_i > min(1, p_i(t_i)/q_i(t_i)) (fp64 on the few
+//      gathered logits), which fixes n; it writes every output except a tempered
+//      sequence's final token, and a record of the final draw's normalisers.
+//   3. sample_kernel: grid (vocab slice, sequence), tempered sequences only. Each block
+//      sums the final draw's weights ([p_n - q_n]_+, or p_B for the bonus) over its
+//      slice; the last block of the sequence to finish (atomic ticket) finds the slice
+//      where the ascending cumulative sum crosses u * S and rescans that slice with a
+//      block-wide scan to pick the token.
 #include <cuda_bf16.h>
 
 #include <cfloat>
@@ -32,7 +34,8 @@ AcceptLayout accept_layout(const spec_accept_args_t& a, size_t base) {
   const size_t nrows = 2 * static_cast<size_t>(a.gamma) - 1;
   L.tickets = base;
   L.partials = ws_round(L.tickets + sizeof(uint32_t) * a.batch);
-  L.slice_sums = ws_round(L.partials + sizeof(RowPartial) * a.batch * nrows * L.nchunk);
+  L.records = ws_round(L.partials + sizeof(RowPartial) * a.batch * nrows * L.nchunk);
+  L.slice_sums = ws_round(L.records + 32 * static_cast<size_t>(a.batch));
   L.end = ws_round(L.slice_sums + sizeof(float4) * a.batch * L.nslice);
   return L;
 }
@@ -44,6 +47,13 @@ struct SliceSum {  // per (sequence, vocab slice) sums of the final draw's weigh
   float e;         // sum of exp((l_p - M_p)/T) (bonus, and the empty-residual fallback)
   int32_t wlast;   // last index with positive residual weight, -1 if none
   int32_t elast;   // last index with positive bonus weight, -1 if none
+};
+
+struct DecideRecord {  // what the sampling kernel needs of a sequence's decisions
+  int32_t n;           // first rejected draft (gamma: all accepted); 0: bad sequence
+  float Mp, invSp;     // max and 1 / sum of row p_n (target row n - 1)
+  float Mq, invSq;     // the same for q_n (drafter row n); unused for the bonus draw
+  int32_t pad[3];
 };
 
 struct AcceptParams {
@@ -60,6 +70,7 @@ struct AcceptParams {
   uint32_t* status;
   uint32_t* tickets;
   RowPartial* partials;
+  DecideRecord* records;
   SliceSum* slices;
 };
 
@@ -324,29 +335,27 @@ __device__ __forceinline__ void final_weights(const AcceptParams& p, const void*
   }
 }
 
-template <bool BF16, bool VEC>
-__global__ void __launch_bounds__(kSampleThreads, 5) decide_sample_kernel(AcceptParams p) {
+// Decisions: one block per sequence merges the chunk statistics of the rows it uses,
+// takes the gamma-1 decisions and writes every output except, for a tempered
+// sequence, the final drawn token (left to the sampling kernel with a record).
+template <bool BF16>
+__global__ void __launch_bounds__(kDecideThreads) decide_kernel(AcceptParams p) {
+  pdl_launch_dependents();
   constexpr int kMaxGamma = 64;
-  constexpr int kPer = kSamplePerThread;
   __shared__ float rM[2 * kMaxGamma], rS[2 * kMaxGamma];
   __shared__ int rA[2 * kMaxGamma];
   __shared__ int s_tok[kMaxGamma];
   __shared__ float s_ptok[kMaxGamma], s_qtok[kMaxGamma];
-  __shared__ int s_bad, s_n, s_last, s_star, s_use_res, s_owner, s_token;
-  __shared__ float s_base, s_target;
-  __shared__ float sh_scan[kSampleThreads / 32 + 1];
+  __shared__ int s_bad, s_n;
 
-  const int b = blockIdx.y, sl = blockIdx.x, tid = threadIdx.x;
+  const int b = blockIdx.x, tid = threadIdx.x;
   const int gamma = p.gamma, V = p.vocab, nrows = 2 * gamma - 1;
   const float T = p.temperature[b];
   const bool greedy = !(T > 0.f);
-  if (greedy && sl != 0) return;  // a greedy sequence draws nothing: slice 0 decides alone
   const float c = greedy ? 0.f : kLog2e / T;
   if (tid == 0) {
     s_bad = 0;
     s_n = gamma;
-    s_owner = INT_MAX;
-    s_token = -1;
   }
   // the block's tokens do not depend on the statistics: their load goes out first
   const int my_tok = tid < gamma ? p.tokens[static_cast<int64_t>(b) * gamma + tid] : 0;
@@ -359,7 +368,7 @@ __global__ void __launch_bounds__(kSampleThreads, 5) decide_sample_kernel(Accept
   const int rows_needed = greedy ? gamma : nrows;
   {
     const int warp = tid >> 5, lane = tid & 31;
-    for (int r = warp; r < rows_needed; r += kSampleThreads / 32) {
+    for (int r = warp; r < rows_needed; r += kDecideThreads / 32) {
       const RowPartial* rp = p.partials + (static_cast<int64_t>(b) * nrows + r) * p.nchunk;
       float M = -INFINITY, S = 0.f;
       int A = INT_MAX;
@@ -390,17 +399,18 @@ __global__ void __launch_bounds__(kSampleThreads, 5) decide_sample_kernel(Accept
 
   const int64_t orow = static_cast<int64_t>(b) * (gamma + 1);
   if (s_bad) {
-    if (sl == 0) {
-      for (int k = tid; k <= gamma; k += kSampleThreads) p.out_tokens[orow + k] = -1;
-      if (p.diag)
-        for (int k = tid; k < 2 * gamma; k += kSampleThreads)
-          p.diag[static_cast<int64_t>(b) * gamma * 2 + k] = NAN;
-      if (tid == 0) {
-        p.num_accepted[b] = -1;
-        p.num_emitted[b] = 0;
-        set_status(p.status, (s_bad & 2) ? SPEC_FLAG_BAD_TOKEN : SPEC_FLAG_BAD_LOGITS);
-        if ((s_bad & 3) == 3) set_status(p.status, SPEC_FLAG_BAD_LOGITS);
-      }
+    for (int k = tid; k <= gamma; k += kDecideThreads) p.out_tokens[orow + k] = -1;
+    if (p.diag)
+      for (int k = tid; k < 2 * gamma; k += kDecideThreads)
+        p.diag[static_cast<int64_t>(b) * gamma * 2 + k] = NAN;
+    if (tid == 0) {
+      p.num_accepted[b] = -1;
+      p.num_emitted[b] = 0;
+      set_status(p.status, (s_bad & 2) ? SPEC_FLAG_BAD_TOKEN : SPEC_FLAG_BAD_LOGITS);
+      if ((s_bad & 3) == 3) set_status(p.status, SPEC_FLAG_BAD_LOGITS);
+      DecideRecord rec = {};
+      rec.n = 0;  // nothing to draw
+      p.records[b] = rec;
     }
     return;
   }
@@ -436,27 +446,59 @@ __global__ void __launch_bounds__(kSampleThreads, 5) decide_sample_kernel(Accept
   __syncthreads();
   const int n = s_n;
 
-  auto write_outputs = [&](int final_token) {
-    for (int k = tid; k <= gamma; k += kSampleThreads)
-      p.out_tokens[orow + k] = k < n ? s_tok[k] : (k == n ? final_token : -1);
-    if (p.diag) {
-      for (int i = tid; i < gamma; i += kSampleThreads) {
-        const int64_t d = (static_cast<int64_t>(b) * gamma + i) * 2;
-        const bool taken = i >= 1 && i <= n && i < gamma;
-        p.diag[d] = i == 0 ? 0.f : (taken ? s_ptok[i] : NAN);
-        p.diag[d + 1] = i == 0 ? 0.f : (taken ? s_qtok[i] : NAN);
-      }
-    }
-    if (tid == 0) {
-      p.num_accepted[b] = n - 1;
-      p.num_emitted[b] = n + 1;
-    }
-  };
-
-  if (greedy) {
-    if (sl == 0) write_outputs(rA[n - 1]);
-    return;
+  // every output but the final token of a tempered sequence
+  for (int k = tid; k <= gamma; k += kDecideThreads) {
+    if (k < n) p.out_tokens[orow + k] = s_tok[k];
+    else if (k > n) p.out_tokens[orow + k] = -1;
+    else if (greedy) p.out_tokens[orow + k] = rA[n - 1];
   }
+  if (p.diag) {
+    for (int i = tid; i < gamma; i += kDecideThreads) {
+      const int64_t d = (static_cast<int64_t>(b) * gamma + i) * 2;
+      const bool taken = i >= 1 && i <= n && i < gamma;
+      p.diag[d] = i == 0 ? 0.f : (taken ? s_ptok[i] : NAN);
+      p.diag[d + 1] = i == 0 ? 0.f : (taken ? s_qtok[i] : NAN);
+    }
+  }
+  if (tid == 0) {
+    p.num_accepted[b] = n - 1;
+    p.num_emitted[b] = n + 1;
+    if (!greedy) {
+      const bool bonus = n == gamma;
+      DecideRecord rec = {};
+      rec.n = n;
+      rec.Mp = rM[n - 1];
+      rec.invSp = 1.f / rS[n - 1];
+      rec.Mq = bonus ? 0.f : rM[gamma + n - 1];
+      rec.invSq = bonus ? 0.f : 1.f / rS[gamma + n - 1];
+      p.records[b] = rec;
+    }
+  }
+}
+
+// Sampling: grid (vocab slice, sequence) for tempered sequences. Each block sums the
+// final draw's weights over its slice; the last block of the sequence (atomic ticket)
+// finds the slice where the ascending cumulative sum crosses u * S and rescans it.
+template <bool BF16, bool VEC>
+__global__ void __launch_bounds__(kSampleThreads, 5) sample_kernel(AcceptParams p) {
+  constexpr int kPer = kSamplePerThread;
+  __shared__ int s_last, s_star, s_use_res, s_owner, s_token;
+  __shared__ float s_base, s_target;
+  __shared__ float sh_scan[kSampleThreads / 32 + 1];
+  const int b = blockIdx.y, sl = blockIdx.x, tid = threadIdx.x;
+  const int gamma = p.gamma, V = p.vocab;
+  const float T = p.temperature[b];
+  if (!(T > 0.f)) return;  // greedy: the decide kernel wrote the whole row
+  const float c = kLog2e / T;
+  if (tid == 0) {
+    s_owner = INT_MAX;
+    s_token = -1;
+  }
+  pdl_wait_prior();  // the decide kernel has finished and its writes are visible
+  const DecideRecord rec = p.records[b];
+  const int n = rec.n;
+  if (n < 1) return;  // bad sequence: nothing to draw
+  const int64_t orow = static_cast<int64_t>(b) * (gamma + 1);
 
   // 3. sums of the final draw's weights over this block's slice
   const bool bonus = n == gamma;
@@ -465,9 +507,7 @@ __global__ void __launch_bounds__(kSampleThreads, 5) decide_sample_kernel(Accept
   const void* qrow = bonus ? prow
                            : static_cast<const char*>(p.drafter) +
                                  (static_cast<int64_t>(b) * gamma + n) * V * (BF16 ? 2 : 4);
-  const float Mp = rM[n - 1], invSp = 1.f / rS[n - 1];
-  const float Mq = bonus ? 0.f : rM[gamma + n - 1];
-  const float invSq = bonus ? 0.f : 1.f / rS[gamma + n - 1];
+  const float Mp = rec.Mp, invSp = rec.invSp, Mq = rec.Mq, invSq = rec.invSq;
 
   float w[kPer], e[kPer];
   int first;
@@ -607,7 +647,7 @@ __global__ void __launch_bounds__(kSampleThreads, 5) decide_sample_kernel(Accept
     }
   }
   __syncthreads();
-  write_outputs(s_token);
+  if (tid == 0) p.out_tokens[orow + n] = s_token;
 }
 
 __global__ void philox_uniforms_kernel(uint64_t seed, uint64_t offset, int64_t n, float* out) {
@@ -652,12 +692,16 @@ cudaError_t launch_typed(const AcceptParams& p, cudaStream_t stream, bool overla
   cfg.numAttrs = overlap_prior ? 1 : 0;
   cudaError_t e = cudaLaunchKernelEx(&cfg, row_stats_kernel<BF16, VEC>, p);
   if (e != cudaSuccess) return e;
-  // decisions and draws: a programmatic dependent of the statistics kernel (it waits
-  // for that kernel's completion before reading the partials)
+  // decisions (a programmatic dependent of the statistics kernel, which it waits for
+  // before reading the partials), then the draws (likewise of the decisions)
+  cfg.gridDim = dim3(p.batch);
+  cfg.blockDim = dim3(kDecideThreads);
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, decide_kernel<BF16>, p);
+  if (e != cudaSuccess) return e;
   cfg.gridDim = dim3(p.nslice, p.batch);
   cfg.blockDim = dim3(kSampleThreads);
-  cfg.numAttrs = 1;
-  e = cudaLaunchKernelEx(&cfg, decide_sample_kernel<BF16, VEC>, p);
+  e = cudaLaunchKernelEx(&cfg, sample_kernel<BF16, VEC>, p);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
@@ -684,6 +728,7 @@ cudaError_t launch_accept(const spec_accept_args_t& a, const AcceptLayout& L, ch
   p.status = reinterpret_cast<uint32_t*>(ws);
   p.tickets = reinterpret_cast<uint32_t*>(ws + L.tickets);
   p.partials = reinterpret_cast<RowPartial*>(ws + L.partials);
+  p.records = reinterpret_cast<DecideRecord*>(ws + L.records);
   p.slices = reinterpret_cast<SliceSum*>(ws + L.slice_sums);
   const bool bf16 = a.logits_dtype == SPEC_BF16;
   const size_t esz = bf16 ? 2 : 4;

@@ -23,6 +23,7 @@ inline size_t ws_round(size_t x) { return (x + kWsAlign - 1) / kWsAlign * kWsAli
 constexpr int kStatsThreads = 128;
 constexpr int kStatsChunk = 4096;                          // vocab elements per row item
 constexpr int kSampleThreads = 128;
+constexpr int kDecideThreads = 256;                        // one block per sequence
 constexpr int kSampleSlice = 4096;                         // vocab elements per sample block
 constexpr int kSamplePerThread = kSampleSlice / kSampleThreads;  // contiguous per thread
 
@@ -36,6 +37,7 @@ struct RowPartial {  // one (sequence, row, vocab chunk) item of the row statist
 struct AcceptLayout {
   size_t tickets;      // uint32 [batch]
   size_t partials;     // RowPartial [batch][2*gamma-1][nchunk]
+  size_t records;      // 32-byte decision record [batch] (n and the final draw's normalisers)
   size_t slice_sums;   // float4 [batch][nslice] = (residual sum, p sum, residual last, p last)
   size_t end;
   int nchunk, nslice;
