@@ -43,15 +43,15 @@ L2_FLUSH_BYTES = 256 << 20
 # while the kernel's sources still hash to what they were when the capture was taken.
 MEASURED_TRAFFIC = {
     ("llama8b", "attention"): {
-        "bytes": 139_722_752,
+        "bytes": 139_693_056,
         "profile": "profiles/attn_tc_kernel_llama8b.md",
         "sources": {
             "paper_2609_04010_gb300/csrc/attn_tc.cu":
-                "9c962f061f9e632752374081c86394ae1ff79d93deed0ac5082bb58729d77ad7",
+                "e108ce0d33e6bfa78a03713b6355cf6386c729aa620c38c7db71fd510c3cbda0",
             "paper_2609_04010_gb300/csrc/attn_common.cuh":
-                "303519f8ceecdf8dc1d87cb5a31f59dc3b88858372f4e4d285e218a5eb6dc155",
+                "92c08340231887aa7a8614c752c7a0fcea3ba600461aec09240162de420f465c",
             "paper_2609_04010_gb300/csrc/common.cuh":
-                "5440eaabb2f9533d39a8abd13d08d2c28cae2a7868c16422ec56a8d35aeb3892",
+                "b59156aa4ea00852b9b5c078bbc03a73954bc83e855e407907568782ed4f9a90",
         },
     },
 }
@@ -380,20 +380,24 @@ def run_ours(args, wl, ai, ci, rank, world, local_rank):
     acc_ms = statistics.mean(timed_loop(acc_g.replay, parts_n))
     eager_ms = statistics.mean(timed_loop(step, parts_n))
 
-    e2e = None
+    e2e = e2e_kv = None
     if not args.no_e2e:
         pin = {k: v.pin_memory() for k, v in host_in.items()}
         outs_h = [torch.empty(x.shape, dtype=x.dtype).pin_memory() for x in (out, lse, na, ot, ne)]
         h2d = sum(v.numel() * v.element_size() for v in pin.values())
         d2h = sum(v.numel() * v.element_size() for v in outs_h)
 
-        def e2e_step():
-            for k in d:
-                d[k].copy_(pin[k], non_blocking=True)
-            step()
-            for hst, src in zip(outs_h, (out, lse, na, ot, ne)):
-                hst.copy_(src, non_blocking=True)
+        def e2e_with(keys):
+            def run():
+                for k in keys:
+                    d[k].copy_(pin[k], non_blocking=True)
+                step()
+                for hst, src in zip(outs_h, (out, lse, na, ot, ne)):
+                    hst.copy_(src, non_blocking=True)
+            return run
 
+        # every input from host memory, the KV cache included
+        e2e_step = e2e_with(list(d))
         for _ in range(3):
             e2e_step()
         n_e2e = max(10, min(args.steps, 200))
@@ -401,6 +405,16 @@ def run_ours(args, wl, ai, ci, rank, world, local_rank):
         e2e = {"value": whole_job_tokens_per_s(world, B, G, e2e_ms), "unit": UNIT,
                "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
                "ms_per_step": e2e_ms}
+        # context: a serving loop keeps the KV cache on the device and copies the rest
+        step_keys = [k for k in d if k not in ("k", "v")]
+        kv_step = e2e_with(step_keys)
+        for _ in range(3):
+            kv_step()
+        kv_ms = max_over_ranks(statistics.mean(timed_loop(kv_step, n_e2e)), world, dev)
+        e2e_kv = {"value": whole_job_tokens_per_s(world, B, G, kv_ms), "unit": UNIT,
+                  "h2d_bytes_per_step": int(sum(pin[k].numel() * pin[k].element_size() for k in step_keys)),
+                  "d2h_bytes_per_step": int(d2h), "ms_per_step": kv_ms,
+                  "note": "KV cache resident on the device; every other input copied from host"}
 
     emitted = sum_over_ranks(float(ne.sum().item()), world, dev)
     tm = traffic_model(ai, ci)
@@ -411,7 +425,7 @@ def run_ours(args, wl, ai, ci, rank, world, local_rank):
     dom_bytes = tm["kv"] if dominant == "attention" else tm["logits"]
     dom_ms = attn_ms if dominant == "attention" else acc_ms
     dom_gbs = dom_bytes / (dom_ms / 1000.0) / 1e9
-    launches_per_step = 3
+    launches_per_step = 4  # attention, row statistics, decisions, draws
     traffic, traffic_src = (None, None)
     if dominant == "attention" and attn_path_name(args.attn_path, binding, ai) == "tensor cores":
         traffic, traffic_src = measured_traffic(args.workload, "attention")
@@ -442,6 +456,7 @@ def run_ours(args, wl, ai, ci, rank, world, local_rank):
     }
     if e2e:
         result["e2e"] = e2e
+        result["e2e_kv_resident"] = e2e_kv
     return result
 
 

@@ -196,7 +196,8 @@ int32_t spec_attn_tensor_core_min_rows(void);
  * every GPU that loads the library keeps until the process exits.
  *   - Arguments: as spec_accept_block (device pointers, same layouts); no workspace.
  *   - Limit: the scratch this batch needs (16 bytes per (sequence, row, 4096-entry
- *     vocab chunk) plus 16 bytes per (sequence, 4096-entry slice), rounded up) must fit
+ *     vocab chunk), 32 bytes per sequence, and 16 bytes per (sequence, 4096-entry
+ *     slice), rounded up) must fit
  *     in SPEC_NOALLOC_SCRATCH_BYTES; otherwise SPEC_ERR_WORKSPACE_TOO_SMALL, with
  *     nothing launched. Other argument errors as spec_accept_block.
  *   - Allocates nothing: no cudaMalloc, cudaFree or allocating library routine. The
