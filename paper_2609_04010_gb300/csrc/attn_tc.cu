@@ -51,6 +51,10 @@ struct TcCfg {
   static constexpr int PB = MT == 1 ? 2 : 1;          // P buffers (double with one M tile)
   static constexpr int STAGES = (D == 128 && MT == 2) || (D == 64 && MT == 1) ? 3 : 4;
   static constexpr int THREADS = 128 + 256;           // 4 producer / MMA warps + 8 softmax
+  // Starting a unit inside a block's range costs about this many tiles of time (its Q
+  // tile, the pipeline refill and the previous unit's epilogue). When blocks hold
+  // several unit starts the work list charges it, so that blocks stay balanced.
+  static constexpr int UNIT_OVERHEAD = MT == 1 ? 3 : 2;
   static constexpr uint32_t Q_BYTES = MT * DH * 16384;  // [MT][DH][128 rows x 128 B]
   static constexpr uint32_t KV_BYTES = DH * 8192;       // one stage of K (or V): [DH][64 x 128 B]
   static constexpr uint32_t P_BYTES = PB * MT * 16384;  // [PB][MT][128 rows x 128 B]
@@ -235,41 +239,58 @@ __device__ __forceinline__ int unit_tiles(int kv_len, const AttnParams& p) {
   return ok ? (kv_len + TK - 1) / TK : 1;  // a malformed sequence keeps one tile to report it
 }
 
+// The work list is virtual: each unit is ovh overhead tiles followed by its real tiles,
+// and a block owns an equal range of virtual tiles. A segment is the part of one unit
+// inside a block's range. Only a range that ends inside a unit's overhead has a segment
+// with no real tile, and then it is the range's last (a first segment without real
+// tiles means the block has no work).
 struct Seg {
   int b, g, rt;      // sequence, KV head, row tile
   int64_t u;         // unit index (b * Hkv + g) * row_tiles + rt
-  int tile0, ntile;  // first tile within the unit and tile count of this segment
-  int unit_tiles;    // tiles of the whole unit
+  int tile0, ntile;  // first real tile within the unit and real tile count of this segment
+  int unit_tiles;    // real tiles of the whole unit
   int kv_len;
   bool len_ok;
-  int64_t unit_start;  // global index of the unit's first tile
+  int64_t unit_start;  // virtual index of the unit's first real tile
+  int64_t vnext;       // virtual index just past this segment
 };
 
-__device__ __forceinline__ Seg locate(int64_t t, int64_t t1, const AttnParams& p,
-                                      const int* pb) {
-  int lo = 0, hi = p.batch;  // largest b with pb[b] <= t
+__device__ __forceinline__ Seg locate(int64_t v, int64_t v1, const AttnParams& p,
+                                      const int* pb, int ovh) {
+  int lo = 0, hi = p.batch;  // largest b with pb[b] <= v
   while (hi - lo > 1) {
     const int mid = (lo + hi) >> 1;
-    if (pb[mid] <= t) lo = mid; else hi = mid;
+    if (pb[mid] <= v) lo = mid; else hi = mid;
   }
   Seg s;
   s.b = lo;
   s.kv_len = p.kv_len[lo];
   s.len_ok = s.kv_len >= p.gamma && s.kv_len <= p.max_keys;
   s.unit_tiles = unit_tiles(s.kv_len, p);
-  const int64_t rem = t - pb[lo];
-  const int ub = static_cast<int>(rem / s.unit_tiles);
-  s.tile0 = static_cast<int>(rem % s.unit_tiles);
+  const int vlen = s.unit_tiles + ovh;
+  const int64_t rem = v - pb[lo];
+  const int ub = static_cast<int>(rem / vlen);
+  const int64_t vstart = v - rem % vlen;  // the unit's first (overhead) virtual tile
   s.g = ub / p.row_tiles;
   s.rt = ub % p.row_tiles;
   s.u = static_cast<int64_t>(lo) * p.hkv * p.row_tiles + ub;
-  s.unit_start = t - s.tile0;
-  const int64_t end = s.unit_start + s.unit_tiles;
-  s.ntile = static_cast<int>((end < t1 ? end : t1) - t);
+  s.unit_start = vstart + ovh;
+  const int64_t vend = vstart + vlen;
+  s.vnext = vend < v1 ? vend : v1;
+  const int64_t lo_real = v > s.unit_start ? v : s.unit_start;
+  s.ntile = s.vnext > lo_real ? static_cast<int>(s.vnext - lo_real) : 0;
+  s.tile0 = s.ntile > 0 ? static_cast<int>(lo_real - s.unit_start) : 0;
   return s;
 }
 
-// Block that owns global tile t when `total` tiles are cut into `ctas` ranges
+// Whether real tiles follow segment s in the range ending at v1. A segment ends at its
+// unit's end or at v1, so the next one starts a unit, whose real tiles begin ovh virtual
+// tiles later; no load is needed.
+__device__ __forceinline__ bool has_more(const Seg& s, int64_t v1, int ovh) {
+  return v1 - s.vnext > ovh;
+}
+
+// Block that owns virtual tile t when `total` virtual tiles are cut into `ctas` ranges
 // [c * total / ctas, (c + 1) * total / ctas).
 __device__ __forceinline__ int owner_of(int64_t t, int64_t total, int ctas) {
   return static_cast<int>(((t + 1) * ctas - 1) / total);
@@ -365,7 +386,7 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
     int carry = 0;
     for (int b0 = 0; b0 < p.batch; b0 += 32) {
       const int b = b0 + lane;
-      int v = b < p.batch ? unit_tiles(p.kv_len[b], p) * per_b : 0;
+      int v = b < p.batch ? (unit_tiles(p.kv_len[b], p) + p.unit_overhead) * per_b : 0;
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
         const int y = __shfl_up_sync(0xffffffffu, v, o);
@@ -386,6 +407,7 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
   const int cta = blockIdx.x;
   const int64_t t0 = cta < ctas ? static_cast<int64_t>(cta) * total / ctas : 0;
   const int64_t t1 = cta < ctas ? static_cast<int64_t>(cta + 1) * total / ctas : 0;
+  const int OVH = p.unit_overhead;
 
   if (pw >= 0) {
     // ============================ KV producers ============================
@@ -407,8 +429,7 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
     };
     const uint32_t box_bytes = static_cast<uint32_t>(p.page_size) * D * 2;  // one page of one head
     uint32_t seg_no = 0;
-    for (int64_t t = t0; t < t1 && ok; ++seg_no) {
-      const Seg s = locate(t, t1, p, pb);
+    for (Seg s = locate(t0, t1, p, pb, OVH); s.ntile > 0 && ok; ++seg_no) {
       const bool bad = !s.len_ok;  // nothing to read
       bool flag = bad;             // ... or a page id out of range (read as page 0)
       for (int k = 0; k < s.ntile && ok; ++k, ++it) {
@@ -447,7 +468,8 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
         seg_flag[seg_no & 7] = flag ? 1 : 0;
         mbar_arrive(flag_bar(seg_no & 7));
       }
-      t += s.ntile;
+      if (!has_more(s, t1, OVH)) break;
+      s = locate(s.vnext, t1, p, pb, OVH);
     }
     if (!ok) {  // drain this block's copies still in flight (bounded)
       for (uint32_t x = it > static_cast<uint32_t>(C::STAGES) ? it - C::STAGES : 0; x < it; ++x) {
@@ -485,9 +507,11 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
       }
       __syncwarp();
     };
-    if (qk_role && p.q_tma && t0 < t1) issue_q(locate(t0, t1, p, pb));
-    for (int64_t t = t0; t < t1 && ok;) {
-      const Seg s = locate(t, t1, p, pb);
+    if (qk_role && p.q_tma) {
+      const Seg s0 = locate(t0, t1, p, pb, OVH);
+      if (s0.ntile > 0) issue_q(s0);
+    }
+    for (Seg s = locate(t0, t1, p, pb, OVH); s.ntile > 0 && ok;) {
       if (qk_role) {
         ok = mbar_wait(p.q_tma ? q_full : seg_ready, seg_no & 1, abort_flag, p.status);
         if (!ok) break;
@@ -533,12 +557,12 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
             issued = true;
           }
           __syncwarp();
-          if (p.q_tma && k == s.ntile - 1 && t + s.ntile < t1) {
+          if (p.q_tma && k == s.ntile - 1 && has_more(s, t1, OVH)) {
             // the segment's last scores are done with its Q tile: fetch the next one
             for (int mt = 0; mt < MT && ok; ++mt)
               ok = mbar_wait(s_full(mt, x & 1), (x >> 1) & 1, abort_flag, p.status);
             if (!ok) break;
-            issue_q(locate(t + s.ntile, t1, p, pb));
+            issue_q(locate(s.vnext, t1, p, pb, OVH));
           }
         } else {
           // O += P V for tile x (its P implies its S, hence its landed stage)
@@ -571,8 +595,9 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
         }
       }
       it += s.ntile;
-      t += s.ntile;
       ++seg_no;
+      if (!has_more(s, t1, OVH)) break;
+      s = locate(s.vnext, t1, p, pb, OVH);
     }
     if (!ok && __any_sync(0xffffffffu, issued)) {  // drain this warp's MMAs (bounded)
       const uint32_t db = drain_bar(qk_role ? 0 : 1);
@@ -629,18 +654,14 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
       if (lane == 0) mbar_arrive(seg_ready);
     };
     uint4 qr[kChunks];
-    Seg s;
     uint32_t seg_no = 0;
-    if (t0 < t1) {
-      s = locate(t0, t1, p, pb);
-      if (!p.q_tma) {
-        load_q(s, qr);
-        store_q(qr);
-      }
+    Seg s = locate(t0, t1, p, pb, OVH);
+    if (s.ntile > 0 && !p.q_tma) {
+      load_q(s, qr);
+      store_q(qr);
     }
-    for (int64_t t = t0; t < t1 && ok;) {
-      const int64_t tn = t + s.ntile;
-      const bool has_next = tn < t1;
+    while (s.ntile > 0 && ok) {
+      const bool has_next = has_more(s, t1, OVH);
       const RowOf ro = row_of(s);
       const int ctx = s.kv_len - p.gamma;
       float m = -INFINITY, l = 0.f;
@@ -733,8 +754,9 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
       // (its last S was read above), so its Q tile can be replaced while this
       // segment's epilogue runs. Its first P V waits for this epilogue (program order).
       Seg sn;
+      sn.ntile = 0;
       if (has_next) {
-        sn = locate(tn, t1, p, pb);
+        sn = locate(s.vnext, t1, p, pb, OVH);
         if (!p.q_tma) {
           load_q(sn, qr);
           store_q(qr);
@@ -820,7 +842,6 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
         *pend_count = *pend_count + 1;
       }
       it += s.ntile;
-      t = tn;
       s = sn;
       ++seg_no;
     }
@@ -930,6 +951,11 @@ cudaError_t launch_typed(const spec_attn_args_t& a, const AttnPlan& P, char* ws,
     return cudaErrorInvalidValue;
   AttnParams p = make_attn_params(a, P, ws);
   p.q_tma = encode_q_map(&mq, a) ? 1 : 0;
+  // Charge unit starts only when blocks hold several of them; when every unit is spread
+  // over several blocks, a block holds at most one start and the charge would mostly
+  // move real tiles away from blocks that pay no boundary.
+  const int64_t units = static_cast<int64_t>(a.batch) * a.num_kv_heads * P.row_tiles;
+  p.unit_overhead = units > P.grid ? Cf::UNIT_OVERHEAD : 0;
   if (!p.q_tma) mq = mk;  // unused
   const size_t smem = Cf::smem_bytes(a.batch);
   cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel<D, MT>,
