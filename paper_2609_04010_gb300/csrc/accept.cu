@@ -357,8 +357,16 @@ __global__ void __launch_bounds__(kDecideThreads) decide_kernel(AcceptParams p) 
     s_bad = 0;
     s_n = gamma;
   }
-  // the block's tokens do not depend on the statistics: their load goes out first
+  // The tokens, the logits at the drafted tokens and the uniforms are inputs, not
+  // results of the statistics kernel: they are read while that kernel still runs.
   const int my_tok = tid < gamma ? p.tokens[static_cast<int64_t>(b) * gamma + tid] : 0;
+  double my_lp = 0.0, my_lq = 0.0;
+  float my_u = 0.f;
+  if (!greedy && tid >= 1 && tid < gamma && my_tok >= 0 && my_tok < V) {
+    my_lp = load_elem<BF16>(p.target, (static_cast<int64_t>(b) * gamma + tid - 1) * V + my_tok);
+    my_lq = load_elem<BF16>(p.drafter, (static_cast<int64_t>(b) * gamma + tid) * V + my_tok);
+    my_u = p.uniforms[static_cast<int64_t>(b) * gamma + tid - 1];
+  }
   pdl_wait_prior();  // the row statistics kernel has finished and its writes are visible
   __syncthreads();
 
@@ -425,16 +433,13 @@ __global__ void __launch_bounds__(kDecideThreads) decide_kernel(AcceptParams p) 
       pt = reject ? 0.f : 1.f;
       qt = 1.f;
     } else {
-      const int64_t prow = static_cast<int64_t>(b) * gamma + (i - 1);
-      const int64_t qrow = static_cast<int64_t>(b) * gamma + i;
-      const double lp = load_elem<BF16>(p.target, prow * V + t);
-      const double lq = load_elem<BF16>(p.drafter, qrow * V + t);
+      const double lp = my_lp, lq = my_lq;  // this thread's token is t (fetched above)
       const double Td = static_cast<double>(T);
       const double pd = exp((lp - static_cast<double>(rM[i - 1])) / Td) / static_cast<double>(rS[i - 1]);
       const double qd = exp((lq - static_cast<double>(rM[gamma + i - 1])) / Td) /
                         static_cast<double>(rS[gamma + i - 1]);
       const double ratio = qd > 0.0 ? pd / qd : INFINITY;
-      const double u = static_cast<double>(p.uniforms[static_cast<int64_t>(b) * gamma + i - 1]);
+      const double u = static_cast<double>(my_u);
       reject = u > fmin(1.0, ratio);
       pt = static_cast<float>(pd);
       qt = static_cast<float>(qd);

@@ -23,7 +23,7 @@ inline size_t ws_round(size_t x) { return (x + kWsAlign - 1) / kWsAlign * kWsAli
 constexpr int kStatsThreads = 128;
 constexpr int kStatsChunk = 4096;                          // vocab elements per row item
 constexpr int kSampleThreads = 128;
-constexpr int kDecideThreads = 256;                        // one block per sequence
+constexpr int kDecideThreads = 512;                        // one block per sequence
 constexpr int kSampleSlice = 4096;                         // vocab elements per sample block
 constexpr int kSamplePerThread = kSampleSlice / kSampleThreads;  // contiguous per thread
 
