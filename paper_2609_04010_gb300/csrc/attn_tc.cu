@@ -403,7 +403,18 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
   const uint32_t tmem = misc[0];
 
   const int64_t total = pb[p.batch];
-  const int ctas = static_cast<int>(total < gridDim.x ? total : gridDim.x);
+  // With no more units than blocks, use a multiple of the unit count: equal-length
+  // units then split into equal parts with no unit boundary inside any block's range
+  // (a few SMs idle; measured faster than spreading boundaries and extra merges over
+  // every SM). Ranges stay equal in tiles, so ragged lengths stay balanced.
+  int ctas = static_cast<int>(total < gridDim.x ? total : gridDim.x);
+  {
+    const int units = p.batch * p.hkv * p.row_tiles;
+    if (units <= static_cast<int>(gridDim.x)) {
+      const int aligned = units * (static_cast<int>(gridDim.x) / units);
+      if (aligned < ctas) ctas = aligned;
+    }
+  }
   const int cta = blockIdx.x;
   const int64_t t0 = cta < ctas ? static_cast<int64_t>(cta) * total / ctas : 0;
   const int64_t t1 = cta < ctas ? static_cast<int64_t>(cta + 1) * total / ctas : 0;
