@@ -65,6 +65,11 @@ def _load():
             lib.oracle_accept_block.argtypes = [i32, i32, i64, i32, P, P, P, P, P, P, P, P,
                                                 P, P, P, P, i32]
             lib.oracle_accept_block.restype = ctypes.c_int
+            lib.oracle_filter_row.argtypes = [P, i64, i32, f64, P, P]
+            lib.oracle_filter_row.restype = ctypes.c_int
+            lib.oracle_accept_block_filtered.argtypes = [i32, i32, i64, i32, P, P, P, P, P, P,
+                                                         P, P, P, P, P, P, P, P, P, i32]
+            lib.oracle_accept_block_filtered.restype = ctypes.c_int
             lib.oracle_verify_attention.argtypes = [i32, i32, i32, i32, i32, i32, i32, i32, f64,
                                                     P, P, P, P, P, P, P, P, i64, P, i32]
             lib.oracle_verify_attention.restype = ctypes.c_int
@@ -177,6 +182,9 @@ def load_variant(src_text: str, tag: str):
     i32, i64 = ctypes.c_int32, ctypes.c_int64
     lib.oracle_accept_probs_many.argtypes = [i64, i32, i64, P, P, P, P, i32, P, P, P, i32]
     lib.oracle_accept_probs_many.restype = ctypes.c_int
+    lib.oracle_accept_block_filtered.argtypes = [i32, i32, i64, i32, P, P, P, P, P, P, P, P,
+                                                 P, P, P, P, P, P, P, i32]
+    lib.oracle_accept_block_filtered.restype = ctypes.c_int
     return lib
 
 
@@ -222,6 +230,60 @@ def accept_block(target_logits, drafter_logits, block_tokens, temperature, unifo
         raise ValueError("invalid arguments to oracle_accept_block")
     return dict(num_accepted=na, out_tokens=ot, num_emitted=ne, diag=diag,
                 accept_margin=am, sample_margin=sm, status=st)
+
+
+def filter_row(p, top_k: int, top_p: float):
+    """Top-k then top-p filtering of one probability row; returns (filtered row, margin)."""
+    lib = _load()
+    pr = _c(p, np.float64)
+    out = np.empty_like(pr)
+    m = np.empty(1, np.float64)
+    rc = lib.oracle_filter_row(_ptr(pr), pr.size, int(top_k), float(top_p), _ptr(out), _ptr(m))
+    if rc:
+        raise ValueError("top_k must be >= 1 and top_p in (0, 1]")
+    return out, float(m[0])
+
+
+def accept_block_filtered(target_logits, drafter_logits, block_tokens, temperature, top_k, top_p,
+                          uniforms, nthreads: int = 0, lib=None):
+    """accept_block with top-k / top-p filtering of both distributions (per sequence).
+
+    Returns the accept_block dict plus filter_margin (the smallest top-p margin of the
+    rows a sequence uses); status 3 marks a top_k / top_p outside its range.
+    """
+    lib = lib or _load()
+    tl = np.ascontiguousarray(target_logits)
+    dl = np.ascontiguousarray(drafter_logits)
+    if tl.dtype == np.float32:
+        dtype = 0
+    elif tl.dtype == np.uint16:
+        dtype = 1
+    else:
+        raise TypeError("logits must be float32 or uint16 (bf16 bits)")
+    if dl.dtype != tl.dtype or dl.shape != tl.shape:
+        raise TypeError("target and drafter logits must match in dtype and shape")
+    batch, gamma, vocab = tl.shape
+    bt = _c(block_tokens, np.int32)
+    T = _c(temperature, np.float32)
+    K = _c(np.broadcast_to(np.asarray(top_k, np.int32), (batch,)), np.int32)
+    P = _c(np.broadcast_to(np.asarray(top_p, np.float32), (batch,)), np.float32)
+    u = _c(uniforms, np.float32)
+    na = np.empty(batch, np.int32)
+    ne = np.empty(batch, np.int32)
+    ot = np.empty((batch, gamma + 1), np.int32)
+    diag = np.empty((batch, gamma, 2), np.float64)
+    am = np.empty((batch, gamma), np.float64)
+    sm = np.empty(batch, np.float64)
+    fm = np.empty(batch, np.float64)
+    st = np.empty(batch, np.int32)
+    rc = lib.oracle_accept_block_filtered(batch, gamma, vocab, dtype, _ptr(tl), _ptr(dl), _ptr(bt),
+                                          _ptr(T), _ptr(K), _ptr(P), _ptr(u), _ptr(na), _ptr(ot),
+                                          _ptr(ne), _ptr(diag), _ptr(am), _ptr(sm), _ptr(fm),
+                                          _ptr(st), int(nthreads))
+    if rc:
+        raise ValueError("invalid arguments to oracle_accept_block_filtered")
+    return dict(num_accepted=na, out_tokens=ot, num_emitted=ne, diag=diag,
+                accept_margin=am, sample_margin=sm, filter_margin=fm, status=st)
 
 
 def verify_attention(q, k_cache, v_cache, page_table, kv_len, gamma: int, softmax_scale=None,

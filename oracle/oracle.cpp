@@ -19,6 +19,9 @@
 //   * temperature T > 0: p = softmax(l_target / T), q = softmax(l_drafter / T).
 //     T == 0: greedy verification (accept iff the draft is the argmax of its target
 //     row; correction and bonus are argmaxes; ties go to the lowest token id).
+//   * filtered verification (the top-k / top-p sampling of the paper's evaluations,
+//     Sec. 5.1, Sec. 5.2, Appendix C.1): p and q are replaced by their top-k, then
+//     top-p filtered and renormalised forms p', q' before the same rule.
 //
 // Every floating-point step is fp64 on exactly decoded inputs; sums are plain
 // left-to-right loops. Each function says which passage it follows.
@@ -192,9 +195,10 @@ int oracle_accept_probs(int32_t gamma, int64_t vocab, const double* p_rows,
     const double qv = q_i[t];
     p_tok[i] = pv;
     q_tok[i] = qv;
-    // q_i(t) = 0 cannot happen for a token drawn from q_i; if it does (underflow),
-    // the ratio is +inf and the draft is accepted.
-    const double ratio = (qv > 0.0) ? pv / qv : kInf;
+    // q_i(t) = 0 cannot happen for a token drawn from q_i; if it does (underflow, or a
+    // draft outside a filtered proposal's support), the ratio is +inf and the draft is
+    // accepted when p_i(t) > 0, and 0 (rejected) when p_i(t) = 0 as well.
+    const double ratio = (qv > 0.0) ? pv / qv : (pv > 0.0 ? kInf : 0.0);
     const double thresh = std::min(1.0, ratio);
     accept_margin[i] = std::fabs(uniforms[i - 1] - thresh);
     if (uniforms[i - 1] > thresh) { n = i; break; }
@@ -335,6 +339,142 @@ int oracle_accept_block(int32_t batch, int32_t gamma, int64_t vocab, int32_t dty
       if (accept_margin) accept_margin[row0 + j] = am[j];
     }
     if (sample_margin) sample_margin[b] = sm;
+  });
+  return 0;
+}
+
+// Top-k / top-p filtering of one probability row (the paper decodes with top-k 50
+// and top-p 0.95, Sec. 5.1, Sec. 5.2 and Appendix C.1; the order of the two filters is
+// not stated, and the common one is taken): tokens are ranked by probability, ties
+// to the lower token id; the first top_k are kept; of those, renormalised, the
+// shortest prefix in rank order whose mass reaches top_p is kept; the kept
+// probabilities are renormalised to sum to 1 and every other token gets 0.
+// out[vocab] receives the filtered row. *margin (may be NULL) receives the distance
+// from top_p to the nearer of the two renormalised cumulative masses that bracket
+// the cut (+inf when the cut is set by top_k alone). Returns 0, or 1 if top_k < 1 or
+// top_p is outside (0, 1].
+int oracle_filter_row(const double* p, int64_t vocab, int32_t top_k, double top_p, double* out,
+                      double* margin) {
+  if (top_k < 1 || !(top_p > 0.0) || top_p > 1.0) return 1;
+  std::vector<int64_t> order(static_cast<size_t>(vocab));
+  for (int64_t x = 0; x < vocab; ++x) order[x] = x;
+  std::stable_sort(order.begin(), order.end(),
+                   [&](int64_t a, int64_t b) { return p[a] > p[b]; });
+  const int64_t k = std::min<int64_t>(top_k, vocab);
+  double mass_k = 0.0;
+  for (int64_t j = 0; j < k; ++j) mass_k += p[order[j]];
+  // shortest prefix of the top-k, renormalised, whose mass reaches top_p (top_p = 1
+  // keeps the whole top-k: no rounding of the running sum may cut its tail)
+  int64_t keep = k;
+  double m = kInf, c = 0.0;
+  for (int64_t j = 0; j < k && top_p < 1.0; ++j) {
+    const double before = c;
+    c += p[order[j]] / mass_k;
+    if (c >= top_p) {
+      keep = j + 1;
+      m = std::min(top_p - before, c - top_p);
+      break;
+    }
+  }
+  if (margin) *margin = m;
+  double kept = 0.0;
+  for (int64_t j = 0; j < keep; ++j) kept += p[order[j]];
+  for (int64_t x = 0; x < vocab; ++x) out[x] = 0.0;
+  for (int64_t j = 0; j < keep; ++j) out[order[j]] = p[order[j]] / kept;
+  return 0;
+}
+
+// oracle_accept_block with top-k / top-p filtering of both the target and the drafter
+// distributions (oracle_filter_row with the sequence's top_k[b], top_p[b]) before the
+// decisions and the final draw; greedy sequences (T = 0) are unchanged, since the
+// filter always keeps the argmax. filter_margin[b] (may be NULL) receives the smallest
+// top-p margin over the rows the sequence uses. A top_k or top_p outside its range
+// counts as bad input (status 3).
+int oracle_accept_block_filtered(int32_t batch, int32_t gamma, int64_t vocab, int32_t dtype,
+                                 const void* target_logits, const void* drafter_logits,
+                                 const int32_t* block_tokens, const float* temperature,
+                                 const int32_t* top_k, const float* top_p, const float* uniforms,
+                                 int32_t* num_accepted, int32_t* out_tokens,
+                                 int32_t* num_emitted, double* diag, double* accept_margin,
+                                 double* sample_margin, double* filter_margin, int32_t* status,
+                                 int32_t nthreads) {
+  if (batch < 0 || gamma < 1 || vocab < 1 || (dtype != 0 && dtype != 1)) return -1;
+  parallel_for(batch, nthreads, [&](int64_t b) {
+    const int64_t row0 = b * gamma;
+    const double T = static_cast<double>(temperature[b]);
+    const bool greedy = !(T > 0.0);
+    const int32_t k = top_k[b];
+    const double tp = static_cast<double>(top_p[b]);
+    std::vector<double> p_rows(static_cast<size_t>(gamma) * vocab);
+    std::vector<double> q_rows(greedy ? 0 : static_cast<size_t>(gamma) * vocab);
+    std::vector<double> raw(static_cast<size_t>(vocab)), sm_row(static_cast<size_t>(vocab));
+    int bad = 0, badf = 0;
+    double fm = kInf;
+    if (k < 1 || !(tp > 0.0) || tp > 1.0) badf = 1;
+    for (int32_t j = 0; j < gamma && !bad; ++j) {
+      for (int64_t x = 0; x < vocab; ++x)
+        raw[x] = load_elem(target_logits, dtype, (row0 + j) * vocab + x);
+      if (greedy) {
+        for (int64_t x = 0; x < vocab; ++x) {
+          if (std::isnan(raw[x])) bad = 1;
+          p_rows[j * vocab + x] = raw[x];
+        }
+      } else {
+        bad |= oracle_softmax(raw.data(), vocab, T, sm_row.data());
+        double m = kInf;
+        if (!bad && !badf) {
+          oracle_filter_row(sm_row.data(), vocab, k, tp, &p_rows[j * vocab], &m);
+          fm = std::min(fm, m);
+        }
+      }
+    }
+    if (!greedy) {
+      for (int32_t j = 1; j < gamma && !bad; ++j) {
+        for (int64_t x = 0; x < vocab; ++x)
+          raw[x] = load_elem(drafter_logits, dtype, (row0 + j) * vocab + x);
+        bad |= oracle_softmax(raw.data(), vocab, T, sm_row.data());
+        double m = kInf;
+        if (!bad && !badf) {
+          oracle_filter_row(sm_row.data(), vocab, k, tp, &q_rows[j * vocab], &m);
+          fm = std::min(fm, m);
+        }
+      }
+    }
+    std::vector<double> u(static_cast<size_t>(gamma));
+    for (int32_t j = 0; j < gamma; ++j) u[j] = static_cast<double>(uniforms[row0 + j]);
+    std::vector<double> ptok(gamma), qtok(gamma), am(gamma);
+    double sm = kInf;
+    int32_t n = 0, ne = 0;
+    int32_t* ot = out_tokens + b * (gamma + 1);
+    int rc = 0;
+    for (int32_t j = 0; j < gamma; ++j)
+      if (block_tokens[row0 + j] < 0 || block_tokens[row0 + j] >= vocab) rc = 2;
+    if (rc == 0 && !bad && !(badf && !greedy))
+      rc = oracle_accept_probs(gamma, vocab, p_rows.data(), greedy ? nullptr : q_rows.data(),
+                               block_tokens + row0, u.data(), greedy ? 1 : 0, &n, ot, &ne,
+                               ptok.data(), qtok.data(), am.data(), &sm);
+    const int code = rc ? rc : (bad ? 1 : ((badf && !greedy) ? 3 : 0));
+    if (status) status[b] = code;
+    if (code) {
+      num_accepted[b] = -1;
+      num_emitted[b] = 0;
+      for (int32_t kk = 0; kk <= gamma; ++kk) ot[kk] = -1;
+      for (int32_t j = 0; j < gamma; ++j) { ptok[j] = kNaN; qtok[j] = kNaN; am[j] = kInf; }
+      sm = kInf;
+      fm = kInf;
+    } else {
+      num_accepted[b] = n - 1;
+      num_emitted[b] = ne;
+    }
+    for (int32_t j = 0; j < gamma; ++j) {
+      if (diag) {
+        diag[(row0 + j) * 2 + 0] = ptok[j];
+        diag[(row0 + j) * 2 + 1] = qtok[j];
+      }
+      if (accept_margin) accept_margin[row0 + j] = am[j];
+    }
+    if (sample_margin) sample_margin[b] = sm;
+    if (filter_margin) filter_margin[b] = greedy ? kInf : fm;
   });
   return 0;
 }

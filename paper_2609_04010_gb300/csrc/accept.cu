@@ -438,7 +438,8 @@ __global__ void __launch_bounds__(kDecideThreads) decide_kernel(AcceptParams p) 
       const double pd = exp((lp - static_cast<double>(rM[i - 1])) / Td) / static_cast<double>(rS[i - 1]);
       const double qd = exp((lq - static_cast<double>(rM[gamma + i - 1])) / Td) /
                         static_cast<double>(rS[gamma + i - 1]);
-      const double ratio = qd > 0.0 ? pd / qd : INFINITY;
+      // q_i(t_i) = 0 (underflow): accept iff p_i(t_i) > 0
+      const double ratio = qd > 0.0 ? pd / qd : (pd > 0.0 ? INFINITY : 0.0);
       const double u = static_cast<double>(my_u);
       reject = u > fmin(1.0, ratio);
       pt = static_cast<float>(pd);
