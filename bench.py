@@ -4,7 +4,8 @@ one GB300 (or N independent replicas under torchrun), through the C ABI.
 
 One step = one spec_verify_step call over one batch of synthetic input (attention of
 the gamma block queries over the paged KV cache for one layer, plus the vocabulary-wide
-softmax and acceptance over target and drafter logits). Inputs are resident in HBM;
+softmax and acceptance over target and drafter logits; a workload with top_k > 0 runs
+spec_verify_step_filtered, the top-k / top-p filtered acceptance). Inputs are resident in HBM;
 L2 is flushed before every timed step, outside the timed events: a 256 MiB write, then
 a read of a different 256 MiB buffer, so the step neither hits its inputs in L2 nor pays
 to write back the flush's dirty lines.
@@ -177,17 +178,23 @@ def traffic_model(ai, ci):
 class OracleStep:
     """One verify step of the oracle over the first ``nseq`` sequences of the workload."""
 
-    def __init__(self, ai, ci):
+    def __init__(self, ai, ci, filt=None):
         import oracle
         self.oracle = oracle
-        self.ai, self.ci = ai, ci
+        self.ai, self.ci, self.filt = ai, ci, filt
 
     def run(self, nseq: int):
         ai, ci, o = self.ai, self.ci, self.oracle
         o.verify_attention(ai.q[:nseq], ai.k_cache, ai.v_cache, ai.page_table[:nseq],
                            ai.kv_len[:nseq], ai.gamma)
-        o.accept_block(ci.target_logits[:nseq], ci.drafter_logits[:nseq],
-                       ci.block_tokens[:nseq], ci.temperature[:nseq], ci.uniforms[:nseq])
+        if self.filt is not None:
+            k, p = self.filt
+            o.accept_block_filtered(ci.target_logits[:nseq], ci.drafter_logits[:nseq],
+                                    ci.block_tokens[:nseq], ci.temperature[:nseq], k[:nseq],
+                                    p[:nseq], ci.uniforms[:nseq])
+        else:
+            o.accept_block(ci.target_logits[:nseq], ci.drafter_logits[:nseq],
+                           ci.block_tokens[:nseq], ci.temperature[:nseq], ci.uniforms[:nseq])
 
     def calibrate(self, budget_s: float):
         """Sequences per step so that one step takes at most about budget_s."""
@@ -197,9 +204,9 @@ class OracleStep:
         return int(max(1, min(self.ci.batch, budget_s // t1))), t1
 
 
-def cpu_baseline(ai, ci, seconds: float):
+def cpu_baseline(ai, ci, seconds: float, filt=None):
     import oracle
-    st = OracleStep(ai, ci)
+    st = OracleStep(ai, ci, filt)
     nseq, _ = st.calibrate(max(0.5, seconds / 4))
     tokens, elapsed, steps = 0, 0.0, 0
     while elapsed < seconds or steps == 0:
@@ -217,7 +224,7 @@ def cpu_baseline(ai, ci, seconds: float):
 
 def reference_arm(args, wl, ai, ci):
     import oracle
-    st = OracleStep(ai, ci)
+    st = OracleStep(ai, ci, wl.filter_params() if wl.top_k > 0 else None)
     nseq, _ = st.calibrate(1.0)
     for _ in range(args.warmup):
         st.run(nseq)
@@ -298,6 +305,10 @@ def run_ours(args, wl, ai, ci, rank, world, local_rank):
                    tl=bf16(ci.target_logits) if ci.is_bf16 else t(ci.target_logits),
                    dl=bf16(ci.drafter_logits) if ci.is_bf16 else t(ci.drafter_logits),
                    tok=t(ci.block_tokens), temp=t(ci.temperature), u=t(ci.uniforms))
+    filtered = wl.top_k > 0
+    if filtered:
+        fk, fp = wl.filter_params()
+        host_in.update(topk=t(fk), topp=t(fp))
     d = {k: v.to(dev) for k, v in host_in.items()}
     B, G = ci.batch, ci.gamma
     out = torch.empty_like(d["q"])
@@ -309,7 +320,11 @@ def run_ours(args, wl, ai, ci, rank, world, local_rank):
             "tensor-cores": binding.ATTN_TENSOR_CORES}[args.attn_path]
     a = binding.attn_args(d["q"], d["k"], d["v"], d["pt"], d["kvl"], out, lse, path=path)
     c = binding.accept_args(d["tl"], d["dl"], d["tok"], d["temp"], d["u"], na, ot, ne, None)
-    ws = binding.new_workspace(binding.workspace_size(a, c), dev)
+    if filtered:
+        f = binding.filter_args(d["topk"], d["topp"], B, max_top_k=wl.top_k)
+        ws = binding.new_workspace(binding.filtered_workspace_size(c, f, a), dev)
+    else:
+        ws = binding.new_workspace(binding.workspace_size(a, c), dev)
     flush_w = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
     flush_r = torch.ones(L2_FLUSH_BYTES // 4, dtype=torch.int32, device=dev)
     flush_sink = torch.empty(1, dtype=torch.int64, device=dev)
@@ -330,9 +345,13 @@ def run_ours(args, wl, ai, ci, rank, world, local_rank):
         torch.cuda.synchronize()
         return [s.elapsed_time(e) for s, e in evs]
 
-    step = lambda: binding.verify_step_args(a, c, ws)
+    if filtered:
+        step = lambda: binding.verify_step_filtered_args(a, c, f, ws)
+        acc_only = lambda: binding.verify_step_filtered_args(None, c, f, ws)
+    else:
+        step = lambda: binding.verify_step_args(a, c, ws)
+        acc_only = lambda: binding.verify_step_args(None, c, ws)
     attn_only = lambda: binding.verify_step_args(a, None, ws)
-    acc_only = lambda: binding.verify_step_args(None, c, ws)
 
     # Device-timed loops replay CUDA graphs of the same C-ABI calls, so that the events
     # bracket GPU work only (the host's launch latency stays outside the timed region;
@@ -425,7 +444,9 @@ def run_ours(args, wl, ai, ci, rank, world, local_rank):
     dom_bytes = tm["kv"] if dominant == "attention" else tm["logits"]
     dom_ms = attn_ms if dominant == "attention" else acc_ms
     dom_gbs = dom_bytes / (dom_ms / 1000.0) / 1e9
-    launches_per_step = 4  # attention, row statistics, decisions, draws
+    # attention, then row statistics, decisions, draws (filtered: lane maxima, top-k /
+    # top-p select, decisions and draw)
+    launches_per_step = 4
     traffic, traffic_src = (None, None)
     if dominant == "attention" and attn_path_name(args.attn_path, binding, ai) == "tensor cores":
         traffic, traffic_src = measured_traffic(args.workload, "attention")
@@ -436,7 +457,9 @@ def run_ours(args, wl, ai, ci, rank, world, local_rank):
         "data": "synthetic (seeded; no weights or datasets)",
         "config": dict(wl.describe(), parallelism=f"replicas x{world}",
                        l2="flushed before every timed step (256 MiB write + 256 MiB read, outside events)",
-                       timing="device: CUDA events around a CUDA-graph replay of one spec_verify_step call per step",
+                       timing="device: CUDA events around a CUDA-graph replay of one "
+                              + ("spec_verify_step_filtered" if filtered else "spec_verify_step")
+                              + " call per step",
                        attention_path=attn_path_name(args.attn_path, binding, ai)),
         "roofline": {"bound": "hbm", "kernel": dominant, "achieved": round(dom_gbs, 1),
                      "peak": peak, "unit": "GB/s", "frac": round(dom_gbs / peak, 4),
@@ -484,7 +507,8 @@ def main():
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         import oracle
         oracle.build()
-        res["cpu_baseline"] = cpu_baseline(ai, ci, args.cpu_seconds)
+        res["cpu_baseline"] = cpu_baseline(ai, ci, args.cpu_seconds,
+                                           wl.filter_params() if wl.top_k > 0 else None)
     if rank == 0:
         print(json.dumps(res), flush=True)
     if world > 1:

@@ -75,6 +75,7 @@ typedef enum {
 #define SPEC_FLAG_BAD_PAGE 0x4u    /* a page id of a visible key outside [0, num_pages)      */
 #define SPEC_FLAG_BAD_KV_LEN 0x8u  /* kv_len outside [gamma, max_pages_per_seq * page_size] */
 #define SPEC_FLAG_TIMEOUT 0x10u    /* a bounded internal wait ran out                        */
+#define SPEC_FLAG_BAD_FILTER 0x20u /* a tempered sequence's top_k or top_p out of range       */
 
 /*
  * Part (a): block-causal verify attention (Sec. 4.1: the block [x^{L+1}, z] is
@@ -186,6 +187,58 @@ const char* spec_status_string(spec_status_t status);
 
 /* The (Hq/Hkv)*gamma at and above which SPEC_ATTN_AUTO picks the tensor-core kernel. */
 int32_t spec_attn_tensor_core_min_rows(void);
+
+/*
+ * Filtered acceptance: spec_accept_block with top-k / top-p filtering of both
+ * distributions, the sampling of the paper's evaluations (top-k 50 and top-p 0.95 for
+ * drafting and verification: Sec. 5.1, Sec. 5.2, Appendix C.1).
+ *
+ * For a tempered sequence b (temperature[b] > 0), every target row and every used
+ * drafter row is replaced by its filtered form before the rule: rank the tokens by
+ * logit, equal logits by lower token id; keep the first k = min(top_k[b], vocab);
+ * of those, keep the shortest rank-order prefix whose mass under their renormalised
+ * distribution reaches top_p[b] (top_p = 1 keeps all k); renormalise over the kept
+ * tokens; every other token has probability 0. The rule of spec_accept_block then runs
+ * on the filtered p' and q', with one addition: a draft with q'_i(t_i) = 0 (outside
+ * the filtered proposal) is accepted iff p'_i(t_i) > 0. The final draw is over the
+ * kept tokens of p'_n in ascending token order. Drafts should be drawn from q' for
+ * the output to follow the filtered target exactly. Greedy sequences (T = 0) are
+ * verified as by spec_accept_block; their top_k / top_p are not read.
+ *   - accept: as spec_accept_block (same layouts, outputs and sentinels); diag holds
+ *     (p'_i(t_i), q'_i(t_i)).
+ *   - filter->top_k: int32 [batch], device; 1 <= top_k[b] <= filter->max_top_k.
+ *   - filter->top_p: fp32 [batch], device; 0 < top_p[b] <= 1.
+ *   - filter->max_top_k: host bound on top_k, 1 .. SPEC_FILTER_MAX_TOP_K; it sizes
+ *     the workspace (spec_filtered_workspace_size).
+ *   - A tempered sequence whose top_k or top_p is out of range sets
+ *     SPEC_FLAG_BAD_FILTER and gets the sentinel outputs; other sequences are unaffected.
+ *   - Precision: the filter and the decisions are evaluated in fp64 on the logits
+ *     (z = l / T); ranking uses the logits themselves, so it is exact.
+ *   - The workspace needs no zero state beyond the status word.
+ */
+#define SPEC_FILTER_MAX_TOP_K 1024
+typedef struct {
+  const int32_t* top_k;  /* [batch]                                                   */
+  const float* top_p;    /* [batch]                                                   */
+  int32_t max_top_k;     /* 1 .. SPEC_FILTER_MAX_TOP_K                                */
+} spec_filter_args_t;
+
+/* Bytes of workspace the filtered calls below need (attn may be NULL; 0 if an
+ * argument is invalid). */
+size_t spec_filtered_workspace_size(const spec_attn_args_t* attn, const spec_accept_args_t* accept,
+                                    const spec_filter_args_t* filter);
+
+/* Part (b) with filtering. */
+spec_status_t spec_accept_block_filtered(const spec_accept_args_t* accept,
+                                         const spec_filter_args_t* filter, void* ws,
+                                         size_t ws_bytes, spec_stream_t stream);
+
+/* The whole verify step with filtering: part (a) (attn may be NULL) and the filtered
+ * part (b) on one stream, as spec_verify_step. */
+spec_status_t spec_verify_step_filtered(const spec_attn_args_t* attn,
+                                        const spec_accept_args_t* accept,
+                                        const spec_filter_args_t* filter, void* ws,
+                                        size_t ws_bytes, spec_stream_t stream);
 
 /*
  * spec_accept_block without a workspace, for callers that cannot allocate device

@@ -28,6 +28,8 @@ STATUS_NAMES = {0: "SPEC_OK", 1: "SPEC_ERR_INVALID_ARGUMENT", 2: "SPEC_ERR_UNSUP
 SPEC_F32, SPEC_BF16 = 0, 1
 ATTN_AUTO, ATTN_CUDA_CORES, ATTN_TENSOR_CORES = 0, 1, 2
 FLAG_BAD_TOKEN, FLAG_BAD_LOGITS, FLAG_BAD_PAGE, FLAG_BAD_KV_LEN, FLAG_TIMEOUT = 1, 2, 4, 8, 16
+FLAG_BAD_FILTER = 32
+FILTER_MAX_TOP_K = 1024
 
 
 class SpecError(RuntimeError):
@@ -54,6 +56,11 @@ class AcceptArgs(ctypes.Structure):
                 ("temperature", ctypes.c_void_p), ("uniforms", ctypes.c_void_p),
                 ("num_accepted", ctypes.c_void_p), ("out_tokens", ctypes.c_void_p),
                 ("num_emitted", ctypes.c_void_p), ("diag", ctypes.c_void_p)]
+
+
+class FilterArgs(ctypes.Structure):
+    _fields_ = [("top_k", ctypes.c_void_p), ("top_p", ctypes.c_void_p),
+                ("max_top_k", ctypes.c_int32)]
 
 
 HEADER = os.path.join(_build.ROOT, "include", "spec_verify.h")
@@ -90,6 +97,12 @@ def lib(build_if_missing: bool = True):
             L.spec_attn_tensor_core_min_rows.restype = i32
             L.spec_accept_block_noalloc.argtypes = [P, P]
             L.spec_accept_block_noalloc.restype = ctypes.c_int
+            L.spec_filtered_workspace_size.argtypes = [P, P, P]
+            L.spec_filtered_workspace_size.restype = ctypes.c_size_t
+            L.spec_accept_block_filtered.argtypes = [P, P, P, ctypes.c_size_t, P]
+            L.spec_accept_block_filtered.restype = ctypes.c_int
+            L.spec_verify_step_filtered.argtypes = [P, P, P, P, ctypes.c_size_t, P]
+            L.spec_verify_step_filtered.restype = ctypes.c_int
             for f in ("spec_workspace_init", "spec_verify_attention", "spec_accept_block",
                       "spec_verify_step", "spec_philox_uniforms", "spec_read_device_status"):
                 getattr(L, f).restype = ctypes.c_int
@@ -235,6 +248,61 @@ def accept_block_noalloc(target_logits, drafter_logits, block_tokens, temperatur
                     num_accepted, out_tokens, num_emitted, diag)
     _raise(lib().spec_accept_block_noalloc(ctypes.byref(a), _stream(stream)),
            "spec_accept_block_noalloc")
+
+
+def filter_args(top_k, top_p, batch: int, max_top_k: Optional[int] = None) -> FilterArgs:
+    """spec_filter_args_t over int32 top_k [batch] and fp32 top_p [batch] device tensors.
+
+    max_top_k defaults to FILTER_MAX_TOP_K (it sizes the workspace)."""
+    _check(top_k, "top_k", torch.int32, (batch,))
+    _check(top_p, "top_p", torch.float32, (batch,))
+    return FilterArgs(top_k.data_ptr(), top_p.data_ptr(),
+                      int(FILTER_MAX_TOP_K if max_top_k is None else max_top_k))
+
+
+def filtered_workspace_size(accept: AcceptArgs, filt: FilterArgs,
+                            attn: Optional[AttnArgs] = None) -> int:
+    n = lib().spec_filtered_workspace_size(None if attn is None else ctypes.byref(attn),
+                                           ctypes.byref(accept), ctypes.byref(filt))
+    if n == 0:
+        raise SpecError(1, "spec_filtered_workspace_size")
+    return int(n)
+
+
+def verify_step_filtered_args(attn: Optional[AttnArgs], acc: AcceptArgs, filt: FilterArgs,
+                              ws: torch.Tensor, stream=None):
+    _raise(lib().spec_verify_step_filtered(None if attn is None else ctypes.byref(attn),
+                                           ctypes.byref(acc), ctypes.byref(filt), _ptr(ws),
+                                           ws.numel(), _stream(stream)),
+           "spec_verify_step_filtered")
+
+
+def accept_block_filtered_args(acc: AcceptArgs, filt: FilterArgs, ws: torch.Tensor, stream=None):
+    _raise(lib().spec_accept_block_filtered(ctypes.byref(acc), ctypes.byref(filt), _ptr(ws),
+                                            ws.numel(), _stream(stream)),
+           "spec_accept_block_filtered")
+
+
+def accept_block_filtered(target_logits, drafter_logits, block_tokens, temperature, top_k, top_p,
+                          uniforms, max_top_k: Optional[int] = None, want_diag=True, ws=None,
+                          stream=None) -> Dict[str, torch.Tensor]:
+    """Top-k / top-p filtered lossless acceptance over a batch (spec_accept_block_filtered).
+
+    top_k: int32 [batch], top_p: fp32 [batch] device tensors. Returns num_accepted,
+    out_tokens, num_emitted, diag."""
+    B, G, _ = target_logits.shape
+    dev = target_logits.device
+    res = dict(num_accepted=torch.empty(B, dtype=torch.int32, device=dev),
+               out_tokens=torch.empty(B, G + 1, dtype=torch.int32, device=dev),
+               num_emitted=torch.empty(B, dtype=torch.int32, device=dev),
+               diag=torch.empty(B, G, 2, dtype=torch.float32, device=dev) if want_diag else None)
+    a = accept_args(target_logits, drafter_logits, block_tokens, temperature, uniforms,
+                    res["num_accepted"], res["out_tokens"], res["num_emitted"], res["diag"])
+    f = filter_args(top_k, top_p, B, max_top_k)
+    if ws is None:
+        ws = new_workspace(filtered_workspace_size(a, f), dev)
+    accept_block_filtered_args(a, f, ws, stream)
+    return res
 
 
 def philox_uniforms(seed: int, n: int, offset: int = 0, device=None, stream=None) -> torch.Tensor:

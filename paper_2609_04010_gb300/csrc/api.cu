@@ -90,6 +90,13 @@ spec_status_t check_accept(const spec_accept_args_t* a) {
   return SPEC_OK;
 }
 
+spec_status_t check_filter(const spec_filter_args_t* f) {
+  if (!f || !f->top_k || !f->top_p) return SPEC_ERR_INVALID_ARGUMENT;
+  if (f->max_top_k < 1) return SPEC_ERR_INVALID_ARGUMENT;
+  if (f->max_top_k > SPEC_FILTER_MAX_TOP_K) return SPEC_ERR_UNSUPPORTED;
+  return SPEC_OK;
+}
+
 }  // namespace
 
 AttnPlan attn_plan(const spec_attn_args_t& a, size_t base, int num_sms, int path_override) {
@@ -153,19 +160,26 @@ size_t attn_region(const spec_attn_args_t& a, size_t base, int sms) {
   return end;
 }
 
-size_t required_bytes(const spec_attn_args_t* attn, const spec_accept_args_t* accept, int sms,
-                      size_t* attn_base) {
+size_t required_bytes(const spec_attn_args_t* attn, const spec_accept_args_t* accept,
+                      const spec_filter_args_t* filter, int sms, size_t* attn_base) {
   size_t end = kWsHeader;
-  if (accept) end = accept_layout(*accept, kWsHeader).end;
+  if (accept)
+    end = filter ? filter_layout(*accept, filter->max_top_k, kWsHeader).end
+                 : accept_layout(*accept, kWsHeader).end;
   if (attn_base) *attn_base = end;
   if (attn) end = attn_region(*attn, end, sms);
   return end;
 }
 
-spec_status_t run(const spec_attn_args_t* attn, const spec_accept_args_t* accept, void* ws,
-                  size_t ws_bytes, spec_stream_t stream_) {
+spec_status_t run(const spec_attn_args_t* attn, const spec_accept_args_t* accept,
+                  const spec_filter_args_t* filter, void* ws, size_t ws_bytes,
+                  spec_stream_t stream_) {
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
   if (!attn && !accept) return SPEC_ERR_INVALID_ARGUMENT;
+  if (filter) {
+    const spec_status_t s = check_filter(filter);
+    if (s != SPEC_OK) return s;
+  }
   if (attn) {
     const spec_status_t s = check_attn(attn);
     if (s != SPEC_OK) return s;
@@ -175,11 +189,15 @@ spec_status_t run(const spec_attn_args_t* attn, const spec_accept_args_t* accept
     if (s != SPEC_OK) return s;
   }
   if (!ws || (reinterpret_cast<uintptr_t>(ws) % kWsAlign) != 0) return SPEC_ERR_INVALID_ARGUMENT;
+  // without attention the size does not depend on the device: check it on the host
+  if (!attn && required_bytes(nullptr, accept, filter, 0, nullptr) > ws_bytes)
+    return SPEC_ERR_WORKSPACE_TOO_SMALL;
   int sms = 0;
   if (!bind_device(stream, &sms)) return SPEC_ERR_CUDA;
   (void)cudaGetLastError();  // a failed call before this one must not fail our launches
   size_t attn_base = 0;
-  if (required_bytes(attn, accept, sms, &attn_base) > ws_bytes) return SPEC_ERR_WORKSPACE_TOO_SMALL;
+  if (required_bytes(attn, accept, filter, sms, &attn_base) > ws_bytes)
+    return SPEC_ERR_WORKSPACE_TOO_SMALL;
   char* w = static_cast<char*>(ws);
   // Attention first; the acceptance kernels follow as programmatic dependents, so they
   // start on the SM resources the attention kernel leaves free and the two parts
@@ -190,20 +208,22 @@ spec_status_t run(const spec_attn_args_t* attn, const spec_accept_args_t* accept
                                                            : launch_attn_simt(*attn, P, w, stream);
     if (e != cudaSuccess) return SPEC_ERR_CUDA;
   }
-  if (accept) {
+  if (accept && filter) {
+    const FilterLayout L = filter_layout(*accept, filter->max_top_k, kWsHeader);
+    if (launch_accept_filtered(*accept, *filter, L, w, stream, attn != nullptr) != cudaSuccess)
+      return SPEC_ERR_CUDA;
+  } else if (accept) {
     const AcceptLayout L = accept_layout(*accept, kWsHeader);
     if (launch_accept(*accept, L, w, sms, stream, attn != nullptr) != cudaSuccess) return SPEC_ERR_CUDA;
   }
   return SPEC_OK;
 }
 
-}  // namespace
-
-extern "C" {
-
-size_t spec_workspace_size(const spec_attn_args_t* attn, const spec_accept_args_t* accept) {
+size_t workspace_bytes(const spec_attn_args_t* attn, const spec_accept_args_t* accept,
+                       const spec_filter_args_t* filter) {
   if (attn && check_attn(attn) != SPEC_OK) return 0;
   if (accept && check_accept(accept) != SPEC_OK) return 0;
+  if (filter && (!accept || check_filter(filter) != SPEC_OK)) return 0;
   // The split count depends on the SM count; size for the larger of the current
   // device's and a 160-SM part so that a workspace fits every device it may meet.
   int dev = 0, sms = 160;
@@ -213,12 +233,20 @@ size_t spec_workspace_size(const spec_attn_args_t* attn, const spec_accept_args_
   } else {
     cudaGetLastError();
   }
-  size_t need = required_bytes(attn, accept, sms, nullptr);
+  size_t need = required_bytes(attn, accept, filter, sms, nullptr);
   for (int s : {148, 152, sms}) {
-    const size_t x = required_bytes(attn, accept, s, nullptr);
+    const size_t x = required_bytes(attn, accept, filter, s, nullptr);
     if (x > need) need = x;
   }
   return need;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t spec_workspace_size(const spec_attn_args_t* attn, const spec_accept_args_t* accept) {
+  return workspace_bytes(attn, accept, nullptr);
 }
 
 spec_status_t spec_workspace_init(void* ws, size_t ws_bytes, spec_stream_t stream) {
@@ -231,18 +259,39 @@ spec_status_t spec_workspace_init(void* ws, size_t ws_bytes, spec_stream_t strea
 spec_status_t spec_verify_attention(const spec_attn_args_t* attn, void* ws, size_t ws_bytes,
                                     spec_stream_t stream) {
   if (!attn) return SPEC_ERR_INVALID_ARGUMENT;
-  return run(attn, nullptr, ws, ws_bytes, stream);
+  return run(attn, nullptr, nullptr, ws, ws_bytes, stream);
 }
 
 spec_status_t spec_accept_block(const spec_accept_args_t* accept, void* ws, size_t ws_bytes,
                                 spec_stream_t stream) {
   if (!accept) return SPEC_ERR_INVALID_ARGUMENT;
-  return run(nullptr, accept, ws, ws_bytes, stream);
+  return run(nullptr, accept, nullptr, ws, ws_bytes, stream);
 }
 
 spec_status_t spec_verify_step(const spec_attn_args_t* attn, const spec_accept_args_t* accept,
                                void* ws, size_t ws_bytes, spec_stream_t stream) {
-  return run(attn, accept, ws, ws_bytes, stream);
+  return run(attn, accept, nullptr, ws, ws_bytes, stream);
+}
+
+size_t spec_filtered_workspace_size(const spec_attn_args_t* attn, const spec_accept_args_t* accept,
+                                    const spec_filter_args_t* filter) {
+  if (!accept || !filter) return 0;
+  return workspace_bytes(attn, accept, filter);
+}
+
+spec_status_t spec_accept_block_filtered(const spec_accept_args_t* accept,
+                                         const spec_filter_args_t* filter, void* ws,
+                                         size_t ws_bytes, spec_stream_t stream) {
+  if (!accept || !filter) return SPEC_ERR_INVALID_ARGUMENT;
+  return run(nullptr, accept, filter, ws, ws_bytes, stream);
+}
+
+spec_status_t spec_verify_step_filtered(const spec_attn_args_t* attn,
+                                        const spec_accept_args_t* accept,
+                                        const spec_filter_args_t* filter, void* ws,
+                                        size_t ws_bytes, spec_stream_t stream) {
+  if (!accept || !filter) return SPEC_ERR_INVALID_ARGUMENT;
+  return run(attn, accept, filter, ws, ws_bytes, stream);
 }
 
 spec_status_t spec_philox_uniforms(uint64_t seed, uint64_t offset, int64_t n, float* out_dev,

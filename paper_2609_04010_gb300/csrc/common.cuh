@@ -45,6 +45,27 @@ struct AcceptLayout {
 
 AcceptLayout accept_layout(const spec_accept_args_t& a, size_t base);
 
+// --- filtered acceptance ---
+constexpr int kFilterMaxTopK = SPEC_FILTER_MAX_TOP_K;
+
+struct FiltRow {    // one (sequence, row) result of the filtered select kernel
+  int32_t nkeep;    // kept tokens (top-k, then top-p)
+  int32_t argmax;   // lowest index of the row maximum
+  uint32_t flags;   // 1: NaN / +inf / no finite logit; 2: top_k or top_p out of range
+  int32_t pad;
+};
+
+struct FilterLayout {
+  size_t lanes;  // uint64 [batch][2*gamma-1][nchunk*32]: lane maxima (order keys)
+  size_t rows;   // FiltRow [batch][2*gamma-1]
+  size_t ids;    // int32 [batch][2*gamma-1][max_top_k]: kept tokens, rank order
+  size_t probs;  // fp64, same layout: their filtered probabilities
+  size_t end;
+  int nchunk, nlanes;
+};
+
+FilterLayout filter_layout(const spec_accept_args_t& a, int max_top_k, size_t base);
+
 // --- attention ---
 struct AttnPlan {
   int path;          // SPEC_ATTN_CUDA_CORES or SPEC_ATTN_TENSOR_CORES
@@ -71,6 +92,9 @@ AttnPlan attn_plan(const spec_attn_args_t& a, size_t base, int num_sms, int path
 // reads none of their inputs and writes none of their outputs).
 cudaError_t launch_accept(const spec_accept_args_t& a, const AcceptLayout& L, char* ws,
                           int num_sms, cudaStream_t stream, bool overlap_prior = false);
+cudaError_t launch_accept_filtered(const spec_accept_args_t& a, const spec_filter_args_t& f,
+                                   const FilterLayout& L, char* ws, cudaStream_t stream,
+                                   bool overlap_prior = false);
 cudaError_t launch_attn_simt(const spec_attn_args_t& a, const AttnPlan& P, char* ws,
                              cudaStream_t stream);
 cudaError_t launch_attn_tc(const spec_attn_args_t& a, const AttnPlan& P, char* ws,

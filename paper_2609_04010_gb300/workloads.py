@@ -142,24 +142,32 @@ class AcceptInputs:
         return self.target_logits.dtype == np.uint16
 
 
-def _gumbel_argmax(rng: np.random.Generator, logits_f32: np.ndarray, T: float) -> int:
+def _gumbel_argmax(rng: np.random.Generator, logits_f32: np.ndarray, T: float,
+                   top_k: int = 0) -> int:
     if not T > 0.0:
         return int(np.argmax(logits_f32))
     u = rng.random(logits_f32.shape[0])
     g = -np.log(-np.log(np.maximum(u, 1e-300)))
-    return int(np.argmax(logits_f32.astype(np.float64) / T + g))
+    score = logits_f32.astype(np.float64) / T + g
+    if top_k > 0 and top_k < logits_f32.shape[0]:
+        # only the top_k largest logits (equal logits by lower id) can be drawn
+        order = np.argsort(-logits_f32, kind="stable")
+        score[order[top_k:]] = -np.inf
+    return int(np.argmax(score))
 
 
 def make_accept_inputs(batch: int, gamma: int, vocab: int, logits_dtype: str = "bf16",
                        target_sigma: float = 3.0, drafter_sigma: float = 1.0,
-                       temperature=1.0, seed: int = 0) -> AcceptInputs:
+                       temperature=1.0, seed: int = 0, draft_top_k: int = 0) -> AcceptInputs:
     """Synthetic logits for the acceptance rule.
 
     Target row j ~ N(0, target_sigma^2) per element.  Drafter row j (j >= 1) is target
     row j-1 plus N(0, drafter_sigma^2) noise (drafter row j proposes block token j,
     whose verifier distribution is target row j-1); drafter row 0 is independent.
     Rows are rounded to bf16 when ``logits_dtype == "bf16"``.  Block token j is drawn
-    from drafter row j at the sequence's temperature (argmax at T = 0).
+    from drafter row j at the sequence's temperature (argmax at T = 0); with
+    ``draft_top_k`` > 0, only among that row's draft_top_k largest logits (the support
+    of a top-k filtered proposal).
     ``temperature`` is a scalar or a sequence cycled over the batch.
     """
     temps = np.resize(np.asarray(temperature, dtype=np.float32).ravel(), batch)
@@ -187,7 +195,7 @@ def make_accept_inputs(batch: int, gamma: int, vocab: int, logits_dtype: str = "
             dl[b] = d32
             dseen = d32
         for j in range(gamma):
-            tokens[b, j] = _gumbel_argmax(rng_s, dseen[j], float(temps[b]))
+            tokens[b, j] = _gumbel_argmax(rng_s, dseen[j], float(temps[b]), draft_top_k)
     u = philox_uniforms(uniform_seed(seed), batch * gamma).reshape(batch, gamma)
     return AcceptInputs(tl, dl, tokens, temps, u)
 
@@ -300,6 +308,8 @@ class Workload:
     ctx: object                      # int or (lo, hi)
     permute_pages: bool = True
     note: str = ""
+    top_k: int = 0        # > 0: top-k / top-p filtered verification (drafts from the top-k)
+    top_p: float = 1.0
 
     def temps(self) -> np.ndarray:
         t = np.asarray(self.temperatures, dtype=np.float32)
@@ -307,17 +317,26 @@ class Workload:
 
     def accept_inputs(self, seed: int = 0) -> AcceptInputs:
         return make_accept_inputs(self.batch, self.gamma, self.vocab, self.logits_dtype,
-                                  self.target_sigma, self.drafter_sigma, self.temps(), seed)
+                                  self.target_sigma, self.drafter_sigma, self.temps(), seed,
+                                  draft_top_k=self.top_k)
+
+    def filter_params(self):
+        """(top_k [batch] int32, top_p [batch] float32) of a filtered workload."""
+        return (np.full(self.batch, self.top_k, np.int32),
+                np.full(self.batch, self.top_p, np.float32))
 
     def attn_inputs(self, seed: int = 0) -> AttnInputs:
         return make_attn_inputs(self.batch, self.gamma, self.num_q_heads, self.num_kv_heads,
                                 self.head_dim, self.page_size, self.ctx, self.permute_pages, seed)
 
     def describe(self) -> Dict[str, object]:
-        return dict(workload=self.name, batch=self.batch, gamma=self.gamma, vocab=self.vocab,
-                    logits_dtype=self.logits_dtype, num_q_heads=self.num_q_heads,
-                    num_kv_heads=self.num_kv_heads, head_dim=self.head_dim,
-                    page_size=self.page_size, ctx=self.ctx)
+        d = dict(workload=self.name, batch=self.batch, gamma=self.gamma, vocab=self.vocab,
+                 logits_dtype=self.logits_dtype, num_q_heads=self.num_q_heads,
+                 num_kv_heads=self.num_kv_heads, head_dim=self.head_dim,
+                 page_size=self.page_size, ctx=self.ctx)
+        if self.top_k > 0:
+            d.update(top_k=self.top_k, top_p=self.top_p)
+        return d
 
 
 WORKLOADS: Dict[str, Workload] = {
@@ -334,6 +353,12 @@ WORKLOADS: Dict[str, Workload] = {
     # 70B-shaped long context: batch 4, gamma 32, 64/8 heads, context 32,768 in 64-token
     # pages, T = 0.7.
     "long70b": Workload("long70b", 4, 32, 128256, "bf16", 3.0, 1.0, (0.7,), 64, 8, 128, 64, 32768),
+    # the paper's evaluation sampling (T = 1, top-k 50, top-p 0.95) on the Llama-3-8B
+    # shape and on the high-batch serving shape (all sequences tempered)
+    "llama8b_topk": Workload("llama8b_topk", 8, 8, 128256, "bf16", 3.0, 1.0, (1.0,), 32, 8, 128,
+                             16, 4096, top_k=50, top_p=0.95),
+    "serve64_topk": Workload("serve64_topk", 64, 16, 128256, "bf16", 3.0, 0.5, (1.0,), 32, 8, 128,
+                             16, (512, 4096), top_k=50, top_p=0.95),
 }
 
 SWEEP_GAMMAS = (1, 2, 4, 8, 16, 32)

@@ -59,13 +59,16 @@ def gpu_attention(inp, path=0, ws=None):
     return out.float().cpu().numpy(), lse.cpu().numpy()
 
 
-def compare_accept(g, o, gamma):
-    """Compares GPU and oracle acceptance outputs; returns (ties, report).
+def compare_accept(g, o, gamma, skip=()):
+    """Compares GPU and oracle acceptance outputs; returns the list of ties.
 
-    Raises AssertionError on any mismatch that is not a tie."""
+    Sequences in ``skip`` are not compared. Raises AssertionError on any mismatch that
+    is not a tie."""
     B = len(o["num_accepted"])
     ties = []
     for b in range(B):
+        if b in skip:
+            continue
         if o["status"][b] != 0:
             assert g["num_accepted"][b] == -1 and g["num_emitted"][b] == 0, b
             assert np.all(g["out_tokens"][b] == -1), b

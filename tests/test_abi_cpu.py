@@ -88,3 +88,49 @@ def test_misaligned_workspace_rejected(lib):
     a = _attn()
     assert lib.spec_verify_attention(ctypes.byref(a), ctypes.c_void_p(4096 + 16), 1 << 30,
                                      None) == 1
+
+
+def _accept(**kw):
+    base = dict(batch=4, gamma=8, vocab=128256, logits_dtype=1)
+    base.update(kw)
+    acc = binding.AcceptArgs(**base)
+    for f in ("target_logits", "drafter_logits", "block_tokens", "temperature", "uniforms",
+              "num_accepted", "out_tokens", "num_emitted"):
+        setattr(acc, f, 4096)
+    return acc
+
+
+@pytest.mark.parametrize("max_top_k,code", [(0, 1), (-5, 1), (1025, 2), (1 << 20, 2)])
+def test_filter_host_checks(lib, max_top_k, code):
+    acc = _accept()
+    f = binding.FilterArgs(4096, 4096, max_top_k)
+    assert lib.spec_accept_block_filtered(ctypes.byref(acc), ctypes.byref(f),
+                                          ctypes.c_void_p(4096), 1 << 30, None) == code
+    assert lib.spec_filtered_workspace_size(None, ctypes.byref(acc), ctypes.byref(f)) == 0
+
+
+def test_filter_null_arguments(lib):
+    acc = _accept()
+    f = binding.FilterArgs(4096, None, 50)
+    assert lib.spec_accept_block_filtered(ctypes.byref(acc), None, ctypes.c_void_p(4096),
+                                          1 << 30, None) == 1
+    assert lib.spec_accept_block_filtered(ctypes.byref(acc), ctypes.byref(f),
+                                          ctypes.c_void_p(4096), 1 << 30, None) == 1
+    assert lib.spec_verify_step_filtered(None, None, None, None, 0, None) == 1
+
+
+def test_filtered_workspace_size_and_too_small(lib):
+    acc = _accept()
+    f50 = binding.FilterArgs(4096, 4096, 50)
+    f1k = binding.FilterArgs(4096, 4096, 1024)
+    n50 = lib.spec_filtered_workspace_size(None, ctypes.byref(acc), ctypes.byref(f50))
+    n1k = lib.spec_filtered_workspace_size(None, ctypes.byref(acc), ctypes.byref(f1k))
+    assert 0 < n50 < n1k and n50 % 256 == 0
+    # rows x max_top_k x (4-byte id + 8-byte probability) separates the two sizes
+    rows = 4 * (2 * 8 - 1)
+    assert n1k - n50 >= rows * (1024 - 50) * 12 - 1024
+    both = lib.spec_filtered_workspace_size(ctypes.byref(_attn()), ctypes.byref(acc),
+                                            ctypes.byref(f50))
+    assert both > n50
+    assert lib.spec_accept_block_filtered(ctypes.byref(acc), ctypes.byref(f50),
+                                          ctypes.c_void_p(4096), n50 - 256, None) == 3
