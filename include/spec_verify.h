@@ -214,7 +214,8 @@ int32_t spec_attn_tensor_core_min_rows(void);
  *     SPEC_FLAG_BAD_FILTER and gets the sentinel outputs; other sequences are unaffected.
  *   - Precision: the filter and the decisions are evaluated in fp64 on the logits
  *     (z = l / T); ranking uses the logits themselves, so it is exact.
- *   - The workspace needs no zero state beyond the status word.
+ *   - Workspace: as for every call, zero-filled once when new; each call leaves its
+ *     per-sequence counters at zero again.
  */
 #define SPEC_FILTER_MAX_TOP_K 1024
 typedef struct {

@@ -164,7 +164,7 @@ size_t required_bytes(const spec_attn_args_t* attn, const spec_accept_args_t* ac
                       const spec_filter_args_t* filter, int sms, size_t* attn_base) {
   size_t end = kWsHeader;
   if (accept)
-    end = filter ? filter_layout(*accept, filter->max_top_k, kWsHeader).end
+    end = filter ? filter_layout(*accept, filter->max_top_k, kWsHeader, sms).end
                  : accept_layout(*accept, kWsHeader).end;
   if (attn_base) *attn_base = end;
   if (attn) end = attn_region(*attn, end, sms);
@@ -209,7 +209,7 @@ spec_status_t run(const spec_attn_args_t* attn, const spec_accept_args_t* accept
     if (e != cudaSuccess) return SPEC_ERR_CUDA;
   }
   if (accept && filter) {
-    const FilterLayout L = filter_layout(*accept, filter->max_top_k, kWsHeader);
+    const FilterLayout L = filter_layout(*accept, filter->max_top_k, kWsHeader, sms);
     if (launch_accept_filtered(*accept, *filter, L, w, stream, attn != nullptr) != cudaSuccess)
       return SPEC_ERR_CUDA;
   } else if (accept) {

@@ -47,8 +47,13 @@ AcceptLayout accept_layout(const spec_accept_args_t& a, size_t base);
 
 // --- filtered acceptance ---
 constexpr int kFilterMaxTopK = SPEC_FILTER_MAX_TOP_K;
+constexpr int kFiltLaneElems = 64;    // contiguous logits per lane (at the smallest lane size)
+constexpr int kFiltMaxLanes = 4096;   // lane maxima one row block keeps in shared memory
+constexpr int kFiltBlocksPerSm = 8;   // row blocks resident per SM (128 threads each)
+constexpr int kFiltMaxSplits = 16;    // blocks one row may be split across
+constexpr int kRowThreads = 128;      // threads of a filtered row block
 
-struct FiltRow {    // one (sequence, row) result of the filtered select kernel
+struct FiltRow {    // one (sequence, row) result of the filtered row kernel
   int32_t nkeep;    // kept tokens (top-k, then top-p)
   int32_t argmax;   // lowest index of the row maximum
   uint32_t flags;   // 1: NaN / +inf / no finite logit; 2: top_k or top_p out of range
@@ -56,15 +61,22 @@ struct FiltRow {    // one (sequence, row) result of the filtered select kernel
 };
 
 struct FilterLayout {
-  size_t lanes;  // uint64 [batch][2*gamma-1][nchunk*32]: lane maxima (order keys)
-  size_t rows;   // FiltRow [batch][2*gamma-1]
-  size_t ids;    // int32 [batch][2*gamma-1][max_top_k]: kept tokens, rank order
-  size_t probs;  // fp64, same layout: their filtered probabilities
+  size_t tickets;  // uint32 [batch]: rows of the sequence finished (reset by the last)
+  size_t rows;     // FiltRow [batch][2*gamma-1]
+  size_t kept;     // (int32 token, fp32 p') [batch][2*gamma-1][max_top_k], rank order
+  size_t row_tickets;  // uint32 [batch][2*gamma-1]: splits of the row finished (splits > 1)
+  size_t lanes_g;  // uint32 [batch][2*gamma-1][nlanes]: lane maxima (splits > 1)
+  size_t parts;    // 16 B [batch][2*gamma-1][splits]: each split's maximum and bad flag
   size_t end;
-  int nchunk, nlanes;
+  int lane_shift;  // lanes hold kFiltLaneElems << lane_shift logits
+  int nlanes;      // ceil(vocab / lane size) <= kFiltMaxLanes
+  int splits;      // blocks per row
+  int lanes_per_split;
+  int cand_cap;    // candidates one block holds (a power of two)
+  int smem_a;      // bytes of the first dynamic shared region
 };
 
-FilterLayout filter_layout(const spec_accept_args_t& a, int max_top_k, size_t base);
+FilterLayout filter_layout(const spec_accept_args_t& a, int max_top_k, size_t base, int sms);
 
 // --- attention ---
 struct AttnPlan {
