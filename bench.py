@@ -444,9 +444,9 @@ def run_ours(args, wl, ai, ci, rank, world, local_rank):
     dom_bytes = tm["kv"] if dominant == "attention" else tm["logits"]
     dom_ms = attn_ms if dominant == "attention" else acc_ms
     dom_gbs = dom_bytes / (dom_ms / 1000.0) / 1e9
-    # attention, then row statistics, decisions, draws (filtered: lane maxima, top-k /
-    # top-p select, decisions and draw)
-    launches_per_step = 4
+    # attention, then row statistics, decisions, draws; a filtered step: attention and
+    # the one filtered acceptance kernel
+    launches_per_step = 2 if filtered else 4
     traffic, traffic_src = (None, None)
     if dominant == "attention" and attn_path_name(args.attn_path, binding, ai) == "tensor cores":
         traffic, traffic_src = measured_traffic(args.workload, "attention")
