@@ -65,6 +65,9 @@ def _load():
             lib.oracle_accept_block.argtypes = [i32, i32, i64, i32, P, P, P, P, P, P, P, P,
                                                 P, P, P, P, i32]
             lib.oracle_accept_block.restype = ctypes.c_int
+            lib.oracle_sample_block.argtypes = [i32, i32, i64, i32, P, P, P, P, P, P, P, P, P, P,
+                                                i32]
+            lib.oracle_sample_block.restype = ctypes.c_int
             lib.oracle_filter_row.argtypes = [P, i64, i32, f64, P, P]
             lib.oracle_filter_row.restype = ctypes.c_int
             lib.oracle_accept_block_filtered.argtypes = [i32, i32, i64, i32, P, P, P, P, P, P,
@@ -284,6 +287,100 @@ def accept_block_filtered(target_logits, drafter_logits, block_tokens, temperatu
         raise ValueError("invalid arguments to oracle_accept_block_filtered")
     return dict(num_accepted=na, out_tokens=ot, num_emitted=ne, diag=diag,
                 accept_margin=am, sample_margin=sm, filter_margin=fm, status=st)
+
+
+def sample_block(drafter_logits, temperature, uniforms, top_k=None, top_p=None,
+                 nthreads: int = 0):
+    """Draft-side sampling of every block token from its drafter row (see
+    ``oracle_sample_block`` in oracle.cpp). Returns a dict of tokens, q_tok, margin,
+    filter_margin, status."""
+    lib = _load()
+    dl = np.ascontiguousarray(drafter_logits)
+    if dl.dtype == np.float32:
+        dtype = 0
+    elif dl.dtype == np.uint16:
+        dtype = 1
+    else:
+        raise TypeError("logits must be float32 or uint16 (bf16 bits)")
+    batch, gamma, vocab = dl.shape
+    T = _c(temperature, np.float32)
+    u = _c(uniforms, np.float32)
+    K = P = None
+    if top_k is not None:
+        K = _c(np.broadcast_to(np.asarray(top_k, np.int32), (batch,)), np.int32)
+        P = _c(np.broadcast_to(np.asarray(top_p, np.float32), (batch,)), np.float32)
+    tok = np.empty((batch, gamma), np.int32)
+    qt = np.empty((batch, gamma), np.float64)
+    mg = np.empty((batch, gamma), np.float64)
+    fm = np.empty((batch, gamma), np.float64)
+    st = np.empty(batch, np.int32)
+    rc = lib.oracle_sample_block(batch, gamma, vocab, dtype, _ptr(dl), _ptr(T),
+                                 None if K is None else _ptr(K), None if P is None else _ptr(P),
+                                 _ptr(u), _ptr(tok), _ptr(qt), _ptr(mg), _ptr(fm), _ptr(st),
+                                 int(nthreads))
+    if rc:
+        raise ValueError("invalid arguments to oracle_sample_block")
+    return dict(tokens=tok, q_tok=qt, margin=mg, filter_margin=fm, status=st)
+
+
+def noise_tokens(words, vocab: int):
+    """Alg. line 1 (z ~ U[V], i.i.d.): token = floor(x * V / 2^32) of each 32-bit random
+    word x, i.e. the word's position in [0, 1) scaled to the vocabulary."""
+    w = np.asarray(words, dtype=np.uint64)
+    return ((w * np.uint64(vocab)) >> np.uint64(32)).astype(np.int32)
+
+
+def commit_kv(kv_len, num_accepted, page_table, page_size: int, gamma: int, free_pages,
+              free_count: int, reserve: bool = True):
+    """Roll a paged KV cache back to the accepted prefix of a verify step, sequence by
+    sequence in batch order (plain loops).
+
+    kv_len[b] = ctx_b + gamma on entry (the block's keys were written for the verify
+    pass). The step keeps x^{L+1} and the n-1 accepted drafts (n = num_accepted + 1), so
+    kv_len becomes ctx_b + n; a sequence whose step failed (num_accepted = -1) keeps
+    ctx_b. The keys past the new length are stale and are overwritten by the next block.
+      * reserve: the sequence keeps its pages and pops, in batch order and from the top
+        of the free list, the pages it lacks for gamma more keys; a sequence that would
+        run the list dry, or whose table cannot hold them, gets none (flag 2; its length
+        is still committed).
+      * otherwise (the sequence stops here): pages wholly past the new length are pushed
+        onto the free list in batch order and their table entries become -1.
+    A sequence with kv_len outside [gamma, max_pages * page_size] or num_accepted outside
+    [-1, gamma - 1] is left unchanged (flag 1).
+
+    Returns (kv_len', page_table', free_pages', free_count', flags[b]: 0, 1 or 2)."""
+    kv = np.array(kv_len, dtype=np.int64)
+    na = np.asarray(num_accepted, dtype=np.int64)
+    table = np.array(page_table, dtype=np.int32, copy=True)
+    free = np.array(free_pages, dtype=np.int32, copy=True)
+    count = int(free_count)
+    B, max_pages = table.shape
+    new = kv.copy()
+    flags = np.zeros(B, np.int32)
+    for b in range(B):
+        if kv[b] < gamma or kv[b] > max_pages * page_size or na[b] < -1 or na[b] > gamma - 1:
+            flags[b] = 1
+            continue
+        new[b] = kv[b] - gamma + (na[b] + 1 if na[b] >= 0 else 0)
+    for b in range(B):
+        if flags[b]:
+            continue
+        have = -(-int(kv[b]) // page_size)
+        if reserve:
+            want = -(-int(new[b] + gamma) // page_size)
+            if want > max_pages or want - have > count:
+                flags[b] = 2
+                continue
+            for i in range(have, want):
+                count -= 1
+                table[b, i] = free[count]
+        else:
+            keep = -(-int(new[b]) // page_size)
+            for i in range(keep, have):
+                free[count] = table[b, i]
+                count += 1
+                table[b, i] = -1
+    return new.astype(np.int32), table, free, count, flags
 
 
 def verify_attention(q, k_cache, v_cache, page_table, kv_len, gamma: int, softmax_scale=None,

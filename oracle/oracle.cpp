@@ -479,6 +479,67 @@ int oracle_accept_block_filtered(int32_t batch, int32_t gamma, int64_t vocab, in
   return 0;
 }
 
+// Draft-side sampling (Alg. "Lossless Psi-Spec decoding (Linear Sampler)": the free
+// clean token x^{L+1} ~ q_0 and the B-1 drafts x~ ~ q, sampled in parallel). Drafter
+// row j of sequence b (q_0 for j = 0, the diffusion rows after it) is softmaxed at the
+// sequence's temperature, top-k / top-p filtered when top_k is not NULL (as in
+// oracle_accept_block_filtered), and block token j is the inverse-CDF draw with
+// uniforms[b][j] in ascending token order. At T = 0 it is the row's lowest-index argmax.
+// Outputs per (b, j): tokens, q_tok (the drawn token's probability; 1 at T = 0), margin
+// (the inverse-CDF margin; +inf at T = 0), filter_margin (the top-p margin; +inf
+// unfiltered or at T = 0). status[b]: 0, 1 (NaN or undefined softmax in a row), 3 (a
+// tempered sequence's top_k / top_p out of range); a flagged sequence's tokens are -1.
+int oracle_sample_block(int32_t batch, int32_t gamma, int64_t vocab, int32_t dtype,
+                        const void* drafter_logits, const float* temperature,
+                        const int32_t* top_k, const float* top_p, const float* uniforms,
+                        int32_t* tokens, double* q_tok, double* margin, double* filter_margin,
+                        int32_t* status, int32_t nthreads) {
+  if (batch < 0 || gamma < 1 || vocab < 1 || (dtype != 0 && dtype != 1)) return -1;
+  parallel_for(batch, nthreads, [&](int64_t b) {
+    const double T = static_cast<double>(temperature[b]);
+    const bool greedy = !(T > 0.0);
+    const bool filtered = top_k != nullptr && !greedy;
+    int code = 0;
+    if (filtered && (top_k[b] < 1 || !(top_p[b] > 0.0f) || top_p[b] > 1.0f)) code = 3;
+    std::vector<double> raw(static_cast<size_t>(vocab)), q(static_cast<size_t>(vocab)),
+        qf(static_cast<size_t>(vocab));
+    std::vector<int32_t> tok(gamma, -1);
+    std::vector<double> qt(gamma, kNaN), mg(gamma, kInf), fm(gamma, kInf);
+    for (int32_t j = 0; j < gamma && code == 0; ++j) {
+      const int64_t row = b * gamma + j;
+      for (int64_t x = 0; x < vocab; ++x) raw[x] = load_elem(drafter_logits, dtype, row * vocab + x);
+      if (greedy) {
+        for (int64_t x = 0; x < vocab; ++x)
+          if (std::isnan(raw[x])) code = 1;
+        if (code) break;
+        tok[j] = static_cast<int32_t>(oracle_argmax(raw.data(), vocab));
+        qt[j] = 1.0;
+        continue;
+      }
+      if (oracle_softmax(raw.data(), vocab, T, q.data())) { code = 1; break; }
+      const double* w = q.data();
+      if (filtered) {
+        oracle_filter_row(q.data(), vocab, top_k[b], static_cast<double>(top_p[b]), qf.data(),
+                          &fm[j]);
+        w = qf.data();
+      }
+      const double u = static_cast<double>(uniforms[row]);
+      const int64_t x = oracle_inverse_cdf(w, vocab, u, &mg[j]);
+      tok[j] = static_cast<int32_t>(x);
+      qt[j] = w[x];
+    }
+    status[b] = code;
+    for (int32_t j = 0; j < gamma; ++j) {
+      const int64_t row = b * gamma + j;
+      tokens[row] = code ? -1 : tok[j];
+      if (q_tok) q_tok[row] = code ? kNaN : qt[j];
+      if (margin) margin[row] = code ? kInf : mg[j];
+      if (filter_margin) filter_margin[row] = code ? kInf : fm[j];
+    }
+  });
+  return 0;
+}
+
 // Block-causal verify attention over a paged KV cache with grouped-query heads
 // (Sec. 4.1: the block is scored while the prefix activations stay in the KV
 // cache; Alg. "Lossless Psi-Spec": p <- x_theta([x^{L+1}, x~]; x) is one causal
