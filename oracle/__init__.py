@@ -339,12 +339,16 @@ def commit_kv(kv_len, num_accepted, page_table, page_size: int, gamma: int, free
     pass). The step keeps x^{L+1} and the n-1 accepted drafts (n = num_accepted + 1), so
     kv_len becomes ctx_b + n; a sequence whose step failed (num_accepted = -1) keeps
     ctx_b. The keys past the new length are stale and are overwritten by the next block.
-      * reserve: the sequence keeps its pages and pops, in batch order and from the top
-        of the free list, the pages it lacks for gamma more keys; a sequence that would
-        run the list dry, or whose table cannot hold them, gets none (flag 2; its length
-        is still committed).
+      * reserve: the sequence keeps its pages and pops from the top of the free list the
+        pages it lacks for gamma more keys. Requests are served in batch order; request
+        b is granted iff the requests of sequences 0..b together fit in the list (a
+        refused request still counts against the later ones, so the grants are a prefix
+        of the batch order). A refused sequence, or one whose table cannot hold the
+        pages, gets none (flag 2; its length is still committed).
       * otherwise (the sequence stops here): pages wholly past the new length are pushed
-        onto the free list in batch order and their table entries become -1.
+        onto the free list in batch order, with the same prefix rule against the list's
+        capacity; their table entries become -1. A sequence whose pages do not fit keeps
+        them (flag 2).
     A sequence with kv_len outside [gamma, max_pages * page_size] or num_accepted outside
     [-1, gamma - 1] is left unchanged (flag 1).
 
@@ -362,25 +366,40 @@ def commit_kv(kv_len, num_accepted, page_table, page_size: int, gamma: int, free
             flags[b] = 1
             continue
         new[b] = kv[b] - gamma + (na[b] + 1 if na[b] >= 0 else 0)
+    capacity = len(free)
+    asked = 0  # pages requested (reserve) or offered (release) by sequences 0..b-1
+    top = count
     for b in range(B):
         if flags[b]:
             continue
         have = -(-int(kv[b]) // page_size)
         if reserve:
             want = -(-int(new[b] + gamma) // page_size)
-            if want > max_pages or want - have > count:
+            if want > max_pages:
                 flags[b] = 2
                 continue
-            for i in range(have, want):
-                count -= 1
-                table[b, i] = free[count]
+            need = want - have
+            if asked + need > count:
+                flags[b] = 2
+                asked += need
+                continue
+            for i in range(need):
+                table[b, have + i] = free[count - 1 - asked - i]
+            asked += need
+            top = count - asked
         else:
             keep = -(-int(new[b]) // page_size)
-            for i in range(keep, have):
-                free[count] = table[b, i]
-                count += 1
-                table[b, i] = -1
-    return new.astype(np.int32), table, free, count, flags
+            give = have - keep
+            if count + asked + give > capacity:
+                flags[b] = 2
+                asked += give
+                continue
+            for i in range(give):
+                free[count + asked + i] = table[b, keep + i]
+                table[b, keep + i] = -1
+            asked += give
+            top = count + asked
+    return new.astype(np.int32), table, free, top, flags
 
 
 def verify_attention(q, k_cache, v_cache, page_table, kv_len, gamma: int, softmax_scale=None,

@@ -205,10 +205,18 @@ def test_commit_conserves_pages(reserve):
             assert np.all(t[b, :pages] >= 0) and np.all(t[b, pages:] == -1)
             if reserve and fl[b] == 0:
                 assert pages == -(-(new[b] + gamma) // P)
-            elif reserve:
-                assert fl[b] == 2 and pages == -(-kv[b] // P)
+            elif fl[b] == 2:
+                assert pages == -(-kv[b] // P)
             else:
                 assert pages == -(-new[b] // P)
+        if reserve:  # once the pool refuses a request, every later request is refused
+            need = np.array([-(-(new[b] + gamma) // P) - -(-kv[b] // P) for b in range(B)])
+            fits = np.array([-(-(new[b] + gamma) // P) <= max_pages for b in range(B)])
+            pool_refused = np.flatnonzero((fl == 2) & fits)
+            if pool_refused.size:
+                later = np.arange(B) > pool_refused[0]
+                assert np.all(fl[later & (fl == 0)] == 0)
+                assert not np.any(later & (fl == 0) & (need > 0))
 
 
 def test_commit_flags_bad_input_and_exhaustion():
@@ -225,3 +233,17 @@ def test_commit_flags_bad_input_and_exhaustion():
     new, t, f, c, fl = oracle.commit_kv(np.array([4, 4]), np.array([3, 3]), table, 4, 4,
                                         np.array([7, 0]), 1, reserve=True)
     assert list(fl) == [0, 2] and list(t[0]) == [1, 7] and list(t[1]) == [2, -1]
+    # a refused request still counts: the third sequence's single page would fit the
+    # list on its own, but the grants are a prefix of the batch order
+    table = np.array([[1, -1, -1], [2, -1, -1], [3, -1, -1]], np.int32)
+    new, t, f, c, fl = oracle.commit_kv(np.array([4, 4, 4]), np.array([0, 3, 3]), table, 4, 4,
+                                        np.array([7, 8, 0]), 2, reserve=True)
+    # needs: 1 (ctx 0 + n 1 + 4 keys = 5 -> 2 pages), 1 (8 keys -> 2), 1
+    assert list(fl) == [0, 0, 2] and list(t[0][:2]) == [1, 8] and list(t[1][:2]) == [2, 7]
+    # release with room for one more page: every step failed, so each sequence drops
+    # back to its context and offers one page; the first fits, the other two do not
+    table = np.array([[1, 2, 3], [4, 5, -1], [6, 7, -1]], np.int32)
+    new, t, f, c, fl = oracle.commit_kv(np.array([12, 8, 8]), np.array([-1, -1, -1]), table, 4,
+                                        4, np.array([9, 0]), 1, reserve=False)
+    assert list(new) == [8, 4, 4] and list(fl) == [0, 2, 2] and c == 2 and list(f) == [9, 3]
+    assert list(t[0]) == [1, 2, -1] and list(t[1]) == [4, 5, -1] and list(t[2]) == [6, 7, -1]
