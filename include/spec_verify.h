@@ -242,6 +242,80 @@ spec_status_t spec_verify_step_filtered(const spec_attn_args_t* attn,
                                         size_t ws_bytes, spec_stream_t stream);
 
 /*
+ * Draft-side sampling (Alg. "Lossless Psi-Spec decoding (Linear Sampler)": sample the
+ * free clean token x^{L+1} ~ q_0 and the B-1 drafts x~ ~ q, in parallel). Block token j
+ * of sequence b is drawn from drafter row j (row 0 = q_0, the AR pathway's
+ * distribution; rows 1.. = q, the diffusion drafter's) at temperature[b]: the smallest
+ * x with C(x) >= uniforms[b][j] * C(vocab-1), C the ascending-token cumulative sum of
+ * softmax(row / T), top-k / top-p filtered first when filter is not NULL (as in
+ * spec_accept_block_filtered); at T = 0 the row's lowest-index argmax. The result is the
+ * block_tokens input of the verify step.
+ *   - A sequence with a row that has NaN, +inf (T > 0) or no finite logit (T > 0) sets
+ *     SPEC_FLAG_BAD_LOGITS and gets block_tokens = -1 (and q_tok = NaN) in every row; a
+ *     tempered sequence with an out-of-range filter sets SPEC_FLAG_BAD_FILTER likewise.
+ *   - Unfiltered draws keep one 8-byte (max, sum) pair per 64 logits (32 without 16-byte
+ *     alignment) in shared memory: vocab up to 1,600,000 (800,000); larger is
+ *     SPEC_ERR_UNSUPPORTED.
+ */
+typedef struct {
+  int32_t batch;               /* >= 1                                                      */
+  int32_t gamma;               /* 1 .. 64                                                   */
+  int32_t vocab;               /* >= 1                                                      */
+  int32_t logits_dtype;        /* spec_dtype_t                                              */
+  const void* drafter_logits;  /* [batch][gamma][vocab]                                     */
+  const float* temperature;    /* [batch]; 0 => argmax                                      */
+  const float* uniforms;       /* [batch][gamma] in (0, 1]; [j] draws block token j         */
+  int32_t* block_tokens;       /* [batch][gamma], written                                   */
+  float* q_tok;                /* [batch][gamma]: the drawn token's (filtered) probability,
+                                  1 at T = 0; or NULL                                       */
+} spec_draft_args_t;
+
+size_t spec_draft_workspace_size(const spec_draft_args_t* draft, const spec_filter_args_t* filter);
+spec_status_t spec_sample_block(const spec_draft_args_t* draft, const spec_filter_args_t* filter,
+                                void* ws, size_t ws_bytes, spec_stream_t stream);
+
+/*
+ * The noise tokens that start a draft pass (Alg. line 1: z ~ U[V], i.i.d.):
+ * out_dev[i] = floor(x * vocab / 2^32), x = the Philox4x32-10 word of
+ * spec_philox_uniforms' definition at index offset + i. n >= 0, vocab >= 1.
+ */
+spec_status_t spec_noise_tokens(uint64_t seed, uint64_t offset, int64_t n, int32_t vocab,
+                                int32_t* out_dev, spec_stream_t stream);
+
+/*
+ * KV commit: roll a paged KV cache back to the accepted prefix of a verify step (the
+ * Algorithm returns [x, x^{L+1}, x~^{1:n-1}, z~]: the block keys past x~^{n-1} are not
+ * part of the sequence). On entry kv_len[b] = ctx_b + gamma (the verify layout); on exit
+ * kv_len[b] = ctx_b + n_b, n_b = num_accepted[b] + 1 (ctx_b if num_accepted[b] = -1,
+ * a failed step). The final token z~ has no key yet: the next pass computes it.
+ *   - reserve = 1: each sequence keeps its pages and takes, from the top of the free
+ *     list, the pages it lacks to hold gamma more keys (the next block). Requests are
+ *     served in batch order while their running total fits the list; a refused request
+ *     still counts against the later ones (flag 2, its length still committed), as does a
+ *     sequence whose table cannot hold the pages.
+ *   - reserve = 0 (the sequence stops): pages wholly past the new length are pushed onto
+ *     the free list in batch order (entries set to -1), under the same prefix rule
+ *     against free_capacity; a sequence whose pages do not fit keeps them (flag 2).
+ *   - kv_len outside [gamma, max_pages_per_seq * page_size] or num_accepted outside
+ *     [-1, gamma-1]: the sequence is left unchanged (flag 1).
+ * All pointers are device memory; one launch of one block, no workspace. The paper
+ * keeps its cache inside its serving framework; this call is that framework's step.
+ */
+typedef struct {
+  int32_t batch, gamma, page_size, max_pages_per_seq;
+  int32_t* kv_len;              /* [batch], read and written                                 */
+  const int32_t* num_accepted;  /* [batch], from the verify step                            */
+  int32_t* page_table;          /* [batch][max_pages_per_seq], read and written             */
+  int32_t* free_pages;          /* [free_capacity]: the free list, its top at free_count     */
+  int32_t* free_count;          /* [1], read and written                                     */
+  int32_t free_capacity;
+  int32_t reserve;              /* 1: reserve for the next block; 0: release                 */
+  int32_t* flags;               /* [batch]: 0, 1 or 2 as above; or NULL                      */
+} spec_commit_args_t;
+
+spec_status_t spec_commit_kv(const spec_commit_args_t* commit, spec_stream_t stream);
+
+/*
  * spec_accept_block without a workspace, for callers that cannot allocate device
  * memory when they verify (for example, code confined to a fixed, pre-planned memory
  * arena, or code that must not call an allocator). It computes exactly what

@@ -379,18 +379,19 @@ def commit_kv(kv_len, num_accepted, page_table, page_size: int, gamma: int, free
                 flags[b] = 2
                 continue
             need = want - have
-            if asked + need > count:
+            if need > 0 and asked + need > count:
                 flags[b] = 2
                 asked += need
                 continue
             for i in range(need):
                 table[b, have + i] = free[count - 1 - asked - i]
             asked += need
-            top = count - asked
+            if need > 0:
+                top = count - asked
         else:
             keep = -(-int(new[b]) // page_size)
             give = have - keep
-            if count + asked + give > capacity:
+            if give > 0 and count + asked + give > capacity:
                 flags[b] = 2
                 asked += give
                 continue
@@ -398,7 +399,8 @@ def commit_kv(kv_len, num_accepted, page_table, page_size: int, gamma: int, free
                 free[count + asked + i] = table[b, keep + i]
                 table[b, keep + i] = -1
             asked += give
-            top = count + asked
+            if give > 0:
+                top = count + asked
     return new.astype(np.int32), table, free, top, flags
 
 

@@ -63,6 +63,22 @@ class FilterArgs(ctypes.Structure):
                 ("max_top_k", ctypes.c_int32)]
 
 
+class DraftArgs(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int32), ("gamma", ctypes.c_int32), ("vocab", ctypes.c_int32),
+                ("logits_dtype", ctypes.c_int32), ("drafter_logits", ctypes.c_void_p),
+                ("temperature", ctypes.c_void_p), ("uniforms", ctypes.c_void_p),
+                ("block_tokens", ctypes.c_void_p), ("q_tok", ctypes.c_void_p)]
+
+
+class CommitArgs(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int32), ("gamma", ctypes.c_int32),
+                ("page_size", ctypes.c_int32), ("max_pages_per_seq", ctypes.c_int32),
+                ("kv_len", ctypes.c_void_p), ("num_accepted", ctypes.c_void_p),
+                ("page_table", ctypes.c_void_p), ("free_pages", ctypes.c_void_p),
+                ("free_count", ctypes.c_void_p), ("free_capacity", ctypes.c_int32),
+                ("reserve", ctypes.c_int32), ("flags", ctypes.c_void_p)]
+
+
 HEADER = os.path.join(_build.ROOT, "include", "spec_verify.h")
 
 
@@ -103,6 +119,14 @@ def lib(build_if_missing: bool = True):
             L.spec_accept_block_filtered.restype = ctypes.c_int
             L.spec_verify_step_filtered.argtypes = [P, P, P, P, ctypes.c_size_t, P]
             L.spec_verify_step_filtered.restype = ctypes.c_int
+            L.spec_draft_workspace_size.argtypes = [P, P]
+            L.spec_draft_workspace_size.restype = ctypes.c_size_t
+            L.spec_sample_block.argtypes = [P, P, P, ctypes.c_size_t, P]
+            L.spec_sample_block.restype = ctypes.c_int
+            L.spec_noise_tokens.argtypes = [u64, u64, i64, i32, P, P]
+            L.spec_noise_tokens.restype = ctypes.c_int
+            L.spec_commit_kv.argtypes = [P, P]
+            L.spec_commit_kv.restype = ctypes.c_int
             for f in ("spec_workspace_init", "spec_verify_attention", "spec_accept_block",
                       "spec_verify_step", "spec_philox_uniforms", "spec_read_device_status"):
                 getattr(L, f).restype = ctypes.c_int
@@ -303,6 +327,81 @@ def accept_block_filtered(target_logits, drafter_logits, block_tokens, temperatu
         ws = new_workspace(filtered_workspace_size(a, f), dev)
     accept_block_filtered_args(a, f, ws, stream)
     return res
+
+
+def draft_args(drafter_logits, temperature, uniforms, block_tokens, q_tok=None) -> DraftArgs:
+    B, G, V = drafter_logits.shape
+    if drafter_logits.dtype == torch.bfloat16:
+        dt = SPEC_BF16
+    elif drafter_logits.dtype == torch.float32:
+        dt = SPEC_F32
+    else:
+        raise TypeError("logits must be bfloat16 or float32")
+    _check(drafter_logits, "drafter_logits", drafter_logits.dtype)
+    _check(temperature, "temperature", torch.float32, (B,))
+    _check(uniforms, "uniforms", torch.float32, (B, G))
+    _check(block_tokens, "block_tokens", torch.int32, (B, G))
+    if q_tok is not None:
+        _check(q_tok, "q_tok", torch.float32, (B, G))
+    return DraftArgs(B, G, V, dt, drafter_logits.data_ptr(), temperature.data_ptr(),
+                     uniforms.data_ptr(), block_tokens.data_ptr(),
+                     None if q_tok is None else q_tok.data_ptr())
+
+
+def draft_workspace_size(d: DraftArgs, filt: Optional[FilterArgs] = None) -> int:
+    n = lib().spec_draft_workspace_size(ctypes.byref(d), None if filt is None else ctypes.byref(filt))
+    if n == 0:
+        raise SpecError(1, "spec_draft_workspace_size")
+    return int(n)
+
+
+def sample_block_args(d: DraftArgs, filt: Optional[FilterArgs], ws: torch.Tensor, stream=None):
+    _raise(lib().spec_sample_block(ctypes.byref(d), None if filt is None else ctypes.byref(filt),
+                                   _ptr(ws), ws.numel(), _stream(stream)), "spec_sample_block")
+
+
+def sample_block(drafter_logits, temperature, uniforms, top_k=None, top_p=None, max_top_k=None,
+                 ws=None, stream=None) -> Dict[str, torch.Tensor]:
+    """Draft-side sampling of every block token from its drafter row (x^{L+1} ~ q_0,
+    drafts ~ q), optionally top-k / top-p filtered. Returns block_tokens and q_tok."""
+    B, G, _ = drafter_logits.shape
+    dev = drafter_logits.device
+    res = dict(block_tokens=torch.empty(B, G, dtype=torch.int32, device=dev),
+               q_tok=torch.empty(B, G, dtype=torch.float32, device=dev))
+    d = draft_args(drafter_logits, temperature, uniforms, res["block_tokens"], res["q_tok"])
+    f = None if top_k is None else filter_args(top_k, top_p, B, max_top_k)
+    if ws is None:
+        ws = new_workspace(draft_workspace_size(d, f), dev)
+    sample_block_args(d, f, ws, stream)
+    return res
+
+
+def noise_tokens(seed: int, n: int, vocab: int, offset: int = 0, device=None,
+                 stream=None) -> torch.Tensor:
+    """The uniform noise tokens z ~ U[V] that start a draft pass (Alg. line 1)."""
+    out = torch.empty(n, dtype=torch.int32, device=device or "cuda")
+    _raise(lib().spec_noise_tokens(ctypes.c_uint64(seed), ctypes.c_uint64(offset), n, int(vocab),
+                                   _ptr(out), _stream(stream)), "spec_noise_tokens")
+    return out
+
+
+def commit_kv(kv_len, num_accepted, page_table, page_size: int, gamma: int, free_pages, free_count,
+              reserve: bool = True, flags=None, stream=None):
+    """spec_commit_kv on device tensors (kv_len, page_table, free_pages, free_count are
+    updated in place; free_count is an int32 tensor of one element)."""
+    B, MP = page_table.shape
+    _check(kv_len, "kv_len", torch.int32, (B,))
+    _check(num_accepted, "num_accepted", torch.int32, (B,))
+    _check(page_table, "page_table", torch.int32)
+    _check(free_pages, "free_pages", torch.int32)
+    _check(free_count, "free_count", torch.int32, (1,))
+    if flags is not None:
+        _check(flags, "flags", torch.int32, (B,))
+    a = CommitArgs(B, int(gamma), int(page_size), MP, kv_len.data_ptr(), num_accepted.data_ptr(),
+                   page_table.data_ptr(), free_pages.data_ptr(), free_count.data_ptr(),
+                   free_pages.numel(), 1 if reserve else 0,
+                   None if flags is None else flags.data_ptr())
+    _raise(lib().spec_commit_kv(ctypes.byref(a), _stream(stream)), "spec_commit_kv")
 
 
 def philox_uniforms(seed: int, n: int, offset: int = 0, device=None, stream=None) -> torch.Tensor:

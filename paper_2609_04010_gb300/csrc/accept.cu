@@ -656,12 +656,10 @@ __global__ void __launch_bounds__(kSampleThreads, 5) sample_kernel(AcceptParams 
   if (tid == 0) p.out_tokens[orow + n] = s_token;
 }
 
-__global__ void philox_uniforms_kernel(uint64_t seed, uint64_t offset, int64_t n, float* out) {
-  // Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11): 10 rounds of two 32x32->64
-  // multiplies by the Philox constants, with the key advanced by the Weyl constants.
-  const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
-  if (i >= n) return;
-  const uint64_t g = offset + static_cast<uint64_t>(i);
+// Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11): 10 rounds of two 32x32->64
+// multiplies by the Philox constants, with the key advanced by the Weyl constants.
+// Returns word g & 3 of the block at counter (g >> 2, 0, 0) under key (seed low, high).
+__device__ __forceinline__ uint32_t philox_word(uint64_t seed, uint64_t g) {
   const uint64_t blk = g >> 2;
   uint32_t c0 = static_cast<uint32_t>(blk), c1 = static_cast<uint32_t>(blk >> 32), c2 = 0, c3 = 0;
   uint32_t k0 = static_cast<uint32_t>(seed), k1 = static_cast<uint32_t>(seed >> 32);
@@ -680,8 +678,23 @@ __global__ void philox_uniforms_kernel(uint64_t seed, uint64_t offset, int64_t n
     c3 = lo0;
   }
   const uint32_t words[4] = {c0, c1, c2, c3};
-  const uint32_t x = words[g & 3];
+  return words[g & 3];
+}
+
+__global__ void philox_uniforms_kernel(uint64_t seed, uint64_t offset, int64_t n, float* out) {
+  const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  const uint32_t x = philox_word(seed, offset + static_cast<uint64_t>(i));
   out[i] = static_cast<float>((x >> 8) + 1u) * 5.9604644775390625e-8f;  // * 2^-24
+}
+
+// Alg. line 1: noise tokens z ~ U[V], token = floor(x * V / 2^32) of the word x.
+__global__ void noise_tokens_kernel(uint64_t seed, uint64_t offset, int64_t n, int32_t vocab,
+                                    int32_t* out) {
+  const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  const uint32_t x = philox_word(seed, offset + static_cast<uint64_t>(i));
+  out[i] = static_cast<int32_t>((static_cast<uint64_t>(x) * static_cast<uint32_t>(vocab)) >> 32);
 }
 
 template <bool BF16, bool VEC>
@@ -746,6 +759,15 @@ cudaError_t launch_accept(const spec_accept_args_t& a, const AcceptLayout& L, ch
                : launch_typed<true, false>(p, stream, overlap_prior);
   return vec ? launch_typed<false, true>(p, stream, overlap_prior)
              : launch_typed<false, false>(p, stream, overlap_prior);
+}
+
+cudaError_t launch_noise(uint64_t seed, uint64_t offset, int64_t n, int32_t vocab, int32_t* out,
+                         cudaStream_t s) {
+  if (n == 0) return cudaSuccess;
+  const int64_t blocks = (n + 255) / 256;
+  (void)cudaGetLastError();  // report this launch's error only
+  noise_tokens_kernel<<<static_cast<unsigned>(blocks), 256, 0, s>>>(seed, offset, n, vocab, out);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_philox(uint64_t seed, uint64_t offset, int64_t n, float* out, cudaStream_t s) {

@@ -34,7 +34,8 @@
 
 namespace specv {
 
-FilterLayout filter_layout(const spec_accept_args_t& a, int max_top_k, size_t base, int sms) {
+FilterLayout filter_layout(const spec_accept_args_t& a, int max_top_k, size_t base, int sms,
+                           bool draw) {
   FilterLayout L;
   L.lane_shift = 0;
   while ((static_cast<int64_t>(a.vocab) + (kFiltLaneElems << L.lane_shift) - 1) /
@@ -42,7 +43,8 @@ FilterLayout filter_layout(const spec_accept_args_t& a, int max_top_k, size_t ba
     ++L.lane_shift;
   const int lane = kFiltLaneElems << L.lane_shift;
   L.nlanes = static_cast<int>((static_cast<int64_t>(a.vocab) + lane - 1) / lane);
-  const int64_t rows = static_cast<int64_t>(a.batch) * (2 * static_cast<int64_t>(a.gamma) - 1);
+  const int64_t rows = static_cast<int64_t>(a.batch) *
+                       (draw ? a.gamma : 2 * static_cast<int64_t>(a.gamma) - 1);
   // split rows across blocks until the grid holds about kFiltBlocksPerSm blocks per SM
   int64_t splits = (static_cast<int64_t>(kFiltBlocksPerSm) * sms + rows - 1) / rows;
   splits = splits < 1 ? 1 : (splits > kFiltMaxSplits ? kFiltMaxSplits : splits);
@@ -76,6 +78,7 @@ constexpr int kRankSortMax = 256;    // candidates ranked by counting; more are 
 constexpr uint32_t kRowBadLogits = 1u, kRowBadFilter = 2u;
 
 struct FiltParams {
+  int mode;  // 0: verify (target and drafter rows); 1: draw every drafter row's token
   int batch, gamma, vocab, max_top_k, lane_shift, nlanes;
   int splits, lanes_per_split;  // blocks per row and the lanes each scans
   int cand_cap;                 // candidates (and lanes to rescan) one block holds
@@ -98,6 +101,8 @@ struct FiltParams {
   uint32_t* row_tickets;  // [batch][2*gamma-1] (splits > 1)
   uint32_t* lanes_g;      // [batch][2*gamma-1][nlanes] lane maxima (splits > 1)
   uint4* parts;           // [batch][2*gamma-1][splits]: (row max candidate, bad) per split
+  int32_t* draw_tokens;   // mode 1: [batch][gamma] block tokens
+  float* draw_q;          // mode 1: [batch][gamma] their filtered probabilities, or NULL
 };
 
 // Small shared arrays of the decision phase (the sequence's last block).
@@ -141,8 +146,11 @@ __device__ __forceinline__ int cand_tok(unsigned long long c) {
   return static_cast<int>(0xffffffffu - static_cast<uint32_t>(c));
 }
 
-// Row r of sequence b: target row r for r < gamma, else drafter row r - gamma + 1.
+// Row r of sequence b. Verify: target row r for r < gamma, else drafter row
+// r - gamma + 1. Draw: drafter row r.
 __device__ __forceinline__ const char* row_ptr(const FiltParams& p, int b, int r, int esz) {
+  if (p.mode == 1)
+    return static_cast<const char*>(p.drafter) + (static_cast<int64_t>(b) * p.gamma + r) * p.vocab * esz;
   const int64_t row = static_cast<int64_t>(b) * p.gamma + (r < p.gamma ? r : r - p.gamma + 1);
   const void* base = r < p.gamma ? p.target : p.drafter;
   return static_cast<const char*>(base) + row * p.vocab * esz;
@@ -605,10 +613,11 @@ __global__ void __launch_bounds__(kRowThreads, 8) filter_row_kernel(FiltParams p
   __shared__ int s_ncand, s_keep, s_bad, s_last;
 
   const int split = blockIdx.x, r = blockIdx.y, b = blockIdx.z, tid = threadIdx.x;
-  const int gamma = p.gamma, nrows = 2 * gamma - 1, V = p.vocab;
+  const int gamma = p.gamma, nrows = p.mode == 1 ? gamma : 2 * gamma - 1, V = p.vocab;
   const float T = p.temperature[b];
   const bool greedy = !(T > 0.f);
-  if (greedy && r >= gamma) return;  // greedy sequences never read drafter rows
+  if (greedy && r >= gamma) return;  // greedy sequences never read drafter rows (verify)
+  const float u_draw = p.mode == 1 ? p.uniforms[static_cast<int64_t>(b) * gamma + r] : 0.f;
   const int64_t rid = static_cast<int64_t>(b) * nrows + r;
   const char* rowp = row_ptr(p, b, r, BF16 ? 2 : 4);
   const int lane_elems = kFiltLaneElems << p.lane_shift;
@@ -934,12 +943,46 @@ __global__ void __launch_bounds__(kRowThreads, 8) filter_row_kernel(FiltParams p
         if (pre[j] / mass >= tp) atomicMin(&s_keep, j + 1);
     __syncthreads();
     const int keep = s_keep;
-    const float S = pre[keep - 1];
-    int2* kept = p.kept + rid * p.max_top_k;
-    for (int j = tid; j < keep; j += kRowThreads)
-      kept[j] = make_int2(cand_tok(ranked[j]), __float_as_int(wsm[j] / S));
+    if (p.mode == 1) {
+      // the draw: the smallest kept token whose cumulative weight over the kept tokens
+      // with ids up to it reaches u * S (every thread sums in the same order)
+      if (tid == 0) {
+        s_misc[0] = INT_MAX;
+        s_misc[1] = -1;
+      }
+      __syncthreads();
+      float Sall = 0.f;
+      for (int i = 0; i < keep; ++i) Sall += wsm[i];
+      const float target = u_draw * Sall;
+      for (int j = tid; j < keep; j += kRowThreads) {
+        const int my = cand_tok(ranked[j]);
+        float C = 0.f;
+        for (int i = 0; i < keep; ++i)
+          if (cand_tok(ranked[i]) <= my) C += wsm[i];
+        if (wsm[j] > 0.f) {
+          atomicMax(&s_misc[1], my);
+          if (C >= target) atomicMin(&s_misc[0], my);
+        }
+      }
+      __syncthreads();
+      const int tok = s_misc[0] != INT_MAX ? s_misc[0] : s_misc[1];  // rounding: last positive
+      for (int j = tid; j < keep; j += kRowThreads)
+        if (cand_tok(ranked[j]) == tok) {
+          p.draw_tokens[static_cast<int64_t>(b) * gamma + r] = tok;
+          if (p.draw_q) p.draw_q[static_cast<int64_t>(b) * gamma + r] = wsm[j] / Sall;
+        }
+    } else {
+      const float S = pre[keep - 1];
+      int2* kept = p.kept + rid * p.max_top_k;
+      for (int j = tid; j < keep; j += kRowThreads)
+        kept[j] = make_int2(cand_tok(ranked[j]), __float_as_int(wsm[j] / S));
+    }
     info.nkeep = keep;
     info.argmax = cand_tok(ranked[0]);
+  } else if (p.mode == 1 && tid == 0) {
+    // a greedy row draws its argmax; a bad row's outputs are set by the sequence's last block
+    p.draw_tokens[static_cast<int64_t>(b) * gamma + r] = info.flags ? -1 : info.argmax;
+    if (p.draw_q) p.draw_q[static_cast<int64_t>(b) * gamma + r] = info.flags ? NAN : 1.f;
   }
   if (tid == 0) p.rows[rid] = info;
 
@@ -955,6 +998,25 @@ __global__ void __launch_bounds__(kRowThreads, 8) filter_row_kernel(FiltParams p
   __syncthreads();
   if (!s_last) return;
   __threadfence();
+  if (p.mode == 1) {
+    // a sequence with a bad row draws nothing: every token -1 (the oracle's convention)
+    if (tid == 0) s_flags[0] = 0;
+    __syncthreads();
+    for (int k = tid; k < gamma; k += kRowThreads)
+      atomicOr(&s_flags[0], static_cast<int>(__ldcg(&p.rows[static_cast<int64_t>(b) * nrows + k].flags)));
+    __syncthreads();
+    if (s_flags[0]) {
+      for (int k = tid; k < gamma; k += kRowThreads) {
+        p.draw_tokens[static_cast<int64_t>(b) * gamma + k] = -1;
+        if (p.draw_q) p.draw_q[static_cast<int64_t>(b) * gamma + k] = NAN;
+      }
+      if (tid == 0) {
+        if (s_flags[0] & kRowBadLogits) set_status(p.status, SPEC_FLAG_BAD_LOGITS);
+        if (s_flags[0] & kRowBadFilter) set_status(p.status, SPEC_FLAG_BAD_FILTER);
+      }
+    }
+    return;
+  }
   DrawLists L;
   const int mk2 = pow2_at_least(p.max_top_k);  // list stride: room for the sort's padding
   L.P_id = reinterpret_cast<int*>(dsm);
@@ -972,7 +1034,7 @@ cudaError_t launch_filtered_typed(const FiltParams& p, cudaStream_t stream, bool
   attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(p.splits, 2 * p.gamma - 1, p.batch);
+  cfg.gridDim = dim3(p.splits, p.mode == 1 ? p.gamma : 2 * p.gamma - 1, p.batch);
   cfg.blockDim = dim3(kRowThreads);
   cfg.dynamicSmemBytes = p.smem_a + static_cast<size_t>(p.cand_cap) * 12;
   cfg.stream = stream;
@@ -987,8 +1049,11 @@ cudaError_t launch_filtered_typed(const FiltParams& p, cudaStream_t stream, bool
 
 cudaError_t launch_accept_filtered(const spec_accept_args_t& a, const spec_filter_args_t& f,
                                    const FilterLayout& L, char* ws, cudaStream_t stream,
-                                   bool overlap_prior) {
+                                   bool overlap_prior, int32_t* draw_tokens, float* draw_q) {
   FiltParams p;
+  p.mode = draw_tokens ? 1 : 0;
+  p.draw_tokens = draw_tokens;
+  p.draw_q = draw_q;
   p.batch = a.batch;
   p.gamma = a.gamma;
   p.vocab = a.vocab;

@@ -90,6 +90,37 @@ spec_status_t check_accept(const spec_accept_args_t* a) {
   return SPEC_OK;
 }
 
+spec_status_t check_draft(const spec_draft_args_t* d) {
+  if (!d) return SPEC_ERR_INVALID_ARGUMENT;
+  if (d->batch < 1 || d->gamma < 1 || d->vocab < 1) return SPEC_ERR_INVALID_ARGUMENT;
+  if (d->logits_dtype != SPEC_F32 && d->logits_dtype != SPEC_BF16) return SPEC_ERR_INVALID_ARGUMENT;
+  if (!d->drafter_logits || !d->temperature || !d->uniforms || !d->block_tokens)
+    return SPEC_ERR_INVALID_ARGUMENT;
+  if (d->gamma > 64 || d->batch > 65535) return SPEC_ERR_UNSUPPORTED;
+  return SPEC_OK;
+}
+
+// The acceptance arguments the filtered row kernel reads in its draw mode.
+spec_accept_args_t draft_as_accept(const spec_draft_args_t& d) {
+  spec_accept_args_t a = {};
+  a.batch = d.batch;
+  a.gamma = d.gamma;
+  a.vocab = d.vocab;
+  a.logits_dtype = d.logits_dtype;
+  a.target_logits = d.drafter_logits;
+  a.drafter_logits = d.drafter_logits;
+  a.temperature = d.temperature;
+  a.uniforms = d.uniforms;
+  return a;
+}
+
+constexpr size_t kDraftMaxSmem = 200 * 1024;  // lane summaries of one unfiltered draw block
+
+size_t draft_bytes(const spec_draft_args_t& d, const spec_filter_args_t* f, int sms, bool vec) {
+  if (f) return filter_layout(draft_as_accept(d), f->max_top_k, kWsHeader, sms, true).end;
+  return draft_layout(d, kWsHeader, sms, vec).end;
+}
+
 spec_status_t check_filter(const spec_filter_args_t* f) {
   if (!f || !f->top_k || !f->top_p) return SPEC_ERR_INVALID_ARGUMENT;
   if (f->max_top_k < 1) return SPEC_ERR_INVALID_ARGUMENT;
@@ -292,6 +323,73 @@ spec_status_t spec_verify_step_filtered(const spec_attn_args_t* attn,
                                         size_t ws_bytes, spec_stream_t stream) {
   if (!accept || !filter) return SPEC_ERR_INVALID_ARGUMENT;
   return run(attn, accept, filter, ws, ws_bytes, stream);
+}
+
+spec_status_t spec_noise_tokens(uint64_t seed, uint64_t offset, int64_t n, int32_t vocab,
+                                int32_t* out_dev, spec_stream_t stream) {
+  if (n < 0 || vocab < 1 || (n > 0 && !out_dev)) return SPEC_ERR_INVALID_ARGUMENT;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  int sms = 0;
+  if (!bind_device(s, &sms)) return SPEC_ERR_CUDA;
+  return launch_noise(seed, offset, n, vocab, out_dev, s) == cudaSuccess ? SPEC_OK : SPEC_ERR_CUDA;
+}
+
+size_t spec_draft_workspace_size(const spec_draft_args_t* draft, const spec_filter_args_t* filter) {
+  if (check_draft(draft) != SPEC_OK || (filter && check_filter(filter) != SPEC_OK)) return 0;
+  int dev = 0, sms = 160;
+  if (cudaGetDevice(&dev) == cudaSuccess) {
+    const int n = device_sm_count(dev);
+    if (n > sms) sms = n;
+  } else {
+    cudaGetLastError();
+  }
+  size_t need = 0;
+  for (int s : {148, 152, sms})
+    for (bool vec : {false, true}) {
+      const size_t x = draft_bytes(*draft, filter, s, vec);
+      if (x > need) need = x;
+    }
+  return need;
+}
+
+spec_status_t spec_sample_block(const spec_draft_args_t* draft, const spec_filter_args_t* filter,
+                                void* ws, size_t ws_bytes, spec_stream_t stream_) {
+  spec_status_t st = check_draft(draft);
+  if (st != SPEC_OK) return st;
+  if (filter && (st = check_filter(filter)) != SPEC_OK) return st;
+  if (!ws || (reinterpret_cast<uintptr_t>(ws) % kWsAlign) != 0) return SPEC_ERR_INVALID_ARGUMENT;
+  const size_t esz = draft->logits_dtype == SPEC_BF16 ? 2 : 4;
+  const bool vec = (static_cast<size_t>(draft->vocab) * esz) % 16 == 0 &&
+                   reinterpret_cast<uintptr_t>(draft->drafter_logits) % 16 == 0;
+  if (!filter && draft_layout(*draft, kWsHeader, 1, vec).smem > kDraftMaxSmem) return SPEC_ERR_UNSUPPORTED;
+  if (draft_bytes(*draft, filter, 1, vec) > ws_bytes) return SPEC_ERR_WORKSPACE_TOO_SMALL;
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  int sms = 0;
+  if (!bind_device(stream, &sms)) return SPEC_ERR_CUDA;
+  (void)cudaGetLastError();
+  if (draft_bytes(*draft, filter, sms, vec) > ws_bytes) return SPEC_ERR_WORKSPACE_TOO_SMALL;
+  char* w = static_cast<char*>(ws);
+  if (filter) {
+    const spec_accept_args_t a = draft_as_accept(*draft);
+    const FilterLayout L = filter_layout(a, filter->max_top_k, kWsHeader, sms, true);
+    return launch_accept_filtered(a, *filter, L, w, stream, false, draft->block_tokens,
+                                  draft->q_tok) == cudaSuccess ? SPEC_OK : SPEC_ERR_CUDA;
+  }
+  const DraftLayout L = draft_layout(*draft, kWsHeader, sms, vec);
+  return launch_draft(*draft, L, w, stream, vec) == cudaSuccess ? SPEC_OK : SPEC_ERR_CUDA;
+}
+
+spec_status_t spec_commit_kv(const spec_commit_args_t* c, spec_stream_t stream) {
+  if (!c || c->batch < 1 || c->gamma < 1 || c->page_size < 1 || c->max_pages_per_seq < 1 ||
+      c->free_capacity < 0 || !c->kv_len || !c->num_accepted || !c->page_table ||
+      !c->free_pages || !c->free_count || (c->reserve != 0 && c->reserve != 1))
+    return SPEC_ERR_INVALID_ARGUMENT;
+  if (static_cast<int64_t>(c->max_pages_per_seq) * c->page_size + c->gamma > INT32_MAX)
+    return SPEC_ERR_UNSUPPORTED;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  int sms = 0;
+  if (!bind_device(s, &sms)) return SPEC_ERR_CUDA;
+  return launch_commit(*c, s) == cudaSuccess ? SPEC_OK : SPEC_ERR_CUDA;
 }
 
 spec_status_t spec_philox_uniforms(uint64_t seed, uint64_t offset, int64_t n, float* out_dev,

@@ -76,7 +76,27 @@ struct FilterLayout {
   int smem_a;      // bytes of the first dynamic shared region
 };
 
-FilterLayout filter_layout(const spec_accept_args_t& a, int max_top_k, size_t base, int sms);
+// draw = true: the layout of the draft-side draw (gamma drafter rows per sequence).
+FilterLayout filter_layout(const spec_accept_args_t& a, int max_top_k, size_t base, int sms,
+                           bool draw = false);
+
+// --- draft-side sampling ---
+struct DraftLayout {
+  size_t tickets;      // uint32 [batch]: rows of the sequence finished (reset by the last)
+  size_t row_flags;    // uint32 [batch][gamma]
+  size_t row_tickets;  // uint32 [batch][gamma]: splits of the row finished (splits > 1)
+  size_t lanes_g;      // float2 [batch][gamma][nlanes]: lane (max, sum) (splits > 1)
+  size_t parts;        // 16 B [batch][gamma][splits]: each split's maximum and bad flag
+  size_t end;
+  size_t smem;         // dynamic shared memory of one block: nlanes x 8 B
+  int lane_elems;      // 64 with 16-byte loads, 32 with element loads
+  int nlanes, splits, lanes_per_split;
+};
+
+DraftLayout draft_layout(const spec_draft_args_t& a, size_t base, int sms, bool vec);
+cudaError_t launch_draft(const spec_draft_args_t& a, const DraftLayout& L, char* ws,
+                         cudaStream_t stream, bool vec);
+cudaError_t launch_commit(const spec_commit_args_t& a, cudaStream_t stream);
 
 // --- attention ---
 struct AttnPlan {
@@ -104,14 +124,19 @@ AttnPlan attn_plan(const spec_attn_args_t& a, size_t base, int num_sms, int path
 // reads none of their inputs and writes none of their outputs).
 cudaError_t launch_accept(const spec_accept_args_t& a, const AcceptLayout& L, char* ws,
                           int num_sms, cudaStream_t stream, bool overlap_prior = false);
+// With draw_tokens set, draws every drafter row's token instead of verifying (only the
+// logits, temperature, uniforms and batch shape of a are read).
 cudaError_t launch_accept_filtered(const spec_accept_args_t& a, const spec_filter_args_t& f,
                                    const FilterLayout& L, char* ws, cudaStream_t stream,
-                                   bool overlap_prior = false);
+                                   bool overlap_prior = false, int32_t* draw_tokens = nullptr,
+                                   float* draw_q = nullptr);
 cudaError_t launch_attn_simt(const spec_attn_args_t& a, const AttnPlan& P, char* ws,
                              cudaStream_t stream);
 cudaError_t launch_attn_tc(const spec_attn_args_t& a, const AttnPlan& P, char* ws,
                            cudaStream_t stream);
 cudaError_t launch_philox(uint64_t seed, uint64_t offset, int64_t n, float* out, cudaStream_t s);
+cudaError_t launch_noise(uint64_t seed, uint64_t offset, int64_t n, int32_t vocab, int32_t* out,
+                         cudaStream_t s);
 
 // Rows of one CUDA-core block and of one tensor-core block.
 constexpr int kSimtRowTile = 16;

@@ -134,3 +134,37 @@ def test_filtered_workspace_size_and_too_small(lib):
     assert both > n50
     assert lib.spec_accept_block_filtered(ctypes.byref(acc), ctypes.byref(f50),
                                           ctypes.c_void_p(4096), 1024, None) == 3
+
+
+def _draft(**kw):
+    base = dict(batch=4, gamma=8, vocab=128256, logits_dtype=1)
+    base.update(kw)
+    d = binding.DraftArgs(**base)
+    for f in ("drafter_logits", "temperature", "uniforms", "block_tokens"):
+        setattr(d, f, 4096)
+    return d
+
+
+@pytest.mark.parametrize("kw,code", [(dict(gamma=65), 2), (dict(batch=0), 1), (dict(vocab=0), 1),
+                                     (dict(logits_dtype=5), 1)])
+def test_draft_host_checks(lib, kw, code):
+    d = _draft(**kw)
+    assert lib.spec_sample_block(ctypes.byref(d), None, ctypes.c_void_p(4096), 1 << 30, None) == code
+    assert lib.spec_draft_workspace_size(ctypes.byref(d), None) == 0
+
+
+def test_draft_workspace_and_other_checks(lib):
+    d = _draft()
+    n = lib.spec_draft_workspace_size(ctypes.byref(d), None)
+    f = binding.FilterArgs(4096, 4096, 50)
+    nf = lib.spec_draft_workspace_size(ctypes.byref(d), ctypes.byref(f))
+    assert n > 0 and nf > 0 and n % 256 == 0
+    assert lib.spec_sample_block(None, None, ctypes.c_void_p(4096), 1 << 30, None) == 1
+    assert lib.spec_sample_block(ctypes.byref(d), None, ctypes.c_void_p(4096), 512, None) == 3
+    assert lib.spec_noise_tokens(1, 0, -1, 10, None, None) == 1
+    assert lib.spec_noise_tokens(1, 0, 5, 0, ctypes.c_void_p(4096), None) == 1
+    assert lib.spec_commit_kv(None, None) == 1
+    c = binding.CommitArgs(4, 8, 16, 10, 4096, 4096, 4096, None, 4096, 100, 1, None)
+    assert lib.spec_commit_kv(ctypes.byref(c), None) == 1  # no free list
+    c = binding.CommitArgs(4, 8, 16, 10, 4096, 4096, 4096, 4096, 4096, 100, 2, None)
+    assert lib.spec_commit_kv(ctypes.byref(c), None) == 1  # reserve must be 0 or 1

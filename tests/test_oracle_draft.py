@@ -240,6 +240,12 @@ def test_commit_flags_bad_input_and_exhaustion():
                                         np.array([7, 8, 0]), 2, reserve=True)
     # needs: 1 (ctx 0 + n 1 + 4 keys = 5 -> 2 pages), 1 (8 keys -> 2), 1
     assert list(fl) == [0, 0, 2] and list(t[0][:2]) == [1, 8] and list(t[1][:2]) == [2, 7]
+    # a request of zero pages after a refused one is served, and the list's top stays
+    # where the last grant left it
+    table = np.array([[1, -1, -1], [2, -1, -1], [3, 4, -1]], np.int32)
+    new, t, f, c, fl = oracle.commit_kv(np.array([4, 4, 8]), np.array([3, 3, -1]), table, 4, 4,
+                                        np.array([5, 0, 0]), 1, reserve=True)
+    assert list(fl) == [0, 2, 0] and c == 0 and list(t[0]) == [1, 5, -1]
     # release with room for one more page: every step failed, so each sequence drops
     # back to its context and offers one page; the first fits, the other two do not
     table = np.array([[1, 2, 3], [4, 5, -1], [6, 7, -1]], np.int32)
