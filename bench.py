@@ -44,15 +44,15 @@ L2_FLUSH_BYTES = 256 << 20
 # while the kernel's sources still hash to what they were when the capture was taken.
 MEASURED_TRAFFIC = {
     ("llama8b", "attention"): {
-        "bytes": 139_693_056,
+        "bytes": 139_308_800,
         "profile": "profiles/attn_tc_kernel_llama8b.md",
         "sources": {
             "paper_2609_04010_gb300/csrc/attn_tc.cu":
-                "e108ce0d33e6bfa78a03713b6355cf6386c729aa620c38c7db71fd510c3cbda0",
+                "194e2351e6d39423418b78a4fb5a4e4d49002d0329417b93b7e5987178d1ee38",
             "paper_2609_04010_gb300/csrc/attn_common.cuh":
-                "92c08340231887aa7a8614c752c7a0fcea3ba600461aec09240162de420f465c",
+                "ed48d4dd71d0521ef69a8e8a78e8c0c0d5d8fe094a7a2784a1b3c0412f23e131",
             "paper_2609_04010_gb300/csrc/common.cuh":
-                "b59156aa4ea00852b9b5c078bbc03a73954bc83e855e407907568782ed4f9a90",
+                "2043c94505012a600bb927d65add0620cd827fe46f727917cd25e3eafbfc73bc",
         },
     },
 }
