@@ -76,6 +76,10 @@ def _load():
             lib.oracle_verify_attention.argtypes = [i32, i32, i32, i32, i32, i32, i32, i32, f64,
                                                     P, P, P, P, P, P, P, P, i64, P, i32]
             lib.oracle_verify_attention.restype = ctypes.c_int
+            lib.oracle_verify_attention_tree.argtypes = [i32, i32, i32, i32, i32, i32, i32, i32,
+                                                         f64, P, P, P, P, P, P, P, P, P, i64, P,
+                                                         i32]
+            lib.oracle_verify_attention_tree.restype = ctypes.c_int
             _lib = lib
     return _lib
 
@@ -404,13 +408,151 @@ def commit_kv(kv_len, num_accepted, page_table, page_size: int, gamma: int, free
     return new.astype(np.int32), table, free, top, flags
 
 
+def _rows_f64(logits):
+    a = np.asarray(logits)
+    if a.dtype == np.uint16:
+        return (a.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    return a.astype(np.float64)
+
+
+def build_tree(drafter_logits, temperature, root_tokens, top_k: int, budget: int):
+    """The tree sampler's candidate tree (Sec. 3.3, "Tree Sampler": the top K tokens at
+    each block position, pruned to the top ``budget`` prefixes by log-probability), by
+    best-first search in plain loops.
+
+    Position d = 1 .. gamma-1 of the block draws from drafter row d; its candidates are
+    the top_k tokens of log q_d = log softmax(row / T) (T = temperature[b], or 1 at
+    T = 0), ranked by probability, equal ones by lower token id. Node 0 is the root (the
+    free token x^{L+1} = root_tokens[b]); a node at depth d < gamma - 1 offers its next
+    unused candidate of position d + 1 as a child, scored score(node) + log q_{d+1}.
+    Each of ``budget`` steps takes the best offered child (equal scores: the lower
+    parent index) as the next node. Since scores only fall along a path, the nodes are
+    the top ``budget`` prefixes and every node's parent precedes it.
+
+    Returns a dict: tokens, parents, depth (int32 [batch][budget+1]), mask (uint64
+    [batch][budget+1]: bit i of node j set iff node i is j or an ancestor of j), score
+    (fp64), margin (fp64 [batch]: the smallest gap between the taken child's score and
+    the best other offer over all steps; +inf if there never was another offer).
+    """
+    dl = _rows_f64(drafter_logits)
+    B, G, V = dl.shape
+    N = budget + 1
+    if N > 64:
+        raise ValueError("a tree holds at most 64 nodes")
+    out = dict(tokens=np.full((B, N), -1, np.int32), parents=np.full((B, N), -1, np.int32),
+               depth=np.zeros((B, N), np.int32), mask=np.zeros((B, N), np.uint64),
+               score=np.zeros((B, N), np.float64), margin=np.full(B, np.inf))
+    for b in range(B):
+        T = float(np.float32(temperature[b]))
+        T = T if T > 0 else 1.0
+        logq, top = [None], [None]
+        for d in range(1, G):
+            z = dl[b, d] / T
+            m = z.max()
+            lq = z - m - np.log(np.exp(z - m).sum())
+            order = sorted(range(V), key=lambda x: (-lq[x], x))[:min(top_k, V)]
+            logq.append(lq)
+            top.append(order)
+        tokens, parents, depth, score = [int(root_tokens[b])], [-1], [0], [0.0]
+        nxt = [0]
+        margin = np.inf
+        for _ in range(budget):
+            offers = []
+            for u in range(len(tokens)):
+                d = depth[u] + 1
+                if d < G and nxt[u] < len(top[d]):
+                    c = top[d][nxt[u]]
+                    offers.append((score[u] + logq[d][c], u, c))
+            if not offers:
+                raise ValueError("the tree ran out of candidates before the budget")
+            best = max(offers, key=lambda o: (o[0], -o[1]))
+            others = [o[0] for o in offers if o is not best]
+            if others:
+                margin = min(margin, best[0] - max(others))
+            sc, u, c = best
+            tokens.append(c)
+            parents.append(u)
+            depth.append(depth[u] + 1)
+            score.append(sc)
+            nxt[u] += 1
+            nxt.append(0)
+        for j in range(N):
+            bits, a = 0, j
+            while a >= 0:
+                bits |= 1 << a
+                a = parents[a]
+            out["mask"][b, j] = np.uint64(bits)
+        out["tokens"][b] = tokens
+        out["parents"][b] = parents
+        out["depth"][b] = depth
+        out["score"][b] = score
+        out["margin"][b] = margin
+    return out
+
+
+def accept_tree_greedy(target_logits, tokens, parents):
+    """Greedy (T = 0) verification of a candidate tree: from the root, move to the child
+    whose token is the lowest-index argmax of the current node's target row (children
+    in node order); stop when there is none, and emit that argmax as the final token.
+    target row j is the verifier's distribution of the token after node j.
+
+    Returns a dict: path (int32 [batch][N], node indices, -1 padded), num_accepted
+    (path length - 1), out_tokens (int32 [batch][N+1]: the path's tokens, then the final
+    token, -1 padded), num_emitted (path length + 1)."""
+    tl = _rows_f64(target_logits)
+    B, N, V = tl.shape
+    path = np.full((B, N), -1, np.int32)
+    out = np.full((B, N + 1), -1, np.int32)
+    na = np.zeros(B, np.int32)
+    ne = np.zeros(B, np.int32)
+    for b in range(B):
+        cur, walk = 0, [0]
+        while True:
+            a = int(np.argmax(tl[b, cur]))
+            nxt = next((c for c in range(N) if parents[b, c] == cur and tokens[b, c] == a), None)
+            if nxt is None:
+                break
+            walk.append(nxt)
+            cur = nxt
+        path[b, :len(walk)] = walk
+        toks = [int(tokens[b, x]) for x in walk] + [int(np.argmax(tl[b, cur]))]
+        out[b, :len(toks)] = toks
+        na[b] = len(walk) - 1
+        ne[b] = len(walk) + 1
+    return dict(path=path, num_accepted=na, out_tokens=out, num_emitted=ne)
+
+
+def compact_tree_kv(k_cache, v_cache, page_table, kv_len, num_nodes: int, path, num_accepted):
+    """Keep the accepted path of a verified tree in the paged KV cache: the block's node
+    keys sit at positions ctx .. ctx + num_nodes - 1 (kv_len = ctx + num_nodes); the key
+    and value of path node path[d] move to position ctx + d for d = 1 .. n - 1
+    (n = num_accepted + 1; the root stays at ctx), and kv_len becomes ctx + n (ctx when
+    num_accepted = -1). Returns new (k_cache, v_cache, kv_len)."""
+    k = np.array(k_cache, copy=True)
+    v = np.array(v_cache, copy=True)
+    kl = np.array(kv_len, dtype=np.int32, copy=True)
+    P = k.shape[2]
+    for b in range(len(kl)):
+        ctx = int(kv_len[b]) - num_nodes
+        n = int(num_accepted[b]) + 1 if num_accepted[b] >= 0 else 0
+        for d in range(1, n):
+            src, dst = ctx + int(path[b, d]), ctx + d
+            ps, pd = page_table[b, src // P], page_table[b, dst // P]
+            k[pd, :, dst % P] = k[ps, :, src % P]
+            v[pd, :, dst % P] = v[ps, :, src % P]
+        kl[b] = ctx + n
+    return k, v, kl
+
+
 def verify_attention(q, k_cache, v_cache, page_table, kv_len, gamma: int, softmax_scale=None,
-                     rows=None, nthreads: int = 0):
+                     rows=None, nthreads: int = 0, tree_mask=None):
     """fp64 block-causal paged GQA attention.
 
     q: uint16 bf16 bits [batch][gamma][Hq][D]; k_cache, v_cache: uint16
     [num_pages][Hkv][page_size][D]; page_table: int32 [batch][max_pages];
     kv_len: int32 [batch].  rows: optional int array [n][3] of (b, j, h) to compute.
+    tree_mask: optional uint64 [batch][gamma]: block query j sees the block keys whose
+    bits are set (tree attention) instead of the first j + 1.
     Returns (out fp64 [batch][gamma][Hq][D], lse fp64 [batch][gamma][Hq], status).
     Rows not listed in ``rows`` are left NaN.
     """
@@ -435,10 +577,11 @@ def verify_attention(q, k_cache, v_cache, page_table, kv_len, gamma: int, softma
     if rows is not None:
         r = _c(rows, np.int32).reshape(-1, 3)
         nrows = r.shape[0]
-    rc = lib.oracle_verify_attention(batch, gamma, Hq, Hkv, D, page_size, pt.shape[1], num_pages,
-                                     scale, _ptr(qa), _ptr(ka), _ptr(va), _ptr(pt), _ptr(kl),
-                                     _ptr(out), _ptr(lse), _ptr(r), nrows, _ptr(st),
-                                     int(nthreads))
+    tm = None if tree_mask is None else _c(tree_mask, np.uint64)
+    rc = lib.oracle_verify_attention_tree(batch, gamma, Hq, Hkv, D, page_size, pt.shape[1],
+                                          num_pages, scale, _ptr(qa), _ptr(ka), _ptr(va),
+                                          _ptr(pt), _ptr(kl), _ptr(tm), _ptr(out), _ptr(lse),
+                                          _ptr(r), nrows, _ptr(st), int(nthreads))
     if rc:
         raise ValueError("invalid arguments to oracle_verify_attention")
     return out, lse, st

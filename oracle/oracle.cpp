@@ -555,13 +555,21 @@ int oracle_sample_block(int32_t batch, int32_t gamma, int64_t vocab, int32_t dty
 // A sequence whose kv_len is outside [gamma, max_pages * page_size] or that maps a
 // visible key to a page id outside [0, num_pages) gets out = 0, lse = -inf and
 // status[b] = 1 (status may be NULL).
-int oracle_verify_attention(int32_t batch, int32_t gamma, int32_t num_q_heads,
-                            int32_t num_kv_heads, int32_t head_dim, int32_t page_size,
-                            int32_t max_pages_per_seq, int32_t num_pages, double softmax_scale,
-                            const uint16_t* q, const uint16_t* k_cache, const uint16_t* v_cache,
-                            const int32_t* page_table, const int32_t* kv_len, double* out,
-                            double* lse, const int32_t* rows, int64_t nrows, int32_t* status,
-                            int32_t nthreads) {
+//
+// tree_mask (may be NULL): [batch][gamma] bit sets for tree verification (Sec. 4.2: for
+// more than one candidate the block is verified "as a prefix tree using tree
+// attention"). Block query j then sees the prefix keys k < ctx and the block keys
+// ctx + i for every bit i set in tree_mask[b][j] (its ancestors and itself), instead
+// of every k <= ctx + j. gamma <= 64 with a mask.
+int oracle_verify_attention_tree(int32_t batch, int32_t gamma, int32_t num_q_heads,
+                                 int32_t num_kv_heads, int32_t head_dim, int32_t page_size,
+                                 int32_t max_pages_per_seq, int32_t num_pages,
+                                 double softmax_scale, const uint16_t* q, const uint16_t* k_cache,
+                                 const uint16_t* v_cache, const int32_t* page_table,
+                                 const int32_t* kv_len, const uint64_t* tree_mask, double* out,
+                                 double* lse, const int32_t* rows, int64_t nrows, int32_t* status,
+                                 int32_t nthreads) {
+  if (tree_mask && gamma > 64) return -1;
   if (batch < 0 || gamma < 1 || num_q_heads < 1 || num_kv_heads < 1 ||
       num_q_heads % num_kv_heads != 0 || head_dim < 1 || page_size < 1)
     return -1;
@@ -601,7 +609,15 @@ int oracle_verify_attention(int32_t batch, int32_t gamma, int32_t num_q_heads,
     }
     const int32_t g = h / group;
     const int32_t ctx = kv_len[b] - gamma;
-    const int32_t nvis = ctx + j + 1;
+    // the visible keys, in increasing order
+    std::vector<int32_t> vis;
+    for (int32_t k = 0; k < ctx; ++k) vis.push_back(k);
+    for (int32_t i = 0; i < gamma; ++i) {
+      const bool seen = tree_mask ? ((tree_mask[static_cast<int64_t>(b) * gamma + j] >> i) & 1u) != 0
+                                  : i <= j;
+      if (seen) vis.push_back(ctx + i);
+    }
+    const int32_t nvis = static_cast<int32_t>(vis.size());
     std::vector<double> qv(D), s(nvis);
     for (int32_t d = 0; d < D; ++d) qv[d] = bf16_bits_to_double(q[orow * D + d]);
     auto kv_offset = [&](int32_t k) {
@@ -610,7 +626,7 @@ int oracle_verify_attention(int32_t batch, int32_t gamma, int32_t num_q_heads,
     };
     double m = -kInf;
     for (int32_t k = 0; k < nvis; ++k) {
-      const int64_t off = kv_offset(k);
+      const int64_t off = kv_offset(vis[k]);
       double dot = 0.0;
       for (int32_t d = 0; d < D; ++d) dot += qv[d] * bf16_bits_to_double(k_cache[off + d]);
       s[k] = dot * softmax_scale;
@@ -623,7 +639,7 @@ int oracle_verify_attention(int32_t batch, int32_t gamma, int32_t num_q_heads,
     }
     std::vector<double> acc(D, 0.0);  // local: a row listed twice is computed twice
     for (int32_t k = 0; k < nvis; ++k) {
-      const int64_t off = kv_offset(k);
+      const int64_t off = kv_offset(vis[k]);
       const double pk = s[k] / l;
       for (int32_t d = 0; d < D; ++d) acc[d] += pk * bf16_bits_to_double(v_cache[off + d]);
     }
@@ -631,6 +647,19 @@ int oracle_verify_attention(int32_t batch, int32_t gamma, int32_t num_q_heads,
     if (lse) lse[orow] = m + std::log(l);
   });
   return 0;
+}
+
+int oracle_verify_attention(int32_t batch, int32_t gamma, int32_t num_q_heads,
+                            int32_t num_kv_heads, int32_t head_dim, int32_t page_size,
+                            int32_t max_pages_per_seq, int32_t num_pages, double softmax_scale,
+                            const uint16_t* q, const uint16_t* k_cache, const uint16_t* v_cache,
+                            const int32_t* page_table, const int32_t* kv_len, double* out,
+                            double* lse, const int32_t* rows, int64_t nrows, int32_t* status,
+                            int32_t nthreads) {
+  return oracle_verify_attention_tree(batch, gamma, num_q_heads, num_kv_heads, head_dim,
+                                      page_size, max_pages_per_seq, num_pages, softmax_scale, q,
+                                      k_cache, v_cache, page_table, kv_len, nullptr, out, lse,
+                                      rows, nrows, status, nthreads);
 }
 
 }  // extern "C"
