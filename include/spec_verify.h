@@ -76,6 +76,7 @@ typedef enum {
 #define SPEC_FLAG_BAD_KV_LEN 0x8u  /* kv_len outside [gamma, max_pages_per_seq * page_size] */
 #define SPEC_FLAG_TIMEOUT 0x10u    /* a bounded internal wait ran out                        */
 #define SPEC_FLAG_BAD_FILTER 0x20u /* a tempered sequence's top_k or top_p out of range       */
+#define SPEC_FLAG_BAD_TREE 0x40u   /* a candidate tree whose parents are not a tree          */
 
 /*
  * Part (a): block-causal verify attention (Sec. 4.1: the block [x^{L+1}, z] is
@@ -91,6 +92,13 @@ typedef enum {
  * Logical key k lives in physical page page_table[b][k / page_size], slot
  * k % page_size. Accumulation is fp32; out is rounded to bf16.
  * A sequence flagged BAD_PAGE or BAD_KV_LEN gets out = 0 and lse = -inf.
+ *
+ * Tree attention (Sec. 4.2: several candidates are verified in one pass, arranged as a
+ * prefix tree under tree attention): with tree_mask set, the gamma block positions are
+ * the nodes of a candidate tree, and block query j sees the prefix keys k < ctx_b and
+ * the block keys ctx_b + i for every bit i set in tree_mask[b][j] (itself and its
+ * ancestors) instead of every k <= ctx_b + j. A mask with bits 0..j set is the causal
+ * block. Device memory, caller-owned; gamma <= 64.
  */
 typedef struct {
   int32_t batch;              /* >= 1                                                       */
@@ -110,6 +118,7 @@ typedef struct {
   const int32_t* kv_len;      /* [batch]                                                    */
   void* out;                  /* bf16 [batch][gamma][Hq][D]                                 */
   float* lse;                 /* fp32 [batch][gamma][Hq], or NULL                           */
+  const uint64_t* tree_mask;  /* [batch][gamma], or NULL: tree attention (below)           */
 } spec_attn_args_t;
 
 /*
@@ -314,6 +323,66 @@ typedef struct {
 } spec_commit_args_t;
 
 spec_status_t spec_commit_kv(const spec_commit_args_t* commit, spec_stream_t stream);
+
+/*
+ * Tree verification (Sec. 4.2: several candidates verified at once as a prefix tree;
+ * Sec. 3.3, "Tree Sampler"), greedy (T = 0).
+ *
+ * A candidate tree of num_nodes <= 64 nodes per sequence: node 0 is the root (the free
+ * token x^{L+1}); parents[b][c] < c is node c's parent (-1 for the root); tokens[b][c]
+ * is its token. The verify pass runs on the nodes as the block (spec_verify_attention
+ * with tree_mask = each node's ancestor bits); target row c (target_logits
+ * [batch][num_nodes][vocab]) is the verifier's distribution of the token after node c.
+ *
+ * spec_accept_tree: from the root, move to the child (lowest node index first) whose
+ * token is the lowest-index argmax of the current node's target row; stop where there
+ * is none. path[b] = the visited nodes (-1 padded), out_tokens[b] = their tokens then
+ * that argmax (-1 padded, num_nodes + 1 entries), num_accepted = path length - 1,
+ * num_emitted = path length + 1. A sequence with a token outside [0, vocab), parents
+ * that are not a tree (SPEC_FLAG_BAD_TREE), or a NaN in a target row gets
+ * num_accepted = -1, num_emitted = 0 and -1 outputs. Sampled (T > 0) tree verification
+ * is not provided: the paper's tree takes the top K tokens per position, and it states
+ * no lossless rule for such candidate sets.
+ */
+typedef struct {
+  int32_t batch, num_nodes, vocab, logits_dtype;
+  const void* target_logits;   /* [batch][num_nodes][vocab]                                */
+  const int32_t* tokens;       /* [batch][num_nodes]                                       */
+  const int32_t* parents;      /* [batch][num_nodes]                                       */
+  int32_t* path;               /* [batch][num_nodes], written                              */
+  int32_t* num_accepted;       /* [batch], written                                         */
+  int32_t* out_tokens;         /* [batch][num_nodes + 1], written                          */
+  int32_t* num_emitted;        /* [batch], written                                         */
+} spec_tree_accept_args_t;
+
+size_t spec_tree_workspace_size(const spec_tree_accept_args_t* tree);
+spec_status_t spec_accept_tree(const spec_tree_accept_args_t* tree, void* ws, size_t ws_bytes,
+                               spec_stream_t stream);
+
+/*
+ * After spec_accept_tree: keep the accepted path in the paged KV cache. The nodes' keys
+ * sit at positions ctx_b .. ctx_b + num_nodes - 1 (kv_len[b] = ctx_b + num_nodes); the
+ * key and value rows (every KV head) of path node path[b][d] move to position ctx_b + d
+ * for d = 1 .. num_accepted[b], and kv_len[b] becomes ctx_b + num_accepted[b] + 1
+ * (ctx_b when num_accepted[b] = -1). The result is that of moving the rows one by one
+ * in increasing d. A sequence with kv_len[b] outside [num_nodes, max_pages_per_seq *
+ * page_size] (SPEC_FLAG_BAD_KV_LEN), num_accepted outside [-1, num_nodes) or a path that
+ * does not start at node 0 and rise strictly below num_nodes (SPEC_FLAG_BAD_TREE), or a
+ * moved row's page id outside [0, num_pages) (SPEC_FLAG_BAD_PAGE) is left unchanged,
+ * kv_len included, and the flag is set in *status (if given). Two launches, no workspace.
+ */
+typedef struct {
+  int32_t batch, num_nodes, num_kv_heads, head_dim, page_size, max_pages_per_seq, num_pages;
+  void* k_cache;                /* bf16 [num_pages][Hkv][page_size][D], updated              */
+  void* v_cache;                /* bf16, same layout, updated                                */
+  const int32_t* page_table;    /* [batch][max_pages_per_seq]                               */
+  int32_t* kv_len;              /* [batch], updated                                          */
+  const int32_t* path;          /* [batch][num_nodes] from spec_accept_tree                 */
+  const int32_t* num_accepted;  /* [batch] from spec_accept_tree                            */
+  uint32_t* status;             /* a status word (e.g. a workspace's first word), or NULL   */
+} spec_tree_commit_args_t;
+
+spec_status_t spec_commit_tree_kv(const spec_tree_commit_args_t* commit, spec_stream_t stream);
 
 /*
  * spec_accept_block without a workspace, for callers that cannot allocate device

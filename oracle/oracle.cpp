@@ -556,9 +556,8 @@ int oracle_sample_block(int32_t batch, int32_t gamma, int64_t vocab, int32_t dty
 // visible key to a page id outside [0, num_pages) gets out = 0, lse = -inf and
 // status[b] = 1 (status may be NULL).
 //
-// tree_mask (may be NULL): [batch][gamma] bit sets for tree verification (Sec. 4.2: for
-// more than one candidate the block is verified "as a prefix tree using tree
-// attention"). Block query j then sees the prefix keys k < ctx and the block keys
+// tree_mask (may be NULL): [batch][gamma] bit sets for tree verification (Sec. 4.2:
+// several candidates verified in one pass as a prefix tree). Block query j then sees the prefix keys k < ctx and the block keys
 // ctx + i for every bit i set in tree_mask[b][j] (its ancestors and itself), instead
 // of every k <= ctx + j. gamma <= 64 with a mask.
 int oracle_verify_attention_tree(int32_t batch, int32_t gamma, int32_t num_q_heads,

@@ -29,6 +29,7 @@ SPEC_F32, SPEC_BF16 = 0, 1
 ATTN_AUTO, ATTN_CUDA_CORES, ATTN_TENSOR_CORES = 0, 1, 2
 FLAG_BAD_TOKEN, FLAG_BAD_LOGITS, FLAG_BAD_PAGE, FLAG_BAD_KV_LEN, FLAG_TIMEOUT = 1, 2, 4, 8, 16
 FLAG_BAD_FILTER = 32
+FLAG_BAD_TREE = 64
 FILTER_MAX_TOP_K = 1024
 
 
@@ -46,7 +47,8 @@ class AttnArgs(ctypes.Structure):
                 ("softmax_scale", ctypes.c_float), ("path", ctypes.c_int32),
                 ("q", ctypes.c_void_p), ("k_cache", ctypes.c_void_p),
                 ("v_cache", ctypes.c_void_p), ("page_table", ctypes.c_void_p),
-                ("kv_len", ctypes.c_void_p), ("out", ctypes.c_void_p), ("lse", ctypes.c_void_p)]
+                ("kv_len", ctypes.c_void_p), ("out", ctypes.c_void_p), ("lse", ctypes.c_void_p),
+                ("tree_mask", ctypes.c_void_p)]
 
 
 class AcceptArgs(ctypes.Structure):
@@ -77,6 +79,25 @@ class CommitArgs(ctypes.Structure):
                 ("page_table", ctypes.c_void_p), ("free_pages", ctypes.c_void_p),
                 ("free_count", ctypes.c_void_p), ("free_capacity", ctypes.c_int32),
                 ("reserve", ctypes.c_int32), ("flags", ctypes.c_void_p)]
+
+
+class TreeAcceptArgs(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int32), ("num_nodes", ctypes.c_int32),
+                ("vocab", ctypes.c_int32), ("logits_dtype", ctypes.c_int32),
+                ("target_logits", ctypes.c_void_p), ("tokens", ctypes.c_void_p),
+                ("parents", ctypes.c_void_p), ("path", ctypes.c_void_p),
+                ("num_accepted", ctypes.c_void_p), ("out_tokens", ctypes.c_void_p),
+                ("num_emitted", ctypes.c_void_p)]
+
+
+class TreeCommitArgs(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int32), ("num_nodes", ctypes.c_int32),
+                ("num_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
+                ("page_size", ctypes.c_int32), ("max_pages_per_seq", ctypes.c_int32),
+                ("num_pages", ctypes.c_int32), ("k_cache", ctypes.c_void_p),
+                ("v_cache", ctypes.c_void_p), ("page_table", ctypes.c_void_p),
+                ("kv_len", ctypes.c_void_p), ("path", ctypes.c_void_p),
+                ("num_accepted", ctypes.c_void_p), ("status", ctypes.c_void_p)]
 
 
 HEADER = os.path.join(_build.ROOT, "include", "spec_verify.h")
@@ -127,6 +148,12 @@ def lib(build_if_missing: bool = True):
             L.spec_noise_tokens.restype = ctypes.c_int
             L.spec_commit_kv.argtypes = [P, P]
             L.spec_commit_kv.restype = ctypes.c_int
+            L.spec_tree_workspace_size.argtypes = [P]
+            L.spec_tree_workspace_size.restype = ctypes.c_size_t
+            L.spec_accept_tree.argtypes = [P, P, ctypes.c_size_t, P]
+            L.spec_accept_tree.restype = ctypes.c_int
+            L.spec_commit_tree_kv.argtypes = [P, P]
+            L.spec_commit_tree_kv.restype = ctypes.c_int
             for f in ("spec_workspace_init", "spec_verify_attention", "spec_accept_block",
                       "spec_verify_step", "spec_philox_uniforms", "spec_read_device_status"):
                 getattr(L, f).restype = ctypes.c_int
@@ -160,7 +187,7 @@ def _raise(code: int, what: str):
 
 
 def attn_args(q, k_cache, v_cache, page_table, kv_len, out, lse=None, softmax_scale=0.0,
-              path=ATTN_AUTO) -> AttnArgs:
+              path=ATTN_AUTO, tree_mask=None) -> AttnArgs:
     B, G, Hq, D = q.shape
     num_pages, Hkv, P, D2 = k_cache.shape
     _check(q, "q", torch.bfloat16)
@@ -171,12 +198,15 @@ def attn_args(q, k_cache, v_cache, page_table, kv_len, out, lse=None, softmax_sc
     _check(out, "out", torch.bfloat16, q.shape)
     if lse is not None:
         _check(lse, "lse", torch.float32, (B, G, Hq))
+    if tree_mask is not None:
+        _check(tree_mask, "tree_mask", torch.int64, (B, G))
     if D2 != D or page_table.dim() != 2 or page_table.shape[0] != B:
         raise ValueError("inconsistent attention shapes")
     return AttnArgs(B, G, Hq, Hkv, D, P, page_table.shape[1], num_pages, float(softmax_scale),
                     int(path), q.data_ptr(), k_cache.data_ptr(), v_cache.data_ptr(),
                     page_table.data_ptr(), kv_len.data_ptr(), out.data_ptr(),
-                    None if lse is None else lse.data_ptr())
+                    None if lse is None else lse.data_ptr(),
+                    None if tree_mask is None else tree_mask.data_ptr())
 
 
 def accept_args(target_logits, drafter_logits, block_tokens, temperature, uniforms, num_accepted,
@@ -235,11 +265,12 @@ def verify_step_args(attn: Optional[AttnArgs], acc: Optional[AcceptArgs], ws: to
 
 
 def verify_attention(q, k_cache, v_cache, page_table, kv_len, softmax_scale=0.0, path=ATTN_AUTO,
-                     want_lse=True, ws=None, stream=None):
-    """Block-causal paged GQA verify attention. Returns (out bf16, lse fp32 or None)."""
+                     want_lse=True, ws=None, stream=None, tree_mask=None):
+    """Block-causal (or, with tree_mask, tree) paged GQA verify attention. Returns
+    (out bf16, lse fp32 or None). tree_mask: int64 [batch][gamma] bit sets."""
     out = torch.empty_like(q)
     lse = torch.empty(q.shape[:3], dtype=torch.float32, device=q.device) if want_lse else None
-    a = attn_args(q, k_cache, v_cache, page_table, kv_len, out, lse, softmax_scale, path)
+    a = attn_args(q, k_cache, v_cache, page_table, kv_len, out, lse, softmax_scale, path, tree_mask)
     if ws is None:
         ws = new_workspace(workspace_size(attn=a), q.device)
     verify_attention_args(a, ws, stream)
@@ -402,6 +433,69 @@ def commit_kv(kv_len, num_accepted, page_table, page_size: int, gamma: int, free
                    free_pages.numel(), 1 if reserve else 0,
                    None if flags is None else flags.data_ptr())
     _raise(lib().spec_commit_kv(ctypes.byref(a), _stream(stream)), "spec_commit_kv")
+
+
+def tree_accept_args(target_logits, tokens, parents, path, num_accepted, out_tokens,
+                     num_emitted) -> TreeAcceptArgs:
+    B, N, V = target_logits.shape
+    if target_logits.dtype == torch.bfloat16:
+        dt = SPEC_BF16
+    elif target_logits.dtype == torch.float32:
+        dt = SPEC_F32
+    else:
+        raise TypeError("logits must be bfloat16 or float32")
+    _check(target_logits, "target_logits", target_logits.dtype)
+    for t, name, shape in ((tokens, "tokens", (B, N)), (parents, "parents", (B, N)),
+                           (path, "path", (B, N)), (num_accepted, "num_accepted", (B,)),
+                           (out_tokens, "out_tokens", (B, N + 1)), (num_emitted, "num_emitted", (B,))):
+        _check(t, name, torch.int32, shape)
+    return TreeAcceptArgs(B, N, V, dt, target_logits.data_ptr(), tokens.data_ptr(),
+                          parents.data_ptr(), path.data_ptr(), num_accepted.data_ptr(),
+                          out_tokens.data_ptr(), num_emitted.data_ptr())
+
+
+def accept_tree_args(t: TreeAcceptArgs, ws: torch.Tensor, stream=None):
+    _raise(lib().spec_accept_tree(ctypes.byref(t), _ptr(ws), ws.numel(), _stream(stream)),
+           "spec_accept_tree")
+
+
+def accept_tree(target_logits, tokens, parents, ws=None, stream=None) -> Dict[str, torch.Tensor]:
+    """Greedy verification of a candidate tree (spec_accept_tree). Returns path,
+    num_accepted, out_tokens, num_emitted."""
+    B, N, _ = target_logits.shape
+    dev = target_logits.device
+    res = dict(path=torch.empty(B, N, dtype=torch.int32, device=dev),
+               num_accepted=torch.empty(B, dtype=torch.int32, device=dev),
+               out_tokens=torch.empty(B, N + 1, dtype=torch.int32, device=dev),
+               num_emitted=torch.empty(B, dtype=torch.int32, device=dev))
+    t = tree_accept_args(target_logits, tokens, parents, res["path"], res["num_accepted"],
+                         res["out_tokens"], res["num_emitted"])
+    if ws is None:
+        n = lib().spec_tree_workspace_size(ctypes.byref(t))
+        if n == 0:
+            raise SpecError(1, "spec_tree_workspace_size")
+        ws = new_workspace(n, dev)
+    accept_tree_args(t, ws, stream)
+    return res
+
+
+def commit_tree_kv(k_cache, v_cache, page_table, kv_len, path, num_accepted, status_ws=None,
+                   stream=None):
+    """spec_commit_tree_kv: move the accepted path's keys and values into place and
+    shorten kv_len (k_cache, v_cache and kv_len are updated in place)."""
+    num_pages, Hkv, P, D = k_cache.shape
+    B, N = path.shape
+    _check(k_cache, "k_cache", torch.bfloat16)
+    _check(v_cache, "v_cache", torch.bfloat16, k_cache.shape)
+    _check(page_table, "page_table", torch.int32)
+    _check(kv_len, "kv_len", torch.int32, (B,))
+    _check(path, "path", torch.int32)
+    _check(num_accepted, "num_accepted", torch.int32, (B,))
+    a = TreeCommitArgs(B, N, Hkv, D, P, page_table.shape[1], num_pages, k_cache.data_ptr(),
+                       v_cache.data_ptr(), page_table.data_ptr(), kv_len.data_ptr(),
+                       path.data_ptr(), num_accepted.data_ptr(),
+                       None if status_ws is None else status_ws.data_ptr())
+    _raise(lib().spec_commit_tree_kv(ctypes.byref(a), _stream(stream)), "spec_commit_tree_kv")
 
 
 def philox_uniforms(seed: int, n: int, offset: int = 0, device=None, stream=None) -> torch.Tensor:

@@ -121,6 +121,17 @@ size_t draft_bytes(const spec_draft_args_t& d, const spec_filter_args_t* f, int 
   return draft_layout(d, kWsHeader, sms, vec).end;
 }
 
+spec_status_t check_tree(const spec_tree_accept_args_t* t) {
+  if (!t) return SPEC_ERR_INVALID_ARGUMENT;
+  if (t->batch < 1 || t->num_nodes < 1 || t->vocab < 1) return SPEC_ERR_INVALID_ARGUMENT;
+  if (t->logits_dtype != SPEC_F32 && t->logits_dtype != SPEC_BF16) return SPEC_ERR_INVALID_ARGUMENT;
+  if (!t->target_logits || !t->tokens || !t->parents || !t->path || !t->num_accepted ||
+      !t->out_tokens || !t->num_emitted)
+    return SPEC_ERR_INVALID_ARGUMENT;
+  if (t->num_nodes > 64 || t->batch > 65535) return SPEC_ERR_UNSUPPORTED;
+  return SPEC_OK;
+}
+
 spec_status_t check_filter(const spec_filter_args_t* f) {
   if (!f || !f->top_k || !f->top_p) return SPEC_ERR_INVALID_ARGUMENT;
   if (f->max_top_k < 1) return SPEC_ERR_INVALID_ARGUMENT;
@@ -377,6 +388,59 @@ spec_status_t spec_sample_block(const spec_draft_args_t* draft, const spec_filte
   }
   const DraftLayout L = draft_layout(*draft, kWsHeader, sms, vec);
   return launch_draft(*draft, L, w, stream, vec) == cudaSuccess ? SPEC_OK : SPEC_ERR_CUDA;
+}
+
+size_t spec_tree_workspace_size(const spec_tree_accept_args_t* t) {
+  if (check_tree(t) != SPEC_OK) return 0;
+  int dev = 0, sms = 160;
+  if (cudaGetDevice(&dev) == cudaSuccess) {
+    const int n = device_sm_count(dev);
+    if (n > sms) sms = n;
+  } else {
+    cudaGetLastError();
+  }
+  size_t need = 0;
+  for (int s : {148, 152, sms})
+    for (bool vec : {false, true}) {
+      const size_t x = tree_layout(t->batch, t->num_nodes, t->vocab, kWsHeader, s, vec).end;
+      if (x > need) need = x;
+    }
+  return need;
+}
+
+spec_status_t spec_accept_tree(const spec_tree_accept_args_t* t, void* ws, size_t ws_bytes,
+                               spec_stream_t stream_) {
+  const spec_status_t st = check_tree(t);
+  if (st != SPEC_OK) return st;
+  if (!ws || (reinterpret_cast<uintptr_t>(ws) % kWsAlign) != 0) return SPEC_ERR_INVALID_ARGUMENT;
+  const size_t esz = t->logits_dtype == SPEC_BF16 ? 2 : 4;
+  const bool vec = (static_cast<size_t>(t->vocab) * esz) % 16 == 0 &&
+                   reinterpret_cast<uintptr_t>(t->target_logits) % 16 == 0;
+  if (tree_layout(t->batch, t->num_nodes, t->vocab, kWsHeader, 1, vec).end > ws_bytes)
+    return SPEC_ERR_WORKSPACE_TOO_SMALL;
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  int sms = 0;
+  if (!bind_device(stream, &sms)) return SPEC_ERR_CUDA;
+  const TreeLayout L = tree_layout(t->batch, t->num_nodes, t->vocab, kWsHeader, sms, vec);
+  if (L.end > ws_bytes) return SPEC_ERR_WORKSPACE_TOO_SMALL;
+  return launch_tree_greedy(*t, L, static_cast<char*>(ws), stream, vec) == cudaSuccess
+             ? SPEC_OK
+             : SPEC_ERR_CUDA;
+}
+
+spec_status_t spec_commit_tree_kv(const spec_tree_commit_args_t* c, spec_stream_t stream) {
+  if (!c || c->batch < 1 || c->num_nodes < 1 || c->num_nodes > 64 || c->num_kv_heads < 1 ||
+      c->page_size < 1 || c->max_pages_per_seq < 1 || c->num_pages < 1 || !c->k_cache ||
+      !c->v_cache || !c->page_table || !c->kv_len || !c->path || !c->num_accepted)
+    return SPEC_ERR_INVALID_ARGUMENT;
+  if (c->head_dim != 64 && c->head_dim != 128) return SPEC_ERR_UNSUPPORTED;
+  if ((reinterpret_cast<uintptr_t>(c->k_cache) | reinterpret_cast<uintptr_t>(c->v_cache)) & 15u)
+    return SPEC_ERR_INVALID_ARGUMENT;
+  if (c->batch > 65535) return SPEC_ERR_UNSUPPORTED;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  int sms = 0;
+  if (!bind_device(s, &sms)) return SPEC_ERR_CUDA;
+  return launch_tree_commit(*c, s) == cudaSuccess ? SPEC_OK : SPEC_ERR_CUDA;
 }
 
 spec_status_t spec_commit_kv(const spec_commit_args_t* c, spec_stream_t stream) {

@@ -32,6 +32,7 @@ struct AttnParams {
   float2* partial_ml;  // [slot][slot_rows] = (m, l); l = -1 marks a bad sequence
   int q_tma;           // tensor-core kernel: Q tiles arrive by TMA (else softmax warps load them)
   int unit_overhead;   // tensor-core kernel: tiles charged per unit start in the work list
+  const uint64_t* tree_mask;  // [batch][gamma] block keys each query sees, or NULL (causal)
 };
 
 inline AttnParams make_attn_params(const spec_attn_args_t& a, const AttnPlan& P, char* ws) {
@@ -66,6 +67,7 @@ inline AttnParams make_attn_params(const spec_attn_args_t& a, const AttnPlan& P,
   p.partial_ml = reinterpret_cast<float2*>(ws + P.partial_ml);
   p.q_tma = 0;
   p.unit_overhead = 0;
+  p.tree_mask = a.tree_mask;
   return p;
 }
 

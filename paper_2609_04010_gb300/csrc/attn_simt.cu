@@ -34,6 +34,7 @@ struct SimtSmem {
   float alpha[RT];
   float m[RT];
   float l[RT];
+  unsigned long long tmask[RT];  // tree attention: the block keys each row sees
   int bad;
   int last;
 };
@@ -111,6 +112,8 @@ __global__ void __launch_bounds__(NT) attn_simt_kernel(AttnParams p) {
   if (tid < RT) {
     sm.m[tid] = -INFINITY;
     sm.l[tid] = 0.f;
+    const int j = min(row0 + tid, p.rows - 1) / p.group;
+    sm.tmask[tid] = p.tree_mask ? p.tree_mask[static_cast<int64_t>(b) * p.gamma + j] : 0ull;
   }
   __syncthreads();
   const bool bad = sm.bad != 0;
@@ -174,7 +177,9 @@ __global__ void __launch_bounds__(NT) attn_simt_kernel(AttnParams p) {
       for (int i = 0; i < RT / 2; ++i) {
         const int r = hr + 2 * i;
         const int j = (row0 + r) / p.group;
-        const bool vis = r < nrows && key <= ctx + j;
+        const int rel = key - ctx;  // block position of the key (negative: the prefix)
+        const bool vis = r < nrows && (p.tree_mask ? (rel < 0 || (rel < 64 && ((sm.tmask[r] >> rel) & 1ull)))
+                                                   : key <= ctx + j);
         sm.s[r][kk] = vis ? acc[i] : -INFINITY;
       }
     }

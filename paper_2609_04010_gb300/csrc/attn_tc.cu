@@ -299,7 +299,8 @@ __device__ __forceinline__ int owner_of(int64_t t, int64_t total, int ctas) {
 // ---------------------------------------------------------------------------------
 // The kernel
 // ---------------------------------------------------------------------------------
-template <int D, int MT>
+// TREE: tree attention (a per-row mask over the block keys) instead of the causal block.
+template <int D, int MT, bool TREE>
 __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
                    const __grid_constant__ CUtensorMap tmap_v,
@@ -675,6 +676,9 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
       const bool has_next = has_more(s, t1, OVH);
       const RowOf ro = row_of(s);
       const int ctx = s.kv_len - p.gamma;
+      // tree attention: the block keys this row sees (one bit per block position)
+      const unsigned long long tmask =
+          TREE ? __ldg(p.tree_mask + static_cast<int64_t>(s.b) * p.gamma + (ro.real ? ro.j : 0)) : 0ull;
       float m = -INFINITY, l = 0.f;
       for (int k = 0; k < s.ntile; ++k) {
         const uint32_t x = it + k;
@@ -700,10 +704,21 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
         const int key0 = (s.tile0 + k) * TK + hf * KH;
         const int lim = ctx + ro.j - key0;  // keys c <= lim are visible
         float tmax = -INFINITY;
+        if (TREE) {
+          const int rel0 = key0 - ctx;  // block position of element 0 (negative: the prefix)
 #pragma unroll
-        for (int c = 0; c < KH; ++c) {
-          v[c] = c <= lim ? v[c] * p.scale_log2 : -INFINITY;
-          tmax = fmaxf(tmax, v[c]);
+          for (int c = 0; c < KH; ++c) {
+            const int rel = rel0 + c;
+            const bool vis = rel < 0 || (rel < 64 && ((tmask >> rel) & 1ull));
+            v[c] = vis ? v[c] * p.scale_log2 : -INFINITY;
+            tmax = fmaxf(tmax, v[c]);
+          }
+        } else {
+#pragma unroll
+          for (int c = 0; c < KH; ++c) {
+            v[c] = c <= lim ? v[c] * p.scale_log2 : -INFINITY;
+            tmax = fmaxf(tmax, v[c]);
+          }
         }
         const float m_new = fmaxf(m, tmax);
         const bool want = k > 0 && m_new > m + 8.f;
@@ -969,11 +984,11 @@ cudaError_t launch_typed(const spec_attn_args_t& a, const AttnPlan& P, char* ws,
   p.unit_overhead = units > P.grid ? Cf::UNIT_OVERHEAD : 0;
   if (!p.q_tma) mq = mk;  // unused
   const size_t smem = Cf::smem_bytes(a.batch);
-  cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel<D, MT>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+  auto kernel = a.tree_mask ? attn_tc_kernel<D, MT, true> : attn_tc_kernel<D, MT, false>;
+  cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  attn_tc_kernel<D, MT><<<P.grid, Cf::THREADS, smem, stream>>>(mk, mv, mq, p);
+  kernel<<<P.grid, Cf::THREADS, smem, stream>>>(mk, mv, mq, p);
   return cudaGetLastError();
 }
 

@@ -98,6 +98,21 @@ cudaError_t launch_draft(const spec_draft_args_t& a, const DraftLayout& L, char*
                          cudaStream_t stream, bool vec);
 cudaError_t launch_commit(const spec_commit_args_t& a, cudaStream_t stream);
 
+// --- tree verification ---
+struct TreeLayout {
+  size_t tickets;      // uint32 [batch]: node rows of the sequence finished
+  size_t row_tickets;  // uint32 [batch][nodes]: splits of the row finished
+  size_t parts;        // 16 B [batch][nodes][splits]
+  size_t argmax;       // int32 [batch][nodes]
+  size_t end;
+  int splits, elems_per_split;
+};
+
+TreeLayout tree_layout(int batch, int nodes, int vocab, size_t base, int sms, bool vec);
+cudaError_t launch_tree_greedy(const spec_tree_accept_args_t& a, const TreeLayout& L, char* ws,
+                               cudaStream_t stream, bool vec);
+cudaError_t launch_tree_commit(const spec_tree_commit_args_t& a, cudaStream_t stream);
+
 // --- attention ---
 struct AttnPlan {
   int path;          // SPEC_ATTN_CUDA_CORES or SPEC_ATTN_TENSOR_CORES

@@ -1,0 +1,226 @@
+"""GPU parity of tree verification with the oracle, through the C ABI: tree attention
+(spec_verify_attention with tree_mask, both kernels), greedy acceptance along a tree
+(spec_accept_tree) and the compaction of the accepted path (spec_commit_tree_kv).
+
+Attention within the tolerances of the block-causal tests; a causal mask reproduces the
+block-causal kernels bit for bit. Acceptance and compaction are integer results:
+bit-exact. Trees come from the oracle's tree sampler on synthetic drafter rows."""
+
+import numpy as np
+import pytest
+import torch
+
+from paper_2609_04010_gb300 import binding
+from paper_2609_04010_gb300 import workloads as W
+
+from helpers import bf16_dev, compare_attention, dev, logits_dev, sample_rows
+
+pytestmark = pytest.mark.gpu
+
+
+def tree_case(oracle_mod, seed, batch, budget, K, gamma_draft, vocab, dtype="bf16", agree=0.8):
+    """A tree built by the oracle from synthetic drafter rows, and target rows that often
+    agree with one of each node's children (so long accepted paths occur)."""
+    rng = np.random.default_rng(seed)
+    inp = W.make_accept_inputs(batch, gamma_draft, vocab, dtype, 3.0, 1.0, 1.0, seed=seed)
+    tree = oracle_mod.build_tree(inp.drafter_logits, inp.temperature, inp.block_tokens[:, 0], K,
+                                 budget)
+    N = budget + 1
+    tl32 = rng.standard_normal((batch, N, vocab)).astype(np.float32) * 3
+    for b in range(batch):
+        for j in range(N):
+            kids = [c for c in range(N) if tree["parents"][b, c] == j]
+            if kids and rng.random() < agree:
+                tl32[b, j, tree["tokens"][b, rng.choice(kids)]] = tl32[b, j].max() + 1.0
+    tl = W.f32_to_bf16_bits(tl32).reshape(tl32.shape) if dtype == "bf16" else tl32
+    return tree, tl
+
+
+def attn_tree_inputs(seed, batch, N, hq, hkv, D, P, ctx):
+    inp = W.make_attn_inputs(batch, N, hq, hkv, D, P, ctx, True, seed)
+    return inp
+
+
+@pytest.mark.parametrize("path", [binding.ATTN_TENSOR_CORES, binding.ATTN_CUDA_CORES])
+@pytest.mark.parametrize("N,hq,hkv,D,P,ctx,batch", [(33, 32, 8, 128, 16, 4096, 1),
+                                                    (61, 32, 8, 128, 16, 2000, 2),
+                                                    (17, 8, 8, 64, 64, (100, 900), 4)])
+def test_tree_attention(oracle_mod, path, N, hq, hkv, D, P, ctx, batch):
+    rng = np.random.default_rng(N * 7 + batch)
+    inp = attn_tree_inputs(N + batch, batch, N, hq, hkv, D, P, ctx)
+    masks = np.zeros((batch, N), np.uint64)
+    for b in range(batch):
+        par = [-1] + [int(rng.integers(max(0, j - 6), j)) for j in range(1, N)]
+        for j in range(N):
+            bits, a = 0, j
+            while a >= 0:
+                bits |= 1 << a
+                a = par[a]
+            masks[b, j] = np.uint64(bits)
+    q, k, v, pt, kl = (bf16_dev(inp.q), bf16_dev(inp.k_cache), bf16_dev(inp.v_cache),
+                       dev(inp.page_table), dev(inp.kv_len))
+    tm = dev(masks.view(np.int64))
+    out, lse = binding.verify_attention(q, k, v, pt, kl, path=path, tree_mask=tm)
+    torch.cuda.synchronize()
+    rows = sample_rows(inp, 200, seed=N)
+    # every node of the first sequence, head 0
+    rows = np.unique(np.concatenate([rows, np.array([[0, j, 0] for j in range(N)], np.int32)]), axis=0)
+    o_out, o_lse, _ = oracle_mod.verify_attention(inp.q, inp.k_cache, inp.v_cache, inp.page_table,
+                                                  inp.kv_len, N, rows=rows, tree_mask=masks)
+    compare_attention(out.float().cpu().numpy(), lse.cpu().numpy(), o_out, o_lse, rows)
+
+
+@pytest.mark.parametrize("path", [binding.ATTN_TENSOR_CORES, binding.ATTN_CUDA_CORES])
+def test_causal_mask_reproduces_block_attention(path):
+    inp = attn_tree_inputs(3, 2, 16, 32, 8, 128, 16, 1000)
+    N = 16
+    causal = np.array([[(1 << (j + 1)) - 1 for j in range(N)]] * 2, np.uint64)
+    args = (bf16_dev(inp.q), bf16_dev(inp.k_cache), bf16_dev(inp.v_cache), dev(inp.page_table),
+            dev(inp.kv_len))
+    a, la = binding.verify_attention(*args, path=path, tree_mask=dev(causal.view(np.int64)))
+    c, lc = binding.verify_attention(*args, path=path)
+    torch.cuda.synchronize()
+    assert torch.equal(a, c) and torch.equal(la, lc)
+
+
+def compare_tree_accept(g, o):
+    for k in ("path", "num_accepted", "out_tokens", "num_emitted"):
+        np.testing.assert_array_equal(g[k], o[k], err_msg=k)
+
+
+def gpu_accept_tree(tl, tree):
+    r = binding.accept_tree(logits_dev(tl), dev(tree["tokens"]), dev(tree["parents"]))
+    torch.cuda.synchronize()
+    return {k: v.cpu().numpy() for k, v in r.items()}
+
+
+@pytest.mark.parametrize("batch,budget,K,G,vocab,dtype", [(1, 32, 32, 16, 128256, "bf16"),
+                                                          (1, 60, 32, 16, 151936, "bf16"),
+                                                          (8, 32, 8, 8, 32000, "f32"),
+                                                          (16, 20, 4, 6, 5000, "bf16"),
+                                                          (3, 7, 2, 4, 33, "f32")])
+def test_tree_greedy_acceptance(oracle_mod, batch, budget, K, G, vocab, dtype):
+    tree, tl = tree_case(oracle_mod, budget + batch, batch, budget, K, G, vocab, dtype)
+    g = gpu_accept_tree(tl, tree)
+    o = oracle_mod.accept_tree_greedy(tl, tree["tokens"], tree["parents"])
+    compare_tree_accept(g, o)
+
+
+def test_tree_full_chain_and_root_only(oracle_mod):
+    # K = 1 makes the tree a chain; sequence 0's target follows it to the end (the longest
+    # path, num_accepted = N - 1), sequence 1's root row prefers a token no child has
+    # (num_accepted = 0), sequence 2 is a one-node tree
+    B, G, V, N = 3, 40, 1000, 33
+    inp = W.make_accept_inputs(B, G, V, "f32", 3.0, 1.0, 1.0, seed=5)
+    tree = oracle_mod.build_tree(inp.drafter_logits, inp.temperature, inp.block_tokens[:, 0], 1, N - 1)
+    assert np.array_equal(tree["parents"][0], np.arange(-1, N - 1))
+    tl = np.random.default_rng(5).standard_normal((B, N, V)).astype(np.float32)
+    for j in range(N - 1):
+        tl[0, j, tree["tokens"][0, j + 1]] = 10.0
+    tl[1, 0, (tree["tokens"][1, 1] + 1) % V] = 10.0
+    g = gpu_accept_tree(tl, tree)
+    o = oracle_mod.accept_tree_greedy(tl, tree["tokens"], tree["parents"])
+    compare_tree_accept(g, o)
+    assert list(o["num_accepted"][:2]) == [N - 1, 0]
+    one = gpu_accept_tree(tl[2:, :1].copy(), {k: tree[k][2:, :1].copy() for k in ("tokens", "parents")})
+    assert one["num_accepted"][0] == 0 and one["num_emitted"][0] == 1 + 1
+    assert one["out_tokens"][0, 1] == int(np.argmax(tl[2, 0]))
+
+
+def test_tree_acceptance_flags_bad_sequences(oracle_mod):
+    tree, tl = tree_case(oracle_mod, 9, 4, 10, 3, 5, 3000, "f32")
+    tree["parents"][1, 5] = 7           # a parent after its child
+    tree["tokens"][2, 3] = 3000         # a token outside the vocabulary
+    tl[3, 4, 11] = np.nan
+    ws = binding.new_workspace(1 << 20)
+    r = binding.accept_tree(logits_dev(tl), dev(tree["tokens"]), dev(tree["parents"]), ws=ws)
+    torch.cuda.synchronize()
+    code, flags = binding.read_device_status(ws)
+    assert flags & binding.FLAG_BAD_TREE and flags & binding.FLAG_BAD_TOKEN
+    assert flags & binding.FLAG_BAD_LOGITS
+    g = {k: v.cpu().numpy() for k, v in r.items()}
+    for b in (1, 2, 3):
+        assert g["num_accepted"][b] == -1 and g["num_emitted"][b] == 0
+        assert np.all(g["out_tokens"][b] == -1) and np.all(g["path"][b] == -1)
+    o = oracle_mod.accept_tree_greedy(tl[:1], tree["tokens"][:1], tree["parents"][:1])
+    np.testing.assert_array_equal(g["out_tokens"][0], o["out_tokens"][0])
+
+
+def commit_case(oracle_mod, inp, N, path, na, expect_flags=0):
+    k2, v2, kl2 = oracle_mod.compact_tree_kv(inp.k_cache, inp.v_cache, inp.page_table, inp.kv_len, N,
+                                             path, na)
+    dk, dv, dkl = bf16_dev(inp.k_cache), bf16_dev(inp.v_cache), dev(inp.kv_len)
+    ws = binding.new_workspace(1024)
+    binding.commit_tree_kv(dk, dv, dev(inp.page_table), dkl, dev(path), dev(na), status_ws=ws)
+    torch.cuda.synchronize()
+    assert binding.read_device_status(ws)[1] == expect_flags
+    np.testing.assert_array_equal(dkl.cpu().numpy(), kl2)
+    np.testing.assert_array_equal(dk.view(torch.int16).cpu().numpy().view(np.uint16), k2)
+    np.testing.assert_array_equal(dv.view(torch.int16).cpu().numpy().view(np.uint16), v2)
+
+
+@pytest.mark.parametrize("D,P", [(128, 16), (64, 64)])
+def test_tree_commit(oracle_mod, D, P):
+    rng = np.random.default_rng(61 + D)
+    batch, N = 6, 33
+    inp = attn_tree_inputs(61, batch, N, 32, 8, D, P, (40, 300))
+    path = np.full((batch, N), -1, np.int32)
+    na = np.array([5, -1, 12, 0, 5, 32], np.int32)
+    for b in range(batch):
+        n = na[b] + 1 if na[b] >= 0 else 0
+        if n:
+            path[b, :n] = np.concatenate([[0], np.sort(rng.choice(np.arange(1, N), n - 1, replace=False))])
+    # a source that is a later position's destination (slot 2 is read by position 1 and
+    # written by position 2), and the whole block kept
+    path[4, :6] = [0, 2, 3, 4, 5, 7]
+    path[5] = np.arange(N)
+    commit_case(oracle_mod, inp, N, path, na)
+
+
+def test_tree_commit_bad_inputs_leave_the_sequence(oracle_mod):
+    batch, N = 4, 9
+    inp = attn_tree_inputs(62, batch, N, 8, 8, 64, 16, 50)
+    path = np.tile(np.arange(N, dtype=np.int32), (batch, 1))
+    path[:, 1:4] = [[2, 5, 7]] * batch
+    na = np.array([3, 3, 3, 3], np.int32)
+    ok = np.array([True, False, False, True])
+    path[1, 2] = 1                   # not rising
+    inp.page_table[2, :] = 10 ** 6   # a page outside the cache
+    expect = oracle_mod.compact_tree_kv(inp.k_cache, inp.v_cache, inp.page_table, inp.kv_len, N,
+                                        np.where(ok[:, None], path, -1), np.where(ok, na, -1))
+    dk, dv, dkl = bf16_dev(inp.k_cache), bf16_dev(inp.v_cache), dev(inp.kv_len)
+    ws = binding.new_workspace(1024)
+    binding.commit_tree_kv(dk, dv, dev(inp.page_table), dkl, dev(path), dev(na), status_ws=ws)
+    torch.cuda.synchronize()
+    flags = binding.read_device_status(ws)[1]
+    assert flags == binding.FLAG_BAD_TREE | binding.FLAG_BAD_PAGE
+    kl = dkl.cpu().numpy()
+    np.testing.assert_array_equal(kl[ok], expect[2][ok])
+    np.testing.assert_array_equal(kl[~ok], inp.kv_len[~ok])
+    np.testing.assert_array_equal(dk.view(torch.int16).cpu().numpy().view(np.uint16), expect[0])
+
+
+def test_tree_step_end_to_end(oracle_mod):
+    # tree attention over the nodes, then greedy acceptance, then the compaction: the
+    # accepted tokens and the compacted cache match the oracle's chain of the same steps
+    batch, budget, K, G, V = 1, 32, 32, 16, 128256
+    N = budget + 1
+    tree, tl = tree_case(oracle_mod, 71, batch, budget, K, G, V)
+    inp = attn_tree_inputs(71, batch, N, 32, 8, 128, 16, 4096)
+    args = (bf16_dev(inp.q), bf16_dev(inp.k_cache), bf16_dev(inp.v_cache), dev(inp.page_table),
+            dev(inp.kv_len))
+    out, lse = binding.verify_attention(*args, tree_mask=dev(tree["mask"].view(np.int64)))
+    g = gpu_accept_tree(tl, tree)
+    o = oracle_mod.accept_tree_greedy(tl, tree["tokens"], tree["parents"])
+    compare_tree_accept(g, o)
+    dk, dv, dkl = args[1], args[2], args[4]
+    binding.commit_tree_kv(dk, dv, args[3], dkl, dev(g["path"]), dev(g["num_accepted"]))
+    torch.cuda.synchronize()
+    k2, v2, kl2 = oracle_mod.compact_tree_kv(inp.k_cache, inp.v_cache, inp.page_table, inp.kv_len,
+                                             N, o["path"], o["num_accepted"])
+    np.testing.assert_array_equal(dkl.cpu().numpy(), kl2)
+    np.testing.assert_array_equal(dk.view(torch.int16).cpu().numpy().view(np.uint16), k2)
+    rows = sample_rows(inp, 100, seed=3)
+    o_out, o_lse, _ = oracle_mod.verify_attention(inp.q, inp.k_cache, inp.v_cache, inp.page_table,
+                                                  inp.kv_len, N, rows=rows, tree_mask=tree["mask"])
+    compare_attention(out.float().cpu().numpy(), lse.cpu().numpy(), o_out, o_lse, rows)
