@@ -385,6 +385,45 @@ typedef struct {
 spec_status_t spec_commit_tree_kv(const spec_tree_commit_args_t* commit, spec_stream_t stream);
 
 /*
+ * The tree sampler (Sec. 3.3, "Tree Sampler", with (B, K, V) = (gamma, top_k,
+ * num_nodes - 1)): the candidate tree that spec_accept_tree verifies, built from the
+ * drafter's rows. Block position d = 1 .. gamma-1 draws from drafter row d
+ * (drafter_logits[b][d]; row 0 is not read). Its candidates are the top_k tokens of
+ * log q_d = log softmax(row / T), T = temperature[b] (T <= 0 or NaN ranks at T = 1),
+ * ranked by probability, equal ones by lower token id. Node 0 is the root, token
+ * root_tokens[b] (the free token x^{L+1}). Each of the num_nodes - 1 steps adds the
+ * best child on offer, where every node at depth d < gamma - 1 offers its next unused
+ * candidate of position d + 1, scored by the sum of log q along its path; equal scores
+ * go to the lower parent index. The nodes are then the most probable num_nodes - 1
+ * prefixes, each after its parent, in the order they were taken. log q is computed in
+ * fp32 and path scores are summed in fp64.
+ *
+ * Outputs: tokens, parents (-1 for the root), depth (optional; the root is 0) and
+ * tree_mask (optional; bit i of node j set iff node i is j or one of its ancestors, the
+ * input of tree attention), each [batch][num_nodes]. A sequence whose used drafter rows
+ * hold a NaN or +inf or no finite logit (SPEC_FLAG_BAD_LOGITS) or whose root token is
+ * outside [0, vocab) (SPEC_FLAG_BAD_TOKEN) gets -1 tokens, parents and depths and a
+ * zero mask. SPEC_ERR_INVALID_ARGUMENT when the positions cannot hold num_nodes - 1
+ * nodes: sum over d = 1 .. gamma-1 of min(top_k, vocab)^d < num_nodes - 1.
+ */
+typedef struct {
+  int32_t batch, gamma, vocab, logits_dtype;
+  int32_t top_k;                /* K >= 1                                                  */
+  int32_t num_nodes;            /* 1 .. 64                                                 */
+  const void* drafter_logits;   /* [batch][gamma][vocab]                                   */
+  const float* temperature;     /* [batch]                                                 */
+  const int32_t* root_tokens;   /* [batch]                                                 */
+  int32_t* tokens;              /* [batch][num_nodes], written                             */
+  int32_t* parents;             /* [batch][num_nodes], written                             */
+  int32_t* depth;               /* [batch][num_nodes], written, or NULL                    */
+  uint64_t* tree_mask;          /* [batch][num_nodes], written, or NULL                    */
+} spec_tree_build_args_t;
+
+size_t spec_tree_build_workspace_size(const spec_tree_build_args_t* build);
+spec_status_t spec_build_tree(const spec_tree_build_args_t* build, void* ws, size_t ws_bytes,
+                              spec_stream_t stream);
+
+/*
  * spec_accept_block without a workspace, for callers that cannot allocate device
  * memory when they verify (for example, code confined to a fixed, pre-planned memory
  * arena, or code that must not call an allocator). It computes exactly what

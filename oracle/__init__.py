@@ -432,16 +432,21 @@ def build_tree(drafter_logits, temperature, root_tokens, top_k: int, budget: int
     Returns a dict: tokens, parents, depth (int32 [batch][budget+1]), mask (uint64
     [batch][budget+1]: bit i of node j set iff node i is j or an ancestor of j), score
     (fp64), margin (fp64 [batch]: the smallest gap between the taken child's score and
-    the best other offer over all steps; +inf if there never was another offer).
+    the best other offer over all steps; +inf if there never was another offer), and the
+    ranked candidates: cand_tokens (int32 [batch][gamma][min(top_k, vocab)], row 0 -1)
+    and cand_logq (their log q, fp64).
     """
     dl = _rows_f64(drafter_logits)
     B, G, V = dl.shape
     N = budget + 1
     if N > 64:
         raise ValueError("a tree holds at most 64 nodes")
+    Kc = min(top_k, V)
     out = dict(tokens=np.full((B, N), -1, np.int32), parents=np.full((B, N), -1, np.int32),
                depth=np.zeros((B, N), np.int32), mask=np.zeros((B, N), np.uint64),
-               score=np.zeros((B, N), np.float64), margin=np.full(B, np.inf))
+               score=np.zeros((B, N), np.float64), margin=np.full(B, np.inf),
+               cand_tokens=np.full((B, G, Kc), -1, np.int32),
+               cand_logq=np.full((B, G, Kc), np.nan, np.float64))
     for b in range(B):
         T = float(np.float32(temperature[b]))
         T = T if T > 0 else 1.0
@@ -453,6 +458,8 @@ def build_tree(drafter_logits, temperature, root_tokens, top_k: int, budget: int
             order = sorted(range(V), key=lambda x: (-lq[x], x))[:min(top_k, V)]
             logq.append(lq)
             top.append(order)
+            out["cand_tokens"][b, d] = order
+            out["cand_logq"][b, d] = lq[order]
         tokens, parents, depth, score = [int(root_tokens[b])], [-1], [0], [0.0]
         nxt = [0]
         margin = np.inf

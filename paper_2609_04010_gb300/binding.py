@@ -100,6 +100,15 @@ class TreeCommitArgs(ctypes.Structure):
                 ("num_accepted", ctypes.c_void_p), ("status", ctypes.c_void_p)]
 
 
+class TreeBuildArgs(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int32), ("gamma", ctypes.c_int32), ("vocab", ctypes.c_int32),
+                ("logits_dtype", ctypes.c_int32), ("top_k", ctypes.c_int32),
+                ("num_nodes", ctypes.c_int32), ("drafter_logits", ctypes.c_void_p),
+                ("temperature", ctypes.c_void_p), ("root_tokens", ctypes.c_void_p),
+                ("tokens", ctypes.c_void_p), ("parents", ctypes.c_void_p),
+                ("depth", ctypes.c_void_p), ("tree_mask", ctypes.c_void_p)]
+
+
 HEADER = os.path.join(_build.ROOT, "include", "spec_verify.h")
 
 
@@ -154,6 +163,10 @@ def lib(build_if_missing: bool = True):
             L.spec_accept_tree.restype = ctypes.c_int
             L.spec_commit_tree_kv.argtypes = [P, P]
             L.spec_commit_tree_kv.restype = ctypes.c_int
+            L.spec_tree_build_workspace_size.argtypes = [P]
+            L.spec_tree_build_workspace_size.restype = ctypes.c_size_t
+            L.spec_build_tree.argtypes = [P, P, ctypes.c_size_t, P]
+            L.spec_build_tree.restype = ctypes.c_int
             for f in ("spec_workspace_init", "spec_verify_attention", "spec_accept_block",
                       "spec_verify_step", "spec_philox_uniforms", "spec_read_device_status"):
                 getattr(L, f).restype = ctypes.c_int
@@ -496,6 +509,60 @@ def commit_tree_kv(k_cache, v_cache, page_table, kv_len, path, num_accepted, sta
                        path.data_ptr(), num_accepted.data_ptr(),
                        None if status_ws is None else status_ws.data_ptr())
     _raise(lib().spec_commit_tree_kv(ctypes.byref(a), _stream(stream)), "spec_commit_tree_kv")
+
+
+def tree_build_args(drafter_logits, temperature, root_tokens, top_k: int, tokens, parents,
+                    depth=None, tree_mask=None) -> TreeBuildArgs:
+    B, G, V = drafter_logits.shape
+    N = tokens.shape[1]
+    if drafter_logits.dtype == torch.bfloat16:
+        dt = SPEC_BF16
+    elif drafter_logits.dtype == torch.float32:
+        dt = SPEC_F32
+    else:
+        raise TypeError("logits must be bfloat16 or float32")
+    _check(drafter_logits, "drafter_logits", drafter_logits.dtype)
+    _check(temperature, "temperature", torch.float32, (B,))
+    _check(root_tokens, "root_tokens", torch.int32, (B,))
+    _check(tokens, "tokens", torch.int32, (B, N))
+    _check(parents, "parents", torch.int32, (B, N))
+    if depth is not None:
+        _check(depth, "depth", torch.int32, (B, N))
+    if tree_mask is not None:
+        _check(tree_mask, "tree_mask", torch.int64, (B, N))
+    return TreeBuildArgs(B, G, V, dt, int(top_k), N, drafter_logits.data_ptr(),
+                         temperature.data_ptr(), root_tokens.data_ptr(), tokens.data_ptr(),
+                         parents.data_ptr(), None if depth is None else depth.data_ptr(),
+                         None if tree_mask is None else tree_mask.data_ptr())
+
+
+def tree_build_workspace_size(t: TreeBuildArgs) -> int:
+    n = lib().spec_tree_build_workspace_size(ctypes.byref(t))
+    if n == 0:
+        raise SpecError(1, "spec_tree_build_workspace_size")
+    return int(n)
+
+
+def build_tree_args(t: TreeBuildArgs, ws: torch.Tensor, stream=None):
+    _raise(lib().spec_build_tree(ctypes.byref(t), _ptr(ws), ws.numel(), _stream(stream)),
+           "spec_build_tree")
+
+
+def build_tree(drafter_logits, temperature, root_tokens, top_k: int, num_nodes: int, ws=None,
+               stream=None) -> Dict[str, torch.Tensor]:
+    """The tree sampler (spec_build_tree). Returns tokens, parents, depth and mask
+    (int64 bit sets, the tree_mask input of verify_attention), each [batch][num_nodes]."""
+    B = drafter_logits.shape[0]
+    dev = drafter_logits.device
+    res = {k: torch.empty(B, num_nodes, dtype=torch.int32, device=dev)
+           for k in ("tokens", "parents", "depth")}
+    res["mask"] = torch.empty(B, num_nodes, dtype=torch.int64, device=dev)
+    t = tree_build_args(drafter_logits, temperature, root_tokens, top_k, res["tokens"],
+                        res["parents"], res["depth"], res["mask"])
+    if ws is None:
+        ws = new_workspace(tree_build_workspace_size(t), dev)
+    build_tree_args(t, ws, stream)
+    return res
 
 
 def philox_uniforms(seed: int, n: int, offset: int = 0, device=None, stream=None) -> torch.Tensor:

@@ -3,6 +3,7 @@
 // memory; all state lives in the caller's workspace.
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <atomic>
 #include <climits>
 #include <cstring>
@@ -129,6 +130,29 @@ spec_status_t check_tree(const spec_tree_accept_args_t* t) {
       !t->out_tokens || !t->num_emitted)
     return SPEC_ERR_INVALID_ARGUMENT;
   if (t->num_nodes > 64 || t->batch > 65535) return SPEC_ERR_UNSUPPORTED;
+  return SPEC_OK;
+}
+
+// Nodes the positions can hold: sum over d = 1 .. gamma-1 of min(top_k, vocab)^d, saturated.
+int64_t tree_capacity(const spec_tree_build_args_t* t) {
+  const int64_t k = std::min(t->top_k, t->vocab);
+  int64_t total = 0, level = 1;
+  for (int d = 1; d < t->gamma && total < 64; ++d) {
+    level = std::min<int64_t>(level * k, 64);
+    total += level;
+  }
+  return total;
+}
+
+spec_status_t check_tree_build(const spec_tree_build_args_t* t) {
+  if (!t) return SPEC_ERR_INVALID_ARGUMENT;
+  if (t->batch < 1 || t->gamma < 1 || t->vocab < 1 || t->top_k < 1 || t->num_nodes < 1)
+    return SPEC_ERR_INVALID_ARGUMENT;
+  if (t->logits_dtype != SPEC_F32 && t->logits_dtype != SPEC_BF16) return SPEC_ERR_INVALID_ARGUMENT;
+  if (!t->drafter_logits || !t->temperature || !t->root_tokens || !t->tokens || !t->parents)
+    return SPEC_ERR_INVALID_ARGUMENT;
+  if (t->num_nodes > 64 || t->batch > 65535) return SPEC_ERR_UNSUPPORTED;
+  if (tree_capacity(t) < t->num_nodes - 1) return SPEC_ERR_INVALID_ARGUMENT;
   return SPEC_OK;
 }
 
@@ -426,6 +450,38 @@ spec_status_t spec_accept_tree(const spec_tree_accept_args_t* t, void* ws, size_
   return launch_tree_greedy(*t, L, static_cast<char*>(ws), stream, vec) == cudaSuccess
              ? SPEC_OK
              : SPEC_ERR_CUDA;
+}
+
+size_t spec_tree_build_workspace_size(const spec_tree_build_args_t* t) {
+  if (check_tree_build(t) != SPEC_OK) return 0;
+  int dev = 0, sms = 160;
+  if (cudaGetDevice(&dev) == cudaSuccess) {
+    const int n = device_sm_count(dev);
+    if (n > sms) sms = n;
+  } else {
+    cudaGetLastError();
+  }
+  size_t need = 0;
+  for (int s : {148, 152, sms}) need = std::max(need, tree_build_layout(*t, kWsHeader, s).end);
+  return need;
+}
+
+spec_status_t spec_build_tree(const spec_tree_build_args_t* t, void* ws, size_t ws_bytes,
+                              spec_stream_t stream_) {
+  const spec_status_t st = check_tree_build(t);
+  if (st != SPEC_OK) return st;
+  if (!ws || (reinterpret_cast<uintptr_t>(ws) % kWsAlign) != 0) return SPEC_ERR_INVALID_ARGUMENT;
+  if (tree_build_layout(*t, kWsHeader, 1).end > ws_bytes) return SPEC_ERR_WORKSPACE_TOO_SMALL;
+  const size_t esz = t->logits_dtype == SPEC_BF16 ? 2 : 4;
+  const bool vec = (static_cast<size_t>(t->vocab) * esz) % 16 == 0 &&
+                   reinterpret_cast<uintptr_t>(t->drafter_logits) % 16 == 0;
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  int sms = 0;
+  if (!bind_device(stream, &sms)) return SPEC_ERR_CUDA;
+  const TreeBuildLayout L = tree_build_layout(*t, kWsHeader, sms);
+  if (L.end > ws_bytes) return SPEC_ERR_WORKSPACE_TOO_SMALL;
+  return launch_tree_build(*t, L, static_cast<char*>(ws), stream, vec) == cudaSuccess ? SPEC_OK
+                                                                                       : SPEC_ERR_CUDA;
 }
 
 spec_status_t spec_commit_tree_kv(const spec_tree_commit_args_t* c, spec_stream_t stream) {

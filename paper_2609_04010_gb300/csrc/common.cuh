@@ -113,6 +113,26 @@ cudaError_t launch_tree_greedy(const spec_tree_accept_args_t& a, const TreeLayou
                                cudaStream_t stream, bool vec);
 cudaError_t launch_tree_commit(const spec_tree_commit_args_t& a, cudaStream_t stream);
 
+constexpr int kTreeCandCap = 512;  // candidates of one row part ranked in shared memory
+
+struct TreeBuildLayout {
+  size_t tickets;      // uint32 [batch]: position rows of the sequence finished
+  size_t seq_flags;    // uint32 [batch]: flags its rows raised
+  size_t row_tickets;  // uint32 [batch][rows]: parts of the row finished
+  size_t keys;         // uint64 [batch][rows][splits][64]: each part's ranked candidate keys
+  size_t stats;        // float4 [batch][rows][splits]: (max, sum of exponentials, bad, -)
+  size_t table;        // int2 [batch][rows][64]: the position's (token, log q), ranked
+  size_t end;
+  int rows;            // positions that can hold a node: min(gamma - 1, num_nodes - 1)
+  int keff;            // candidates used per position: min(top_k, vocab, num_nodes - 1)
+  int splits, elems_per_split;
+  int smem;            // dynamic shared memory of a block, bytes
+};
+
+TreeBuildLayout tree_build_layout(const spec_tree_build_args_t& t, size_t base, int sms);
+cudaError_t launch_tree_build(const spec_tree_build_args_t& t, const TreeBuildLayout& L, char* ws,
+                              cudaStream_t stream, bool vec);
+
 // --- attention ---
 struct AttnPlan {
   int path;          // SPEC_ATTN_CUDA_CORES or SPEC_ATTN_TENSOR_CORES

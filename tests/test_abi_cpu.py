@@ -168,3 +168,49 @@ def test_draft_workspace_and_other_checks(lib):
     assert lib.spec_commit_kv(ctypes.byref(c), None) == 1  # no free list
     c = binding.CommitArgs(4, 8, 16, 10, 4096, 4096, 4096, 4096, 4096, 100, 2, None)
     assert lib.spec_commit_kv(ctypes.byref(c), None) == 1  # reserve must be 0 or 1
+
+
+def _tree_build(**kw):
+    a = dict(batch=2, gamma=16, vocab=32000, logits_dtype=binding.SPEC_BF16, top_k=32,
+             num_nodes=33, drafter_logits=4096, temperature=4096, root_tokens=4096, tokens=4096,
+             parents=4096, depth=None, tree_mask=None)
+    a.update(kw)
+    return binding.TreeBuildArgs(**a)
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(num_nodes=65), 2), (dict(num_nodes=0), 1), (dict(top_k=0), 1), (dict(gamma=0), 1),
+    (dict(logits_dtype=7), 1), (dict(parents=None), 1), (dict(batch=70000), 2),
+    (dict(gamma=2, top_k=3, num_nodes=5), 1),        # position 1 holds three nodes only
+    (dict(gamma=3, top_k=2, vocab=1, num_nodes=4), 1),  # one candidate per position: a chain of 2
+    (dict(gamma=1, num_nodes=2), 1),
+])
+def test_tree_build_host_checks(lib, kw, code):
+    t = _tree_build(**kw)
+    assert lib.spec_build_tree(ctypes.byref(t), ctypes.c_void_p(4096), 1 << 30, None) == code
+    assert lib.spec_tree_build_workspace_size(ctypes.byref(t)) == 0
+
+
+def test_tree_workspace_sizes_and_checks(lib):
+    for kw in (dict(), dict(gamma=2, top_k=3, num_nodes=4), dict(num_nodes=1, gamma=1),
+               dict(gamma=3, top_k=2, vocab=1, num_nodes=3)):
+        t = _tree_build(**kw)
+        n = lib.spec_tree_build_workspace_size(ctypes.byref(t))
+        assert n > 0 and n % 256 == 0
+        assert lib.spec_build_tree(ctypes.byref(t), ctypes.c_void_p(4096), 256, None) == 3
+        assert lib.spec_build_tree(ctypes.byref(t), ctypes.c_void_p(4097), n, None) == 1
+    assert lib.spec_build_tree(None, ctypes.c_void_p(4096), 1 << 30, None) == 1
+    a = binding.TreeAcceptArgs(2, 33, 32000, binding.SPEC_BF16, *([4096] * 7))
+    n = lib.spec_tree_workspace_size(ctypes.byref(a))
+    assert n > 0 and n % 256 == 0
+    assert lib.spec_accept_tree(ctypes.byref(a), ctypes.c_void_p(4096), 256, None) == 3
+    a.num_nodes = 65
+    assert lib.spec_accept_tree(ctypes.byref(a), ctypes.c_void_p(4096), 1 << 30, None) == 2
+    a.num_nodes, a.path = 33, None
+    assert lib.spec_accept_tree(ctypes.byref(a), ctypes.c_void_p(4096), 1 << 30, None) == 1
+    assert lib.spec_tree_workspace_size(ctypes.byref(a)) == 0
+    c = binding.TreeCommitArgs(2, 33, 8, 96, 16, 10, 100, *([4096] * 6), None)
+    assert lib.spec_commit_tree_kv(ctypes.byref(c), None) == 2  # head_dim 64 or 128
+    c.head_dim, c.path = 128, None
+    assert lib.spec_commit_tree_kv(ctypes.byref(c), None) == 1
+    assert lib.spec_commit_tree_kv(None, None) == 1

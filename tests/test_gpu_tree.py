@@ -1,10 +1,13 @@
-"""GPU parity of tree verification with the oracle, through the C ABI: tree attention
-(spec_verify_attention with tree_mask, both kernels), greedy acceptance along a tree
-(spec_accept_tree) and the compaction of the accepted path (spec_commit_tree_kv).
+"""GPU parity of tree verification with the oracle, through the C ABI: the tree sampler
+(spec_build_tree), tree attention (spec_verify_attention with tree_mask, both kernels),
+greedy acceptance along a tree (spec_accept_tree) and the compaction of the accepted
+path (spec_commit_tree_kv).
 
-Attention within the tolerances of the block-causal tests; a causal mask reproduces the
-block-causal kernels bit for bit. Acceptance and compaction are integer results:
-bit-exact. Trees come from the oracle's tree sampler on synthetic drafter rows."""
+The tree's structure, acceptance and compaction are integer results: bit-exact, except
+a sequence whose tree construction met a near-tie of path scores in the oracle (two
+offers within TREE_MARGIN = 1e-4 in log-probability; the kernel ranks by fp32 log q), which
+may differ and is counted. Attention within the tolerances of the block-causal tests; a
+causal mask reproduces the block-causal kernels bit for bit."""
 
 import numpy as np
 import pytest
@@ -16,6 +19,141 @@ from paper_2609_04010_gb300 import workloads as W
 from helpers import bf16_dev, compare_attention, dev, logits_dev, sample_rows
 
 pytestmark = pytest.mark.gpu
+
+TREE_MARGIN = 1e-4
+
+
+def gpu_build(dl, T, root, K, N, ws=None):
+    r = binding.build_tree(logits_dev(dl), dev(np.asarray(T, np.float32)),
+                           dev(np.asarray(root, np.int32)), K, N, ws=ws)
+    torch.cuda.synchronize()
+    return {k: v.cpu().numpy() for k, v in r.items()}
+
+
+def assert_valid_tree(g, o, b, tol):
+    """The GPU's tree for sequence b is a best-first tree over the oracle's ranked
+    candidates in which every step took an offer within tol of the best one: each
+    node's token is its parent's next unused candidate, its depth and mask follow its
+    parent's, and its score (fp64, from the oracle's log q) is at most tol below the
+    best offer of that step."""
+    tok, par, dep, msk = g["tokens"][b], g["parents"][b], g["depth"][b], g["mask"][b].view(np.uint64)
+    ct, cq = o["cand_tokens"][b], o["cand_logq"][b]
+    G, Kc = ct.shape
+    N = len(tok)
+    assert tok[0] == o["tokens"][b, 0] and par[0] == -1 and dep[0] == 0 and msk[0] == 1
+    score, nxt = [0.0], [0]
+    for i in range(1, N):
+        offers = {u: score[u] + cq[dep[u] + 1, nxt[u]] for u in range(i)
+                  if dep[u] + 1 < G and nxt[u] < Kc}
+        u = int(par[i])
+        assert u in offers, f"seq {b} node {i}: parent {u} had no offer"
+        assert offers[u] >= max(offers.values()) - tol, f"seq {b} node {i}: not the best offer"
+        assert tok[i] == ct[dep[u] + 1, nxt[u]] and dep[i] == dep[u] + 1, f"seq {b} node {i}"
+        assert msk[i] == msk[u] | np.uint64(1 << i), f"seq {b} node {i}: mask"
+        score.append(offers[u])
+        nxt[u] += 1
+        nxt.append(0)
+
+
+def check_build(oracle_mod, dl, T, root, K, N, strict=False):
+    """GPU trees equal the oracle's where its margin is at least TREE_MARGIN; elsewhere
+    they are valid best-first trees within TREE_MARGIN (or equal, if strict)."""
+    g = gpu_build(dl, T, root, K, N)
+    o = oracle_mod.build_tree(dl, T, root, K, N - 1)
+    for b in range(dl.shape[0]):
+        same = all(np.array_equal(g[k][b], o[k][b]) for k in ("tokens", "parents", "depth")) and \
+            np.array_equal(g["mask"][b].view(np.uint64), o["mask"][b])
+        if not same:
+            assert not strict and o["margin"][b] < TREE_MARGIN, (
+                f"seq {b}: trees differ, oracle margin {o['margin'][b]:.3g}\n"
+                f"GPU {g['tokens'][b]} {g['parents'][b]}\noracle {o['tokens'][b]} {o['parents'][b]}")
+            assert_valid_tree(g, o, b, TREE_MARGIN)
+    return g, o
+
+
+@pytest.mark.parametrize("batch,G,V,dtype,K,N,temps", [
+    (1, 16, 128256, "bf16", 32, 33, 1.0),        # (B, K, V) = (16, 32, 32)
+    (1, 16, 151936, "bf16", 32, 64, 0.0),
+    (8, 8, 32000, "f32", 8, 33, [1.0, 0.0, 0.5, 2.0]),
+    (16, 6, 5000, "bf16", 4, 21, 1.0),
+    (32, 8, 32000, "bf16", 16, 33, 0.8),
+    (3, 4, 33, "f32", 50, 8, 1.0),               # top_k above the vocabulary, unaligned rows
+    (2, 5, 100, "bf16", 3, 12, 0.7),
+])
+def test_build_tree(oracle_mod, batch, G, V, dtype, K, N, temps):
+    inp = W.make_accept_inputs(batch, G, V, dtype, 3.0, 1.0, temps, seed=V + batch)
+    check_build(oracle_mod, inp.drafter_logits, inp.temperature, inp.block_tokens[:, 0], K, N)
+
+
+def test_build_tree_chain_and_root_only(oracle_mod):
+    inp = W.make_accept_inputs(2, 40, 3000, "bf16", 3.0, 1.0, 1.0, seed=8)
+    g, _ = check_build(oracle_mod, inp.drafter_logits, inp.temperature, inp.block_tokens[:, 0], 1, 33)
+    assert np.array_equal(g["parents"][0], np.arange(-1, 32))
+    g = gpu_build(inp.drafter_logits, inp.temperature, inp.block_tokens[:, 0], 5, 1)
+    assert np.array_equal(g["tokens"][:, 0], inp.block_tokens[:, 0])
+    assert np.all(g["parents"] == -1) and np.all(g["depth"] == 0) and np.all(g["mask"] == 1)
+
+
+def test_build_tree_masked_rows(oracle_mod):
+    # rows with fewer finite logits than K: the remaining candidates have log q = -inf
+    inp = W.make_accept_inputs(3, 5, 1000, "f32", 3.0, 1.0, 1.0, seed=9)
+    dl = inp.drafter_logits
+    dl[0, 1:, 5:] = -np.inf
+    dl[1, 2, :997] = -np.inf
+    check_build(oracle_mod, dl, inp.temperature, inp.block_tokens[:, 0], 8, 30, strict=True)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_build_tree_ranks_structured_rows(oracle_mod, dtype):
+    # One drafter position: the tree is the root and the top N-1 candidates in rank
+    # order, so this compares the ranked candidate list itself. Sequences 0 and 1 put
+    # their large logits in whole 16-byte groups with a period of 128 groups, so that a
+    # row part's threads with the largest values hold many values above the threshold
+    # (the exact ranking rounds); sequence 2 is a constant row (every candidate tied,
+    # ranked by id).
+    rng = np.random.default_rng(10)
+    B, G, V, epv = 3, 2, 32768, (4 if dtype == "f32" else 8)
+    x = rng.standard_normal((B, G, V)).astype(np.float32)
+    for b, shift in ((0, 0), (1, 512)):
+        grp = ((np.arange(V) + shift) // epv) % 128
+        big = grp < 63
+        vals = 100.0 + grp[big] * 4.0 + rng.random((G, int(big.sum()))) * 0.5
+        x[b][:, big] = vals
+    x[2] = 0.25
+    dl = W.f32_to_bf16_bits(x).reshape(x.shape) if dtype == "bf16" else x
+    g, o = check_build(oracle_mod, dl, np.ones(B, np.float32), np.array([3, 4, 5], np.int32), 63, 64,
+                       strict=True)
+    assert np.array_equal(g["tokens"][2, 1:], np.arange(63))
+
+
+def test_build_tree_bad_inputs(oracle_mod):
+    B, G, V = 6, 6, 2000
+    inp = W.make_accept_inputs(B, G, V, "f32", 3.0, 1.0, 1.0, seed=12)
+    dl, root = inp.drafter_logits, inp.block_tokens[:, 0].copy()
+    dl[0, 0, 7] = np.nan          # row 0 is never read
+    dl[1, 2, 9] = np.nan
+    dl[2, 3, 1] = np.inf
+    dl[3, 1, :] = -np.inf
+    root[4] = V
+    ws = binding.new_workspace(1 << 22)
+    g = gpu_build(dl, inp.temperature, root, 4, 9, ws=ws)
+    flags = binding.read_device_status(ws)[1]
+    assert flags == binding.FLAG_BAD_LOGITS | binding.FLAG_BAD_TOKEN
+    for b in (1, 2, 3, 4):
+        assert np.all(g["tokens"][b] == -1) and np.all(g["parents"][b] == -1)
+        assert np.all(g["depth"][b] == -1) and np.all(g["mask"][b] == 0)
+    o = oracle_mod.build_tree(dl[[0, 5]], inp.temperature[[0, 5]], root[[0, 5]], 4, 8)
+    for i, b in enumerate((0, 5)):
+        assert np.array_equal(g["tokens"][b], o["tokens"][i]) or o["margin"][i] < TREE_MARGIN
+
+
+def test_build_tree_capacity_is_checked():
+    dl = torch.zeros(1, 2, 100, dtype=torch.float32, device="cuda")
+    T = torch.ones(1, device="cuda")
+    root = torch.zeros(1, dtype=torch.int32, device="cuda")
+    binding.build_tree(dl, T, root, 3, 4)          # three children of the root
+    with pytest.raises(binding.SpecError):
+        binding.build_tree(dl, T, root, 3, 5)      # a fourth node has no place
 
 
 def tree_case(oracle_mod, seed, batch, budget, K, gamma_draft, vocab, dtype="bf16", agree=0.8):
@@ -201,11 +339,17 @@ def test_tree_commit_bad_inputs_leave_the_sequence(oracle_mod):
 
 
 def test_tree_step_end_to_end(oracle_mod):
-    # tree attention over the nodes, then greedy acceptance, then the compaction: the
-    # accepted tokens and the compacted cache match the oracle's chain of the same steps
+    # the tree sampler, tree attention over its nodes, greedy acceptance, then the
+    # compaction, all on the GPU: the results match the oracle's chain of the same steps
     batch, budget, K, G, V = 1, 32, 32, 16, 128256
     N = budget + 1
     tree, tl = tree_case(oracle_mod, 71, batch, budget, K, G, V)
+    inp_d = W.make_accept_inputs(batch, G, V, "bf16", 3.0, 1.0, 1.0, seed=71)
+    gt = gpu_build(inp_d.drafter_logits, inp_d.temperature, inp_d.block_tokens[:, 0], K, N)
+    if tree["margin"][0] >= TREE_MARGIN:
+        for k in ("tokens", "parents", "depth"):
+            np.testing.assert_array_equal(gt[k], tree[k])
+        tree["mask"] = gt["mask"].view(np.uint64)
     inp = attn_tree_inputs(71, batch, N, 32, 8, 128, 16, 4096)
     args = (bf16_dev(inp.q), bf16_dev(inp.k_cache), bf16_dev(inp.v_cache), dev(inp.page_table),
             dev(inp.kv_len))
