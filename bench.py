@@ -88,6 +88,9 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-draft", action="store_true",
                     help="skip the draft-side timing (block sampling, KV commit)")
+    ap.add_argument("--no-tree", action="store_true",
+                    help="skip the tree verification timing (tree sampler, tree attention, "
+                         "greedy tree acceptance, KV compaction)")
     ap.add_argument("--cpu-seconds", type=float, default=10.0,
                     help="CPU time budget of the oracle baseline sample")
     return ap.parse_args()
@@ -476,6 +479,9 @@ def run_ours(args, wl, ai, ci, rank, world, local_rank):
                  "timing": "CUDA-graph replays; sample_block with L2 flushed, commit_kv with its "
                            "inputs restored before each replay"}
 
+    tree = None if args.no_tree else time_tree(wl, ai, ci, binding, dev, graph_of, timed_loop,
+                                               parts_n, stream)
+
     emitted = sum_over_ranks(float(ne.sum().item()), world, dev)
     tm = traffic_model(ai, ci)
     peak, peak_src = measured_peaks()
@@ -523,7 +529,97 @@ def run_ours(args, wl, ai, ci, rank, world, local_rank):
         result["e2e_kv_resident"] = e2e_kv
     if draft:
         result["draft"] = draft
+    if tree:
+        result["tree"] = tree
     return result
+
+
+TREE_BLOCK, TREE_TOP_K, TREE_NODES = 16, 32, 33   # the tree sampler's (B, K, V) = (16, 32, 32)
+
+
+def time_tree(wl, ai, ci, binding, dev, graph_of, timed_loop, n, stream):
+    """Tree verification for one request (the setting the tree sampler serves) on the
+    workload's vocabulary, heads and context, with the tree sampler's (B, K, V) =
+    (16, 32, 32): the tree built from a 16-position drafter block, tree attention over
+    its 33 nodes, greedy acceptance and the KV compaction, each a CUDA-graph replay of
+    its C-ABI call with L2 flushed before it."""
+    import torch
+    from paper_2609_04010_gb300 import workloads as W
+
+    B, V = 1, ci.vocab
+    N = TREE_NODES
+    ti = W.make_accept_inputs(B, N, V, "bf16", 3.0, 1.0, 1.0, seed=21)
+    at = W.make_attn_inputs(B, N, ai.q.shape[2], ai.k_cache.shape[1], ai.q.shape[3], ai.page_size,
+                            wl.ctx, True, seed=22)
+
+    def bf16(a):
+        return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16).to(dev)
+
+    def t(a):
+        return torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+
+    dl = bf16(ti.drafter_logits[:, :TREE_BLOCK])
+    tl = bf16(ti.target_logits)
+    temp, root = t(ti.temperature), t(ti.block_tokens[:, 0])
+    tok, par = (torch.empty(B, N, dtype=torch.int32, device=dev) for _ in range(2))
+    depth = torch.empty(B, N, dtype=torch.int32, device=dev)
+    mask = torch.empty(B, N, dtype=torch.int64, device=dev)
+    bargs = binding.tree_build_args(dl, temp, root, TREE_TOP_K, tok, par, depth, mask)
+    ws_b = binding.new_workspace(binding.tree_build_workspace_size(bargs), dev)
+    build_call = lambda: binding.build_tree_args(bargs, ws_b)
+    build_call()
+    q, k, v, pt, kvl = bf16(at.q), bf16(at.k_cache), bf16(at.v_cache), t(at.page_table), t(at.kv_len)
+    out = torch.empty_like(q)
+    lse = torch.empty(q.shape[:3], dtype=torch.float32, device=dev)
+    aargs = binding.attn_args(q, k, v, pt, kvl, out, lse, tree_mask=mask)
+    ws_a = binding.new_workspace(binding.workspace_size(aargs, None), dev)
+    attn_call = lambda: binding.verify_attention_args(aargs, ws_a)
+    path, na = torch.empty(B, N, dtype=torch.int32, device=dev), torch.empty(B, dtype=torch.int32, device=dev)
+    ot, ne = torch.empty(B, N + 1, dtype=torch.int32, device=dev), torch.empty(B, dtype=torch.int32, device=dev)
+    targs = binding.tree_accept_args(tl, tok, par, path, na, ot, ne)
+    ws_t = binding.new_workspace(binding.tree_workspace_size(targs), dev)
+    accept_call = lambda: binding.accept_tree_args(targs, ws_t)
+    verify_call = lambda: (attn_call(), accept_call())
+    gs = {name: graph_of(fn) for name, fn in (("build", build_call), ("attention", attn_call),
+                                              ("accept", accept_call), ("verify", verify_call))}
+    ms = {name: statistics.mean(timed_loop(g.replay, n)) for name, g in gs.items()}
+    torch.cuda.synchronize()
+    for ws in (ws_b, ws_a, ws_t):
+        code, flags = binding.read_device_status(ws)
+        if code != 0:
+            raise RuntimeError(f"tree timing: device status {code} flags {flags}")
+    # compaction: the accepted path moves into place; kv_len restored before each replay
+    kv0 = kvl.clone()
+    commit_call = lambda: binding.commit_tree_kv(k, v, pt, kvl, path, na)
+    commit_g = graph_of(commit_call)
+    commit_times = []
+    for _ in range(max(20, min(n, 200))):
+        kvl.copy_(kv0)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        commit_g.replay()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        commit_times.append(e0.elapsed_time(e1))
+    rows = min(TREE_BLOCK - 1, N - 1)
+    build_bytes = B * rows * V * 2
+    accept_bytes = B * N * V * 2
+    kv_bytes = int(2 * at.kv_len.astype(np.int64).sum() * at.k_cache.shape[1] * at.q.shape[3] * 2)
+    peak = measured_peaks()[0]
+
+    def gbs(nbytes, t_ms):
+        return round(nbytes / (t_ms / 1000.0) / 1e9, 1)
+
+    return {"shape": {"batch": B, "vocab": V, "drafter_block": TREE_BLOCK, "top_k": TREE_TOP_K,
+                      "num_nodes": N, "context": str(wl.ctx)},
+            "build_tree_ms": ms["build"], "build_tree_gbs": gbs(build_bytes, ms["build"]),
+            "build_tree_frac_of_measured": round(build_bytes / (ms["build"] / 1000.0) / 1e9 / peak, 4),
+            "tree_attention_ms": ms["attention"], "tree_attention_gbs": gbs(kv_bytes, ms["attention"]),
+            "accept_tree_ms": ms["accept"], "accept_tree_gbs": gbs(accept_bytes, ms["accept"]),
+            "verify_ms": ms["verify"], "commit_tree_kv_ms": statistics.median(commit_times),
+            "algorithmic_bytes": {"build_tree": build_bytes, "tree_attention": kv_bytes,
+                                  "accept_tree": accept_bytes},
+            "timing": "CUDA-graph replays, L2 flushed before each (commit: kv_len restored)"}
 
 
 def main():

@@ -396,7 +396,7 @@ spec_status_t spec_commit_tree_kv(const spec_tree_commit_args_t* commit, spec_st
  * candidate of position d + 1, scored by the sum of log q along its path; equal scores
  * go to the lower parent index. The nodes are then the most probable num_nodes - 1
  * prefixes, each after its parent, in the order they were taken. log q is computed in
- * fp32 and path scores are summed in fp64.
+ * fp32 and path scores are summed in double-float (two fp32 words, about 48 bits).
  *
  * Outputs: tokens, parents (-1 for the root), depth (optional; the root is 0) and
  * tree_mask (optional; bit i of node j set iff node i is j or one of its ancestors, the

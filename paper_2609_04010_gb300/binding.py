@@ -467,6 +467,13 @@ def tree_accept_args(target_logits, tokens, parents, path, num_accepted, out_tok
                           out_tokens.data_ptr(), num_emitted.data_ptr())
 
 
+def tree_workspace_size(t: TreeAcceptArgs) -> int:
+    n = lib().spec_tree_workspace_size(ctypes.byref(t))
+    if n == 0:
+        raise SpecError(1, "spec_tree_workspace_size")
+    return int(n)
+
+
 def accept_tree_args(t: TreeAcceptArgs, ws: torch.Tensor, stream=None):
     _raise(lib().spec_accept_tree(ctypes.byref(t), _ptr(ws), ws.numel(), _stream(stream)),
            "spec_accept_tree")
@@ -484,10 +491,7 @@ def accept_tree(target_logits, tokens, parents, ws=None, stream=None) -> Dict[st
     t = tree_accept_args(target_logits, tokens, parents, res["path"], res["num_accepted"],
                          res["out_tokens"], res["num_emitted"])
     if ws is None:
-        n = lib().spec_tree_workspace_size(ctypes.byref(t))
-        if n == 0:
-            raise SpecError(1, "spec_tree_workspace_size")
-        ws = new_workspace(n, dev)
+        ws = new_workspace(tree_workspace_size(t), dev)
     accept_tree_args(t, ws, stream)
     return res
 

@@ -358,7 +358,7 @@ __global__ void tree_commit_len_kernel(spec_tree_commit_args_t a) {
 // the parts' (max, sum of exponentials) into the row's log-normaliser and writes the
 // position's ranked (token, log q) table; the sequence's last row block selects the
 // tree's nodes best first, one warp holding the offers of two nodes per lane (path
-// scores are fp64 sums of the fp32 log q).
+// scores are double-float sums of the fp32 log q).
 // ---------------------------------------------------------------------------------
 struct BuildParams {
   int batch, gamma, vocab, rows, keff, nodes, splits, eps;
@@ -401,9 +401,10 @@ __device__ __forceinline__ void merge_ms(float& m, float& s, float m2, float s2,
   s = t;
 }
 
-// Calls f(x, index) on each of this thread's logits of [e_begin, e_end) of the row.
+// Calls f(x, base) on this thread's logits of [e_begin, e_end) of the row, a 16-byte
+// group at a time (x[q] is logit base + q; groups of one where rows are not aligned).
 template <bool BF16, bool VEC, class F>
-__device__ __forceinline__ void for_part(const char* rowp, int e_begin, int e_end, int tid, F&& f) {
+__device__ __forceinline__ void for_groups(const char* rowp, int e_begin, int e_end, int tid, F&& f) {
   if (VEC) {
     constexpr int kEpv = BF16 ? 8 : 4;
     const uint4* rv = reinterpret_cast<const uint4*>(rowp);
@@ -420,12 +421,12 @@ __device__ __forceinline__ void for_part(const char* rowp, int e_begin, int e_en
         const int vi = v0 + k * kThreads;
         if (vi < vend) {
           const uint32_t wv[4] = {dv[k].x, dv[k].y, dv[k].z, dv[k].w};
+          float x[kEpv];
 #pragma unroll
-          for (int q = 0; q < kEpv; ++q) {
-            const float x = BF16 ? __uint_as_float((q & 1) ? (wv[q >> 1] & 0xffff0000u) : (wv[q >> 1] << 16))
-                                 : __uint_as_float(wv[q]);
-            f(x, vi * kEpv + q);
-          }
+          for (int q = 0; q < kEpv; ++q)
+            x[q] = BF16 ? __uint_as_float((q & 1) ? (wv[q >> 1] & 0xffff0000u) : (wv[q >> 1] << 16))
+                        : __uint_as_float(wv[q]);
+          f(x, vi * kEpv);
         }
       }
     }
@@ -438,10 +439,61 @@ __device__ __forceinline__ void for_part(const char* rowp, int e_begin, int e_en
         x[k] = ei < e_end ? load_elem<BF16>(rowp, ei) : 0.f;
       }
 #pragma unroll
-      for (int k = 0; k < kPartUnroll; ++k)
-        if (e0 + k * kThreads < e_end) f(x[k], e0 + k * kThreads);
+      for (int k = 0; k < kPartUnroll; ++k) {
+        const float one[1] = {x[k]};
+        if (e0 + k * kThreads < e_end) f(one, e0 + k * kThreads);
+      }
     }
   }
+}
+
+// Sorts one key per lane of the warp into descending order (bitonic network).
+__device__ __forceinline__ unsigned long long warp_sort_desc(unsigned long long v, int lane) {
+#pragma unroll
+  for (int k = 2; k <= 32; k <<= 1) {
+#pragma unroll
+    for (int j = k >> 1; j > 0; j >>= 1) {
+      const unsigned long long o = __shfl_xor_sync(0xffffffffu, v, j);
+      const bool keep_max = ((lane & j) == 0) == ((lane & k) == 0);
+      v = keep_max ? (o > v ? o : v) : (o < v ? o : v);
+    }
+  }
+  return v;
+}
+
+// The 64 largest of two descending lists of 64 keys (a0, a1 and b0, b1: the lane's
+// entries lane and lane + 32 of each), descending, as the lane's two entries. The elementwise
+// maximum of one list and the other reversed is bitonic and holds the 64 largest; a
+// bitonic merge (half-cleaners of 32, 16, .., 1) sorts it.
+__device__ __noinline__ ulonglong2 merge_top64(unsigned long long a0, unsigned long long a1,
+                                               unsigned long long b0, unsigned long long b1, int lane) {
+  const unsigned long long rb0 = __shfl_sync(0xffffffffu, b1, 31 - lane);
+  const unsigned long long rb1 = __shfl_sync(0xffffffffu, b0, 31 - lane);
+  unsigned long long c0 = a0 > rb0 ? a0 : rb0;
+  unsigned long long c1 = a1 > rb1 ? a1 : rb1;
+  {
+    const unsigned long long hi = c0 > c1 ? c0 : c1, lo = c0 > c1 ? c1 : c0;
+    c0 = hi;
+    c1 = lo;
+  }
+#pragma unroll
+  for (int j = 16; j > 0; j >>= 1) {
+    const unsigned long long o0 = __shfl_xor_sync(0xffffffffu, c0, j);
+    const unsigned long long o1 = __shfl_xor_sync(0xffffffffu, c1, j);
+    const bool lower = (lane & j) == 0;
+    c0 = lower ? (c0 > o0 ? c0 : o0) : (c0 < o0 ? c0 : o0);
+    c1 = lower ? (c1 > o1 ? c1 : o1) : (c1 < o1 ? c1 : o1);
+  }
+  return make_ulonglong2(c0, c1);
+}
+
+// x[q] for a q known only at run time, by selects (no local-memory copy of x).
+template <int E>
+__device__ __forceinline__ float pick(const float (&x)[E], int q) {
+  float v = x[0];
+#pragma unroll
+  for (int j = 1; j < E; ++j) v = j == q ? x[j] : v;
+  return v;
 }
 
 __device__ __forceinline__ unsigned long long block_max_u64(unsigned long long v, unsigned long long* s_red) {
@@ -459,29 +511,197 @@ __device__ __forceinline__ unsigned long long block_max_u64(unsigned long long v
   return v;
 }
 
+// (ah + al) + b as a normalised double-float (rh + rl): the exact sum of ah and b by
+// Knuth's two-sum, then the low parts folded in (a fast two-sum). Path scores keep
+// about 48 bits this way without fp64 arithmetic, whose latency is high on this part.
+__device__ __forceinline__ void df_add(float ah, float al, float b, float& rh, float& rl) {
+  const float s = __fadd_rn(ah, b);
+  if (!(s > -INFINITY)) {  // a -inf term
+    rh = s;
+    rl = 0.f;
+    return;
+  }
+  const float bb = __fsub_rn(s, ah);
+  const float e = __fadd_rn(__fsub_rn(ah, __fsub_rn(s, bb)), __fsub_rn(b, bb));
+  const float t = __fadd_rn(e, al);
+  rh = __fadd_rn(s, t);
+  rl = __fsub_rn(t, __fsub_rn(rh, s));
+}
+
 struct TreeNode {
   int dep, nx, tok, par;   // dep < 0: no node in this slot
-  double sc, osc;          // path score; score of the current offer (sums of fp32 log q)
+  float sh, sl;            // path score as an unevaluated sum sh + sl (double-float)
+  float oh, ol;            // score of the current offer, the same way
   int otk;                 // token of the current offer
   unsigned long long key;  // order key of the offer's score, 0 if none
   unsigned long long msk;  // ancestor bits
 };
 
-__device__ __forceinline__ unsigned long long order_key64(double x) {
-  unsigned long long f = static_cast<unsigned long long>(__double_as_longlong(x));
-  if (f == 0x8000000000000000ull) f = 0ull;
-  return (f >> 63) ? ~f : (f | 0x8000000000000000ull);
+// The node's next offer, its candidate nx of position dep + 1 (table row dep): its score
+// (oh + ol) and token, and the key (0 if there is none) that orders normalised
+// double-floats: high parts first, then low parts.
+__device__ __forceinline__ unsigned long long offer_of(const TreeNode& n, const int2* tab, int rows, int K,
+                                                       float& oh, float& ol, int& otk) {
+  if (n.dep < 0 || n.dep >= rows || n.nx >= K) return 0ull;
+  const int2 e = tab[n.dep * K + n.nx];
+  df_add(n.sh, n.sl, __int_as_float(e.y), oh, ol);
+  otk = e.x;
+  return (static_cast<unsigned long long>(order_key(oh)) << 32) | order_key(ol);
 }
 
-// The node's next offer: its candidate nx of position dep + 1 (table row dep).
-__device__ __forceinline__ void refresh_offer(TreeNode& n, const int2* tab, int rows, int K) {
-  n.key = 0ull;
-  if (n.dep >= 0 && n.dep < rows && n.nx < K) {
-    const int2 e = tab[n.dep * K + n.nx];
-    n.osc = n.sc + static_cast<double>(__int_as_float(e.y));
-    n.otk = e.x;
-    n.key = order_key64(n.osc);
+// Best-first selection of the tree's nodes by one warp. The root (node 0) is kept in
+// every lane; node c >= 1 is slot (c - 1) / 32 of lane (c - 1) % 32. Each step takes the
+// best offer (largest high word of its key; on a tie the largest low word, then the
+// lowest node index, the root first), makes it node i, and moves its parent to its next
+// candidate.
+template <int SLOTS>
+__device__ __forceinline__ void select_nodes(const BuildParams& p, const int2* tab, int K, int b,
+                                             uint32_t flags, int lane) {
+  const int N = p.nodes;
+  const int64_t base = static_cast<int64_t>(b) * N;
+  TreeNode root, n[SLOTS];
+  root.dep = 0;
+  root.nx = 0;
+  root.tok = flags ? -1 : p.root[b];
+  root.par = -1;
+  root.msk = 1ull;
+  root.sh = root.sl = 0.f;
+  root.oh = root.ol = 0.f;
+  root.otk = -1;
+  root.key = 0ull;
+#pragma unroll
+  for (int h = 0; h < SLOTS; ++h) {
+    n[h].dep = -1;
+    n[h].nx = 0;
+    n[h].tok = -1;
+    n[h].par = -1;
+    n[h].msk = 0ull;
+    n[h].sh = n[h].sl = 0.f;
+    n[h].oh = n[h].ol = 0.f;
+    n[h].otk = -1;
+    n[h].key = 0ull;
   }
+  if (!flags) {
+    root.key = offer_of(root, tab, p.rows, K, root.oh, root.ol, root.otk);
+    for (int i = 1; i < N; ++i) {
+      const uint32_t rh = static_cast<uint32_t>(root.key >> 32);
+      uint32_t hl = 0u;
+#pragma unroll
+      for (int h = 0; h < SLOTS; ++h) hl = max(hl, static_cast<uint32_t>(n[h].key >> 32));
+      const uint32_t Mh = max(__reduce_max_sync(0xffffffffu, hl), rh);
+      if (Mh == 0u) {  // no offer left: excluded by the host's capacity check
+        flags |= SPEC_FLAG_BAD_TREE;
+        break;
+      }
+      unsigned bal[SLOTS];
+      int ties = rh == Mh;
+#pragma unroll
+      for (int h = 0; h < SLOTS; ++h) {
+        bal[h] = __ballot_sync(0xffffffffu, static_cast<uint32_t>(n[h].key >> 32) == Mh);
+        ties += __popc(bal[h]);
+      }
+      bool root_wins = rh == Mh;
+      if (ties > 1) {
+        const uint32_t rl = rh == Mh ? static_cast<uint32_t>(root.key) : 0u;
+        uint32_t ll = 0u;
+#pragma unroll
+        for (int h = 0; h < SLOTS; ++h)
+          if (static_cast<uint32_t>(n[h].key >> 32) == Mh) ll = max(ll, static_cast<uint32_t>(n[h].key));
+        const uint32_t Ml = max(__reduce_max_sync(0xffffffffu, ll), rl);
+        root_wins = rh == Mh && rl == Ml;
+#pragma unroll
+        for (int h = 0; h < SLOTS; ++h)
+          bal[h] = __ballot_sync(0xffffffffu, static_cast<uint32_t>(n[h].key >> 32) == Mh &&
+                                                  static_cast<uint32_t>(n[h].key) == Ml);
+      }
+      // the winner u and its offer (score, token), depth and ancestor bits
+      int u = 0, hs = 0;
+      if (!root_wins) {
+#pragma unroll
+        for (int h = SLOTS - 1; h >= 0; --h)
+          if (bal[h]) {
+            u = 1 + 32 * h + __ffs(bal[h]) - 1;
+            hs = h;
+          }
+      }
+      const int src = (u - 1) & 31;
+      float oh = root.oh, ol = root.ol;
+      int otk = root.otk, pdep = 0;
+      unsigned long long pm = 1ull;
+      {
+        float soh = n[0].oh, sol = n[0].ol;
+        int sotk = n[0].otk, sdep = n[0].dep;
+        unsigned long long smsk = n[0].msk;
+#pragma unroll
+        for (int h = 1; h < SLOTS; ++h)
+          if (hs == h) {
+            soh = n[h].oh;
+            sol = n[h].ol;
+            sotk = n[h].otk;
+            sdep = n[h].dep;
+            smsk = n[h].msk;
+          }
+        soh = __shfl_sync(0xffffffffu, soh, src);
+        sol = __shfl_sync(0xffffffffu, sol, src);
+        sotk = __shfl_sync(0xffffffffu, sotk, src);
+        sdep = __shfl_sync(0xffffffffu, sdep, src);
+        smsk = __shfl_sync(0xffffffffu, smsk, src);
+        if (u != 0) {
+          oh = soh;
+          ol = sol;
+          otk = sotk;
+          pdep = sdep;
+          pm = smsk;
+        }
+      }
+      // node i takes the offer; its parent moves to its next candidate
+      const int ci = (i - 1) & 31, ch = (i - 1) >> 5;
+#pragma unroll
+      for (int h = 0; h < SLOTS; ++h) {
+        const bool is_new = lane == ci && ch == h;
+        const bool adv = u != 0 && lane == src && hs == h;
+        if (is_new) {
+          n[h].dep = pdep + 1;
+          n[h].nx = 0;
+          n[h].tok = otk;
+          n[h].par = u;
+          n[h].sh = oh;
+          n[h].sl = ol;
+          n[h].msk = pm | (1ull << i);
+        }
+        if (adv) ++n[h].nx;
+        float ph = 0.f, pl = 0.f;
+        int pt = -1;
+        const unsigned long long k = offer_of(n[h], tab, p.rows, K, ph, pl, pt);
+        if (is_new || adv) {
+          n[h].key = k;
+          n[h].oh = ph;
+          n[h].ol = pl;
+          n[h].otk = pt;
+        }
+      }
+      if (u == 0) {
+        ++root.nx;
+        root.key = offer_of(root, tab, p.rows, K, root.oh, root.ol, root.otk);
+      }
+    }
+  }
+  if (lane == 0) {
+    p.tokens[base] = flags ? -1 : root.tok;
+    p.parents[base] = -1;
+    if (p.depth) p.depth[base] = flags ? -1 : 0;
+    if (p.mask) p.mask[base] = flags ? 0ull : 1ull;
+  }
+#pragma unroll
+  for (int h = 0; h < SLOTS; ++h) {
+    const int c = 1 + lane + 32 * h;
+    if (c >= N) continue;
+    p.tokens[base + c] = flags ? -1 : n[h].tok;
+    p.parents[base + c] = flags ? -1 : n[h].par;
+    if (p.depth) p.depth[base + c] = flags ? -1 : n[h].dep;
+    if (p.mask) p.mask[base + c] = flags ? 0ull : n[h].msk;
+  }
+  if (lane == 0 && flags) set_status(p.status, flags);
 }
 
 template <bool BF16, bool VEC>
@@ -490,9 +710,11 @@ __global__ void __launch_bounds__(kThreads) tree_build_kernel(BuildParams p) {
   __shared__ unsigned long long s_tmax[kThreads];
   __shared__ unsigned long long s_tau;
   __shared__ float s_wm[kThreads / 32], s_ws[kThreads / 32];
+  __shared__ int s_wcnt[kThreads / 32];
   __shared__ int s_count, s_bad, s_last;
   __shared__ uint32_t s_flags;
   const int split = blockIdx.x, r = blockIdx.y, b = blockIdx.z, tid = threadIdx.x;
+  const int lane = tid & 31, w = tid >> 5;
   const int K = p.keff, S = p.splits;
   const int64_t rid = static_cast<int64_t>(b) * p.rows + r;
   const char* rowp = static_cast<const char*>(p.logits) +
@@ -508,49 +730,138 @@ __global__ void __launch_bounds__(kThreads) tree_build_kernel(BuildParams p) {
   }
   __syncthreads();
 
-  // pass 1: the thread's largest key, its (max, sum), NaN or +inf seen
-  unsigned long long kmax = 0ull;
+  // pass 1, a 16-byte group at a time: the thread's maximum and its lowest index, the
+  // sum of 2^((x - max) c2) (rescaled when the maximum rises), NaN or +inf seen (a NaN
+  // sum, or a NaN among logits that are all -inf so far)
   float m = -INFINITY, s = 0.f;
-  bool bad = false;
-  for_part<BF16, VEC>(rowp, e_begin, e_end, tid, [&](float x, int i) {
-    bad |= !(x < INFINITY);
-    const unsigned long long k = cand_key(x, i);
-    kmax = k > kmax ? k : kmax;
-    if (x > m) {
-      s = s * ex2((m - x) * c2) + 1.f;
-      m = x;
-    } else if (x > -INFINITY) {
-      s += ex2((x - m) * c2);
+  int mi = -1;
+  bool nan_seen = false;
+  for_groups<BF16, VEC>(rowp, e_begin, e_end, tid, [&](const auto& x, int base) {
+    constexpr int E = sizeof(x) / sizeof(float);
+    float vmax = x[0];
+#pragma unroll
+    for (int q = 1; q < E; ++q) vmax = fmaxf(vmax, x[q]);
+    if (mi < 0) mi = base;  // the first logit: the maximum of a part of -inf
+    if (vmax > m) {
+      unsigned eq = 0u;
+#pragma unroll
+      for (int q = 0; q < E; ++q) eq |= (x[q] == vmax ? 1u : 0u) << q;
+      const int q0 = __ffs(eq) - 1;
+      s *= ex2((m - vmax) * c2);
+      m = vmax;
+      mi = base + q0;
+    }
+    if (m > -INFINITY) {
+      const float mc = m * c2;
+#pragma unroll
+      for (int q = 0; q < E; ++q) s += ex2(fmaf(x[q], c2, -mc));
+    } else {
+#pragma unroll
+      for (int q = 0; q < E; ++q) nan_seen |= x[q] != x[q];
     }
   });
-  s_tmax[tid] = kmax;
-  if (bad) s_bad = 1;
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    const float m2 = __shfl_xor_sync(0xffffffffu, m, o), s2 = __shfl_xor_sync(0xffffffffu, s, o);
-    merge_ms(m, s, m2, s2, c2);
-  }
-  if ((tid & 31) == 0) {
-    s_wm[tid >> 5] = m;
-    s_ws[tid >> 5] = s;
-  }
-  __syncthreads();
-  // tau: the K-th largest thread maximum (0 where fewer threads hold logits); the part's
-  // top K keys are among the keys >= tau, which lie in the K threads at or above it
+  if (nan_seen || s != s) s_bad = 1;
+  const unsigned long long L0 = mi >= 0 ? cand_key(m, mi) : 0ull;
+  // tau: the K-th largest of the threads' maximum keys (0 if fewer threads hold
+  // logits); the part's top K keys are among the keys >= tau. Each warp sorts its 32
+  // keys; a key's rank is its place in its warp plus the keys above it in the others.
   {
-    int rank = 0;
-    for (int j = 0; j < kThreads; ++j) rank += s_tmax[j] > kmax;
-    if (rank == K - 1) s_tau = kmax;
+    const unsigned long long v = warp_sort_desc(L0, lane);
+    s_tmax[tid] = v;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float m2 = __shfl_xor_sync(0xffffffffu, m, o), s2 = __shfl_xor_sync(0xffffffffu, s, o);
+      merge_ms(m, s, m2, s2, c2);
+    }
+    if (lane == 0) {
+      s_wm[w] = m;
+      s_ws[w] = s;
+    }
+    __syncthreads();
+    int rank = lane;
+#pragma unroll
+    for (int w2 = 0; w2 < kThreads / 32; ++w2) {
+      if (w2 == w) continue;
+      const unsigned long long* run = s_tmax + w2 * 32;
+      int lo = 0, hi = 32;
+      while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (run[mid] > v) lo = mid + 1;
+        else hi = mid;
+      }
+      rank += lo;
+    }
+    if (rank == K - 1) s_tau = v;
   }
   __syncthreads();
   const unsigned long long tau = s_tau;
-  for_part<BF16, VEC>(rowp, e_begin, e_end, tid, [&](float x, int i) {
-    const unsigned long long k = cand_key(x, i);
-    if (k >= tau) {
-      const int slot = atomicAdd(&s_count, 1);
-      if (slot < kTreeCandCap) s_dyn[slot] = k;
+  // pass 2: the keys >= tau (logit above tv, or equal with index at most ti), kept in
+  // four registers per thread and placed by a block scan; a thread with more (or tau =
+  // 0: every logit is one) sends the block to shared-memory atomics instead
+  const float tv = tau ? key_value(tau) : -INFINITY;
+  const int ti = tau ? key_index(tau) : INT_MAX;
+  unsigned long long c0 = 0ull, c1 = 0ull, c2k = 0ull, c3 = 0ull;
+  int cnt = 0;
+  if (tau != 0ull) {
+    for_groups<BF16, VEC>(rowp, e_begin, e_end, tid, [&](const auto& x, int base) {
+      constexpr int E = sizeof(x) / sizeof(float);
+      float vmax = x[0];
+#pragma unroll
+      for (int q = 1; q < E; ++q) vmax = fmaxf(vmax, x[q]);
+      if (vmax >= tv) {
+        unsigned cm = 0u;
+#pragma unroll
+        for (int q = 0; q < E; ++q)
+          cm |= ((x[q] > tv || (x[q] == tv && base + q <= ti)) ? 1u : 0u) << q;
+        while (cm) {
+          const int q = __ffs(cm) - 1;
+          cm &= cm - 1;
+          const unsigned long long k = cand_key(pick(x, q), base + q);
+          if (cnt == 0) c0 = k;
+          else if (cnt == 1) c1 = k;
+          else if (cnt == 2) c2k = k;
+          else if (cnt == 3) c3 = k;
+          ++cnt;
+        }
+      }
+    });
+  }
+  if (!__syncthreads_or(tau == 0ull || cnt > 4)) {
+    int incl = cnt;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += y;
     }
-  });
+    if (lane == 31) s_wcnt[w] = incl;
+    __syncthreads();
+    int off = incl - cnt;
+    for (int w2 = 0; w2 < w; ++w2) off += s_wcnt[w2];
+    if (cnt > 0) s_dyn[off] = c0;
+    if (cnt > 1) s_dyn[off + 1] = c1;
+    if (cnt > 2) s_dyn[off + 2] = c2k;
+    if (cnt > 3) s_dyn[off + 3] = c3;
+    if (tid == kThreads - 1) s_count = off + cnt;
+  } else {
+    for_groups<BF16, VEC>(rowp, e_begin, e_end, tid, [&](const auto& x, int base) {
+      constexpr int E = sizeof(x) / sizeof(float);
+      float vmax = x[0];
+#pragma unroll
+      for (int q = 1; q < E; ++q) vmax = fmaxf(vmax, x[q]);
+      if (vmax >= tv) {
+        unsigned cm = 0u;
+#pragma unroll
+        for (int q = 0; q < E; ++q)
+          cm |= ((x[q] > tv || (x[q] == tv && base + q <= ti)) ? 1u : 0u) << q;
+        while (cm) {
+          const int q = __ffs(cm) - 1;
+          cm &= cm - 1;
+          const int slot = atomicAdd(&s_count, 1);
+          if (slot < kTreeCandCap) s_dyn[slot] = cand_key(pick(x, q), base + q);
+        }
+      }
+    });
+  }
   __syncthreads();
   const int C = s_count;
   unsigned long long* out = p.keys + (rid * S + split) * 64;
@@ -567,9 +878,13 @@ __global__ void __launch_bounds__(kThreads) tree_build_kernel(BuildParams p) {
     unsigned long long prev = ~0ull;
     for (int rk = 0; rk < K; ++rk) {
       unsigned long long best = 0ull;
-      for_part<BF16, VEC>(rowp, e_begin, e_end, tid, [&](float x, int i) {
-        const unsigned long long k = cand_key(x, i);
-        if (k < prev && k > best) best = k;
+      for_groups<BF16, VEC>(rowp, e_begin, e_end, tid, [&](const auto& x, int base) {
+        constexpr int E = sizeof(x) / sizeof(float);
+#pragma unroll
+        for (int q = 0; q < E; ++q) {
+          const unsigned long long k = cand_key(x[q], base + q);
+          if (k < prev && k > best) best = k;
+        }
       });
       best = block_max_u64(best, s_tmax);
       if (tid == 0) out[rk] = best;
@@ -578,7 +893,7 @@ __global__ void __launch_bounds__(kThreads) tree_build_kernel(BuildParams p) {
   }
   if (tid == 0) {
     float M = s_wm[0], Sum = s_ws[0];
-    for (int w = 1; w < kThreads / 32; ++w) merge_ms(M, Sum, s_wm[w], s_ws[w], c2);
+    for (int w2 = 1; w2 < kThreads / 32; ++w2) merge_ms(M, Sum, s_wm[w2], s_ws[w2], c2);
     p.stats[rid * S + split] = make_float4(M, Sum, __uint_as_float(static_cast<uint32_t>(s_bad)), 0.f);
   }
 
@@ -593,40 +908,43 @@ __global__ void __launch_bounds__(kThreads) tree_build_kernel(BuildParams p) {
   __syncthreads();
   if (!s_last) return;
   __threadfence();
-  unsigned long long* in = s_dyn;
-  unsigned long long* nxt = s_dyn + S * K;
-  for (int i = tid; i < S * K; i += kThreads)
-    in[i] = __ldcg(p.keys + (rid * S + i / K) * 64 + i % K);
-  __syncthreads();
-  // pairwise merges of sorted (descending) lists, each kept to its top K: a key's place
-  // is its place in its list plus the keys of the partner list above it (ties, only
-  // the zero padding, go to the even list)
-  for (int n = S; n > 1; n = (n + 1) / 2) {
-    for (int t = tid; t < n * K; t += kThreads) {
-      const int l = t / K, i = t % K, partner = l ^ 1;
-      const unsigned long long key = in[t];
-      if (partner >= n) {
-        nxt[(l >> 1) * K + i] = key;
-        continue;
-      }
-      const unsigned long long* P = in + partner * K;
-      int lo = 0, hi = K;
-      while (lo < hi) {
-        const int mid = (lo + hi) >> 1;
-        if ((l & 1) ? P[mid] >= key : P[mid] > key) lo = mid + 1;
-        else hi = mid;
-      }
-      if (i + lo < K) nxt[(l >> 1) * K + i + lo] = key;
+  // warp w merges parts w, w + 4, w + 8, w + 12 (entries K..63 read as 0), then warp 0
+  // merges the four results; warp 1 merges the normalisers meanwhile
+  unsigned long long a0, a1;
+  {
+    const unsigned long long* kb = p.keys + rid * S * 64;
+    unsigned long long x0[4], x1[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const int l = w + 4 * j;
+      x0[j] = (l < S && lane < K) ? __ldcg(kb + l * 64 + lane) : 0ull;
+      x1[j] = (l < S && lane + 32 < K) ? __ldcg(kb + l * 64 + 32 + lane) : 0ull;
     }
-    __syncthreads();
-    unsigned long long* t2 = in;
-    in = nxt;
-    nxt = t2;
+    a0 = x0[0];
+    a1 = x1[0];
+#pragma unroll
+    for (int j = 1; j < 4; ++j)
+      if (w + 4 * j < S) {
+        const ulonglong2 m2 = merge_top64(a0, a1, x0[j], x1[j], lane);
+        a0 = m2.x;
+        a1 = m2.y;
+      }
   }
-  if (tid < 32) {
+  s_dyn[w * 64 + lane] = a0;
+  s_dyn[w * 64 + 32 + lane] = a1;
+  __syncthreads();
+  if (w == 0) {
+#pragma unroll
+    for (int w2 = 1; w2 < kThreads / 32; ++w2)
+      if (w2 < S) {
+        const ulonglong2 m2 = merge_top64(a0, a1, s_dyn[w2 * 64 + lane], s_dyn[w2 * 64 + 32 + lane], lane);
+        a0 = m2.x;
+        a1 = m2.y;
+      }
+  } else if (w == 1) {
     float M = -INFINITY, Sum = 0.f;
     uint32_t anybad = 0;
-    for (int l = tid; l < S; l += 32) {
+    for (int l = lane; l < S; l += 32) {
       const float4 st = __ldcg(p.stats + rid * S + l);
       merge_ms(M, Sum, st.x, st.y, c2);
       anybad |= __float_as_uint(st.z);
@@ -637,21 +955,21 @@ __global__ void __launch_bounds__(kThreads) tree_build_kernel(BuildParams p) {
       merge_ms(M, Sum, m2, s2, c2);
     }
     anybad = __reduce_or_sync(0xffffffffu, anybad);
-    if (tid == 0) {
+    if (lane == 0) {
       s_wm[0] = M;
       s_ws[0] = Sum;
       s_bad = (anybad || !(M > -INFINITY)) ? 1 : 0;
     }
   }
   __syncthreads();
-  {
-    const float M = s_wm[0], lnS = logf(s_ws[0]);
+  if (w == 0) {
     // log q = (x - max) / T - log sum exp((x_j - max) / T)
-    if (tid < K) {
-      const unsigned long long k = in[tid];
-      p.table[rid * 64 + tid] = make_int2(key_index(k), __float_as_int((key_value(k) - M) * invT - lnS));
-    }
-    if (tid == 0 && s_bad) atomicOr(&p.seq_flags[b], SPEC_FLAG_BAD_LOGITS);
+    const float M = s_wm[0], lnS = logf(s_ws[0]);
+    int2* trow = p.table + rid * 64;
+    if (lane < K) trow[lane] = make_int2(key_index(a0), __float_as_int((key_value(a0) - M) * invT - lnS));
+    if (lane + 32 < K)
+      trow[lane + 32] = make_int2(key_index(a1), __float_as_int((key_value(a1) - M) * invT - lnS));
+    if (lane == 0 && s_bad) atomicOr(&p.seq_flags[b], SPEC_FLAG_BAD_LOGITS);
   }
 
   // the sequence's last row block selects the nodes
@@ -677,77 +995,8 @@ __global__ void __launch_bounds__(kThreads) tree_build_kernel(BuildParams p) {
   }
   __syncthreads();
   if (tid >= 32) return;
-  const int lane = tid, N = p.nodes;
-  const int64_t base = static_cast<int64_t>(b) * N;
-  uint32_t flags = s_flags;
-  TreeNode n0, n1;
-  n0.dep = n1.dep = -1;
-  n0.key = n1.key = 0ull;
-  n0.nx = n1.nx = 0;
-  n0.tok = n1.tok = -1;
-  n0.par = n1.par = -1;
-  n0.msk = n1.msk = 0ull;
-  n0.sc = n1.sc = 0.0;
-  if (!flags) {
-    if (lane == 0) {
-      n0.dep = 0;
-      n0.tok = p.root[b];
-      n0.msk = 1ull;
-      refresh_offer(n0, tab, p.rows, K);
-    }
-    for (int i = 1; i < N; ++i) {
-      // the best offer: the largest key, then the lowest node index
-      const unsigned long long kl = n0.key > n1.key ? n0.key : n1.key;
-      const uint32_t Mh = __reduce_max_sync(0xffffffffu, static_cast<uint32_t>(kl >> 32));
-      const uint32_t Ml = __reduce_max_sync(
-          0xffffffffu, static_cast<uint32_t>(kl >> 32) == Mh ? static_cast<uint32_t>(kl) : 0u);
-      const unsigned long long M = (static_cast<unsigned long long>(Mh) << 32) | Ml;
-      if (M == 0ull) {  // no offer left: excluded by the host's capacity check
-        flags |= SPEC_FLAG_BAD_TREE;
-        break;
-      }
-      const unsigned b0 = __ballot_sync(0xffffffffu, n0.key == M);
-      const int u = b0 ? __ffs(b0) - 1 : 32 + __ffs(__ballot_sync(0xffffffffu, n1.key == M)) - 1;
-      const int src = u & 31;
-      const bool hs = u >= 32;
-      const double osc = __shfl_sync(0xffffffffu, hs ? n1.osc : n0.osc, src);
-      const int otk = __shfl_sync(0xffffffffu, hs ? n1.otk : n0.otk, src);
-      const int pdep = __shfl_sync(0xffffffffu, hs ? n1.dep : n0.dep, src);
-      const unsigned long long pm = __shfl_sync(0xffffffffu, hs ? n1.msk : n0.msk, src);
-      if (lane == src) {
-        if (hs) {
-          ++n1.nx;
-          refresh_offer(n1, tab, p.rows, K);
-        } else {
-          ++n0.nx;
-          refresh_offer(n0, tab, p.rows, K);
-        }
-      }
-      if (lane == (i & 31)) {
-        TreeNode c;
-        c.dep = pdep + 1;
-        c.nx = 0;
-        c.tok = otk;
-        c.par = u;
-        c.sc = osc;
-        c.msk = pm | (1ull << i);
-        refresh_offer(c, tab, p.rows, K);
-        if (i >= 32) n1 = c;
-        else n0 = c;
-      }
-    }
-  }
-#pragma unroll
-  for (int h = 0; h < 2; ++h) {
-    const int c = lane + 32 * h;
-    if (c >= N) continue;
-    const TreeNode& n = h ? n1 : n0;
-    p.tokens[base + c] = flags ? -1 : n.tok;
-    p.parents[base + c] = flags ? -1 : n.par;
-    if (p.depth) p.depth[base + c] = flags ? -1 : n.dep;
-    if (p.mask) p.mask[base + c] = flags ? 0ull : n.msk;
-  }
-  if (lane == 0 && flags) set_status(p.status, flags);
+  if (p.nodes <= 33) select_nodes<1>(p, tab, K, b, s_flags, lane);
+  else select_nodes<2>(p, tab, K, b, s_flags, lane);
 }
 
 // num_nodes = 1: the tree is its root
@@ -838,7 +1087,7 @@ TreeBuildLayout tree_build_layout(const spec_tree_build_args_t& t, size_t base, 
   L.table = ws_round(L.stats + 16 * nrows * L.splits);
   L.end = ws_round(L.table + 64 * 8 * nrows);
   const int k = L.keff;
-  L.smem = static_cast<int>(8 * std::max(std::max(kTreeCandCap, 2 * L.splits * k), L.rows * k));
+  L.smem = static_cast<int>(8 * std::max(std::max(kTreeCandCap, 4 * 64), L.rows * k));
   return L;
 }
 
