@@ -44,15 +44,15 @@ L2_FLUSH_BYTES = 256 << 20
 # while the kernel's sources still hash to what they were when the capture was taken.
 MEASURED_TRAFFIC = {
     ("llama8b", "attention"): {
-        "bytes": 139_308_800,
+        "bytes": 138_946_816,
         "profile": "profiles/attn_tc_kernel_llama8b.md",
         "sources": {
             "paper_2609_04010_gb300/csrc/attn_tc.cu":
-                "194e2351e6d39423418b78a4fb5a4e4d49002d0329417b93b7e5987178d1ee38",
+                "b783408626c37f9be4931410fdbb20774331ab9dd36b11b6207f343fab9737e5",
             "paper_2609_04010_gb300/csrc/attn_common.cuh":
-                "ed48d4dd71d0521ef69a8e8a78e8c0c0d5d8fe094a7a2784a1b3c0412f23e131",
+                "fcccb38e95b02d314a545f1bc6bab2f21d76dea3e287ecd0ac3833d50a3798cc",
             "paper_2609_04010_gb300/csrc/common.cuh":
-                "2043c94505012a600bb927d65add0620cd827fe46f727917cd25e3eafbfc73bc",
+                "fb34291b5c1d1b7986c17ea7c68c55fcec41cefae83e63c137374784cb8cac46",
         },
     },
 }
