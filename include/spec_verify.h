@@ -424,6 +424,40 @@ spec_status_t spec_build_tree(const spec_tree_build_args_t* build, void* ws, siz
                               spec_stream_t stream);
 
 /*
+ * The target's LM head with the row statistics of the acceptance fused into it (the
+ * verifier pass of Sec. 4.2 scores the block rows with the target's output layer;
+ * Appendix B.3's rule reads p = softmax(logits / T) through its normaliser, its
+ * maximum and the logit of a drafted token): logits = hidden_states . weight^T on the
+ * tensor cores (bf16 operands, fp32 accumulation), reduced per row as they leave the
+ * accumulator, so the [rows][vocab] logits need not be written.
+ *
+ * Row r belongs to sequence r / rows_per_seq, whose temperature is T. Outputs per row:
+ * row_max = max_v l_v; row_sum = sum_v exp((l_v - row_max) / T) (T <= 0 or NaN sums at
+ * T = 1); row_argmax = the lowest index of the maximum; token_logit (if given) = l at
+ * tokens[r] (NaN where tokens is NULL or tokens[r] is outside [0, vocab)). logits (if
+ * given) receives every logit as bf16 [rows][vocab] (the rounding of the fp32 value).
+ * A row with a NaN or an infinite logit sets SPEC_FLAG_BAD_LOGITS and gets
+ * row_argmax = -1. Device memory, caller-owned; hidden_states and weight 16-byte
+ * aligned, hidden a multiple of 8.
+ */
+typedef struct {
+  int32_t rows, hidden, vocab, rows_per_seq;
+  const void* hidden_states;   /* bf16 [rows][hidden]                                    */
+  const void* weight;          /* bf16 [vocab][hidden]: output row v of the LM head       */
+  const float* temperature;    /* [rows / rows_per_seq]                                   */
+  const int32_t* tokens;       /* [rows], or NULL                                         */
+  float* row_max;              /* [rows], written                                         */
+  float* row_sum;              /* [rows], written                                         */
+  int32_t* row_argmax;         /* [rows], written                                         */
+  float* token_logit;          /* [rows], written, or NULL                                */
+  void* logits;                /* bf16 [rows][vocab], written, or NULL                    */
+} spec_lm_head_args_t;
+
+size_t spec_lm_head_workspace_size(const spec_lm_head_args_t* lm);
+spec_status_t spec_lm_head_stats(const spec_lm_head_args_t* lm, void* ws, size_t ws_bytes,
+                                 spec_stream_t stream);
+
+/*
  * spec_accept_block without a workspace, for callers that cannot allocate device
  * memory when they verify (for example, code confined to a fixed, pre-planned memory
  * arena, or code that must not call an allocator). It computes exactly what

@@ -551,6 +551,45 @@ def compact_tree_kv(k_cache, v_cache, page_table, kv_len, num_nodes: int, path, 
     return k, v, kl
 
 
+def lm_head_stats(hidden, weight, temperature, rows_per_seq: int, tokens=None, rows=None,
+                  chunk: int = 8192):
+    """The target's LM head and the acceptance's row statistics (Sec. 4.2 verifier pass;
+    Appendix B.3 reads p = softmax(l / T) through its normaliser, maximum and drafted
+    logits): l = hidden . weight^T in fp64 on the exactly decoded bf16 operands (a
+    matmul per chunk of vocab rows), then per row r (sequence r // rows_per_seq):
+    max, the lowest index of the max, sum_v exp((l_v - max) / T) (T <= 0 sums at T = 1)
+    and l at tokens[r] (NaN where tokens is None or the token is outside [0, vocab)).
+
+    hidden: uint16 bf16 bits [rows][H]; weight: uint16 [vocab][H]; rows: optional row
+    indices to compute. Returns a dict: row_max, row_sum, row_argmax, token_logit (over
+    the selected rows), logits (fp64 [selected rows][vocab]) and abs_bound (fp64, per
+    row: max_v sum_i |h_i w_vi|, which bounds a logit's accumulation error)."""
+    h = _rows_f64(hidden)
+    sel = np.arange(h.shape[0]) if rows is None else np.asarray(rows, dtype=np.int64)
+    hs = h[sel]
+    V = weight.shape[0]
+    logits = np.empty((len(sel), V), np.float64)
+    bound = np.zeros(len(sel), np.float64)
+    for v0 in range(0, V, chunk):
+        w = _rows_f64(weight[v0:v0 + chunk])
+        logits[:, v0:v0 + chunk] = hs @ w.T
+        bound = np.maximum(bound, (np.abs(hs) @ np.abs(w).T).max(axis=1))
+    out = dict(row_max=np.empty(len(sel)), row_sum=np.empty(len(sel)),
+               row_argmax=np.empty(len(sel), np.int64), token_logit=np.full(len(sel), np.nan),
+               logits=logits, abs_bound=bound)
+    for i, r in enumerate(sel):
+        T = float(np.float32(temperature[r // rows_per_seq]))
+        T = T if T > 0 else 1.0
+        l = logits[i]
+        m = l.max()
+        out["row_max"][i] = m
+        out["row_argmax"][i] = int(np.argmax(l))
+        out["row_sum"][i] = np.exp((l - m) / T).sum()
+        if tokens is not None and 0 <= int(tokens[r]) < V:
+            out["token_logit"][i] = l[int(tokens[r])]
+    return out
+
+
 def verify_attention(q, k_cache, v_cache, page_table, kv_len, gamma: int, softmax_scale=None,
                      rows=None, nthreads: int = 0, tree_mask=None):
     """fp64 block-causal paged GQA attention.

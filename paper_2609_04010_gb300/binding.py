@@ -109,6 +109,15 @@ class TreeBuildArgs(ctypes.Structure):
                 ("depth", ctypes.c_void_p), ("tree_mask", ctypes.c_void_p)]
 
 
+class LmHeadArgs(ctypes.Structure):
+    _fields_ = [("rows", ctypes.c_int32), ("hidden", ctypes.c_int32), ("vocab", ctypes.c_int32),
+                ("rows_per_seq", ctypes.c_int32), ("hidden_states", ctypes.c_void_p),
+                ("weight", ctypes.c_void_p), ("temperature", ctypes.c_void_p),
+                ("tokens", ctypes.c_void_p), ("row_max", ctypes.c_void_p),
+                ("row_sum", ctypes.c_void_p), ("row_argmax", ctypes.c_void_p),
+                ("token_logit", ctypes.c_void_p), ("logits", ctypes.c_void_p)]
+
+
 HEADER = os.path.join(_build.ROOT, "include", "spec_verify.h")
 
 
@@ -163,6 +172,10 @@ def lib(build_if_missing: bool = True):
             L.spec_accept_tree.restype = ctypes.c_int
             L.spec_commit_tree_kv.argtypes = [P, P]
             L.spec_commit_tree_kv.restype = ctypes.c_int
+            L.spec_lm_head_workspace_size.argtypes = [P]
+            L.spec_lm_head_workspace_size.restype = ctypes.c_size_t
+            L.spec_lm_head_stats.argtypes = [P, P, ctypes.c_size_t, P]
+            L.spec_lm_head_stats.restype = ctypes.c_int
             L.spec_tree_build_workspace_size.argtypes = [P]
             L.spec_tree_build_workspace_size.restype = ctypes.c_size_t
             L.spec_build_tree.argtypes = [P, P, ctypes.c_size_t, P]
@@ -567,6 +580,62 @@ def build_tree(drafter_logits, temperature, root_tokens, top_k: int, num_nodes: 
         ws = new_workspace(tree_build_workspace_size(t), dev)
     build_tree_args(t, ws, stream)
     return res
+
+
+def lm_head_args(hidden_states, weight, temperature, rows_per_seq: int, out: Dict[str, torch.Tensor],
+                 tokens=None) -> LmHeadArgs:
+    R, H = hidden_states.shape
+    V, H2 = weight.shape
+    if H2 != H:
+        raise ValueError("weight and hidden states disagree on the hidden size")
+    _check(hidden_states, "hidden_states", torch.bfloat16)
+    _check(weight, "weight", torch.bfloat16)
+    _check(temperature, "temperature", torch.float32)
+    if tokens is not None:
+        _check(tokens, "tokens", torch.int32, (R,))
+    for k in ("row_max", "row_sum"):
+        _check(out[k], k, torch.float32, (R,))
+    _check(out["row_argmax"], "row_argmax", torch.int32, (R,))
+    if out.get("token_logit") is not None:
+        _check(out["token_logit"], "token_logit", torch.float32, (R,))
+    if out.get("logits") is not None:
+        _check(out["logits"], "logits", torch.bfloat16, (R, V))
+    return LmHeadArgs(R, H, V, int(rows_per_seq), hidden_states.data_ptr(), weight.data_ptr(),
+                      temperature.data_ptr(), _ptr(tokens), out["row_max"].data_ptr(),
+                      out["row_sum"].data_ptr(), out["row_argmax"].data_ptr(),
+                      _ptr(out.get("token_logit")), _ptr(out.get("logits")))
+
+
+def lm_head_workspace_size(a: LmHeadArgs) -> int:
+    n = lib().spec_lm_head_workspace_size(ctypes.byref(a))
+    if n == 0:
+        raise SpecError(1, "spec_lm_head_workspace_size")
+    return int(n)
+
+
+def lm_head_stats_args(a: LmHeadArgs, ws: torch.Tensor, stream=None):
+    _raise(lib().spec_lm_head_stats(ctypes.byref(a), _ptr(ws), ws.numel(), _stream(stream)),
+           "spec_lm_head_stats")
+
+
+def lm_head_stats(hidden_states, weight, temperature, rows_per_seq: int, tokens=None,
+                  want_logits: bool = False, ws=None, stream=None) -> Dict[str, torch.Tensor]:
+    """spec_lm_head_stats: the LM head's logits reduced per row (max, sum of
+    exp((l - max) / T), lowest-index argmax, the token's logit); the logits themselves
+    (bf16) only if want_logits."""
+    R = hidden_states.shape[0]
+    V = weight.shape[0]
+    dev = hidden_states.device
+    out = dict(row_max=torch.empty(R, dtype=torch.float32, device=dev),
+               row_sum=torch.empty(R, dtype=torch.float32, device=dev),
+               row_argmax=torch.empty(R, dtype=torch.int32, device=dev),
+               token_logit=torch.empty(R, dtype=torch.float32, device=dev) if tokens is not None else None,
+               logits=torch.empty(R, V, dtype=torch.bfloat16, device=dev) if want_logits else None)
+    a = lm_head_args(hidden_states, weight, temperature, rows_per_seq, out, tokens)
+    if ws is None:
+        ws = new_workspace(lm_head_workspace_size(a), dev)
+    lm_head_stats_args(a, ws, stream)
+    return {k: v for k, v in out.items() if v is not None}
 
 
 def philox_uniforms(seed: int, n: int, offset: int = 0, device=None, stream=None) -> torch.Tensor:

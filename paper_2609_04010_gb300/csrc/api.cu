@@ -156,6 +156,19 @@ spec_status_t check_tree_build(const spec_tree_build_args_t* t) {
   return SPEC_OK;
 }
 
+spec_status_t check_lm_head(const spec_lm_head_args_t* a) {
+  if (!a) return SPEC_ERR_INVALID_ARGUMENT;
+  if (a->rows < 1 || a->hidden < 8 || a->hidden % 8 != 0 || a->vocab < 1 || a->rows_per_seq < 1)
+    return SPEC_ERR_INVALID_ARGUMENT;
+  if (!a->hidden_states || !a->weight || !a->temperature || !a->row_max || !a->row_sum ||
+      !a->row_argmax)
+    return SPEC_ERR_INVALID_ARGUMENT;
+  if ((reinterpret_cast<uintptr_t>(a->hidden_states) | reinterpret_cast<uintptr_t>(a->weight)) & 15u)
+    return SPEC_ERR_INVALID_ARGUMENT;
+  if ((a->rows + kLmTileM - 1) / kLmTileM > 65535) return SPEC_ERR_UNSUPPORTED;
+  return SPEC_OK;
+}
+
 spec_status_t check_filter(const spec_filter_args_t* f) {
   if (!f || !f->top_k || !f->top_p) return SPEC_ERR_INVALID_ARGUMENT;
   if (f->max_top_k < 1) return SPEC_ERR_INVALID_ARGUMENT;
@@ -482,6 +495,24 @@ spec_status_t spec_build_tree(const spec_tree_build_args_t* t, void* ws, size_t 
   if (L.end > ws_bytes) return SPEC_ERR_WORKSPACE_TOO_SMALL;
   return launch_tree_build(*t, L, static_cast<char*>(ws), stream, vec) == cudaSuccess ? SPEC_OK
                                                                                        : SPEC_ERR_CUDA;
+}
+
+size_t spec_lm_head_workspace_size(const spec_lm_head_args_t* a) {
+  if (check_lm_head(a) != SPEC_OK) return 0;
+  return lm_layout(*a, kWsHeader).end;
+}
+
+spec_status_t spec_lm_head_stats(const spec_lm_head_args_t* a, void* ws, size_t ws_bytes,
+                                 spec_stream_t stream_) {
+  const spec_status_t st = check_lm_head(a);
+  if (st != SPEC_OK) return st;
+  if (!ws || (reinterpret_cast<uintptr_t>(ws) % kWsAlign) != 0) return SPEC_ERR_INVALID_ARGUMENT;
+  const LmLayout L = lm_layout(*a, kWsHeader);
+  if (L.end > ws_bytes) return SPEC_ERR_WORKSPACE_TOO_SMALL;
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  int sms = 0;
+  if (!bind_device(stream, &sms)) return SPEC_ERR_CUDA;
+  return launch_lm_head(*a, L, static_cast<char*>(ws), stream) == cudaSuccess ? SPEC_OK : SPEC_ERR_CUDA;
 }
 
 spec_status_t spec_commit_tree_kv(const spec_tree_commit_args_t* c, spec_stream_t stream) {

@@ -253,6 +253,32 @@ def _bf16_normals(rng: np.random.Generator, shape, chunk: int = 1 << 24) -> np.n
     return out.reshape(shape)
 
 
+def make_lm_inputs(rows: int, hidden: int, vocab: int, rows_per_seq: int, sigma: float = 3.0,
+                   temperature=1.0, seed: int = 0, chunk: int = 1 << 14):
+    """Synthetic LM-head operands: hidden states ~ N(0, 1) rounded to bf16, and weight
+    entries uniform with variance sigma^2 / hidden, cut to bf16 by dropping the low 16
+    bits of the fp32 value (one cheap pass over the 10^8..10^9 entries of a real head),
+    so that logits are about N(0, sigma^2); per-sequence temperatures (cycled from
+    `temperature`) and one token per row. Returns (hidden uint16 [rows][hidden], weight
+    uint16 [vocab][hidden], temperature float32 [rows // rows_per_seq], tokens int32
+    [rows])."""
+    ss = np.random.SeedSequence([seed, 41])
+    g_h, g_w, g_t = (np.random.Generator(np.random.PCG64(c)) for c in ss.spawn(3))
+    h = f32_to_bf16_bits(g_h.standard_normal((rows, hidden), dtype=np.float32)).reshape(rows, hidden)
+    w = np.empty((vocab, hidden), np.uint16)
+    half = np.float32(np.sqrt(3.0) * sigma / np.sqrt(hidden))  # U(-a, a) has variance a^2 / 3
+    for v0 in range(0, vocab, chunk):
+        n = min(chunk, vocab - v0)
+        x = g_w.random((n, hidden), dtype=np.float32)
+        x *= np.float32(2) * half
+        x -= half
+        w[v0:v0 + n] = (x.view(np.uint32) >> np.uint32(16)).astype(np.uint16)
+    nseq = (rows + rows_per_seq - 1) // rows_per_seq
+    temps = np.resize(np.asarray(temperature, np.float32), nseq).astype(np.float32)
+    tokens = g_t.integers(0, vocab, rows).astype(np.int32)
+    return h, w, temps, tokens
+
+
 def make_attn_inputs(batch: int, gamma: int, num_q_heads: int, num_kv_heads: int, head_dim: int,
                      page_size: int, ctx, permute_pages: bool = True, seed: int = 0,
                      extra_pages: int = 0) -> AttnInputs:
