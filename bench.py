@@ -88,6 +88,8 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-draft", action="store_true",
                     help="skip the draft-side timing (block sampling, KV commit)")
+    ap.add_argument("--no-lm-head", action="store_true",
+                    help="skip the fused LM head + row statistics timing")
     ap.add_argument("--no-tree", action="store_true",
                     help="skip the tree verification timing (tree sampler, tree attention, "
                          "greedy tree acceptance, KV compaction)")
@@ -481,6 +483,8 @@ def run_ours(args, wl, ai, ci, rank, world, local_rank):
 
     tree = None if args.no_tree else time_tree(wl, ai, ci, binding, dev, graph_of, timed_loop,
                                                parts_n, stream)
+    lm_head = None if args.no_lm_head else time_lm_head(ai, ci, binding, dev, graph_of, timed_loop,
+                                                        parts_n)
 
     emitted = sum_over_ranks(float(ne.sum().item()), world, dev)
     tm = traffic_model(ai, ci)
@@ -531,7 +535,48 @@ def run_ours(args, wl, ai, ci, rank, world, local_rank):
         result["draft"] = draft
     if tree:
         result["tree"] = tree
+    if lm_head:
+        result["lm_head"] = lm_head
     return result
+
+
+def time_lm_head(ai, ci, binding, dev, graph_of, timed_loop, n):
+    """The fused LM head + row statistics on the step's rows (batch x gamma hidden states)
+    with the workload's head (hidden = query heads x head dim, the vocabulary), random
+    bf16 operands made on the device: one graph replay of spec_lm_head_stats per timed
+    launch, L2 flushed before each (the weight is larger than L2 anyway)."""
+    import torch
+
+    R = ci.batch * ci.gamma
+    H = ai.q.shape[2] * ai.q.shape[3]
+    V = ci.vocab
+    g = torch.Generator(device=dev)
+    g.manual_seed(31)
+    hidden = torch.randn(R, H, generator=g, device=dev, dtype=torch.float32).to(torch.bfloat16)
+    weight = (torch.randn(V, H, generator=g, device=dev, dtype=torch.float32) * (3.0 / H ** 0.5)).to(torch.bfloat16)
+    temp = torch.ones(ci.batch, dtype=torch.float32, device=dev)
+    tok = torch.randint(0, V, (R,), generator=g, device=dev, dtype=torch.int32)
+    out = dict(row_max=torch.empty(R, dtype=torch.float32, device=dev),
+               row_sum=torch.empty(R, dtype=torch.float32, device=dev),
+               row_argmax=torch.empty(R, dtype=torch.int32, device=dev),
+               token_logit=torch.empty(R, dtype=torch.float32, device=dev))
+    a = binding.lm_head_args(hidden, weight, temp, ci.gamma, out, tok)
+    ws = binding.new_workspace(binding.lm_head_workspace_size(a), dev)
+    gr = graph_of(lambda: binding.lm_head_stats_args(a, ws))
+    ms = statistics.mean(timed_loop(gr.replay, n))
+    code, flags = binding.read_device_status(ws)
+    if code != 0:
+        raise RuntimeError(f"lm head: device status {code} flags {flags}")
+    nbytes = (V + R) * H * 2
+    peak = measured_peaks()[0]
+    gbs = nbytes / (ms / 1000.0) / 1e9
+    del weight
+    torch.cuda.empty_cache()
+    return {"shape": {"rows": R, "hidden": H, "vocab": V},
+            "lm_head_ms": ms, "algorithmic_bytes": int(nbytes), "achieved_gbs": round(gbs, 1),
+            "frac_of_measured": round(gbs / peak, 4),
+            "useful_tflops": round(2.0 * R * H * V / (ms / 1000.0) / 1e12, 1),
+            "timing": "CUDA-graph replays of spec_lm_head_stats, L2 flushed before each"}
 
 
 TREE_BLOCK, TREE_TOP_K, TREE_NODES = 16, 32, 33   # the tree sampler's (B, K, V) = (16, 32, 32)

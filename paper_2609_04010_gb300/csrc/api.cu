@@ -9,6 +9,7 @@
 #include <cstring>
 
 #include "common.cuh"
+#include "lm_head.cuh"
 
 namespace specv {
 

@@ -133,18 +133,6 @@ TreeBuildLayout tree_build_layout(const spec_tree_build_args_t& t, size_t base, 
 cudaError_t launch_tree_build(const spec_tree_build_args_t& t, const TreeBuildLayout& L, char* ws,
                               cudaStream_t stream, bool vec);
 
-// --- fused LM head + row statistics ---
-constexpr int kLmTileN = 256;  // vocab rows per tile (MMA N)
-constexpr int kLmTileM = 128;  // hidden-state rows per tile (MMA M)
-struct LmLayout {
-  size_t parts;  // 16 B [rows][vocab tiles]: (max, sum, argmax, token logit) per tile
-  size_t end;
-  int ntiles_n, ntiles_m;
-};
-LmLayout lm_layout(const spec_lm_head_args_t& a, size_t base);
-cudaError_t launch_lm_head(const spec_lm_head_args_t& a, const LmLayout& L, char* ws,
-                           cudaStream_t stream);
-
 // --- attention ---
 struct AttnPlan {
   int path;          // SPEC_ATTN_CUDA_CORES or SPEC_ATTN_TENSOR_CORES

@@ -2,10 +2,10 @@
 // the verifier pass scores the block rows; Appendix B.3: the rule reads p through its
 // normaliser, maximum and the logits of drafted tokens).
 //
-// lm_head_kernel: one block per (256-row vocab tile, 128-row hidden-state tile). Warp 0
-// streams 64-column slices of the hidden states and of the weight rows by TMA (128-byte
-// swizzle, out-of-range rows read as zeros) into a 4-stage ring; warp 1 issues
-// tcgen05.mma (M = 128, N = 256, K = 16) into a 256-column fp32 TMEM accumulator; warps
+// lm_head_kernel: one block per (224-row vocab tile, 128-row hidden-state tile), two
+// blocks per SM. Warp 0 streams 64-column slices of the hidden states and of the weight
+// rows by TMA (128-byte swizzle, out-of-range rows read as zeros) into a 2-stage ring;
+// warp 1 issues tcgen05.mma (M = 128, N = 224, K = 16) into an fp32 TMEM accumulator; warps
 // 2..5 then read one logit row each (a warp reaches the TMEM lanes of its own
 // sub-partition) and reduce it, 32 columns at a time, to (max, sum of
 // exp((l - max) / T), lowest-index argmax, logit of the row's token), optionally
@@ -17,6 +17,7 @@
 #include <climits>
 #include <cmath>
 
+#include "lm_head.cuh"
 #include "tc_ptx.cuh"
 
 namespace specv {
@@ -35,7 +36,7 @@ namespace {
 using namespace tcx;
 
 constexpr int kBK = 64;      // hidden elements per stage: one 128-byte swizzle span
-constexpr int kStages = 4;
+constexpr int kStages = 2;  // 88 KB of shared memory: two blocks per SM, one streams while the other reduces
 constexpr uint32_t kABytes = kLmTileM * 128;  // 16 KB of hidden states per stage
 constexpr uint32_t kBBytes = kLmTileN * 128;  // 32 KB of weight rows per stage
 constexpr uint32_t kOffA = 0;
@@ -44,6 +45,9 @@ constexpr uint32_t kOffBar = kOffB + kStages * kBBytes;      // full[S], empty[S
 constexpr uint32_t kOffMisc = kOffBar + (2 * kStages + 1) * 8;  // TMEM base, abort flag
 constexpr size_t kSmem = kOffMisc + 16 + 1024;                // + 1 KB alignment slack
 constexpr int kThreads = 192;  // warp 0 TMA, warp 1 MMA, warps 2..5 reduce
+// TMEM columns to allocate: a power of two >= 32 that holds the N fp32 accumulator columns
+constexpr uint32_t kTmemCols = kLmTileN <= 32 ? 32 : kLmTileN <= 64 ? 64 : kLmTileN <= 128 ? 128
+                             : kLmTileN <= 256 ? 256 : 512;
 
 struct LmPart {
   float m, s;   // tile maximum and sum of 2^((l - m) * c2)
@@ -86,7 +90,7 @@ __device__ __forceinline__ void merge_part(float& m, float& s, int& a, float m2,
   m = M;
 }
 
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kThreads)
     lm_head_kernel(const __grid_constant__ CUtensorMap map_h, const __grid_constant__ CUtensorMap map_w,
                    LmParams p) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
@@ -111,7 +115,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     *abort_flag = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
-  if (warp == 1) tmem_alloc(smem_u32(misc), kLmTileN);
+  if (warp == 1) tmem_alloc(smem_u32(misc), kTmemCols);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -237,7 +241,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem, kLmTileN);
+    tmem_dealloc(tmem, kTmemCols);
   }
 }
 
