@@ -214,3 +214,32 @@ def test_tree_workspace_sizes_and_checks(lib):
     c.head_dim, c.path = 128, None
     assert lib.spec_commit_tree_kv(ctypes.byref(c), None) == 1
     assert lib.spec_commit_tree_kv(None, None) == 1
+
+
+def _lm(**kw):
+    a = dict(rows=64, hidden=4096, vocab=128256, rows_per_seq=8, hidden_states=4096, weight=4096,
+             temperature=4096, tokens=None, row_max=4096, row_sum=4096, row_argmax=4096,
+             token_logit=None, logits=None)
+    a.update(kw)
+    return binding.LmHeadArgs(**a)
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(rows=0), 1), (dict(hidden=12), 1), (dict(hidden=4), 1), (dict(vocab=0), 1),
+    (dict(rows_per_seq=0), 1), (dict(weight=None), 1), (dict(row_argmax=None), 1),
+    (dict(hidden_states=4104), 1), (dict(weight=4100), 1), (dict(rows=128 * 65536), 2),
+])
+def test_lm_head_host_checks(lib, kw, code):
+    a = _lm(**kw)
+    assert lib.spec_lm_head_stats(ctypes.byref(a), ctypes.c_void_p(4096), 1 << 30, None) == code
+    assert lib.spec_lm_head_workspace_size(ctypes.byref(a)) == 0
+
+
+def test_lm_head_workspace(lib):
+    a = _lm()
+    n = lib.spec_lm_head_workspace_size(ctypes.byref(a))
+    # a status header and 16 bytes per row and 224-row vocab tile
+    assert n >= 256 + 16 * 64 * ((128256 + 223) // 224) and n % 256 == 0
+    assert lib.spec_lm_head_stats(ctypes.byref(a), ctypes.c_void_p(4096), n - 256, None) == 3
+    assert lib.spec_lm_head_stats(ctypes.byref(a), ctypes.c_void_p(4097), n, None) == 1
+    assert lib.spec_lm_head_stats(None, ctypes.c_void_p(4096), n, None) == 1
