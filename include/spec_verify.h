@@ -172,8 +172,13 @@ spec_status_t spec_verify_attention(const spec_attn_args_t* attn, void* ws, size
 spec_status_t spec_accept_block(const spec_accept_args_t* accept, void* ws, size_t ws_bytes,
                                 spec_stream_t stream);
 
-/* The whole verify step: parts (a) and (b) on one stream (they share no data: the
- * logits are inputs). Either argument may be NULL to run only the other part. */
+/* The whole verify step: parts (a) and (b), ordered on `stream` (they share no data:
+ * the logits are inputs). Either argument may be NULL to run only the other part. With
+ * both, part (b) runs on a second stream of the calling host thread (created on its
+ * first such call and kept for the thread's life) between a fork event recorded on
+ * `stream` and a join event that `stream` waits for, so the two parts overlap; this
+ * also holds under stream capture. The filtered step (spec_verify_step_filtered) does
+ * the same. */
 spec_status_t spec_verify_step(const spec_attn_args_t* attn, const spec_accept_args_t* accept,
                                void* ws, size_t ws_bytes, spec_stream_t stream);
 

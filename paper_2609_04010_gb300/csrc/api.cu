@@ -49,6 +49,36 @@ bool bind_device(cudaStream_t stream, int* sms) {
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
+// A second stream of this host thread on a device, with a fork and a join event, made on
+// first use and kept for the thread's life. Per thread, so that calls from different
+// threads never record the same event; a call's fork and join also work under stream
+// capture (the side stream joins the capture through the fork event).
+struct SideStream {
+  cudaStream_t stream = nullptr;
+  cudaEvent_t fork = nullptr, join = nullptr;
+};
+
+SideStream* side_stream(int dev) {
+  thread_local SideStream cache[kMaxDevices];
+  if (dev < 0 || dev >= kMaxDevices) return nullptr;
+  SideStream& ss = cache[dev];
+  if (!ss.stream) {
+    cudaStream_t st = nullptr;
+    cudaEvent_t f = nullptr, j = nullptr;
+    if (cudaStreamCreateWithFlags(&st, cudaStreamNonBlocking) != cudaSuccess) return nullptr;
+    if (cudaEventCreateWithFlags(&f, cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&j, cudaEventDisableTiming) != cudaSuccess) {
+      if (f) cudaEventDestroy(f);
+      cudaStreamDestroy(st);
+      return nullptr;
+    }
+    ss.stream = st;
+    ss.fork = f;
+    ss.join = j;
+  }
+  return &ss;
+}
+
 spec_status_t check_attn(const spec_attn_args_t* a) {
   if (!a) return SPEC_ERR_INVALID_ARGUMENT;
   if (a->batch < 1 || a->gamma < 1 || a->num_q_heads < 1 || a->num_kv_heads < 1 ||
@@ -279,9 +309,21 @@ spec_status_t run(const spec_attn_args_t* attn, const spec_accept_args_t* accept
   if (required_bytes(attn, accept, filter, sms, &attn_base) > ws_bytes)
     return SPEC_ERR_WORKSPACE_TOO_SMALL;
   char* w = static_cast<char*>(ws);
-  // Attention first; the acceptance kernels follow as programmatic dependents, so they
-  // start on the SM resources the attention kernel leaves free and the two parts
-  // overlap (they share no data: the logits are inputs).
+  // A whole step forks: the acceptance kernels run on this thread's side stream beside
+  // the attention kernel (they share no data: the logits are inputs), on the SM
+  // resources it leaves free, and the caller's stream waits for both. On one stream the
+  // decisions, which wait for their inputs with griddepcontrol.wait, would also wait for
+  // the attention kernel before them.
+  cudaStream_t acc_stream = stream;
+  SideStream* side = nullptr;
+  if (attn && accept) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || !(side = side_stream(dev))) return SPEC_ERR_CUDA;
+    if (cudaEventRecord(side->fork, stream) != cudaSuccess ||
+        cudaStreamWaitEvent(side->stream, side->fork, 0) != cudaSuccess)
+      return SPEC_ERR_CUDA;
+    acc_stream = side->stream;
+  }
   if (attn) {
     const AttnPlan P = attn_plan(*attn, attn_base, sms, attn->path);
     const cudaError_t e = P.path == SPEC_ATTN_TENSOR_CORES ? launch_attn_tc(*attn, P, w, stream)
@@ -290,12 +332,15 @@ spec_status_t run(const spec_attn_args_t* attn, const spec_accept_args_t* accept
   }
   if (accept && filter) {
     const FilterLayout L = filter_layout(*accept, filter->max_top_k, kWsHeader, sms);
-    if (launch_accept_filtered(*accept, *filter, L, w, stream, attn != nullptr) != cudaSuccess)
+    if (launch_accept_filtered(*accept, *filter, L, w, acc_stream, false) != cudaSuccess)
       return SPEC_ERR_CUDA;
   } else if (accept) {
     const AcceptLayout L = accept_layout(*accept, kWsHeader);
-    if (launch_accept(*accept, L, w, sms, stream, attn != nullptr) != cudaSuccess) return SPEC_ERR_CUDA;
+    if (launch_accept(*accept, L, w, sms, acc_stream, false) != cudaSuccess) return SPEC_ERR_CUDA;
   }
+  if (side && (cudaEventRecord(side->join, side->stream) != cudaSuccess ||
+               cudaStreamWaitEvent(stream, side->join, 0) != cudaSuccess))
+    return SPEC_ERR_CUDA;
   return SPEC_OK;
 }
 
