@@ -324,19 +324,42 @@ spec_status_t run(const spec_attn_args_t* attn, const spec_accept_args_t* accept
       return SPEC_ERR_CUDA;
     acc_stream = side->stream;
   }
-  if (attn) {
+  // Order of the two launches: the acceptance first when its logits are a sizeable
+  // share of the step's bytes (at least a sixth of the most KV the attention can read):
+  // its statistics then stream on the whole GPU before the attention blocks take it,
+  // and the decisions and draws run beside the attention. Otherwise the attention first
+  // (its start would wait for a comparatively short statistics pass).
+  bool accept_first = false;
+  if (side) {
+    const size_t esz = accept->logits_dtype == SPEC_BF16 ? 2 : 4;
+    const double logits = static_cast<double>(accept->batch) * (2.0 * accept->gamma - 1) *
+                          accept->vocab * static_cast<double>(esz);
+    const double kv = static_cast<double>(attn->batch) * attn->max_pages_per_seq * attn->page_size *
+                      attn->num_kv_heads * attn->head_dim * 4.0;
+    accept_first = 6.0 * logits >= kv;
+  }
+  auto launch_attention = [&]() -> bool {
+    if (!attn) return true;
     const AttnPlan P = attn_plan(*attn, attn_base, sms, attn->path);
     const cudaError_t e = P.path == SPEC_ATTN_TENSOR_CORES ? launch_attn_tc(*attn, P, w, stream)
                                                            : launch_attn_simt(*attn, P, w, stream);
-    if (e != cudaSuccess) return SPEC_ERR_CUDA;
-  }
-  if (accept && filter) {
-    const FilterLayout L = filter_layout(*accept, filter->max_top_k, kWsHeader, sms);
-    if (launch_accept_filtered(*accept, *filter, L, w, acc_stream, false) != cudaSuccess)
-      return SPEC_ERR_CUDA;
-  } else if (accept) {
-    const AcceptLayout L = accept_layout(*accept, kWsHeader);
-    if (launch_accept(*accept, L, w, sms, acc_stream, false) != cudaSuccess) return SPEC_ERR_CUDA;
+    return e == cudaSuccess;
+  };
+  auto launch_acceptance = [&]() -> bool {
+    if (accept && filter) {
+      const FilterLayout L = filter_layout(*accept, filter->max_top_k, kWsHeader, sms);
+      return launch_accept_filtered(*accept, *filter, L, w, acc_stream, false) == cudaSuccess;
+    }
+    if (accept) {
+      const AcceptLayout L = accept_layout(*accept, kWsHeader);
+      return launch_accept(*accept, L, w, sms, acc_stream, false) == cudaSuccess;
+    }
+    return true;
+  };
+  if (accept_first) {
+    if (!launch_acceptance() || !launch_attention()) return SPEC_ERR_CUDA;
+  } else {
+    if (!launch_attention() || !launch_acceptance()) return SPEC_ERR_CUDA;
   }
   if (side && (cudaEventRecord(side->join, side->stream) != cudaSuccess ||
                cudaStreamWaitEvent(stream, side->join, 0) != cudaSuccess))
