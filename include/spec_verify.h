@@ -449,7 +449,7 @@ typedef struct {
   int32_t rows, hidden, vocab, rows_per_seq;
   const void* hidden_states;   /* bf16 [rows][hidden]                                    */
   const void* weight;          /* bf16 [vocab][hidden]: output row v of the LM head       */
-  const float* temperature;    /* [rows / rows_per_seq]                                   */
+  const float* temperature;    /* [ceil(rows / rows_per_seq)]                             */
   const int32_t* tokens;       /* [rows], or NULL                                         */
   float* row_max;              /* [rows], written                                         */
   float* row_sum;              /* [rows], written                                         */

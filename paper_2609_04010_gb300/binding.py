@@ -590,7 +590,7 @@ def lm_head_args(hidden_states, weight, temperature, rows_per_seq: int, out: Dic
         raise ValueError("weight and hidden states disagree on the hidden size")
     _check(hidden_states, "hidden_states", torch.bfloat16)
     _check(weight, "weight", torch.bfloat16)
-    _check(temperature, "temperature", torch.float32)
+    _check(temperature, "temperature", torch.float32, ((R + rows_per_seq - 1) // rows_per_seq,))
     if tokens is not None:
         _check(tokens, "tokens", torch.int32, (R,))
     for k in ("row_max", "row_sum"):
