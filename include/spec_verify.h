@@ -135,6 +135,13 @@ typedef struct {
  * C the ascending-token cumulative sum of p_B (n = gamma) or of [p_n - q_n]_+.
  * With T = 0 (greedy): n = the first i whose token is not the lowest-index argmax of
  * target row i-1, and the final token is that argmax of target row n-1.
+ *
+ * The classic speculative-decoding convention (k drafts d_1..d_k drawn from q_1..q_k,
+ * k + 1 target rows p_1..p_{k+1}, the last one the bonus) is this call with
+ * gamma = k + 1: block tokens [the last emitted token, d_1, .., d_k], target rows
+ * p_1..p_{k+1}, drafter rows [any row, q_1, .., q_k] (row 0 is never read, so it may
+ * hold anything, even NaN), uniforms [u_1, .., u_k, u_draw]; out_tokens[0] echoes the
+ * last emitted token and num_accepted counts accepted drafts.
  * Outputs: out_tokens[b] = [t_0, t_1 .. t_{n-1}, final, -1 ...] (gamma+1 entries),
  * num_accepted[b] = n - 1 in [0, gamma-1], num_emitted[b] = n + 1 in [2, gamma+1].
  * A sequence flagged BAD_TOKEN or BAD_LOGITS gets num_accepted = -1,

@@ -181,3 +181,31 @@ def test_gpu_output_distribution_chi_square():
     o = np.append(obs[~small], obs[small].sum())
     e = np.append(exp[~small], exp[small].sum())
     assert stats.chisquare(o, e).pvalue > 1e-3
+
+
+def test_unused_drafter_row_is_never_read():
+    # the classic convention's spare leading drafter row may hold anything, even NaN:
+    # the unfiltered and the filtered acceptance give the same outputs and raise no flag
+    from helpers import dev, logits_dev
+    inp = W.workload("llama8b").accept_inputs(seed=3)
+    dl = inp.drafter_logits.copy()
+    dl[:, 0, :] = np.uint16(0x7FC0) if dl.dtype == np.uint16 else np.nan
+    B = inp.batch
+    tl, tok, T, u = (logits_dev(inp.target_logits), dev(inp.block_tokens), dev(inp.temperature),
+                     dev(inp.uniforms))
+    top_k, top_p = dev(np.full(B, 50, np.int32)), dev(np.full(B, 0.95, np.float32))
+    for filtered in (False, True):
+        outs = []
+        for d in (inp.drafter_logits, dl):
+            ws = binding.new_workspace(1 << 28)
+            if filtered:
+                r = binding.accept_block_filtered(tl, logits_dev(d), tok, T, top_k, top_p, u,
+                                                  max_top_k=50, ws=ws)
+            else:
+                r = binding.accept_block(tl, logits_dev(d), tok, T, u, ws=ws)
+            torch.cuda.synchronize()
+            assert binding.read_device_status(ws) == (0, 0)
+            outs.append({k: v.cpu().numpy() for k, v in r.items() if v is not None})
+        for k in ("num_accepted", "out_tokens", "num_emitted"):
+            np.testing.assert_array_equal(outs[0][k], outs[1][k])
+        assert np.all(outs[1]["out_tokens"][:, 0] == inp.block_tokens[:, 0])
