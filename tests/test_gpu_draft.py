@@ -177,13 +177,15 @@ def test_commit_matches_oracle(oracle_mod, reserve):
 
 def test_commit_worked_examples_on_gpu(oracle_mod):
     # the hand-worked cases of the oracle's pins, including a request of zero pages after
-    # a refused one (it is served, and the list's top stays at the last grant)
+    # a refused one (it is served, and the list's top stays at the last grant) and a
+    # request that fits only if an earlier refused one is not counted (it is refused)
     cases = [
         (np.array([[10, 11, 12, -1], [20, 21, 22, -1], [30, 31, -1, -1]]), [9, 12, 7], [1, 3, -1],
          4, 4, [40, 41, 42] + [0] * 13, 3),
         (np.array([[1, -1, -1], [2, -1, -1], [3, -1, -1]]), [4, 4, 4], [0, 3, 3], 4, 4, [7, 8, 0], 2),
         (np.array([[1, 2, 3], [4, 5, -1], [6, 7, -1]]), [12, 8, 8], [-1, -1, -1], 4, 4, [9, 0], 1),
         (np.array([[1, -1, -1], [2, -1, -1], [3, 4, -1]]), [4, 4, 8], [3, 3, -1], 4, 4, [5, 0, 0], 1),
+        (np.array([[1, 2, -1, -1], [3, 4, -1, -1]]), [8, 8], [7, 0], 4, 8, [9, 0], 1),
     ]
     for table, kv, na, P, G, free, count in cases:
         for reserve in (True, False):

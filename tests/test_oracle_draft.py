@@ -131,8 +131,8 @@ def test_sample_flags_bad_inputs(oracle_mod):
 # ---------------------------------------------------------------------------------
 # noise tokens
 # ---------------------------------------------------------------------------------
-def test_noise_tokens_closed_forms():
-    import oracle
+def test_noise_tokens_closed_forms(oracle_mod):
+    oracle = oracle_mod
     words = W.philox_words(11, 4096)
     for k in (1, 8, 17):
         np.testing.assert_array_equal(oracle.noise_tokens(words, 1 << k),
@@ -148,8 +148,8 @@ def test_noise_tokens_closed_forms():
 # ---------------------------------------------------------------------------------
 # KV commit
 # ---------------------------------------------------------------------------------
-def test_commit_worked_example():
-    import oracle
+def test_commit_worked_example(oracle_mod):
+    oracle = oracle_mod
     # page size 4, gamma 4; three sequences of ctx 5, 8, 3 (kv_len = ctx + 4).
     table = np.array([[10, 11, 12, -1], [20, 21, 22, -1], [30, 31, -1, -1]], np.int32)
     kv = np.array([9, 12, 7], np.int32)
@@ -183,8 +183,8 @@ def _random_pool(rng, B, P, max_pages, gamma, spare):
 
 
 @pytest.mark.parametrize("reserve", [True, False])
-def test_commit_conserves_pages(reserve):
-    import oracle
+def test_commit_conserves_pages(oracle_mod, reserve):
+    oracle = oracle_mod
     rng = np.random.default_rng(37)
     for trial in range(50):
         B, P, gamma = int(rng.integers(1, 20)), int(rng.choice([4, 16])), int(rng.integers(1, 9))
@@ -219,8 +219,8 @@ def test_commit_conserves_pages(reserve):
                 assert not np.any(later & (fl == 0) & (need > 0))
 
 
-def test_commit_flags_bad_input_and_exhaustion():
-    import oracle
+def test_commit_flags_bad_input_and_exhaustion(oracle_mod):
+    oracle = oracle_mod
     table = np.array([[1, 2, -1], [3, -1, -1], [4, -1, -1]], np.int32)
     kv = np.array([6, 2, 3], np.int32)     # gamma 3: the second has kv_len < gamma
     na = np.array([2, 0, 5], np.int32)     # the third's num_accepted > gamma - 1
@@ -233,13 +233,22 @@ def test_commit_flags_bad_input_and_exhaustion():
     new, t, f, c, fl = oracle.commit_kv(np.array([4, 4]), np.array([3, 3]), table, 4, 4,
                                         np.array([7, 0]), 1, reserve=True)
     assert list(fl) == [0, 2] and list(t[0]) == [1, 7] and list(t[1]) == [2, -1]
-    # a refused request still counts: the third sequence's single page would fit the
-    # list on its own, but the grants are a prefix of the batch order
+    # batch order: the first two take the list's two pages, so the third's single page,
+    # which would fit the list on its own, is refused
     table = np.array([[1, -1, -1], [2, -1, -1], [3, -1, -1]], np.int32)
     new, t, f, c, fl = oracle.commit_kv(np.array([4, 4, 4]), np.array([0, 3, 3]), table, 4, 4,
                                         np.array([7, 8, 0]), 2, reserve=True)
     # needs: 1 (ctx 0 + n 1 + 4 keys = 5 -> 2 pages), 1 (8 keys -> 2), 1
     assert list(fl) == [0, 0, 2] and list(t[0][:2]) == [1, 8] and list(t[1][:2]) == [2, 7]
+    # a refused request still counts against the later ones (gamma 8, one free page): the
+    # first asks for 2 pages (ctx 0 + n 8 + 8 keys -> 4 pages, has 2) and is refused; the
+    # second's single page (ctx 0 + n 1 + 8 keys -> 3 pages) would fit, but the requests
+    # of sequences 0 and 1 together do not
+    table = np.array([[1, 2, -1, -1], [3, 4, -1, -1]], np.int32)
+    new, t, f, c, fl = oracle.commit_kv(np.array([8, 8]), np.array([7, 0]), table, 4, 8,
+                                        np.array([9, 0]), 1, reserve=True)
+    assert list(fl) == [2, 2] and list(new) == [8, 1] and c == 1
+    assert np.array_equal(t, table)
     # a request of zero pages after a refused one is served, and the list's top stays
     # where the last grant left it
     table = np.array([[1, -1, -1], [2, -1, -1], [3, 4, -1]], np.int32)

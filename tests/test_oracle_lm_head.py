@@ -87,7 +87,20 @@ def test_token_logit_and_row_subset(oracle_mod):
         else:
             assert o["token_logit"][r] == o["logits"][r, tok[r]]
     sub = oracle_mod.lm_head_stats(h, w, T, 3, tokens=tok, rows=[7, 1], chunk=64)
-    for key in ("row_max", "row_sum", "row_argmax"):
+    for key in ("row_max", "row_sum", "row_argmax", "token_logit"):
         np.testing.assert_array_equal(sub[key], o[key][[7, 1]])
     # the bound on a logit's accumulation error dominates every logit
     assert np.all(np.abs(o["logits"]).max(axis=1) <= o["abs_bound"] + 1e-12)
+
+
+def test_each_row_takes_its_sequence_temperature(oracle_mod):
+    # rows_per_seq = 2: rows 2s and 2s + 1 use temperature[s]; the sum is the closed form
+    # exp(logsumexp(l / T) - max / T) at that T (T <= 0 at T = 1)
+    h, w, _, _ = W.make_lm_inputs(6, 32, 200, 2, seed=5)
+    T = np.array([1.0, 0.5, 0.0], np.float32)
+    o = oracle_mod.lm_head_stats(h, w, T, 2)
+    l = o["logits"]
+    for r in range(6):
+        t = float(T[r // 2]) if T[r // 2] > 0 else 1.0
+        want = np.exp(special.logsumexp(l[r] / t) - l[r].max() / t)
+        np.testing.assert_allclose(o["row_sum"][r], want, rtol=1e-12)

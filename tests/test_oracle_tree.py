@@ -65,6 +65,24 @@ def test_tree_is_the_best_prefixes(oracle_mod, K, G, budget):
             np.testing.assert_allclose(tree["score"][b, j], scores[node_prefix(tree, b, j)], rtol=1e-12)
 
 
+def test_tie_rules_worked_example(oracle_mod):
+    # Worked by hand (K = 2, budget 6, T = 1). Position 1's tokens 0 and 1 tie at the
+    # top, position 2's tokens 1 and 2 tie behind token 0. Equal candidates rank by the
+    # lower token id; equal offers go to the lower parent index.
+    #   step 1: root offers token 0 (the lower id of the tie)          -> node 1
+    #   step 2: root's token 1 (same score) beats node 1's child       -> node 2
+    #   step 3: nodes 1 and 2 offer token 0 at the same score; node 1  -> node 3
+    #   step 4: node 2's token 0 beats node 1's token 1                -> node 4
+    #   step 5: nodes 1 and 2 offer token 1 at the same score; node 1  -> node 5
+    #   step 6: node 2's token 1                                       -> node 6
+    dl = np.array([[[0, 0, 0], [0, 0, -10], [5, 0, 0]]], np.float32)
+    tree = oracle_mod.build_tree(dl, np.ones(1, np.float32), np.array([2]), 2, 6)
+    assert list(tree["tokens"][0]) == [2, 0, 1, 0, 0, 1, 1]
+    assert list(tree["parents"][0]) == [-1, 0, 0, 1, 2, 1, 2]
+    assert list(tree["cand_tokens"][0, 1]) == [0, 1] and list(tree["cand_tokens"][0, 2]) == [0, 1]
+    assert tree["margin"][0] == 0.0
+
+
 def test_tree_structure(oracle_mod):
     rng = np.random.default_rng(51)
     B, G, V, K, budget = 8, 16, 200, 8, 40
