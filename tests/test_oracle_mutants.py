@@ -13,6 +13,7 @@ import types
 import numpy as np
 import pytest
 
+import test_oracle_accept as ACC
 import test_oracle_attention as ATT
 import test_oracle_draft as DRAFT
 import test_oracle_lm_head as LM
@@ -115,6 +116,19 @@ def _commit_pins(m):
 
 
 PACKAGE_MUTANTS = {
+    # --- the building blocks (oracle.cpp) ---
+    # equal maxima go to the highest token id
+    "argmax_ties_to_last": (dict(cpp=("if (row[x] > row[best]) best = x;",
+                                      "if (row[x] >= row[best]) best = x;")),
+                            DRAFT.test_sample_greedy_is_lowest_argmax),
+    # the exponent drops the temperature (the maximum keeps it)
+    "softmax_temperature_dropped": (dict(cpp=("p[x] = std::exp(logits[x] / temperature - m);",
+                                              "p[x] = std::exp(logits[x] - m);")),
+                                    ACC.test_softmax_matches_scipy),
+    # the draw compares unnormalised cumulative weights with u instead of u * S
+    "inverse_cdf_unscaled_target": (dict(cpp=("const double target = u * S;",
+                                              "const double target = u;")),
+                                    ACC.test_inverse_cdf_matches_searchsorted),
     # --- verify attention (oracle.cpp) ---
     # a block query does not see its own key
     "attn_query_misses_own_key": (dict(cpp=(": i <= j;", ": i < j;")), _dense_attention_pin),
