@@ -14,6 +14,10 @@
 #include "common.cuh"
 
 namespace specv {
+
+// The argument check of spec_accept_block (api.cu): the same limits and error codes.
+spec_status_t check_accept(const spec_accept_args_t* a);
+
 namespace {
 
 constexpr size_t kScratchBytes = SPEC_NOALLOC_SCRATCH_BYTES;
@@ -47,14 +51,8 @@ using namespace specv;
 
 extern "C" spec_status_t spec_accept_block_noalloc(const spec_accept_args_t* accept,
                                                    spec_stream_t stream_) {
-  if (!accept) return SPEC_ERR_INVALID_ARGUMENT;
-  if (accept->batch < 1 || accept->gamma < 1 || accept->vocab < 1 || accept->gamma > 64 ||
-      accept->batch > 65535 ||
-      (accept->logits_dtype != SPEC_F32 && accept->logits_dtype != SPEC_BF16) ||
-      !accept->target_logits || !accept->drafter_logits || !accept->block_tokens ||
-      !accept->temperature || !accept->uniforms || !accept->num_accepted || !accept->out_tokens ||
-      !accept->num_emitted)
-    return SPEC_ERR_INVALID_ARGUMENT;
+  const spec_status_t st = check_accept(accept);
+  if (st != SPEC_OK) return st;
   // The same scratch layout spec_accept_block uses inside a caller's workspace.
   const AcceptLayout L = accept_layout(*accept, kWsHeader);
   if (L.end > kScratchBytes) return SPEC_ERR_WORKSPACE_TOO_SMALL;  // beyond the fixed array

@@ -106,22 +106,6 @@ spec_status_t check_attn(const spec_attn_args_t* a) {
   return SPEC_OK;
 }
 
-spec_status_t check_accept(const spec_accept_args_t* a) {
-  if (!a) return SPEC_ERR_INVALID_ARGUMENT;
-  if (a->batch < 1 || a->gamma < 1 || a->vocab < 1) return SPEC_ERR_INVALID_ARGUMENT;
-  if (a->logits_dtype != SPEC_F32 && a->logits_dtype != SPEC_BF16) return SPEC_ERR_INVALID_ARGUMENT;
-  if (!a->target_logits || !a->drafter_logits || !a->block_tokens || !a->temperature ||
-      !a->uniforms || !a->num_accepted || !a->out_tokens || !a->num_emitted)
-    return SPEC_ERR_INVALID_ARGUMENT;
-  if (a->gamma > 64 || a->batch > 65535) return SPEC_ERR_UNSUPPORTED;
-  const int64_t nchunk = (static_cast<int64_t>(a->vocab) + kStatsChunk - 1) / kStatsChunk;
-  if (static_cast<int64_t>(a->batch) * (2 * a->gamma - 1) * nchunk > INT32_MAX)
-    return SPEC_ERR_UNSUPPORTED;
-  const int64_t nslice = (static_cast<int64_t>(a->vocab) + kSampleSlice - 1) / kSampleSlice;
-  if (nslice > 65535) return SPEC_ERR_UNSUPPORTED;
-  return SPEC_OK;
-}
-
 spec_status_t check_draft(const spec_draft_args_t* d) {
   if (!d) return SPEC_ERR_INVALID_ARGUMENT;
   if (d->batch < 1 || d->gamma < 1 || d->vocab < 1) return SPEC_ERR_INVALID_ARGUMENT;
@@ -208,6 +192,23 @@ spec_status_t check_filter(const spec_filter_args_t* f) {
 }
 
 }  // namespace
+
+// Also the host check of spec_accept_block_noalloc (accept_noalloc.cu).
+spec_status_t check_accept(const spec_accept_args_t* a) {
+  if (!a) return SPEC_ERR_INVALID_ARGUMENT;
+  if (a->batch < 1 || a->gamma < 1 || a->vocab < 1) return SPEC_ERR_INVALID_ARGUMENT;
+  if (a->logits_dtype != SPEC_F32 && a->logits_dtype != SPEC_BF16) return SPEC_ERR_INVALID_ARGUMENT;
+  if (!a->target_logits || !a->drafter_logits || !a->block_tokens || !a->temperature ||
+      !a->uniforms || !a->num_accepted || !a->out_tokens || !a->num_emitted)
+    return SPEC_ERR_INVALID_ARGUMENT;
+  if (a->gamma > 64 || a->batch > 65535) return SPEC_ERR_UNSUPPORTED;
+  const int64_t nchunk = (static_cast<int64_t>(a->vocab) + kStatsChunk - 1) / kStatsChunk;
+  if (static_cast<int64_t>(a->batch) * (2 * a->gamma - 1) * nchunk > INT32_MAX)
+    return SPEC_ERR_UNSUPPORTED;
+  const int64_t nslice = (static_cast<int64_t>(a->vocab) + kSampleSlice - 1) / kSampleSlice;
+  if (nslice > 65535) return SPEC_ERR_UNSUPPORTED;
+  return SPEC_OK;
+}
 
 AttnPlan attn_plan(const spec_attn_args_t& a, size_t base, int num_sms, int path_override) {
   AttnPlan P;

@@ -47,6 +47,7 @@ def test_host_side_argument_checks(lib):
     assert lib.spec_accept_block(ctypes.byref(acc), None, 0, None) == 1
     assert lib.spec_philox_uniforms(1, 0, -1, None, None) == 1
     assert lib.spec_read_device_status(None, None, None) == 1
+    assert lib.spec_workspace_init(None, 1024, None) == 1
 
 
 def _attn(**kw):
@@ -243,3 +244,17 @@ def test_lm_head_workspace(lib):
     assert lib.spec_lm_head_stats(ctypes.byref(a), ctypes.c_void_p(4096), n - 256, None) == 3
     assert lib.spec_lm_head_stats(ctypes.byref(a), ctypes.c_void_p(4097), n, None) == 1
     assert lib.spec_lm_head_stats(None, ctypes.c_void_p(4096), n, None) == 1
+
+
+def test_fused_step_checks_both_parts_before_any_launch(lib):
+    # a valid attention half does not hide a bad acceptance half, nor the reverse
+    attn = _attn()
+    good = _accept()
+    bad_gamma = _accept(gamma=65)
+    assert lib.spec_verify_step(ctypes.byref(attn), ctypes.byref(bad_gamma), None, 0, None) == 2
+    bad_batch = _accept(batch=0)
+    assert lib.spec_verify_step(ctypes.byref(attn), ctypes.byref(bad_batch), None, 0, None) == 1
+    bad_attn = _attn(num_kv_heads=3)
+    assert lib.spec_verify_step(ctypes.byref(bad_attn), ctypes.byref(good), None, 0, None) == 1
+    # both halves valid: the missing workspace is the error
+    assert lib.spec_verify_step(ctypes.byref(attn), ctypes.byref(good), None, 0, None) == 1

@@ -28,6 +28,28 @@ def test_oversized_batch_is_rejected_without_launch():
     assert binding.lib().spec_accept_block_noalloc(ctypes.byref(a), None) == 3
 
 
+def _fake_accept(batch, gamma, vocab, dtype=binding.SPEC_BF16, skip=()):
+    a = binding.AcceptArgs(batch, gamma, vocab, dtype)
+    for f in ("target_logits", "drafter_logits", "block_tokens", "temperature", "uniforms",
+              "num_accepted", "out_tokens", "num_emitted"):
+        if f not in skip:
+            setattr(a, f, 4096)  # fake aligned addresses: never dereferenced by the checks
+    return a
+
+
+@pytest.mark.parametrize("args,code", [
+    ((0, 4, 1000), 1), ((2, 0, 1000), 1), ((2, 4, 0), 1), ((2, 4, 1000, 7), 1),
+    ((2, 4, 1000, binding.SPEC_BF16, ("uniforms",)), 1), ((2, 65, 1000), 2),
+    ((65536, 1, 1000), 2), ((1, 1, 65536 * 4096 + 1), 2)])
+def test_argument_errors_match_the_workspace_entry_point(args, code):
+    # the same host check as spec_accept_block, before any device call
+    lib = binding.lib()
+    a = _fake_accept(*args)
+    assert lib.spec_accept_block_noalloc(ctypes.byref(a), None) == code
+    assert lib.spec_accept_block(ctypes.byref(a), None, 0, None) == code
+    assert lib.spec_accept_block_noalloc(None, None) == 1
+
+
 @pytest.mark.gpu
 def test_matches_workspace_entry_point_twice():
     def one(inp):
