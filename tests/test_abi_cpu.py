@@ -6,6 +6,7 @@ import ctypes
 import subprocess
 
 import pytest
+import torch
 
 from paper_2609_04010_gb300 import binding, build
 
@@ -258,3 +259,46 @@ def test_fused_step_checks_both_parts_before_any_launch(lib):
     assert lib.spec_verify_step(ctypes.byref(bad_attn), ctypes.byref(good), None, 0, None) == 1
     # both halves valid: the missing workspace is the error
     assert lib.spec_verify_step(ctypes.byref(attn), ctypes.byref(good), None, 0, None) == 1
+
+
+def _cpu_calls():
+    """Every tensor-taking binding call, on small CPU tensors of the right dtypes and
+    shapes (B = 2 sequences, gamma 4, vocab 64)."""
+    B, G, V, Hq, Hkv, D, P = 2, 4, 64, 8, 2, 64, 16
+    bf = lambda *s: torch.zeros(*s, dtype=torch.bfloat16)
+    i32 = lambda *s: torch.zeros(*s, dtype=torch.int32)
+    f32 = lambda *s: torch.ones(*s, dtype=torch.float32)
+    tl, dl = bf(B, G, V), bf(B, G, V)
+    tok, T, u = i32(B, G), f32(B), f32(B, G)
+    q, kc, vc = bf(B, G, Hq, D), bf(4, Hkv, P, D), bf(4, Hkv, P, D)
+    table, kv = i32(B, 2), torch.full((B,), 20, dtype=torch.int32)
+    return {
+        "verify_attention": lambda: binding.verify_attention(q, kc, vc, table, kv),
+        "accept_block": lambda: binding.accept_block(tl, dl, tok, T, u),
+        "accept_block_noalloc": lambda: binding.accept_block_noalloc(
+            tl, dl, tok, T, u, i32(B), i32(B, G + 1), i32(B)),
+        "accept_block_filtered": lambda: binding.accept_block_filtered(
+            tl, dl, tok, T, i32(B) + 5, f32(B), u, max_top_k=8),
+        "sample_block": lambda: binding.sample_block(dl, T, u),
+        "build_tree": lambda: binding.build_tree(dl, T, i32(B), 2, 5),
+        "accept_tree": lambda: binding.accept_tree(tl, tok, i32(B, G) - 1),
+        "lm_head_stats": lambda: binding.lm_head_stats(bf(8, 64), bf(V, 64), f32(2), 4),
+        "commit_kv": lambda: binding.commit_kv(kv, i32(B), table, P, G, i32(8), i32(1)),
+        "commit_tree_kv": lambda: binding.commit_tree_kv(kc, vc, table, kv, i32(B, G), i32(B)),
+    }
+
+
+HOST_TENSOR_CALLS = ["accept_block", "accept_block_filtered", "accept_block_noalloc", "accept_tree",
+                     "build_tree", "commit_kv", "commit_tree_kv", "lm_head_stats", "sample_block",
+                     "verify_attention"]
+
+
+def test_host_tensor_cases_cover_the_table():
+    assert sorted(_cpu_calls()) == HOST_TENSOR_CALLS
+
+
+@pytest.mark.parametrize("name", HOST_TENSOR_CALLS)
+def test_binding_rejects_host_tensors(lib, name):
+    # a host pointer must never reach a kernel: every call checks its tensors first
+    with pytest.raises(ValueError, match="CUDA tensor"):
+        _cpu_calls()[name]()
