@@ -80,8 +80,12 @@ def parse_args():
     ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", default="llama8b",
+    ap.add_argument("--workload", default="serve64",
                     help="tiny | llama8b | serve64 | long70b | sweep_g<G>_b<B>_s<S>_t<T>")
+    ap.add_argument("--also", default="llama8b,long70b,tiny",
+                    help="comma-separated workloads whose fused step is also timed in the same "
+                         "run (device time, rooflines, clocks), reported under 'workloads'; "
+                         "'' for none")
     ap.add_argument("--attn-path", choices=["auto", "cuda-cores", "tensor-cores"], default="auto",
                     help="attention kernel (auto: tensor cores from the library's row crossover)")
     ap.add_argument("--no-e2e", action="store_true")
@@ -293,6 +297,57 @@ def attn_path_name(choice, binding, ai):
     return choice.replace("-", " ")
 
 
+class StepSetup:
+    """One workload's inputs on the device, its outputs, argument structs and workspace,
+    and the three C-ABI calls the bench times: the fused step, attention alone and
+    acceptance alone."""
+
+    def __init__(self, args, wl, ai, ci, binding, dev):
+        import torch
+
+        def bf16(a):
+            return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16)
+
+        def t(a):
+            return torch.from_numpy(np.ascontiguousarray(a))
+
+        host_in = dict(q=bf16(ai.q), k=bf16(ai.k_cache), v=bf16(ai.v_cache), pt=t(ai.page_table),
+                       kvl=t(ai.kv_len),
+                       tl=bf16(ci.target_logits) if ci.is_bf16 else t(ci.target_logits),
+                       dl=bf16(ci.drafter_logits) if ci.is_bf16 else t(ci.drafter_logits),
+                       tok=t(ci.block_tokens), temp=t(ci.temperature), u=t(ci.uniforms))
+        filtered = wl.top_k > 0
+        if filtered:
+            fk, fp = wl.filter_params()
+            host_in.update(topk=t(fk), topp=t(fp))
+        d = {k: v.to(dev) for k, v in host_in.items()}
+        B, G = ci.batch, ci.gamma
+        out = torch.empty_like(d["q"])
+        lse = torch.empty(d["q"].shape[:3], dtype=torch.float32, device=dev)
+        na = torch.empty(B, dtype=torch.int32, device=dev)
+        ot = torch.empty(B, G + 1, dtype=torch.int32, device=dev)
+        ne = torch.empty(B, dtype=torch.int32, device=dev)
+        path = {"auto": binding.ATTN_AUTO, "cuda-cores": binding.ATTN_CUDA_CORES,
+                "tensor-cores": binding.ATTN_TENSOR_CORES}[args.attn_path]
+        a = binding.attn_args(d["q"], d["k"], d["v"], d["pt"], d["kvl"], out, lse, path=path)
+        c = binding.accept_args(d["tl"], d["dl"], d["tok"], d["temp"], d["u"], na, ot, ne, None)
+        if filtered:
+            f = binding.filter_args(d["topk"], d["topp"], B, max_top_k=wl.top_k)
+            ws = binding.new_workspace(binding.filtered_workspace_size(c, f, a), dev)
+        else:
+            ws = binding.new_workspace(binding.workspace_size(a, c), dev)
+        self.host_in, self.d, self.out, self.lse = host_in, d, out, lse
+        self.na, self.ot, self.ne = na, ot, ne
+        self.a, self.c, self.f, self.ws, self.filtered = a, c, (f if filtered else None), ws, filtered
+        if filtered:
+            self.step = lambda: binding.verify_step_filtered_args(a, c, f, ws)
+            self.acc_only = lambda: binding.verify_step_filtered_args(None, c, f, ws)
+        else:
+            self.step = lambda: binding.verify_step_args(a, c, ws)
+            self.acc_only = lambda: binding.verify_step_args(None, c, ws)
+        self.attn_only = lambda: binding.verify_step_args(a, None, ws)
+
+
 def run_ours(args, wl, ai, ci, rank, world, local_rank):
     import torch
     from paper_2609_04010_gb300 import binding, build
@@ -300,38 +355,10 @@ def run_ours(args, wl, ai, ci, rank, world, local_rank):
     build.build()
     torch.cuda.set_device(local_rank)
     dev = torch.device("cuda", local_rank)
-
-    def bf16(a):
-        return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16)
-
-    def t(a):
-        return torch.from_numpy(np.ascontiguousarray(a))
-
-    host_in = dict(q=bf16(ai.q), k=bf16(ai.k_cache), v=bf16(ai.v_cache), pt=t(ai.page_table),
-                   kvl=t(ai.kv_len),
-                   tl=bf16(ci.target_logits) if ci.is_bf16 else t(ci.target_logits),
-                   dl=bf16(ci.drafter_logits) if ci.is_bf16 else t(ci.drafter_logits),
-                   tok=t(ci.block_tokens), temp=t(ci.temperature), u=t(ci.uniforms))
-    filtered = wl.top_k > 0
-    if filtered:
-        fk, fp = wl.filter_params()
-        host_in.update(topk=t(fk), topp=t(fp))
-    d = {k: v.to(dev) for k, v in host_in.items()}
+    S = StepSetup(args, wl, ai, ci, binding, dev)
+    host_in, d, out, lse, na, ot, ne = S.host_in, S.d, S.out, S.lse, S.na, S.ot, S.ne
+    a, c, f, ws, filtered = S.a, S.c, S.f, S.ws, S.filtered
     B, G = ci.batch, ci.gamma
-    out = torch.empty_like(d["q"])
-    lse = torch.empty(d["q"].shape[:3], dtype=torch.float32, device=dev)
-    na = torch.empty(B, dtype=torch.int32, device=dev)
-    ot = torch.empty(B, G + 1, dtype=torch.int32, device=dev)
-    ne = torch.empty(B, dtype=torch.int32, device=dev)
-    path = {"auto": binding.ATTN_AUTO, "cuda-cores": binding.ATTN_CUDA_CORES,
-            "tensor-cores": binding.ATTN_TENSOR_CORES}[args.attn_path]
-    a = binding.attn_args(d["q"], d["k"], d["v"], d["pt"], d["kvl"], out, lse, path=path)
-    c = binding.accept_args(d["tl"], d["dl"], d["tok"], d["temp"], d["u"], na, ot, ne, None)
-    if filtered:
-        f = binding.filter_args(d["topk"], d["topp"], B, max_top_k=wl.top_k)
-        ws = binding.new_workspace(binding.filtered_workspace_size(c, f, a), dev)
-    else:
-        ws = binding.new_workspace(binding.workspace_size(a, c), dev)
     flush_w = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device=dev)
     flush_r = torch.ones(L2_FLUSH_BYTES // 4, dtype=torch.int32, device=dev)
     flush_sink = torch.empty(1, dtype=torch.int64, device=dev)
@@ -352,13 +379,7 @@ def run_ours(args, wl, ai, ci, rank, world, local_rank):
         torch.cuda.synchronize()
         return [s.elapsed_time(e) for s, e in evs]
 
-    if filtered:
-        step = lambda: binding.verify_step_filtered_args(a, c, f, ws)
-        acc_only = lambda: binding.verify_step_filtered_args(None, c, f, ws)
-    else:
-        step = lambda: binding.verify_step_args(a, c, ws)
-        acc_only = lambda: binding.verify_step_args(None, c, ws)
-    attn_only = lambda: binding.verify_step_args(a, None, ws)
+    step, acc_only, attn_only = S.step, S.acc_only, S.attn_only
 
     # Device-timed loops replay CUDA graphs of the same C-ABI calls, so that the events
     # bracket GPU work only (the host's launch latency stays outside the timed region;
@@ -528,6 +549,11 @@ def run_ours(args, wl, ai, ci, rank, world, local_rank):
         "emitted_tokens_per_s": emitted / (ms / 1000.0),
         "clocks": clk,
     }
+    others = [x for x in (n.strip() for n in args.also.split(",")) if x and x != args.workload]
+    if others:
+        result["workloads"] = {n: time_other_workload(n, args, binding, dev, rank, graph_of,
+                                                      timed_loop, local_rank)
+                               for n in others}
     if e2e:
         result["e2e"] = e2e
         result["e2e_kv_resident"] = e2e_kv
@@ -538,6 +564,59 @@ def run_ours(args, wl, ai, ci, rank, world, local_rank):
     if lm_head:
         result["lm_head"] = lm_head
     return result
+
+
+def time_other_workload(name, args, binding, dev, rank, graph_of, timed_loop, local_rank):
+    """The fused verify step of another named workload, timed in the same run: CUDA-graph
+    replays with L2 flushed before each (as the headline), the attention and acceptance
+    alone, the step's and the attention's rooflines, and the clocks during its loop."""
+    import torch
+    from paper_2609_04010_gb300 import workloads as W
+
+    wl = W.workload(name)
+    ai, ci = wl.attn_inputs(seed=rank), wl.accept_inputs(seed=rank)
+    S = StepSetup(args, wl, ai, ci, binding, dev)
+    gs = {k: graph_of(fn) for k, fn in (("step", S.step), ("attention", S.attn_only),
+                                         ("accept", S.acc_only))}
+    n = max(20, min(args.steps, 500))
+    clocks = ClockSampler(local_rank if "CUDA_VISIBLE_DEVICES" not in os.environ else
+                          int(os.environ["CUDA_VISIBLE_DEVICES"].split(",")[local_rank]))
+    clocks.start()
+    time.sleep(0.3)
+    for _ in range(max(3, args.warmup)):
+        gs["step"].replay()
+    torch.cuda.synchronize()
+    ms = {k: statistics.mean(timed_loop(g.replay, n)) for k, g in gs.items()}
+    clk = clocks.stop()
+    code, flags = binding.read_device_status(S.ws)
+    if code != 0:
+        raise RuntimeError(f"{name}: device status {code} flags {flags}")
+    tm = traffic_model(ai, ci)
+    peak, peak_src = measured_peaks()
+    step_gbs = tm["baseline"] / (ms["step"] / 1000.0) / 1e9
+    attn_gbs = tm["kv"] / (ms["attention"] / 1000.0) / 1e9
+    emitted = int(S.ne.sum().item())
+    res = {"ms_per_step": ms["step"],
+           "value": whole_job_tokens_per_s(1, ci.batch, ci.gamma, ms["step"]), "unit": UNIT,
+           "config": wl.describe(),
+           "attention_path": attn_path_name(args.attn_path, binding, ai),
+           "attention_roofline": {"bound": "hbm", "achieved": round(attn_gbs, 1), "peak": peak,
+                                  "unit": "GB/s", "frac": round(attn_gbs / peak, 4),
+                                  "peak_source": peak_src,
+                                  "algorithmic_bytes_per_launch": int(tm["kv"]),
+                                  "launch_ms": ms["attention"]},
+           "step_roofline": {"bytes": int(tm["baseline"]), "strict_bytes": int(tm["strict"]),
+                             "achieved_gbs": round(step_gbs, 1),
+                             "frac_of_measured": round(step_gbs / peak, 4),
+                             "frac_of_8tbs": round(step_gbs / NOMINAL_HBM_GBS, 4)},
+           "parts_ms": {"attention": ms["attention"], "accept": ms["accept"]},
+           "emitted_tokens_per_s": emitted / (ms["step"] / 1000.0),
+           "gpu_launches": (2 if S.filtered else 4) * n,
+           "clocks": clk,
+           "timing": "CUDA-graph replays of one spec_verify_step call, L2 flushed before each"}
+    del S, gs
+    torch.cuda.empty_cache()
+    return res
 
 
 def time_lm_head(ai, ci, binding, dev, graph_of, timed_loop, n):

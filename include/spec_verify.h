@@ -18,9 +18,16 @@
  *
  * Conventions shared by every entry point
  *   - Every tensor argument is a DEVICE pointer owned by the caller, row-major and
- *     densely packed in the layout stated beside it. The library allocates no
- *     memory, keeps no state between calls, and never synchronizes the stream
- *     (except spec_read_device_status). Calls are asynchronous on `stream`.
+ *     densely packed in the layout stated beside it. The library allocates no device
+ *     memory and never synchronizes the stream (except spec_read_device_status).
+ *     Calls are asynchronous on `stream`.
+ *   - Each call makes the device of `stream` current while it runs and restores the
+ *     calling thread's current device before it returns.
+ *   - State kept between calls: cached SM counts, the driver's tensor-map encoder,
+ *     and, for the fused steps only, one side stream with two events per (host
+ *     thread, device, caller stream), at most 16 per thread (the least recently
+ *     used one that is not under capture is released to make room). Calls on
+ *     different streams never wait for each other's work.
  *   - `ws` is a caller-owned device workspace of at least spec_workspace_size()
  *     bytes, 256-byte aligned. A new workspace must be zero-filled once (e.g.
  *     spec_workspace_init); every call leaves its internal counters at zero again.
@@ -181,11 +188,11 @@ spec_status_t spec_accept_block(const spec_accept_args_t* accept, void* ws, size
 
 /* The whole verify step: parts (a) and (b), ordered on `stream` (they share no data:
  * the logits are inputs). Either argument may be NULL to run only the other part. With
- * both, part (b) runs on a second stream of the calling host thread (created on its
- * first such call and kept for the thread's life) between a fork event recorded on
+ * both, part (b) runs on a second stream that belongs to the calling host thread and
+ * to `stream` (created on the first such call) between a fork event recorded on
  * `stream` and a join event that `stream` waits for, so the two parts overlap; this
- * also holds under stream capture. The filtered step (spec_verify_step_filtered) does
- * the same. */
+ * also holds under stream capture. Steps issued on different streams therefore never
+ * wait for each other. The filtered step (spec_verify_step_filtered) does the same. */
 spec_status_t spec_verify_step(const spec_attn_args_t* attn, const spec_accept_args_t* accept,
                                void* ws, size_t ws_bytes, spec_stream_t stream);
 

@@ -57,20 +57,15 @@ extern "C" spec_status_t spec_accept_block_noalloc(const spec_accept_args_t* acc
   const AcceptLayout L = accept_layout(*accept, kWsHeader);
   if (L.end > kScratchBytes) return SPEC_ERR_WORKSPACE_TOO_SMALL;  // beyond the fixed array
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
-  int dev = 0;
-  if (stream_device(stream, &dev) != cudaSuccess) return SPEC_ERR_CUDA;
-  int cur = -1;
-  if (cudaGetDevice(&cur) != cudaSuccess) return SPEC_ERR_CUDA;
-  if (cur != dev && cudaSetDevice(dev) != cudaSuccess) return SPEC_ERR_CUDA;
+  // the stream's device is current until this call returns; the caller's is restored
+  DeviceScope scope(stream);
+  if (!scope.ok) return SPEC_ERR_CUDA;
   void* ptr = nullptr;
-  if (scratch_address(dev, &ptr) != cudaSuccess) return SPEC_ERR_CUDA;
+  if (scratch_address(scope.dev, &ptr) != cudaSuccess) return SPEC_ERR_CUDA;
   (void)cudaGetLastError();  // a failed call before this one must not fail our launches
   char* ws = static_cast<char*>(ptr);
   // The status word and the tickets must start at zero; the array keeps whatever the
   // previous call (possibly an interrupted one) left, so clear them on the stream.
   if (cudaMemsetAsync(ws, 0, L.partials, stream) != cudaSuccess) return SPEC_ERR_CUDA;
-  int sms = 0;
-  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
-    return SPEC_ERR_CUDA;
-  return launch_accept(*accept, L, ws, sms, stream) == cudaSuccess ? SPEC_OK : SPEC_ERR_CUDA;
+  return launch_accept(*accept, L, ws, scope.sms, stream) == cudaSuccess ? SPEC_OK : SPEC_ERR_CUDA;
 }

@@ -13,6 +13,23 @@
 
 namespace specv {
 
+namespace {
+constexpr int kSmCacheDevices = 64;
+std::atomic<int> g_sms[kSmCacheDevices];  // cached multiprocessor counts (0 = unknown)
+}  // namespace
+
+int device_sm_count(int dev) {
+  if (dev < 0 || dev >= kSmCacheDevices) return 148;
+  int n = g_sms[dev].load(std::memory_order_relaxed);
+  if (n > 0) return n;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) {
+    (void)cudaGetLastError();
+    n = 148;
+  }
+  g_sms[dev].store(n, std::memory_order_relaxed);
+  return n;
+}
+
 // (Hq/Hkv) * gamma at and above which SPEC_ATTN_AUTO picks the tensor-core kernel.
 // Measured on GB300: the tensor-core kernel is never slower, from 4 rows per kv head
 // (equal time, both latency-bound) to 32 (6x faster: the CUDA-core kernel re-reads
@@ -23,60 +40,71 @@ int tc_min_rows() { return kTcMinRows; }
 
 namespace {
 
-constexpr int kMaxDevices = 64;
-std::atomic<int> g_sm_count[kMaxDevices];  // cached multiprocessor counts (0 = unknown)
-
-int device_sm_count(int dev) {
-  if (dev < 0 || dev >= kMaxDevices) return 148;
-  int n = g_sm_count[dev].load(std::memory_order_relaxed);
-  if (n > 0) return n;
-  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0)
-    n = 148;
-  g_sm_count[dev].store(n, std::memory_order_relaxed);
-  return n;
-}
-
-// Makes the stream's device current for this library's runtime; returns its SM count.
-bool bind_device(cudaStream_t stream, int* sms) {
-  int dev = 0;
-  if (stream_device(stream, &dev) != cudaSuccess) return false;
-  int cur = -1;
-  if (cudaGetDevice(&cur) != cudaSuccess) return false;
-  if (cur != dev && cudaSetDevice(dev) != cudaSuccess) return false;
-  *sms = device_sm_count(dev);
-  return true;
-}
-
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-// A second stream of this host thread on a device, with a fork and a join event, made on
-// first use and kept for the thread's life. Per thread, so that calls from different
-// threads never record the same event; a call's fork and join also work under stream
-// capture (the side stream joins the capture through the fork event).
+// The fused step's second stream: one per (host thread, device, caller stream), with a
+// fork and a join event, made on first use. Keyed on the caller's stream so that two
+// steps issued on two different streams never queue behind each other on a shared side
+// stream; per thread, so that calls from different threads never record the same
+// event. A call's fork and join also work under stream capture (the side stream joins
+// the capture through the fork event). A thread keeps at most kSideCacheSize of them;
+// the least recently used one that is not capturing is released to make room (a
+// stream or event released with work pending is freed once that work completes).
 struct SideStream {
+  int dev = -1;
+  cudaStream_t caller = nullptr;
   cudaStream_t stream = nullptr;
   cudaEvent_t fork = nullptr, join = nullptr;
+  uint64_t last_use = 0;
 };
+constexpr int kSideCacheSize = 16;
 
-SideStream* side_stream(int dev) {
-  thread_local SideStream cache[kMaxDevices];
-  if (dev < 0 || dev >= kMaxDevices) return nullptr;
-  SideStream& ss = cache[dev];
-  if (!ss.stream) {
-    cudaStream_t st = nullptr;
-    cudaEvent_t f = nullptr, j = nullptr;
-    if (cudaStreamCreateWithFlags(&st, cudaStreamNonBlocking) != cudaSuccess) return nullptr;
-    if (cudaEventCreateWithFlags(&f, cudaEventDisableTiming) != cudaSuccess ||
-        cudaEventCreateWithFlags(&j, cudaEventDisableTiming) != cudaSuccess) {
-      if (f) cudaEventDestroy(f);
-      cudaStreamDestroy(st);
-      return nullptr;
+void release_side(SideStream& ss) {
+  if (ss.fork) cudaEventDestroy(ss.fork);
+  if (ss.join) cudaEventDestroy(ss.join);
+  if (ss.stream) cudaStreamDestroy(ss.stream);
+  ss = SideStream();
+}
+
+SideStream* side_stream(int dev, cudaStream_t caller) {
+  thread_local SideStream cache[kSideCacheSize];
+  thread_local uint64_t clock = 0;
+  ++clock;
+  SideStream* victim = nullptr;
+  for (SideStream& ss : cache) {
+    if (ss.stream && ss.dev == dev && ss.caller == caller) {
+      ss.last_use = clock;
+      return &ss;
     }
-    ss.stream = st;
-    ss.fork = f;
-    ss.join = j;
   }
-  return &ss;
+  for (SideStream& ss : cache) {
+    if (!ss.stream) {
+      victim = &ss;
+      break;
+    }
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(ss.stream, &cs) != cudaSuccess || cs != cudaStreamCaptureStatusNone)
+      continue;
+    if (!victim || ss.last_use < victim->last_use) victim = &ss;
+  }
+  if (!victim) return nullptr;
+  if (victim->stream) release_side(*victim);
+  cudaStream_t st = nullptr;
+  cudaEvent_t f = nullptr, j = nullptr;
+  if (cudaStreamCreateWithFlags(&st, cudaStreamNonBlocking) != cudaSuccess) return nullptr;
+  if (cudaEventCreateWithFlags(&f, cudaEventDisableTiming) != cudaSuccess ||
+      cudaEventCreateWithFlags(&j, cudaEventDisableTiming) != cudaSuccess) {
+    if (f) cudaEventDestroy(f);
+    cudaStreamDestroy(st);
+    return nullptr;
+  }
+  victim->dev = dev;
+  victim->caller = caller;
+  victim->stream = st;
+  victim->fork = f;
+  victim->join = j;
+  victim->last_use = clock;
+  return victim;
 }
 
 spec_status_t check_attn(const spec_attn_args_t* a) {
@@ -303,23 +331,28 @@ spec_status_t run(const spec_attn_args_t* attn, const spec_accept_args_t* accept
   // without attention the size does not depend on the device: check it on the host
   if (!attn && required_bytes(nullptr, accept, filter, 0, nullptr) > ws_bytes)
     return SPEC_ERR_WORKSPACE_TOO_SMALL;
-  int sms = 0;
-  if (!bind_device(stream, &sms)) return SPEC_ERR_CUDA;
+  DeviceScope scope(stream);
+  if (!scope.ok) return SPEC_ERR_CUDA;
+  const int sms = scope.sms;
   (void)cudaGetLastError();  // a failed call before this one must not fail our launches
   size_t attn_base = 0;
   if (required_bytes(attn, accept, filter, sms, &attn_base) > ws_bytes)
     return SPEC_ERR_WORKSPACE_TOO_SMALL;
   char* w = static_cast<char*>(ws);
-  // A whole step forks: the acceptance kernels run on this thread's side stream beside
-  // the attention kernel (they share no data: the logits are inputs), on the SM
-  // resources it leaves free, and the caller's stream waits for both. On one stream the
-  // decisions, which wait for their inputs with griddepcontrol.wait, would also wait for
-  // the attention kernel before them.
+  // A whole step forks: the acceptance kernels run on a side stream (this thread's, for
+  // this caller stream) beside the attention kernel (they share no data: the logits are
+  // inputs), on the SM resources it leaves free, and the caller's stream waits for both.
+  // On one stream the decisions, which wait for their inputs with griddepcontrol.wait,
+  // would also wait for the attention kernel before them.
   cudaStream_t acc_stream = stream;
   SideStream* side = nullptr;
   if (attn && accept) {
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || !(side = side_stream(dev))) return SPEC_ERR_CUDA;
+    // Without a side stream (it could not be created) both parts run on `stream`, in
+    // order: the same results, without the overlap.
+    side = side_stream(scope.dev, stream);
+    if (!side) (void)cudaGetLastError();
+  }
+  if (side) {
     if (cudaEventRecord(side->fork, stream) != cudaSuccess ||
         cudaStreamWaitEvent(side->stream, side->fork, 0) != cudaSuccess)
       return SPEC_ERR_CUDA;
@@ -447,8 +480,8 @@ spec_status_t spec_noise_tokens(uint64_t seed, uint64_t offset, int64_t n, int32
                                 int32_t* out_dev, spec_stream_t stream) {
   if (n < 0 || vocab < 1 || (n > 0 && !out_dev)) return SPEC_ERR_INVALID_ARGUMENT;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  int sms = 0;
-  if (!bind_device(s, &sms)) return SPEC_ERR_CUDA;
+  DeviceScope scope(s);
+  if (!scope.ok) return SPEC_ERR_CUDA;
   return launch_noise(seed, offset, n, vocab, out_dev, s) == cudaSuccess ? SPEC_OK : SPEC_ERR_CUDA;
 }
 
@@ -482,8 +515,9 @@ spec_status_t spec_sample_block(const spec_draft_args_t* draft, const spec_filte
   if (!filter && draft_layout(*draft, kWsHeader, 1, vec).smem > kDraftMaxSmem) return SPEC_ERR_UNSUPPORTED;
   if (draft_bytes(*draft, filter, 1, vec) > ws_bytes) return SPEC_ERR_WORKSPACE_TOO_SMALL;
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
-  int sms = 0;
-  if (!bind_device(stream, &sms)) return SPEC_ERR_CUDA;
+  DeviceScope scope(stream);
+  if (!scope.ok) return SPEC_ERR_CUDA;
+  const int sms = scope.sms;
   (void)cudaGetLastError();
   if (draft_bytes(*draft, filter, sms, vec) > ws_bytes) return SPEC_ERR_WORKSPACE_TOO_SMALL;
   char* w = static_cast<char*>(ws);
@@ -526,8 +560,9 @@ spec_status_t spec_accept_tree(const spec_tree_accept_args_t* t, void* ws, size_
   if (tree_layout(t->batch, t->num_nodes, t->vocab, kWsHeader, 1, vec).end > ws_bytes)
     return SPEC_ERR_WORKSPACE_TOO_SMALL;
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
-  int sms = 0;
-  if (!bind_device(stream, &sms)) return SPEC_ERR_CUDA;
+  DeviceScope scope(stream);
+  if (!scope.ok) return SPEC_ERR_CUDA;
+  const int sms = scope.sms;
   const TreeLayout L = tree_layout(t->batch, t->num_nodes, t->vocab, kWsHeader, sms, vec);
   if (L.end > ws_bytes) return SPEC_ERR_WORKSPACE_TOO_SMALL;
   return launch_tree_greedy(*t, L, static_cast<char*>(ws), stream, vec) == cudaSuccess
@@ -559,8 +594,9 @@ spec_status_t spec_build_tree(const spec_tree_build_args_t* t, void* ws, size_t 
   const bool vec = (static_cast<size_t>(t->vocab) * esz) % 16 == 0 &&
                    reinterpret_cast<uintptr_t>(t->drafter_logits) % 16 == 0;
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
-  int sms = 0;
-  if (!bind_device(stream, &sms)) return SPEC_ERR_CUDA;
+  DeviceScope scope(stream);
+  if (!scope.ok) return SPEC_ERR_CUDA;
+  const int sms = scope.sms;
   const TreeBuildLayout L = tree_build_layout(*t, kWsHeader, sms);
   if (L.end > ws_bytes) return SPEC_ERR_WORKSPACE_TOO_SMALL;
   return launch_tree_build(*t, L, static_cast<char*>(ws), stream, vec) == cudaSuccess ? SPEC_OK
@@ -580,8 +616,8 @@ spec_status_t spec_lm_head_stats(const spec_lm_head_args_t* a, void* ws, size_t 
   const LmLayout L = lm_layout(*a, kWsHeader);
   if (L.end > ws_bytes) return SPEC_ERR_WORKSPACE_TOO_SMALL;
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
-  int sms = 0;
-  if (!bind_device(stream, &sms)) return SPEC_ERR_CUDA;
+  DeviceScope scope(stream);
+  if (!scope.ok) return SPEC_ERR_CUDA;
   return launch_lm_head(*a, L, static_cast<char*>(ws), stream) == cudaSuccess ? SPEC_OK : SPEC_ERR_CUDA;
 }
 
@@ -595,8 +631,8 @@ spec_status_t spec_commit_tree_kv(const spec_tree_commit_args_t* c, spec_stream_
     return SPEC_ERR_INVALID_ARGUMENT;
   if (c->batch > 65535) return SPEC_ERR_UNSUPPORTED;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  int sms = 0;
-  if (!bind_device(s, &sms)) return SPEC_ERR_CUDA;
+  DeviceScope scope(s);
+  if (!scope.ok) return SPEC_ERR_CUDA;
   return launch_tree_commit(*c, s) == cudaSuccess ? SPEC_OK : SPEC_ERR_CUDA;
 }
 
@@ -608,8 +644,8 @@ spec_status_t spec_commit_kv(const spec_commit_args_t* c, spec_stream_t stream) 
   if (static_cast<int64_t>(c->max_pages_per_seq) * c->page_size + c->gamma > INT32_MAX)
     return SPEC_ERR_UNSUPPORTED;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  int sms = 0;
-  if (!bind_device(s, &sms)) return SPEC_ERR_CUDA;
+  DeviceScope scope(s);
+  if (!scope.ok) return SPEC_ERR_CUDA;
   return launch_commit(*c, s) == cudaSuccess ? SPEC_OK : SPEC_ERR_CUDA;
 }
 
@@ -617,16 +653,16 @@ spec_status_t spec_philox_uniforms(uint64_t seed, uint64_t offset, int64_t n, fl
                                    spec_stream_t stream) {
   if (n < 0 || (n > 0 && !out_dev)) return SPEC_ERR_INVALID_ARGUMENT;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  int sms = 0;
-  if (!bind_device(s, &sms)) return SPEC_ERR_CUDA;
+  DeviceScope scope(s);
+  if (!scope.ok) return SPEC_ERR_CUDA;
   return launch_philox(seed, offset, n, out_dev, s) == cudaSuccess ? SPEC_OK : SPEC_ERR_CUDA;
 }
 
 spec_status_t spec_read_device_status(void* ws, spec_stream_t stream, uint32_t* flags_out) {
   if (!ws || !flags_out) return SPEC_ERR_INVALID_ARGUMENT;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  int sms = 0;
-  if (!bind_device(s, &sms)) return SPEC_ERR_CUDA;
+  DeviceScope scope(s);
+  if (!scope.ok) return SPEC_ERR_CUDA;
   uint32_t flags = 0;
   if (cudaMemcpyAsync(&flags, ws, sizeof(flags), cudaMemcpyDeviceToHost, s) != cudaSuccess)
     return SPEC_ERR_CUDA;

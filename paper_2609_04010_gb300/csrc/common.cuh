@@ -194,6 +194,30 @@ inline cudaError_t stream_device(cudaStream_t stream, int* dev) {
   }
   return cudaGetDevice(dev);
 }
+// Cached multiprocessor count of a device (asked once per device).
+int device_sm_count(int dev);
+
+// Makes the device of `stream` current for the duration of one entry point and puts
+// the caller's current device back when it goes out of scope, so that no call changes
+// which device the calling thread has current. `ok` is false when the device could
+// not be found or selected.
+struct DeviceScope {
+  int dev = 0, prev = -1, sms = 0;
+  bool ok = false;
+  explicit DeviceScope(cudaStream_t stream) {
+    if (cudaGetDevice(&prev) != cudaSuccess) { prev = -1; return; }
+    if (stream_device(stream, &dev) != cudaSuccess) return;
+    if (dev != prev && cudaSetDevice(dev) != cudaSuccess) return;
+    sms = device_sm_count(dev);
+    ok = true;
+  }
+  ~DeviceScope() {
+    if (prev >= 0 && dev != prev) cudaSetDevice(prev);
+  }
+  DeviceScope(const DeviceScope&) = delete;
+  DeviceScope& operator=(const DeviceScope&) = delete;
+};
+
 int tc_ctas_per_sm(int head_dim, int rows_per_cta, int batch);
 size_t tc_smem_bytes(int head_dim, int rows_per_cta, int batch);
 constexpr int kTcMaxBatch = 4096;  // batch prefix sums live in shared memory

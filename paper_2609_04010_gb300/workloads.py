@@ -423,3 +423,129 @@ def logits_bytes_strict(temps: np.ndarray, gamma: int, vocab: int, elem_bytes: i
     t = np.asarray(temps)
     rows = gamma * len(t) + (gamma - 1) * int((t > 0).sum())
     return rows * vocab * elem_bytes
+
+
+# ---------------------------------------------------------------------------------
+# Device-side generators for sizes the host generator cannot fill quickly
+# ---------------------------------------------------------------------------------
+# The sweep's largest points hold billions of random values (batch 128 with contexts up
+# to 16,384, or 128 x 32 x 151,936 logits per side). These generators draw the same
+# distributions on the GPU with torch's seeded generator; the tests copy to the host
+# only what the oracle needs. Like the rest of this module they draw inputs and compute
+# nothing of the verify step.
+def _torch_gen(seed: int, stream: int, device):
+    import torch
+    g = torch.Generator(device=device)
+    g.manual_seed((int(seed) * 1_000_003 + int(stream) * 7_919) & 0x7FFF_FFFF_FFFF_FFFF)
+    return g
+
+
+@dataclasses.dataclass
+class DeviceAttnInputs:
+    q: object            # torch bf16 [batch][gamma][Hq][D] on the device
+    k_cache: object      # torch bf16 [num_pages][Hkv][page_size][D]
+    v_cache: object
+    page_table: object   # torch int32 [batch][max_pages]
+    kv_len: object       # torch int32 [batch]
+    page_table_host: np.ndarray
+    kv_len_host: np.ndarray
+    gamma: int
+
+    def host(self) -> AttnInputs:
+        """The same inputs as host arrays (bf16 as uint16 bits), for the oracle."""
+        import torch
+
+        def bits(t):
+            return t.contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+        return AttnInputs(bits(self.q), bits(self.k_cache), bits(self.v_cache),
+                          self.page_table_host.copy(), self.kv_len_host.copy())
+
+
+def make_attn_inputs_device(batch: int, gamma: int, num_q_heads: int, num_kv_heads: int,
+                            head_dim: int, page_size: int, ctx, seed: int = 0,
+                            device="cuda") -> DeviceAttnInputs:
+    """make_attn_inputs' shapes and distributions (contexts uniform on lo..hi, a seeded
+    permutation of physical pages, Q, K, V ~ N(0, 1) rounded to bf16), with Q, K and V
+    drawn on the device. Contexts and the page table come from the host streams of
+    make_attn_inputs, so they equal its own for the same arguments."""
+    import torch
+    if isinstance(ctx, (tuple, list)):
+        lo, hi = int(ctx[0]), int(ctx[1])
+        ctxs = _rng(seed, STREAM_CTX).integers(lo, hi + 1, size=batch).astype(np.int32)
+    else:
+        ctxs = np.full(batch, int(ctx), dtype=np.int32)
+    kv_len = (ctxs + gamma).astype(np.int32)
+    pages = (kv_len + page_size - 1) // page_size
+    total = int(pages.sum())
+    phys = _rng(seed, STREAM_PAGES).permutation(total).astype(np.int32)
+    pt = np.full((batch, int(pages.max())), -1, dtype=np.int32)
+    cur = 0
+    for b in range(batch):
+        pt[b, :pages[b]] = phys[cur:cur + pages[b]]
+        cur += int(pages[b])
+
+    def normals(stream, shape):
+        g = _torch_gen(seed, stream, device)
+        return torch.randn(*shape, generator=g, device=device, dtype=torch.float32).to(torch.bfloat16)
+
+    q = normals(STREAM_Q, (batch, gamma, num_q_heads, head_dim))
+    k = normals(STREAM_K, (total, num_kv_heads, page_size, head_dim))
+    v = normals(STREAM_V, (total, num_kv_heads, page_size, head_dim))
+    return DeviceAttnInputs(q, k, v, torch.from_numpy(pt).to(device),
+                            torch.from_numpy(kv_len).to(device), pt, kv_len, gamma)
+
+
+@dataclasses.dataclass
+class DeviceAcceptInputs:
+    target_logits: object   # torch bf16 [batch][gamma][vocab] on the device
+    drafter_logits: object
+    block_tokens: object    # torch int32 [batch][gamma]
+    temperature: object     # torch float32 [batch]
+    uniforms: object        # torch float32 [batch][gamma]
+
+    def host(self, nseq: int) -> AcceptInputs:
+        """The first nseq sequences as host arrays (bf16 as uint16 bits), for the oracle."""
+        import torch
+
+        def bits(t):
+            return t[:nseq].contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+        return AcceptInputs(bits(self.target_logits), bits(self.drafter_logits),
+                            self.block_tokens[:nseq].cpu().numpy(),
+                            self.temperature[:nseq].cpu().numpy(),
+                            self.uniforms[:nseq].cpu().numpy())
+
+
+def make_accept_inputs_device(batch: int, gamma: int, vocab: int, target_sigma: float = 3.0,
+                              drafter_sigma: float = 1.0, temperature=1.0, seed: int = 0,
+                              device="cuda", chunk: int = 8) -> DeviceAcceptInputs:
+    """make_accept_inputs' distributions with bf16 logits drawn on the device: target rows
+    ~ N(0, target_sigma^2), drafter row j >= 1 = target row j-1 + N(0, drafter_sigma^2),
+    drafter row 0 independent, both rounded to bf16; block token j drawn from drafter
+    row j at the sequence's temperature by Gumbel-max (argmax at T = 0, lowest index on
+    ties). The uniforms are the host Philox stream of make_accept_inputs, bit for bit."""
+    import torch
+    temps = np.resize(np.asarray(temperature, dtype=np.float32).ravel(), batch)
+    g = _torch_gen(seed, STREAM_TARGET, device)
+    tl = torch.empty(batch, gamma, vocab, dtype=torch.bfloat16, device=device)
+    dl = torch.empty_like(tl)
+    tok = torch.empty(batch, gamma, dtype=torch.int32, device=device)
+    for b0 in range(0, batch, chunk):
+        n = min(chunk, batch - b0)
+        t32 = torch.randn(n, gamma, vocab, generator=g, device=device) * target_sigma
+        d32 = torch.empty_like(t32)
+        d32[:, 0] = torch.randn(n, vocab, generator=g, device=device) * target_sigma
+        if gamma > 1:
+            d32[:, 1:] = t32[:, :-1] + torch.randn(n, gamma - 1, vocab, generator=g,
+                                                   device=device) * drafter_sigma
+        tl[b0:b0 + n] = t32.to(torch.bfloat16)
+        dl[b0:b0 + n] = d32.to(torch.bfloat16)
+        dseen = dl[b0:b0 + n].float()
+        T = torch.from_numpy(temps[b0:b0 + n]).to(device).view(n, 1, 1)
+        u = torch.rand(n, gamma, vocab, generator=g, device=device).clamp_min(1e-30)
+        gumbel = -torch.log(-torch.log(u))
+        score = torch.where(T > 0, dseen / torch.where(T > 0, T, torch.ones_like(T)) + gumbel, dseen)
+        tok[b0:b0 + n] = torch.argmax(score, dim=-1).to(torch.int32)
+        del t32, d32, dseen, u, gumbel, score
+    uni = philox_uniforms(uniform_seed(seed), batch * gamma).reshape(batch, gamma)
+    return DeviceAcceptInputs(tl, dl, tok, torch.from_numpy(temps).to(device),
+                              torch.from_numpy(uni).to(device))

@@ -209,3 +209,43 @@ def test_unused_drafter_row_is_never_read():
         for k in ("num_accepted", "out_tokens", "num_emitted"):
             np.testing.assert_array_equal(outs[0][k], outs[1][k])
         assert np.all(outs[1]["out_tokens"][:, 0] == inp.block_tokens[:, 0])
+
+
+def test_gpu_mean_accepted_matches_closed_form():
+    """The GPU's accepted-draft counts over 200,000 seeded steps against the closed form
+    (Leviathan et al.'s acceptance rate, the TV link of Sec. 3.2): with fixed rows,
+    P(a >= k) = prod_{i <= k} alpha_i, alpha_i = sum_x min(p_{i-1}(x), q_i(x)), and
+    E[a] = sum_k P(a >= k). The mean and every tail probability must lie within 5
+    standard errors."""
+    from scipy import special
+    rng = np.random.default_rng(33)
+    gamma, V, T = 6, 64, 1.0
+    target = (rng.standard_normal((gamma, V)) * 2.0).astype(np.float32)
+    drafter = np.empty_like(target)
+    drafter[0] = rng.standard_normal(V).astype(np.float32)
+    drafter[1:] = target[:-1] + rng.standard_normal((gamma - 1, V)).astype(np.float32) * 0.7
+    p = special.softmax(target.astype(np.float64) / T, axis=-1)
+    q = special.softmax(drafter.astype(np.float64) / T, axis=-1)
+    alpha = np.array([np.minimum(p[i - 1], q[i]).sum() for i in range(1, gamma)])
+    tail = np.cumprod(alpha)                 # P(a >= k), k = 1 .. gamma-1
+    expect = tail.sum()
+    N, chunk = 200_000, 50_000
+    tl = torch.from_numpy(np.broadcast_to(target, (chunk, gamma, V)).copy()).cuda()
+    dl = torch.from_numpy(np.broadcast_to(drafter, (chunk, gamma, V)).copy()).cuda()
+    temp = torch.full((chunk,), T, dtype=torch.float32, device="cuda")
+    counts = []
+    for c in range(N // chunk):
+        tok = np.zeros((chunk, gamma), np.int32)
+        for i in range(gamma):
+            tok[:, i] = rng.choice(V, size=chunk, p=q[i])
+        u = binding.philox_uniforms(W.uniform_seed(5000 + c), chunk * gamma).view(chunk, gamma)
+        r = binding.accept_block(tl, dl, torch.from_numpy(tok).cuda(), temp, u, want_diag=False)
+        counts.append(r["num_accepted"].cpu().numpy())
+    a = np.concatenate(counts).astype(np.float64)
+    se = a.std() / np.sqrt(N)
+    assert abs(a.mean() - expect) < 5 * se, (a.mean(), expect, se)
+    for k in range(1, gamma):
+        f = (a >= k).mean()
+        se_k = np.sqrt(tail[k - 1] * (1 - tail[k - 1]) / N)
+        assert abs(f - tail[k - 1]) < 5 * se_k + 1e-12, (k, f, tail[k - 1])
+    print(f"mean accepted {a.mean():.4f} vs closed form {expect:.4f} (se {se:.4f})")

@@ -65,6 +65,19 @@ def test_named_workloads_sampled(oracle_mod, name):
     print(f"{name}: max abs err {err:.2e}, lse err {lerr:.2e}")
 
 
+@pytest.mark.parametrize("name", ["llama8b", "serve64"])
+def test_named_workload_every_row(oracle_mod, name):
+    """Full-size workloads in the benchmark's launch configuration, every (sequence,
+    block position, head) row element-wise against the oracle (2,048 rows at llama8b,
+    32,768 at serve64)."""
+    inp = W.workload(name).attn_inputs(seed=0)
+    g_out, g_lse = gpu_attention(inp, binding.ATTN_AUTO)
+    o_out, o_lse, st = oracle_attn(oracle_mod, inp)
+    assert np.all(st == 0)
+    err, lerr = compare_attention(g_out, g_lse, o_out, o_lse)
+    print(f"{name} every row: max abs err {err:.2e}, lse err {lerr:.2e}")
+
+
 @pytest.mark.parametrize("path", PATHS)
 def test_page_order_invariance_bitwise(path):
     inp = W.make_attn_inputs(3, 8, 32, 8, 128, 16, (50, 400), permute_pages=False, seed=11)

@@ -117,3 +117,53 @@ def test_step_replays_in_a_cuda_graph(name, path):
         assert binding.read_device_status(ws1) == (0, 0)
         for k in eager:
             assert torch.equal(eager[k].nan_to_num(-7), graphed[k].nan_to_num(-7)), k
+
+
+def test_steps_on_two_streams_are_independent(oracle_mod):
+    """Two fused steps issued from one host thread on two streams: each matches the
+    oracle, the second finishes while the first stream is still held by a bounded
+    spinning kernel (the two steps share no side stream, so neither waits for the
+    other), and the calling thread's current device is unchanged."""
+    wl = W.workload("tiny")
+    ai, ci = wl.attn_inputs(seed=5), wl.accept_inputs(seed=5)
+    at, ct = attn_tensors(ai), accept_tensors(ci)
+    B, G = ci.batch, ci.gamma
+
+    def outputs():
+        return dict(out=torch.empty_like(at[0]),
+                    lse=torch.empty(at[0].shape[:3], dtype=torch.float32, device="cuda"),
+                    num_accepted=torch.empty(B, dtype=torch.int32, device="cuda"),
+                    out_tokens=torch.empty(B, G + 1, dtype=torch.int32, device="cuda"),
+                    num_emitted=torch.empty(B, dtype=torch.int32, device="cuda"),
+                    diag=torch.empty(B, G, 2, dtype=torch.float32, device="cuda"))
+
+    res = [outputs(), outputs()]
+    args = []
+    for r in res:
+        a = binding.attn_args(*at, r["out"], r["lse"])
+        c = binding.accept_args(*ct, r["num_accepted"], r["out_tokens"], r["num_emitted"],
+                                r["diag"])
+        args.append((a, c, binding.new_workspace(binding.workspace_size(a, c))))
+    s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
+    dev_before = torch.cuda.current_device()
+    for (a, c, ws), s in zip(args, (s1, s2)):  # first calls make each stream's side stream
+        binding.verify_step_args(a, c, ws, stream=s)
+    torch.cuda.synchronize()
+    with torch.cuda.stream(s1):
+        torch.cuda._sleep(1_000_000_000)  # about half a second of clock cycles on s1
+    binding.verify_step_args(*args[0], stream=s1)
+    binding.verify_step_args(*args[1], stream=s2)
+    s2.synchronize()
+    first_still_busy = not s1.query()
+    s1.synchronize()
+    assert first_still_busy
+    assert torch.cuda.current_device() == dev_before
+    o = oracle_mod.accept_block(ci.target_logits, ci.drafter_logits, ci.block_tokens,
+                                ci.temperature, ci.uniforms)
+    o_out, o_lse, _ = oracle_mod.verify_attention(ai.q, ai.k_cache, ai.v_cache, ai.page_table,
+                                                  ai.kv_len, ai.gamma)
+    for (a, c, ws), r in zip(args, res):
+        assert binding.read_device_status(ws) == (0, 0)
+        compare_accept({k: v.cpu().numpy() for k, v in r.items() if k not in ("out", "lse")},
+                       o, G)
+        compare_attention(r["out"].float().cpu().numpy(), r["lse"].cpu().numpy(), o_out, o_lse)

@@ -2,7 +2,8 @@
 
 Each test checks the oracle against something other than itself:
   * exact losslessness, by enumerating every draft and every cell of the uniforms on
-    probability rows whose entries are multiples of 1/16 (the paper's claim that the
+    probability rows whose entries are multiples of 1/8 (vocabulary 8, gamma 3) or of
+    1/16 (vocabulary 4, gamma 3) (the paper's claim that the
     verify step "preserves the base model's target distribution", Sec. 4.2);
   * the closed-form acceptance rate alpha_i = sum_x min(p_i(x), q_i(x)) = 1 - TV
     (the Total Variation link the paper cites in Sec. 3.2, Eq. "tv-loss");
@@ -93,6 +94,19 @@ def rows16(*rows):
     return a
 
 
+def rows8(*rows):
+    a = np.array(rows, dtype=np.float64) / 8.0
+    assert np.allclose(a.sum(axis=1), 1.0)
+    return a
+
+
+# vocabulary 8, gamma 3: rows whose entries are multiples of 1/8, so that every
+# threshold of the rule is a fraction with denominator <= 8 and Farey(8) cells suffice
+GENERIC8_P = rows8([2, 1, 0, 1, 1, 0, 2, 1], [0, 1, 3, 1, 0, 1, 1, 1], [1, 1, 1, 1, 1, 1, 1, 1])
+GENERIC8_Q = rows8([1, 1, 1, 1, 1, 1, 1, 1], [1, 2, 0, 1, 2, 1, 0, 1], [3, 0, 1, 1, 0, 1, 1, 1])
+SPARSE8_P = rows8([0, 4, 0, 0, 4, 0, 0, 0], [8, 0, 0, 0, 0, 0, 0, 0], [0, 0, 3, 0, 0, 0, 0, 5])
+SPARSE8_Q = rows8([0, 0, 0, 8, 0, 0, 0, 0], [1, 1, 1, 0, 0, 0, 0, 5], [0, 2, 2, 0, 0, 4, 0, 0])
+
 GENERIC_P = rows16([5, 3, 6, 2], [1, 7, 4, 4], [8, 2, 3, 3])
 GENERIC_Q = rows16([4, 4, 4, 4], [4, 4, 2, 6], [2, 6, 6, 2])
 SPARSE_P = rows16([0, 8, 8, 0], [16, 0, 0, 0], [3, 0, 0, 13])
@@ -105,6 +119,27 @@ def test_lossless_exact_enumeration(oracle_mod, p_rows, q_rows):
     P, _ = exact_output_distribution(oracle_mod, p_rows, q_rows, 16)
     assert abs(P.sum() - 1.0) < 1e-12
     np.testing.assert_allclose(P, target_product(p_rows), rtol=0, atol=1e-12)
+
+
+@pytest.mark.parametrize("p_rows,q_rows", [(GENERIC8_P, GENERIC8_Q), (SPARSE8_P, SPARSE8_Q)],
+                         ids=["generic", "sparse"])
+def test_lossless_exact_enumeration_vocab8(oracle_mod, p_rows, q_rows):
+    # every one of the 8^2 draft pairs and every Farey(8) cell of the three uniforms
+    P, A = exact_output_distribution(oracle_mod, p_rows, q_rows, 8)
+    assert abs(P.sum() - 1.0) < 1e-12
+    np.testing.assert_allclose(P, target_product(p_rows), rtol=0, atol=1e-12)
+    # an immediate rejection and a later one are both taken; on the generic rows also
+    # the full acceptance (the sparse q_2 has no mass where p_1 has any)
+    assert A[1].sum() > 0 and A[2].sum() > 0
+    assert (A[3].sum() > 0) == (p_rows is GENERIC8_P)
+
+
+def test_negative_control_vocab8(oracle_mod):
+    greedy = np.zeros_like(GENERIC8_Q)
+    for i in range(GENERIC8_Q.shape[0]):
+        greedy[i, int(np.argmax(GENERIC8_Q[i]))] = 1.0
+    P, _ = exact_output_distribution(oracle_mod, GENERIC8_P, GENERIC8_Q, 8, draft_weights=greedy)
+    assert np.abs(P - target_product(GENERIC8_P)).max() > 1e-2
 
 
 def test_identical_drafter_accepts_everything(oracle_mod):

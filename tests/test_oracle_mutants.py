@@ -19,7 +19,8 @@ import test_oracle_draft as DRAFT
 import test_oracle_lm_head as LM
 import test_oracle_tree as TREE
 
-from test_oracle_accept import GENERIC_P, GENERIC_Q, exact_output_distribution, target_product
+from test_oracle_accept import (GENERIC8_P, GENERIC8_Q, GENERIC_P, GENERIC_Q,
+                                exact_output_distribution, target_product)
 from test_oracle_filtered import P_FILT, filtered_output_distribution
 
 MUTANTS = {
@@ -47,8 +48,10 @@ def test_mutant_breaks_losslessness(oracle_mod, name):
     src = oracle_mod.source_text()
     assert src.count(before) == 1, f"mutation site for {name} not found in oracle.cpp"
     lib = oracle_mod.load_variant(src.replace(before, after), name)
-    P, _ = exact_output_distribution(oracle_mod, GENERIC_P, GENERIC_Q, 16, lib=lib)
-    assert np.abs(P - target_product(GENERIC_P)).max() > 1e-4
+    # caught by the enumeration at vocabulary 4 (1/16 rows) and at vocabulary 8 (1/8 rows)
+    for p_rows, q_rows, denom in ((GENERIC_P, GENERIC_Q, 16), (GENERIC8_P, GENERIC8_Q, 8)):
+        P, _ = exact_output_distribution(oracle_mod, p_rows, q_rows, denom, lib=lib)
+        assert np.abs(P - target_product(p_rows)).max() > 1e-4, (name, p_rows.shape)
 
 
 FILTER_MUTANTS = {

@@ -3,9 +3,9 @@ allocate device memory (its scratch is a fixed device array inside the library).
 
 Collected last on purpose, so that a run stopping at the first failure has already run
 every other test. The GPU test calls the entry point twice in a row through the C ABI
-and checks each result against spec_accept_block with a caller workspace, within the
-acceptance tolerances the other tests use (the two share their kernels, so the tokens
-agree bit for bit)."""
+and checks each result against spec_accept_block with a caller workspace (the two share
+their kernels, so the tokens agree bit for bit) and against the fp64 oracle, within the
+acceptance tolerances the other tests use (tokens bit-exact except counted ties)."""
 
 import ctypes
 
@@ -51,7 +51,9 @@ def test_argument_errors_match_the_workspace_entry_point(args, code):
 
 
 @pytest.mark.gpu
-def test_matches_workspace_entry_point_twice():
+def test_matches_workspace_entry_point_twice(oracle_mod):
+    from helpers import compare_accept
+
     def one(inp):
         dev = lambda x: torch.from_numpy(np.ascontiguousarray(x)).cuda()
         bf = lambda x: torch.from_numpy(x.view(np.int16)).view(torch.bfloat16).cuda()
@@ -72,6 +74,13 @@ def test_matches_workspace_entry_point_twice():
         assert np.array_equal(np.isnan(d_new), np.isnan(d_ref))
         ok = ~np.isnan(d_ref)
         np.testing.assert_allclose(d_new[ok], d_ref[ok], rtol=1e-5, atol=0)
+        # and against the oracle on the same inputs
+        o = oracle_mod.accept_block(inp.target_logits, inp.drafter_logits, inp.block_tokens,
+                                    inp.temperature, inp.uniforms)
+        g = {k: v.cpu().numpy() for k, v in out.items()}
+        ties = compare_accept(g, o, G)
+        assert len(ties) <= 1, ties
+        assert torch.cuda.current_device() == 0  # the caller's current device is kept
 
     # two calls in a row on different batches: the second must not see the first's scratch
     one(W.make_accept_inputs(8, 8, 40000, "bf16", 3.0, 1.0, [1.0, 0.0, 0.7], seed=31))
