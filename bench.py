@@ -86,8 +86,11 @@ def parse_args():
                     help="comma-separated workloads whose fused step is also timed in the same "
                          "run (device time, rooflines, clocks), reported under 'workloads'; "
                          "'' for none")
-    ap.add_argument("--attn-path", choices=["auto", "cuda-cores", "tensor-cores"], default="auto",
-                    help="attention kernel (auto: tensor cores from the library's row crossover)")
+    ap.add_argument("--attn-path", choices=["auto", "cuda-cores", "tensor-cores", "keys-on-lanes"],
+                    default="auto",
+                    help="attention kernel (auto: the row-tile tensor-core kernel from the "
+                         "library's row crossover; keys-on-lanes: the transposed tensor-core "
+                         "kernel where it applies)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-draft", action="store_true",
@@ -291,9 +294,16 @@ def whole_job_tokens_per_s(world: int, batch: int, gamma: int, ms: float) -> flo
 # our arm
 # ----------------------------------------------------------------------------------
 def attn_path_name(choice, binding, ai):
+    """The attention kernel the library picks for this workload and --attn-path."""
+    group = ai.num_q_heads // ai.num_kv_heads
+    rows = group * ai.gamma
     if choice == "auto":
-        rows = (ai.num_q_heads // ai.num_kv_heads) * ai.gamma
-        return "tensor cores" if rows >= binding.tensor_core_min_rows() else "CUDA cores"
+        choice = "tensor-cores" if rows >= binding.tensor_core_min_rows() else "cuda-cores"
+    if choice == "keys-on-lanes":
+        kl = ai.head_dim == 128 and rows <= 64 and 64 % group == 0 and ai.batch <= 2048
+        return "tensor cores, keys on lanes" if kl else "tensor cores, row tiles"
+    if choice == "tensor-cores":
+        return "tensor cores, row tiles"
     return choice.replace("-", " ")
 
 
@@ -328,7 +338,8 @@ class StepSetup:
         ot = torch.empty(B, G + 1, dtype=torch.int32, device=dev)
         ne = torch.empty(B, dtype=torch.int32, device=dev)
         path = {"auto": binding.ATTN_AUTO, "cuda-cores": binding.ATTN_CUDA_CORES,
-                "tensor-cores": binding.ATTN_TENSOR_CORES}[args.attn_path]
+                "tensor-cores": binding.ATTN_TENSOR_CORES,
+                "keys-on-lanes": binding.ATTN_TENSOR_CORES_KEYS_ON_LANES}[args.attn_path]
         a = binding.attn_args(d["q"], d["k"], d["v"], d["pt"], d["kvl"], out, lse, path=path)
         c = binding.accept_args(d["tl"], d["dl"], d["tok"], d["temp"], d["u"], na, ot, ne, None)
         if filtered:
@@ -520,7 +531,7 @@ def run_ours(args, wl, ai, ci, rank, world, local_rank):
     # the one filtered acceptance kernel
     launches_per_step = 2 if filtered else 4
     traffic, traffic_src = (None, None)
-    if dominant == "attention" and attn_path_name(args.attn_path, binding, ai) == "tensor cores":
+    if dominant == "attention" and attn_path_name(args.attn_path, binding, ai).startswith("tensor"):
         traffic, traffic_src = measured_traffic(args.workload, "attention")
     result = {
         "metric": METRIC, "value": whole_job_tokens_per_s(world, B, G, ms), "unit": UNIT,

@@ -73,7 +73,14 @@ typedef enum { SPEC_F32 = 0, SPEC_BF16 = 1 } spec_dtype_t;
 typedef enum {
   SPEC_ATTN_AUTO = 0,          /* tensor cores when (Hq/Hkv)*gamma >= the crossover, else CUDA cores */
   SPEC_ATTN_CUDA_CORES = 1,    /* fp32 CUDA-core kernel                                  */
-  SPEC_ATTN_TENSOR_CORES = 2   /* tcgen05 (TMEM accumulators, TMA-staged KV pages)       */
+  SPEC_ATTN_TENSOR_CORES = 2,  /* tcgen05 (TMEM accumulators, TMA-staged KV pages), the
+                                  row-tile kernel (M = 128 query rows per tile)           */
+  SPEC_ATTN_TENSOR_CORES_KEYS_ON_LANES = 3  /* tcgen05 with the keys of a tile on the MMA's
+                                  M dimension (S^T = K Q^T, O^T = V^T P^T), where it applies
+                                  (head_dim 128, at most 64 query rows per KV head, 64 %
+                                  group == 0, batch <= 2048, no tree mask), else as 2; same
+                                  results within the tolerance. Measured slower than 2 on
+                                  GB300 at the named workloads, so AUTO does not pick it */
 } spec_attn_path_t;
 
 /* Device status word bits. */

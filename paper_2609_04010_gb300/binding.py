@@ -26,7 +26,7 @@ STATUS_NAMES = {0: "SPEC_OK", 1: "SPEC_ERR_INVALID_ARGUMENT", 2: "SPEC_ERR_UNSUP
                 3: "SPEC_ERR_WORKSPACE_TOO_SMALL", 4: "SPEC_ERR_CUDA", 5: "SPEC_ERR_DEVICE_INPUT",
                 6: "SPEC_ERR_TIMEOUT"}
 SPEC_F32, SPEC_BF16 = 0, 1
-ATTN_AUTO, ATTN_CUDA_CORES, ATTN_TENSOR_CORES = 0, 1, 2
+ATTN_AUTO, ATTN_CUDA_CORES, ATTN_TENSOR_CORES, ATTN_TENSOR_CORES_KEYS_ON_LANES = 0, 1, 2, 3
 FLAG_BAD_TOKEN, FLAG_BAD_LOGITS, FLAG_BAD_PAGE, FLAG_BAD_KV_LEN, FLAG_TIMEOUT = 1, 2, 4, 8, 16
 FLAG_BAD_FILTER = 32
 FLAG_BAD_TREE = 64

@@ -119,8 +119,11 @@ spec_status_t check_attn(const spec_attn_args_t* a) {
     return SPEC_ERR_INVALID_ARGUMENT;
   if (!(a->softmax_scale == 0.f || (a->softmax_scale > 0.f && a->softmax_scale < 1e30f)))
     return SPEC_ERR_INVALID_ARGUMENT;
-  if (a->path < SPEC_ATTN_AUTO || a->path > SPEC_ATTN_TENSOR_CORES) return SPEC_ERR_INVALID_ARGUMENT;
-  if (a->path == SPEC_ATTN_TENSOR_CORES && a->batch > kTcMaxBatch) return SPEC_ERR_UNSUPPORTED;
+  if (a->path < SPEC_ATTN_AUTO || a->path > SPEC_ATTN_TENSOR_CORES_KEYS_ON_LANES)
+    return SPEC_ERR_INVALID_ARGUMENT;
+  if ((a->path == SPEC_ATTN_TENSOR_CORES || a->path == SPEC_ATTN_TENSOR_CORES_KEYS_ON_LANES) &&
+      a->batch > kTcMaxBatch)
+    return SPEC_ERR_UNSUPPORTED;
   if (a->gamma > 64) return SPEC_ERR_UNSUPPORTED;
   if (a->head_dim != 64 && a->head_dim != 128) return SPEC_ERR_UNSUPPORTED;
   if (a->page_size != 16 && a->page_size != 32 && a->page_size != 64) return SPEC_ERR_UNSUPPORTED;
@@ -245,6 +248,12 @@ AttnPlan attn_plan(const spec_attn_args_t& a, size_t base, int num_sms, int path
   if (path == SPEC_ATTN_AUTO)
     path = (P.rows >= tc_min_rows() && a.batch <= kTcMaxBatch) ? SPEC_ATTN_TENSOR_CORES
                                                                : SPEC_ATTN_CUDA_CORES;
+  // the keys-on-lanes kernel, when asked for, takes the KV groups of at most 64 query rows
+  const int group = a.num_q_heads / a.num_kv_heads;
+  P.keys_on_lanes = path == SPEC_ATTN_TENSOR_CORES_KEYS_ON_LANES && a.head_dim == 128 &&
+                    P.rows <= kKlMaxRows && kKlMaxRows % group == 0 && a.batch <= kKlMaxBatch &&
+                    !a.tree_mask;
+  if (path == SPEC_ATTN_TENSOR_CORES_KEYS_ON_LANES) path = SPEC_ATTN_TENSOR_CORES;
   P.path = path;
   P.max_keys = a.max_pages_per_seq * a.page_size;
   int64_t units;
@@ -263,6 +272,17 @@ AttnPlan attn_plan(const spec_attn_args_t& a, size_t base, int num_sms, int path
     P.grid = 0;
     P.slot_rows = P.rows_per_cta;
     P.slots = P.nsplit > 1 ? units * P.nsplit : 0;
+  } else if (P.keys_on_lanes) {
+    // persistent grid, one block per SM; one unit per (sequence, KV head)
+    P.rows_per_cta = kKlMaxRows;
+    P.key_tile = kKlKeyTile;
+    P.row_tiles = 1;
+    units = static_cast<int64_t>(a.batch) * a.num_kv_heads;
+    P.nsplit = 1;
+    P.tiles_per_split = 0;
+    P.grid = num_sms;
+    P.slot_rows = P.rows;
+    P.slots = units + P.grid;
   } else {
     // persistent grid; the tile list of all units is cut into equal ranges
     P.rows_per_cta = P.rows <= 128 ? 128 : kTcMaxRows;
@@ -291,8 +311,8 @@ namespace {
 
 size_t attn_region(const spec_attn_args_t& a, size_t base, int sms) {
   size_t end = base;
-  for (int path : {SPEC_ATTN_CUDA_CORES, SPEC_ATTN_TENSOR_CORES}) {
-    if (path == SPEC_ATTN_TENSOR_CORES && a.batch > kTcMaxBatch) continue;
+  for (int path : {SPEC_ATTN_CUDA_CORES, SPEC_ATTN_TENSOR_CORES, SPEC_ATTN_TENSOR_CORES_KEYS_ON_LANES}) {
+    if (path != SPEC_ATTN_CUDA_CORES && a.batch > kTcMaxBatch) continue;
     const AttnPlan P = attn_plan(a, base, sms, path);
     if (P.end > end) end = P.end;
   }
@@ -375,8 +395,9 @@ spec_status_t run(const spec_attn_args_t* attn, const spec_accept_args_t* accept
   auto launch_attention = [&]() -> bool {
     if (!attn) return true;
     const AttnPlan P = attn_plan(*attn, attn_base, sms, attn->path);
-    const cudaError_t e = P.path == SPEC_ATTN_TENSOR_CORES ? launch_attn_tc(*attn, P, w, stream)
-                                                           : launch_attn_simt(*attn, P, w, stream);
+    const cudaError_t e = P.path != SPEC_ATTN_TENSOR_CORES ? launch_attn_simt(*attn, P, w, stream)
+                          : P.keys_on_lanes                 ? launch_attn_kl(*attn, P, w, stream)
+                                                            : launch_attn_tc(*attn, P, w, stream);
     return e == cudaSuccess;
   };
   auto launch_acceptance = [&]() -> bool {

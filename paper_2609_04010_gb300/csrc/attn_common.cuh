@@ -4,6 +4,7 @@
 // base-2 max m and its sum l; the merge rescales by 2^{m_s - max m}).
 #pragma once
 
+#include <cuda.h>  // CUtensorMap
 #include <cuda_bf16.h>
 
 #include <cmath>
@@ -71,7 +72,80 @@ inline AttnParams make_attn_params(const spec_attn_args_t& a, const AttnPlan& P,
   return p;
 }
 
+// Tensor maps of the tensor-core kernels (attn_tc.cu): the K or V cache with one page of
+// one KV head per box, and Q with one tile of tile_rows query rows of one KV group per
+// box (false if group does not divide tile_rows or the encoder is missing).
+bool encode_cache_map(CUtensorMap* map, const void* base, const spec_attn_args_t& a);
+bool encode_q_map(CUtensorMap* map, const spec_attn_args_t& a, int tile_rows);
+
 #ifdef __CUDACC__
+// ---------------------------------------------------------------------------------
+// Work list of the persistent tensor-core kernels (TK keys per tile)
+// ---------------------------------------------------------------------------------
+template <int TK>
+__device__ __forceinline__ int unit_tiles(int kv_len, const AttnParams& p) {
+  const bool ok = kv_len >= p.gamma && kv_len <= p.max_keys;
+  return ok ? (kv_len + TK - 1) / TK : 1;  // a malformed sequence keeps one tile to report it
+}
+
+// The work list is virtual: each unit is ovh overhead tiles followed by its real tiles,
+// and a block owns an equal range of virtual tiles. A segment is the part of one unit
+// inside a block's range. Only a range that ends inside a unit's overhead has a segment
+// with no real tile, and then it is the range's last (a first segment without real
+// tiles means the block has no work).
+struct Seg {
+  int b, g, rt;      // sequence, KV head, row tile
+  int64_t u;         // unit index (b * Hkv + g) * row_tiles + rt
+  int tile0, ntile;  // first real tile within the unit and real tile count of this segment
+  int unit_tiles;    // real tiles of the whole unit
+  int kv_len;
+  bool len_ok;
+  int64_t unit_start;  // virtual index of the unit's first real tile
+  int64_t vnext;       // virtual index just past this segment
+};
+
+template <int TK>
+__device__ __forceinline__ Seg locate(int64_t v, int64_t v1, const AttnParams& p,
+                                      const int* pb, int ovh) {
+  int lo = 0, hi = p.batch;  // largest b with pb[b] <= v
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (pb[mid] <= v) lo = mid; else hi = mid;
+  }
+  Seg s;
+  s.b = lo;
+  s.kv_len = p.kv_len[lo];
+  s.len_ok = s.kv_len >= p.gamma && s.kv_len <= p.max_keys;
+  s.unit_tiles = unit_tiles<TK>(s.kv_len, p);
+  const int vlen = s.unit_tiles + ovh;
+  const int64_t rem = v - pb[lo];
+  const int ub = static_cast<int>(rem / vlen);
+  const int64_t vstart = v - rem % vlen;  // the unit's first (overhead) virtual tile
+  s.g = ub / p.row_tiles;
+  s.rt = ub % p.row_tiles;
+  s.u = static_cast<int64_t>(lo) * p.hkv * p.row_tiles + ub;
+  s.unit_start = vstart + ovh;
+  const int64_t vend = vstart + vlen;
+  s.vnext = vend < v1 ? vend : v1;
+  const int64_t lo_real = v > s.unit_start ? v : s.unit_start;
+  s.ntile = s.vnext > lo_real ? static_cast<int>(s.vnext - lo_real) : 0;
+  s.tile0 = s.ntile > 0 ? static_cast<int>(lo_real - s.unit_start) : 0;
+  return s;
+}
+
+// Whether real tiles follow segment s in the range ending at v1. A segment ends at its
+// unit's end or at v1, so the next one starts a unit, whose real tiles begin ovh virtual
+// tiles later; no load is needed.
+__device__ __forceinline__ bool has_more(const Seg& s, int64_t v1, int ovh) {
+  return v1 - s.vnext > ovh;
+}
+
+// Block that owns virtual tile t when `total` virtual tiles are cut into `ctas` ranges
+// [c * total / ctas, (c + 1) * total / ctas).
+__device__ __forceinline__ int owner_of(int64_t t, int64_t total, int ctas) {
+  return static_cast<int>(((t + 1) * ctas - 1) / total);
+}
+
 // 8 consecutive output dims of unit row `row` (row = j * group + head-in-group).
 template <int D>
 __device__ __forceinline__ void write_out_row(const AttnParams& p, int b, int g, int row, int d0,

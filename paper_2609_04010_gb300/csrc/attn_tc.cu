@@ -111,71 +111,6 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
 }
 
 // ---------------------------------------------------------------------------------
-// Work list
-// ---------------------------------------------------------------------------------
-__device__ __forceinline__ int unit_tiles(int kv_len, const AttnParams& p) {
-  const bool ok = kv_len >= p.gamma && kv_len <= p.max_keys;
-  return ok ? (kv_len + TK - 1) / TK : 1;  // a malformed sequence keeps one tile to report it
-}
-
-// The work list is virtual: each unit is ovh overhead tiles followed by its real tiles,
-// and a block owns an equal range of virtual tiles. A segment is the part of one unit
-// inside a block's range. Only a range that ends inside a unit's overhead has a segment
-// with no real tile, and then it is the range's last (a first segment without real
-// tiles means the block has no work).
-struct Seg {
-  int b, g, rt;      // sequence, KV head, row tile
-  int64_t u;         // unit index (b * Hkv + g) * row_tiles + rt
-  int tile0, ntile;  // first real tile within the unit and real tile count of this segment
-  int unit_tiles;    // real tiles of the whole unit
-  int kv_len;
-  bool len_ok;
-  int64_t unit_start;  // virtual index of the unit's first real tile
-  int64_t vnext;       // virtual index just past this segment
-};
-
-__device__ __forceinline__ Seg locate(int64_t v, int64_t v1, const AttnParams& p,
-                                      const int* pb, int ovh) {
-  int lo = 0, hi = p.batch;  // largest b with pb[b] <= v
-  while (hi - lo > 1) {
-    const int mid = (lo + hi) >> 1;
-    if (pb[mid] <= v) lo = mid; else hi = mid;
-  }
-  Seg s;
-  s.b = lo;
-  s.kv_len = p.kv_len[lo];
-  s.len_ok = s.kv_len >= p.gamma && s.kv_len <= p.max_keys;
-  s.unit_tiles = unit_tiles(s.kv_len, p);
-  const int vlen = s.unit_tiles + ovh;
-  const int64_t rem = v - pb[lo];
-  const int ub = static_cast<int>(rem / vlen);
-  const int64_t vstart = v - rem % vlen;  // the unit's first (overhead) virtual tile
-  s.g = ub / p.row_tiles;
-  s.rt = ub % p.row_tiles;
-  s.u = static_cast<int64_t>(lo) * p.hkv * p.row_tiles + ub;
-  s.unit_start = vstart + ovh;
-  const int64_t vend = vstart + vlen;
-  s.vnext = vend < v1 ? vend : v1;
-  const int64_t lo_real = v > s.unit_start ? v : s.unit_start;
-  s.ntile = s.vnext > lo_real ? static_cast<int>(s.vnext - lo_real) : 0;
-  s.tile0 = s.ntile > 0 ? static_cast<int>(lo_real - s.unit_start) : 0;
-  return s;
-}
-
-// Whether real tiles follow segment s in the range ending at v1. A segment ends at its
-// unit's end or at v1, so the next one starts a unit, whose real tiles begin ovh virtual
-// tiles later; no load is needed.
-__device__ __forceinline__ bool has_more(const Seg& s, int64_t v1, int ovh) {
-  return v1 - s.vnext > ovh;
-}
-
-// Block that owns virtual tile t when `total` virtual tiles are cut into `ctas` ranges
-// [c * total / ctas, (c + 1) * total / ctas).
-__device__ __forceinline__ int owner_of(int64_t t, int64_t total, int ctas) {
-  return static_cast<int>(((t + 1) * ctas - 1) / total);
-}
-
-// ---------------------------------------------------------------------------------
 // The kernel
 // ---------------------------------------------------------------------------------
 // TREE: tree attention (a per-row mask over the block keys) instead of the causal block.
@@ -266,7 +201,7 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
     int carry = 0;
     for (int b0 = 0; b0 < p.batch; b0 += 32) {
       const int b = b0 + lane;
-      int v = b < p.batch ? (unit_tiles(p.kv_len[b], p) + p.unit_overhead) * per_b : 0;
+      int v = b < p.batch ? (unit_tiles<TK>(p.kv_len[b], p) + p.unit_overhead) * per_b : 0;
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
         const int y = __shfl_up_sync(0xffffffffu, v, o);
@@ -320,7 +255,7 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
     };
     const uint32_t box_bytes = static_cast<uint32_t>(p.page_size) * D * 2;  // one page of one head
     uint32_t seg_no = 0;
-    for (Seg s = locate(t0, t1, p, pb, OVH); s.ntile > 0 && ok; ++seg_no) {
+    for (Seg s = locate<TK>(t0, t1, p, pb, OVH); s.ntile > 0 && ok; ++seg_no) {
       const bool bad = !s.len_ok;  // nothing to read
       bool flag = bad;             // ... or a page id out of range (read as page 0)
       for (int k = 0; k < s.ntile && ok; ++k, ++it) {
@@ -360,7 +295,7 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
         mbar_arrive(flag_bar(seg_no & 7));
       }
       if (!has_more(s, t1, OVH)) break;
-      s = locate(s.vnext, t1, p, pb, OVH);
+      s = locate<TK>(s.vnext, t1, p, pb, OVH);
     }
     if (!ok) {  // drain this block's copies still in flight (bounded)
       for (uint32_t x = it > static_cast<uint32_t>(C::STAGES) ? it - C::STAGES : 0; x < it; ++x) {
@@ -399,10 +334,10 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
       __syncwarp();
     };
     if (qk_role && p.q_tma) {
-      const Seg s0 = locate(t0, t1, p, pb, OVH);
+      const Seg s0 = locate<TK>(t0, t1, p, pb, OVH);
       if (s0.ntile > 0) issue_q(s0);
     }
-    for (Seg s = locate(t0, t1, p, pb, OVH); s.ntile > 0 && ok;) {
+    for (Seg s = locate<TK>(t0, t1, p, pb, OVH); s.ntile > 0 && ok;) {
       if (qk_role) {
         ok = mbar_wait(p.q_tma ? q_full : seg_ready, seg_no & 1, abort_flag, p.status);
         if (!ok) break;
@@ -453,7 +388,7 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
             for (int mt = 0; mt < MT && ok; ++mt)
               ok = mbar_wait(s_full(mt, x & 1), (x >> 1) & 1, abort_flag, p.status);
             if (!ok) break;
-            issue_q(locate(s.vnext, t1, p, pb, OVH));
+            issue_q(locate<TK>(s.vnext, t1, p, pb, OVH));
           }
         } else {
           // O += P V for tile x (its P implies its S, hence its landed stage)
@@ -488,7 +423,7 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
       it += s.ntile;
       ++seg_no;
       if (!has_more(s, t1, OVH)) break;
-      s = locate(s.vnext, t1, p, pb, OVH);
+      s = locate<TK>(s.vnext, t1, p, pb, OVH);
     }
     if (!ok && __any_sync(0xffffffffu, issued)) {  // drain this warp's MMAs (bounded)
       const uint32_t db = drain_bar(qk_role ? 0 : 1);
@@ -546,7 +481,7 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
     };
     uint4 qr[kChunks];
     uint32_t seg_no = 0;
-    Seg s = locate(t0, t1, p, pb, OVH);
+    Seg s = locate<TK>(t0, t1, p, pb, OVH);
     if (s.ntile > 0 && !p.q_tma) {
       load_q(s, qr);
       store_q(qr);
@@ -661,7 +596,7 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
       Seg sn;
       sn.ntile = 0;
       if (has_next) {
-        sn = locate(s.vnext, t1, p, pb, OVH);
+        sn = locate<TK>(s.vnext, t1, p, pb, OVH);
         if (!p.q_tma) {
           load_q(sn, qr);
           store_q(qr);
@@ -787,48 +722,6 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
 // ---------------------------------------------------------------------------------
 // Host side
 // ---------------------------------------------------------------------------------
-// K or V cache viewed as a 5-D tensor of bf16 whose box is one page of one KV head:
-// (64 columns; 8 rows at stride D*2 bytes; D/64 column halves at stride 128 bytes;
-// page/8 groups of 8 rows at stride 8*D*2 bytes; page * Hkv + head at stride page*D*2).
-// The box lands in shared memory as [row group][column half][8 rows][128 B], so the
-// 8-row groups of a 64-key tile sit at a uniform stride whatever the page size.
-bool encode_cache_map(CUtensorMap* map, const void* base, const spec_attn_args_t& a) {
-  EncodeTiledFn enc = encoder();
-  if (!enc) return false;
-  const cuuint64_t D = static_cast<cuuint64_t>(a.head_dim);
-  const cuuint64_t dims[5] = {64, 8, D / 64, static_cast<cuuint64_t>(a.page_size / 8),
-                              static_cast<cuuint64_t>(a.num_pages) * a.num_kv_heads};
-  const cuuint64_t strides[4] = {D * 2, 128, 8 * D * 2, static_cast<cuuint64_t>(a.page_size) * D * 2};
-  const cuuint32_t box[5] = {64, 8, static_cast<cuuint32_t>(D / 64),
-                             static_cast<cuuint32_t>(a.page_size / 8), 1};
-  const cuuint32_t estr[5] = {1, 1, 1, 1, 1};
-  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void*>(base), dims, strides, box,
-             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
-// Q [batch][gamma][Hq][D] viewed as a 4-D tensor (64 columns; D/64 column halves at
-// stride 128 bytes; Hq heads at stride D*2; batch*gamma block positions at stride
-// Hq*D*2) whose box is one M tile of one column half: the group's heads at 128/group
-// consecutive block positions, landing as 128 rows of 128 bytes (row = j * group + head)
-// with the 128-byte swizzle. Needs group to divide 128; positions past the end read
-// zeros and only fill padding rows.
-bool encode_q_map(CUtensorMap* map, const spec_attn_args_t& a) {
-  const int group = a.num_q_heads / a.num_kv_heads;
-  if (group < 1 || 128 % group != 0) return false;
-  EncodeTiledFn enc = encoder();
-  if (!enc) return false;
-  const cuuint64_t D = static_cast<cuuint64_t>(a.head_dim);
-  const cuuint64_t dims[4] = {64, D / 64, static_cast<cuuint64_t>(a.num_q_heads),
-                              static_cast<cuuint64_t>(a.batch) * a.gamma};
-  const cuuint64_t strides[3] = {128, D * 2, static_cast<cuuint64_t>(a.num_q_heads) * D * 2};
-  const cuuint32_t box[4] = {64, 1, static_cast<cuuint32_t>(group), static_cast<cuuint32_t>(128 / group)};
-  const cuuint32_t estr[4] = {1, 1, 1, 1};
-  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(a.q), dims, strides, box,
-             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
 template <int D, int MT>
 cudaError_t launch_typed(const spec_attn_args_t& a, const AttnPlan& P, char* ws,
                          cudaStream_t stream) {
@@ -837,7 +730,7 @@ cudaError_t launch_typed(const spec_attn_args_t& a, const AttnPlan& P, char* ws,
   if (!encode_cache_map(&mk, a.k_cache, a) || !encode_cache_map(&mv, a.v_cache, a))
     return cudaErrorInvalidValue;
   AttnParams p = make_attn_params(a, P, ws);
-  p.q_tma = encode_q_map(&mq, a) ? 1 : 0;
+  p.q_tma = encode_q_map(&mq, a, 128) ? 1 : 0;
   // Charge unit starts only when blocks hold several of them; when every unit is spread
   // over several blocks, a block holds at most one start and the charge would mostly
   // move real tiles away from blocks that pay no boundary.
@@ -854,6 +747,49 @@ cudaError_t launch_typed(const spec_attn_args_t& a, const AttnPlan& P, char* ws,
 }
 
 }  // namespace
+
+// K or V cache viewed as a 5-D tensor of bf16 whose box is one page of one KV head:
+// (64 columns; 8 rows at stride D*2 bytes; D/64 column halves at stride 128 bytes;
+// page/8 groups of 8 rows at stride 8*D*2 bytes; page * Hkv + head at stride page*D*2).
+// The box lands in shared memory as [row group][column half][8 rows][128 B], so the
+// 8-row groups of a 64-key tile sit at a uniform stride whatever the page size.
+bool encode_cache_map(CUtensorMap* map, const void* base, const spec_attn_args_t& a) {
+  tcx::EncodeTiledFn enc = tcx::encoder();
+  if (!enc) return false;
+  const cuuint64_t D = static_cast<cuuint64_t>(a.head_dim);
+  const cuuint64_t dims[5] = {64, 8, D / 64, static_cast<cuuint64_t>(a.page_size / 8),
+                              static_cast<cuuint64_t>(a.num_pages) * a.num_kv_heads};
+  const cuuint64_t strides[4] = {D * 2, 128, 8 * D * 2, static_cast<cuuint64_t>(a.page_size) * D * 2};
+  const cuuint32_t box[5] = {64, 8, static_cast<cuuint32_t>(D / 64),
+                             static_cast<cuuint32_t>(a.page_size / 8), 1};
+  const cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void*>(base), dims, strides, box,
+             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Q [batch][gamma][Hq][D] viewed as a 4-D tensor (64 columns; D/64 column halves at
+// stride 128 bytes; Hq heads at stride D*2; batch*gamma block positions at stride
+// Hq*D*2) whose box is one tile of one column half: the group's heads at
+// tile_rows/group consecutive block positions, landing as tile_rows rows of 128 bytes
+// (row = j * group + head) with the 128-byte swizzle. Needs group to divide tile_rows;
+// positions past the end read zeros and only fill padding rows.
+bool encode_q_map(CUtensorMap* map, const spec_attn_args_t& a, int tile_rows) {
+  const int group = a.num_q_heads / a.num_kv_heads;
+  if (group < 1 || tile_rows % group != 0) return false;
+  tcx::EncodeTiledFn enc = tcx::encoder();
+  if (!enc) return false;
+  const cuuint64_t D = static_cast<cuuint64_t>(a.head_dim);
+  const cuuint64_t dims[4] = {64, D / 64, static_cast<cuuint64_t>(a.num_q_heads),
+                              static_cast<cuuint64_t>(a.batch) * a.gamma};
+  const cuuint64_t strides[3] = {128, D * 2, static_cast<cuuint64_t>(a.num_q_heads) * D * 2};
+  const cuuint32_t box[4] = {64, 1, static_cast<cuuint32_t>(group),
+                             static_cast<cuuint32_t>(tile_rows / group)};
+  const cuuint32_t estr[4] = {1, 1, 1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(a.q), dims, strides, box,
+             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
 
 size_t tc_smem_bytes(int head_dim, int rows_per_cta, int batch) {
   const bool two = rows_per_cta > 128;

@@ -136,6 +136,7 @@ cudaError_t launch_tree_build(const spec_tree_build_args_t& t, const TreeBuildLa
 // --- attention ---
 struct AttnPlan {
   int path;          // SPEC_ATTN_CUDA_CORES or SPEC_ATTN_TENSOR_CORES
+  int keys_on_lanes; // tensor cores: the keys-on-lanes kernel (attn_kl.cu), else row tiles
   int rows;          // (Hq/Hkv) * gamma
   int rows_per_cta;  // rows one block handles (a row tile)
   int row_tiles;     // ceil(rows / rows_per_cta)
@@ -169,6 +170,8 @@ cudaError_t launch_attn_simt(const spec_attn_args_t& a, const AttnPlan& P, char*
                              cudaStream_t stream);
 cudaError_t launch_attn_tc(const spec_attn_args_t& a, const AttnPlan& P, char* ws,
                            cudaStream_t stream);
+cudaError_t launch_attn_kl(const spec_attn_args_t& a, const AttnPlan& P, char* ws,
+                           cudaStream_t stream);
 cudaError_t launch_philox(uint64_t seed, uint64_t offset, int64_t n, float* out, cudaStream_t s);
 cudaError_t launch_noise(uint64_t seed, uint64_t offset, int64_t n, int32_t vocab, int32_t* out,
                          cudaStream_t s);
@@ -179,6 +182,12 @@ constexpr int kSimtKeyTile = 64;
 constexpr int kSimtThreads = 128;
 constexpr int kTcKeyTile = 64;
 constexpr int kTcMaxRows = 256;  // two M = 128 tiles per block
+// The keys-on-lanes tensor-core kernel (attn_kl.cu): 128 keys per tile, at most 64 query
+// rows per KV head, head_dim 128, batch prefix sums in shared memory.
+constexpr int kKlKeyTile = 128;
+constexpr int kKlMaxRows = 64;
+constexpr int kKlMaxBatch = 2048;
+size_t kl_smem_bytes(int rows, int batch);
 
 int tc_min_rows();
 

@@ -63,7 +63,7 @@ def _attn(**kw):
 
 @pytest.mark.parametrize("kw,code", [
     (dict(head_dim=96), 2), (dict(page_size=8), 2), (dict(gamma=65), 2),
-    (dict(num_q_heads=30), 1), (dict(batch=0), 1), (dict(path=7), 1),
+    (dict(num_q_heads=30), 1), (dict(batch=0), 1), (dict(path=7), 1), (dict(path=4), 1),
     (dict(softmax_scale=-1.0), 1),
 ])
 def test_attention_shape_limits(lib, kw, code):

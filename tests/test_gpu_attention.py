@@ -13,7 +13,9 @@ from helpers import attn_tensors, compare_attention, gpu_attention, sample_rows
 
 pytestmark = pytest.mark.gpu
 
-PATHS = [binding.ATTN_CUDA_CORES, binding.ATTN_TENSOR_CORES]
+# the CUDA-core kernel, the row-tile tensor-core kernel (AUTO's choice) and the
+# keys-on-lanes tensor-core kernel (where it applies; elsewhere the row-tile one)
+PATHS = [binding.ATTN_CUDA_CORES, binding.ATTN_TENSOR_CORES, binding.ATTN_TENSOR_CORES_KEYS_ON_LANES]
 
 SMALL = [
     dict(batch=2, gamma=4, num_q_heads=8, num_kv_heads=8, head_dim=64, page_size=16, ctx=(0, 300)),
@@ -34,6 +36,16 @@ SMALL = [
     # a group that does not divide 128, with two M tiles
     dict(batch=2, gamma=64, num_q_heads=6, num_kv_heads=2, head_dim=128, page_size=32,
          ctx=(5, 200)),
+    # keys-on-lanes shapes: group 1 with 64-token pages, 48 rows (not a multiple of 32),
+    # group 2 with 64 rows, and contexts shorter than one 128-key tile
+    dict(batch=3, gamma=4, num_q_heads=8, num_kv_heads=8, head_dim=128, page_size=64,
+         ctx=(0, 700)),
+    dict(batch=2, gamma=12, num_q_heads=16, num_kv_heads=4, head_dim=128, page_size=16,
+         ctx=(127, 385)),
+    dict(batch=5, gamma=32, num_q_heads=16, num_kv_heads=8, head_dim=128, page_size=32,
+         ctx=(1, 260)),
+    dict(batch=4, gamma=16, num_q_heads=32, num_kv_heads=8, head_dim=128, page_size=16,
+         ctx=(0, 100)),
 ]
 
 
@@ -93,9 +105,10 @@ def test_page_order_invariance_bitwise(path):
     np.testing.assert_array_equal(lse, base_lse)
 
 
+@pytest.mark.parametrize("head_dim", [64, 128])
 @pytest.mark.parametrize("path", PATHS)
-def test_bad_pages_and_lengths(oracle_mod, path):
-    inp = W.make_attn_inputs(4, 4, 8, 2, 64, 16, (20, 90), seed=12)
+def test_bad_pages_and_lengths(oracle_mod, path, head_dim):
+    inp = W.make_attn_inputs(4, 4, 8, 2, head_dim, 16, (20, 300), seed=12)
     inp.page_table[1, 2] = inp.num_pages + 5
     inp.kv_len[2] = 2  # shorter than the block
     t = attn_tensors(inp)

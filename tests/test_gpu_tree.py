@@ -208,15 +208,19 @@ def test_tree_attention(oracle_mod, path, N, hq, hkv, D, P, ctx, batch):
     compare_attention(out.float().cpu().numpy(), lse.cpu().numpy(), o_out, o_lse, rows)
 
 
-@pytest.mark.parametrize("path", [binding.ATTN_TENSOR_CORES, binding.ATTN_CUDA_CORES])
-def test_causal_mask_reproduces_block_attention(path):
+# tree attention runs on the row-tile tensor-core kernel (or the CUDA-core one); its
+# block-causal mode is the reference for a causal mask
+@pytest.mark.parametrize("path,causal_path", [
+    (binding.ATTN_TENSOR_CORES, binding.ATTN_TENSOR_CORES),
+    (binding.ATTN_CUDA_CORES, binding.ATTN_CUDA_CORES)])
+def test_causal_mask_reproduces_block_attention(path, causal_path):
     inp = attn_tree_inputs(3, 2, 16, 32, 8, 128, 16, 1000)
     N = 16
     causal = np.array([[(1 << (j + 1)) - 1 for j in range(N)]] * 2, np.uint64)
     args = (bf16_dev(inp.q), bf16_dev(inp.k_cache), bf16_dev(inp.v_cache), dev(inp.page_table),
             dev(inp.kv_len))
     a, la = binding.verify_attention(*args, path=path, tree_mask=dev(causal.view(np.int64)))
-    c, lc = binding.verify_attention(*args, path=path)
+    c, lc = binding.verify_attention(*args, path=causal_path)
     torch.cuda.synchronize()
     assert torch.equal(a, c) and torch.equal(la, lc)
 
