@@ -529,6 +529,94 @@ def accept_tree_greedy(target_logits, tokens, parents):
     return dict(path=path, num_accepted=na, out_tokens=out, num_emitted=ne)
 
 
+def accept_tree_sampled(target_logits, tokens, parents, temperature, uniforms):
+    """Sampled (T > 0) verification of a candidate tree whose nodes are deterministic
+    candidates (Sec. 4.2: candidates verified at once as a prefix tree, with the
+    standard rejection correction; Sec. 3.3, "Tree Sampler"), lossless for the target.
+
+    At the current node (the root first) with target distribution p = softmax(row / T)
+    of its target row, its children are tried in node order. A child is a point-mass
+    proposal (q = one-hot at its token), so the rule min(1, p'/q) accepts it with
+    probability p'(token), where p' is what is left of p at this node: p with the
+    tokens of the children rejected so far removed, renormalised (the residual
+    Norm([p' - q]_+) of a rejected point mass). Child c is accepted iff
+    uniforms[c] <= p'(tokens[c]); the walk then moves to c. If no child is accepted (or
+    the node has none), the final token is the inverse-CDF draw from p' with
+    uniforms[0]. A sequence with T <= 0 takes the greedy walk (accept_tree_greedy).
+
+    target_logits [batch][N][V] (float32, or uint16 bf16 bits), tokens / parents int32
+    [batch][N] (parents[0] = -1, parents[c] < c), temperature float32 [batch], uniforms
+    float32 [batch][N] in (0, 1]. Returns a dict: path, num_accepted, out_tokens,
+    num_emitted (as accept_tree_greedy), accept_margin float64 [batch][N] (|u - p'| of
+    each test taken at node c's entry, +inf elsewhere), sample_margin float64 [batch]
+    (the final draw's inverse-CDF margin over the remaining mass), status int32 [batch]
+    (0; 1: a node row with NaN, or for a tempered sequence +inf or no finite logit; 2: a
+    token outside [0, V) or parents that are not a tree; such a sequence gets -1
+    outputs and num_emitted 0)."""
+    tl = _rows_f64(target_logits)
+    B, N, V = tl.shape
+    tok = np.asarray(tokens, dtype=np.int64)
+    par = np.asarray(parents, dtype=np.int64)
+    T = np.asarray(temperature, dtype=np.float32)
+    u = np.asarray(uniforms, dtype=np.float32).astype(np.float64)
+    path = np.full((B, N), -1, np.int32)
+    out = np.full((B, N + 1), -1, np.int32)
+    na = np.full(B, -1, np.int32)
+    ne = np.zeros(B, np.int32)
+    am = np.full((B, N), np.inf)
+    sm = np.full(B, np.inf)
+    st = np.zeros(B, np.int32)
+    for b in range(B):
+        if (np.any(tok[b] < 0) or np.any(tok[b] >= V) or par[b, 0] != -1 or
+                any(not (0 <= par[b, c] < c) for c in range(1, N))):
+            st[b] = 2
+            continue
+        tempered = float(T[b]) > 0.0
+        # every node row must be usable: no NaN; tempered rows also no +inf and a finite max
+        rows_bad = np.isnan(tl[b]).any() or (tempered and (
+            np.isposinf(tl[b]).any() or not np.isfinite(tl[b].max(axis=1)).all()))
+        if rows_bad:
+            st[b] = 1
+            continue
+        if not tempered:
+            g = accept_tree_greedy(tl[b:b + 1], tok[b:b + 1], par[b:b + 1])
+            path[b], out[b], na[b], ne[b] = g["path"][0], g["out_tokens"][0], \
+                g["num_accepted"][0], g["num_emitted"][0]
+            continue
+        cur, walk, final = 0, [0], None
+        while True:
+            prob = softmax(tl[b, cur], float(T[b]))
+            w = prob.copy()
+            nxt = None
+            for c in range(1, N):
+                if par[b, c] != cur:
+                    continue
+                S = w.sum()
+                ratio = w[tok[b, c]] / S if S > 0.0 else 1.0
+                am[b, c] = abs(u[b, c] - min(1.0, ratio))
+                if u[b, c] <= ratio:
+                    nxt = c
+                    break
+                w[tok[b, c]] = 0.0  # the rejected candidate leaves the distribution
+            if nxt is not None:
+                walk.append(nxt)
+                cur = nxt
+                continue
+            S = w.sum()
+            if not S > 0.0:  # only through rounding: draw from p itself
+                w, S = prob, prob.sum()
+            final, margin = inverse_cdf(w, u[b, 0])
+            sm[b] = margin / S
+            break
+        path[b, :len(walk)] = walk
+        toks = [int(tok[b, x]) for x in walk] + [int(final)]
+        out[b, :len(toks)] = toks
+        na[b] = len(walk) - 1
+        ne[b] = len(walk) + 1
+    return dict(path=path, num_accepted=na, out_tokens=out, num_emitted=ne, accept_margin=am,
+                sample_margin=sm, status=st)
+
+
 def compact_tree_kv(k_cache, v_cache, page_table, kv_len, num_nodes: int, path, num_accepted):
     """Keep the accepted path of a verified tree in the paged KV cache: the block's node
     keys sit at positions ctx .. ctx + num_nodes - 1 (kv_len = ctx + num_nodes); the key

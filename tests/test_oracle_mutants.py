@@ -214,6 +214,14 @@ PACKAGE_MUTANTS = {
         "toks = [int(tokens[b, x]) for x in walk] + [int(np.argmax(tl[b, cur]))]",
         "toks = [int(tokens[b, x]) for x in walk] + [int(np.argmax(tl[b, 0]))]")),
         TREE.test_greedy_walk_is_the_deepest_matching_path),
+    # the sampled walk's final draw reuses the last node's test uniform
+    "tree_sampled_draw_reuses_uniform": (dict(py=("final, margin = inverse_cdf(w, u[b, 0])",
+                                                  "final, margin = inverse_cdf(w, u[b, N - 1])")),
+                                         lambda m: TREE.test_sampled_tree_acceptance_is_lossless(m, "tree4")),
+    # every node's children tested against the root's target row
+    "tree_sampled_root_row_only": (dict(py=("prob = softmax(tl[b, cur], float(T[b]))",
+                                            "prob = softmax(tl[b, 0], float(T[b]))")),
+                                   lambda m: TREE.test_sampled_tree_acceptance_is_lossless(m, "tree4")),
     # path rows moved one slot too low (over the root)
     "compact_destination_shifted": (dict(py=("src, dst = ctx + int(path[b, d]), ctx + d",
                                              "src, dst = ctx + int(path[b, d]), ctx + d - 1")),

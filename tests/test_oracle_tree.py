@@ -272,3 +272,168 @@ def test_compaction_moves_the_path(oracle_mod):
         # prefix keys untouched
         for t in range(ctx):
             np.testing.assert_array_equal(k2[table[b, t // P], :, t % P], k[table[b, t // P], :, t % P])
+
+
+# ---------------------------------------------------------------------------------
+# sampled (T > 0) tree acceptance
+# ---------------------------------------------------------------------------------
+from test_oracle_accept import uniform_cells  # noqa: E402
+
+
+def tree_output_law(oracle_mod, p_rows, tokens, parents, denom, lib_mod=None):
+    """Exact law of the emitted tokens (after the root) of one sampled tree verification:
+    every combination of Farey(denom) cells of the N uniforms, weighted by the cells'
+    widths, through the oracle (one sequence per combination). Rows are probability
+    rows whose entries are multiples of 1/denom, given as log-probabilities at T = 1, so
+    every threshold the rule compares a uniform with is such a fraction."""
+    import itertools
+    m = oracle_mod if lib_mod is None else lib_mod
+    N, V = p_rows.shape
+    mids, widths = uniform_cells(denom)
+    combos = np.array(list(itertools.product(range(len(mids)), repeat=N)))
+    U = mids[combos].astype(np.float32)
+    Wt = np.prod(widths[combos], axis=1)
+    with np.errstate(divide="ignore"):
+        logits = np.log(p_rows).astype(np.float32)
+    B = len(U)
+    r = m.accept_tree_sampled(np.broadcast_to(logits, (B, N, V)).copy(),
+                              np.broadcast_to(tokens, (B, N)).copy(),
+                              np.broadcast_to(parents, (B, N)).copy(),
+                              np.ones(B, np.float32), U)
+    assert np.all(r["status"] == 0)
+    law = {}
+    for b in range(B):
+        seq = tuple(int(x) for x in r["out_tokens"][b, 1:r["num_emitted"][b]])
+        law[seq] = law.get(seq, 0.0) + Wt[b]
+    return law
+
+
+def target_tree_law(p_rows, tokens, parents):
+    """The law the target model gives the emitted tokens: from the root, draw x ~ p of the
+    current node; if x is the token of one of its children, move there and draw again,
+    else stop."""
+    N, V = p_rows.shape
+    law = {}
+
+    def walk(node, prefix, prob):
+        for x in range(V):
+            if p_rows[node, x] == 0.0:
+                continue
+            child = next((c for c in range(1, N) if parents[c] == node and tokens[c] == x), None)
+            if child is None:
+                law[prefix + (x,)] = law.get(prefix + (x,), 0.0) + prob * p_rows[node, x]
+            else:
+                walk(child, prefix + (x,), prob * p_rows[node, x])
+    walk(0, (), 1.0)
+    return law
+
+
+def assert_same_law(a, b, tol=1e-12):
+    keys = set(a) | set(b)
+    for k in keys:
+        assert abs(a.get(k, 0.0) - b.get(k, 0.0)) <= tol, (k, a.get(k, 0.0), b.get(k, 0.0))
+
+
+# a root with two children, the first of which has a child (V = 4, rows in quarters)
+TREE4_P = np.array([[1, 2, 1, 0], [2, 1, 1, 0], [0, 1, 1, 2], [1, 1, 1, 1]], np.float64) / 4
+TREE4_TOK = np.array([3, 1, 0, 2], np.int32)    # root token, then the nodes' tokens
+TREE4_PAR = np.array([-1, 0, 0, 1], np.int32)
+# a root with three children covering most of its mass (V = 6, rows in sixths)
+TREE6_P = np.array([[1, 2, 0, 2, 1, 0], [1, 1, 1, 1, 1, 1], [0, 0, 3, 3, 0, 0],
+                    [6, 0, 0, 0, 0, 0]], np.float64) / 6
+TREE6_TOK = np.array([0, 3, 1, 4], np.int32)
+TREE6_PAR = np.array([-1, 0, 0, 0], np.int32)
+
+
+@pytest.mark.parametrize("case", ["tree4", "tree6"])
+def test_sampled_tree_acceptance_is_lossless(oracle_mod, case):
+    p, tok, par, denom = ((TREE4_P, TREE4_TOK, TREE4_PAR, 4) if case == "tree4"
+                          else (TREE6_P, TREE6_TOK, TREE6_PAR, 6))
+    got = tree_output_law(oracle_mod, p, tok, par, denom)
+    assert abs(sum(got.values()) - 1.0) < 1e-12
+    assert_same_law(got, target_tree_law(p, tok, par))
+    # every branch is reached: a child accepted at depth 2, a later sibling accepted, and
+    # a final draw after rejections
+    assert any(len(k) == 3 for k in got) or case == "tree6"
+    assert any(len(k) == 2 for k in got) and any(len(k) == 1 for k in got)
+
+
+def test_sampled_tree_without_renormalisation_is_caught(oracle_mod):
+    # power check: the rule run on p instead of the renormalised residual p' (the rejected
+    # candidates kept) must fail the same exact comparison
+    import types
+    src = open(oracle_mod.__file__).read()
+    site = "                w[tok[b, c]] = 0.0  # the rejected candidate leaves the distribution\n"
+    assert src.count(site) == 1
+    mod = types.ModuleType("oracle_no_renorm")
+    mod.__file__ = oracle_mod.__file__
+    exec(compile(src.replace(site, ""), oracle_mod.__file__, "exec"), mod.__dict__)
+    got = tree_output_law(oracle_mod, TREE6_P, TREE6_TOK, TREE6_PAR, 6, lib_mod=mod)
+    want = target_tree_law(TREE6_P, TREE6_TOK, TREE6_PAR)
+    assert max(abs(got.get(k, 0.0) - want.get(k, 0.0)) for k in set(got) | set(want)) > 1e-3
+
+
+def test_sampled_chain_equals_linear_rule_with_point_mass_drafts(oracle_mod):
+    # a chain tree (one child per node) proposes its tokens with certainty: the linear rule
+    # with one-hot drafter rows (q = point mass at the draft) takes the same decisions;
+    # the tree tests node c with uniforms[c] and draws with uniforms[0], the linear rule
+    # tests draft i with uniforms[i - 1] and draws with uniforms[gamma - 1]
+    rng = np.random.default_rng(5)
+    B, N, V = 300, 5, 12
+    tl = (rng.standard_normal((B, N, V)) * 1.5).astype(np.float32)
+    T = rng.choice([1.0, 0.7, 1.6], size=B).astype(np.float32)
+    tok = np.zeros((B, N), np.int32)
+    for b in range(B):
+        for c in range(N):
+            tok[b, c] = rng.integers(V) if rng.random() < 0.5 else int(np.argmax(tl[b, max(c - 1, 0)]))
+    par = np.broadcast_to(np.arange(-1, N - 1, dtype=np.int32), (B, N)).copy()
+    u_tree = rng.random((B, N)).astype(np.float32)
+    t = oracle_mod.accept_tree_sampled(tl, tok, par, T, u_tree)
+    dl = np.full((B, N, V), -np.inf, np.float32)
+    for b in range(B):
+        for c in range(N):
+            dl[b, c, tok[b, c]] = 0.0
+    u_lin = np.concatenate([u_tree[:, 1:], u_tree[:, :1]], axis=1)
+    lin = oracle_mod.accept_block(tl[:, :N], dl, tok, T, u_lin)
+    np.testing.assert_array_equal(t["num_accepted"], lin["num_accepted"])
+    np.testing.assert_array_equal(t["out_tokens"], lin["out_tokens"])
+    np.testing.assert_array_equal(t["num_emitted"], lin["num_emitted"])
+
+
+def test_sampled_tree_greedy_and_low_temperature_limits(oracle_mod):
+    rng = np.random.default_rng(6)
+    B, N, V = 40, 9, 30
+    tl = (rng.standard_normal((B, N, V)) * 3).astype(np.float32)
+    par = np.array([-1, 0, 0, 1, 1, 2, 3, 3, 5], np.int32)
+    tok = np.zeros((B, N), np.int32)
+    for b in range(B):
+        for c in range(1, N):  # half the children match their parent's argmax
+            p = par[c]
+            tok[b, c] = int(np.argmax(tl[b, p])) if rng.random() < 0.6 else rng.integers(V)
+    parents = np.broadcast_to(par, (B, N)).copy()
+    g = oracle_mod.accept_tree_greedy(tl, tok, parents)
+    u = rng.uniform(0.05, 0.95, (B, N)).astype(np.float32)
+    for T in (0.0, -1.0, 1e-3):
+        s = oracle_mod.accept_tree_sampled(tl, tok, parents, np.full(B, T, np.float32), u)
+        assert np.all(s["status"] == 0)
+        for k in ("path", "num_accepted", "out_tokens", "num_emitted"):
+            np.testing.assert_array_equal(s[k], g[k], err_msg=f"T={T} {k}")
+
+
+def test_sampled_tree_flags_bad_inputs(oracle_mod):
+    rng = np.random.default_rng(7)
+    B, N, V = 5, 4, 16
+    tl = rng.standard_normal((B, N, V)).astype(np.float32)
+    tok = rng.integers(0, V, (B, N)).astype(np.int32)
+    par = np.broadcast_to(np.array([-1, 0, 0, 1], np.int32), (B, N)).copy()
+    T = np.array([1.0, 1.0, 1.0, 0.0, 1.0], np.float32)
+    tok[1, 2] = V                 # token outside the vocabulary
+    par[2, 3] = 3                 # not a tree
+    tl[3, 2, 5] = np.nan          # NaN row, greedy sequence
+    tl[4, 1, :] = -np.inf         # no finite logit, tempered sequence
+    r = oracle_mod.accept_tree_sampled(tl, tok, par, T, rng.random((B, N)).astype(np.float32))
+    assert list(r["status"]) == [0, 2, 2, 1, 1]
+    for b in (1, 2, 3, 4):
+        assert r["num_accepted"][b] == -1 and r["num_emitted"][b] == 0
+        assert np.all(r["out_tokens"][b] == -1) and np.all(r["path"][b] == -1)
+    assert r["num_emitted"][0] == r["num_accepted"][0] + 2
