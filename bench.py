@@ -715,11 +715,18 @@ def time_tree(wl, ai, ci, binding, dev, graph_of, timed_loop, n, stream):
     ws_t = binding.new_workspace(binding.tree_workspace_size(targs), dev)
     accept_call = lambda: binding.accept_tree_args(targs, ws_t)
     verify_call = lambda: (attn_call(), accept_call())
+    # sampled acceptance at T = 1 (the paper's temperature-1 tree setting) on the same tree
+    t_one = torch.ones(B, dtype=torch.float32, device=dev)
+    u_tree = binding.philox_uniforms(W.uniform_seed(23), B * N).view(B, N)
+    sargs = binding.tree_accept_args(tl, tok, par, path, na, ot, ne, t_one, u_tree)
+    ws_s = binding.new_workspace(binding.tree_workspace_size(sargs), dev)
+    sampled_call = lambda: binding.accept_tree_args(sargs, ws_s)
     gs = {name: graph_of(fn) for name, fn in (("build", build_call), ("attention", attn_call),
-                                              ("accept", accept_call), ("verify", verify_call))}
+                                              ("accept", accept_call), ("verify", verify_call),
+                                              ("accept_sampled", sampled_call))}
     ms = {name: statistics.mean(timed_loop(g.replay, n)) for name, g in gs.items()}
     torch.cuda.synchronize()
-    for ws in (ws_b, ws_a, ws_t):
+    for ws in (ws_b, ws_a, ws_t, ws_s):
         code, flags = binding.read_device_status(ws)
         if code != 0:
             raise RuntimeError(f"tree timing: device status {code} flags {flags}")
@@ -751,6 +758,8 @@ def time_tree(wl, ai, ci, binding, dev, graph_of, timed_loop, n, stream):
             "build_tree_frac_of_measured": round(build_bytes / (ms["build"] / 1000.0) / 1e9 / peak, 4),
             "tree_attention_ms": ms["attention"], "tree_attention_gbs": gbs(kv_bytes, ms["attention"]),
             "accept_tree_ms": ms["accept"], "accept_tree_gbs": gbs(accept_bytes, ms["accept"]),
+            "accept_tree_sampled_ms": ms["accept_sampled"],
+            "accept_tree_sampled_gbs": gbs(accept_bytes, ms["accept_sampled"]),
             "verify_ms": ms["verify"], "commit_tree_kv_ms": statistics.median(commit_times),
             "algorithmic_bytes": {"build_tree": build_bytes, "tree_attention": kv_bytes,
                                   "accept_tree": accept_bytes},

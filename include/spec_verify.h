@@ -351,8 +351,9 @@ typedef struct {
 spec_status_t spec_commit_kv(const spec_commit_args_t* commit, spec_stream_t stream);
 
 /*
- * Tree verification (Sec. 4.2: several candidates verified at once as a prefix tree;
- * Sec. 3.3, "Tree Sampler"), greedy (T = 0).
+ * Tree verification (Sec. 4.2: several candidates verified at once as a prefix tree,
+ * with the standard speculative-decoding rejection correction; Sec. 3.3, "Tree
+ * Sampler"), greedy (T = 0) or sampled (T > 0).
  *
  * A candidate tree of num_nodes <= 64 nodes per sequence: node 0 is the root (the free
  * token x^{L+1}); parents[b][c] < c is node c's parent (-1 for the root); tokens[b][c]
@@ -360,15 +361,24 @@ spec_status_t spec_commit_kv(const spec_commit_args_t* commit, spec_stream_t str
  * with tree_mask = each node's ancestor bits); target row c (target_logits
  * [batch][num_nodes][vocab]) is the verifier's distribution of the token after node c.
  *
- * spec_accept_tree: from the root, move to the child (lowest node index first) whose
- * token is the lowest-index argmax of the current node's target row; stop where there
- * is none. path[b] = the visited nodes (-1 padded), out_tokens[b] = their tokens then
- * that argmax (-1 padded, num_nodes + 1 entries), num_accepted = path length - 1,
+ * spec_accept_tree, greedy sequences (temperature NULL, or temperature[b] <= 0): from
+ * the root, move to the child (lowest node index first) whose token is the lowest-index
+ * argmax of the current node's target row; stop where there is none; the final token is
+ * that argmax.
+ * Sampled sequences (temperature[b] > 0): at the current node, with p = softmax(target
+ * row / T), its children are tried in node order as point-mass proposals: child c is
+ * accepted iff uniforms[b][c] <= p'(tokens[b][c]), where p' is p with the tokens of the
+ * children rejected so far at this node removed and renormalised (min(1, p'/q) with q
+ * the point mass; its residual Norm([p' - q]_+) removes the token). On acceptance the
+ * walk moves to c. If none is accepted, or the node has no child, the final token is
+ * drawn from p' by inverse CDF in ascending token order with uniforms[b][0]. The
+ * emitted tokens then follow the target's own distribution exactly (lossless).
+ * Outputs: path[b] = the visited nodes (-1 padded), out_tokens[b] = their tokens then
+ * the final token (-1 padded, num_nodes + 1 entries), num_accepted = path length - 1,
  * num_emitted = path length + 1. A sequence with a token outside [0, vocab), parents
- * that are not a tree (SPEC_FLAG_BAD_TREE), or a NaN in a target row gets
- * num_accepted = -1, num_emitted = 0 and -1 outputs. Sampled (T > 0) tree verification
- * is not provided: the paper's tree takes the top K tokens per position, and it states
- * no lossless rule for such candidate sets.
+ * that are not a tree (SPEC_FLAG_BAD_TREE), a NaN in a target row, or (sampled) a
+ * target row with +inf or no finite logit (SPEC_FLAG_BAD_LOGITS) gets
+ * num_accepted = -1, num_emitted = 0 and -1 outputs.
  */
 typedef struct {
   int32_t batch, num_nodes, vocab, logits_dtype;
@@ -379,6 +389,9 @@ typedef struct {
   int32_t* num_accepted;       /* [batch], written                                         */
   int32_t* out_tokens;         /* [batch][num_nodes + 1], written                          */
   int32_t* num_emitted;        /* [batch], written                                         */
+  const float* temperature;    /* [batch], or NULL: every sequence greedy                  */
+  const float* uniforms;       /* [batch][num_nodes] in (0, 1] (needed with temperature):
+                                  [c] tests node c, [0] draws the final token              */
 } spec_tree_accept_args_t;
 
 size_t spec_tree_workspace_size(const spec_tree_accept_args_t* tree);

@@ -87,7 +87,8 @@ class TreeAcceptArgs(ctypes.Structure):
                 ("target_logits", ctypes.c_void_p), ("tokens", ctypes.c_void_p),
                 ("parents", ctypes.c_void_p), ("path", ctypes.c_void_p),
                 ("num_accepted", ctypes.c_void_p), ("out_tokens", ctypes.c_void_p),
-                ("num_emitted", ctypes.c_void_p)]
+                ("num_emitted", ctypes.c_void_p), ("temperature", ctypes.c_void_p),
+                ("uniforms", ctypes.c_void_p)]
 
 
 class TreeCommitArgs(ctypes.Structure):
@@ -462,7 +463,7 @@ def commit_kv(kv_len, num_accepted, page_table, page_size: int, gamma: int, free
 
 
 def tree_accept_args(target_logits, tokens, parents, path, num_accepted, out_tokens,
-                     num_emitted) -> TreeAcceptArgs:
+                     num_emitted, temperature=None, uniforms=None) -> TreeAcceptArgs:
     B, N, V = target_logits.shape
     if target_logits.dtype == torch.bfloat16:
         dt = SPEC_BF16
@@ -475,9 +476,16 @@ def tree_accept_args(target_logits, tokens, parents, path, num_accepted, out_tok
                            (path, "path", (B, N)), (num_accepted, "num_accepted", (B,)),
                            (out_tokens, "out_tokens", (B, N + 1)), (num_emitted, "num_emitted", (B,))):
         _check(t, name, torch.int32, shape)
+    if (temperature is None) != (uniforms is None):
+        raise ValueError("temperature and uniforms go together")
+    if temperature is not None:
+        _check(temperature, "temperature", torch.float32, (B,))
+        _check(uniforms, "uniforms", torch.float32, (B, N))
     return TreeAcceptArgs(B, N, V, dt, target_logits.data_ptr(), tokens.data_ptr(),
                           parents.data_ptr(), path.data_ptr(), num_accepted.data_ptr(),
-                          out_tokens.data_ptr(), num_emitted.data_ptr())
+                          out_tokens.data_ptr(), num_emitted.data_ptr(),
+                          None if temperature is None else temperature.data_ptr(),
+                          None if uniforms is None else uniforms.data_ptr())
 
 
 def tree_workspace_size(t: TreeAcceptArgs) -> int:
@@ -492,9 +500,11 @@ def accept_tree_args(t: TreeAcceptArgs, ws: torch.Tensor, stream=None):
            "spec_accept_tree")
 
 
-def accept_tree(target_logits, tokens, parents, ws=None, stream=None) -> Dict[str, torch.Tensor]:
-    """Greedy verification of a candidate tree (spec_accept_tree). Returns path,
-    num_accepted, out_tokens, num_emitted."""
+def accept_tree(target_logits, tokens, parents, ws=None, stream=None, temperature=None,
+                uniforms=None) -> Dict[str, torch.Tensor]:
+    """Verification of a candidate tree (spec_accept_tree): greedy, or sampled for the
+    sequences with temperature > 0 (temperature float32 [batch] and uniforms float32
+    [batch][num_nodes] together). Returns path, num_accepted, out_tokens, num_emitted."""
     B, N, _ = target_logits.shape
     dev = target_logits.device
     res = dict(path=torch.empty(B, N, dtype=torch.int32, device=dev),
@@ -502,7 +512,7 @@ def accept_tree(target_logits, tokens, parents, ws=None, stream=None) -> Dict[st
                out_tokens=torch.empty(B, N + 1, dtype=torch.int32, device=dev),
                num_emitted=torch.empty(B, dtype=torch.int32, device=dev))
     t = tree_accept_args(target_logits, tokens, parents, res["path"], res["num_accepted"],
-                         res["out_tokens"], res["num_emitted"])
+                         res["out_tokens"], res["num_emitted"], temperature, uniforms)
     if ws is None:
         ws = new_workspace(tree_workspace_size(t), dev)
     accept_tree_args(t, ws, stream)

@@ -176,6 +176,7 @@ spec_status_t check_tree(const spec_tree_accept_args_t* t) {
       !t->out_tokens || !t->num_emitted)
     return SPEC_ERR_INVALID_ARGUMENT;
   if (t->num_nodes > 64 || t->batch > 65535) return SPEC_ERR_UNSUPPORTED;
+  if (t->temperature && !t->uniforms) return SPEC_ERR_INVALID_ARGUMENT;
   return SPEC_OK;
 }
 

@@ -102,8 +102,9 @@ cudaError_t launch_commit(const spec_commit_args_t& a, cudaStream_t stream);
 struct TreeLayout {
   size_t tickets;      // uint32 [batch]: node rows of the sequence finished
   size_t row_tickets;  // uint32 [batch][nodes]: splits of the row finished
-  size_t parts;        // 16 B [batch][nodes][splits]
+  size_t parts;        // 16 B [batch][nodes][splits]: (argmax key, max key, bad, sum of 2^..)
   size_t argmax;       // int32 [batch][nodes]
+  size_t rowstat;      // float2 [batch][nodes]: (max logit, sum of 2^((l - max) log2e / T))
   size_t end;
   int splits, elems_per_split;
 };

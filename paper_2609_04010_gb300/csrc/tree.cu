@@ -3,10 +3,16 @@
 // candidate tree from the drafter's rows, greedy acceptance along it, and the
 // compaction of the accepted path's keys and values.
 //
-// tree_greedy_kernel: grid (splits, nodes, sequences) of 128-thread blocks. Each block
-// finds the lowest-index argmax of its part of a node's target row; the row's last block
-// (ticket) merges the parts, and the sequence's last block walks the tree from the root,
-// moving to the child whose token is the current node's argmax.
+// tree_greedy_kernel (tree acceptance): grid (splits, nodes, sequences) of 128-thread
+// blocks. Each block finds the lowest-index argmax of its part of a node's target row
+// and, for a tempered sequence, the part's sum of 2^((l - max) log2e / T); the row's
+// last block (ticket) merges the parts, and the sequence's last block walks the tree
+// from the root. Greedy: to the child whose token is the current node's argmax.
+// Sampled: the children are tried in node order as point-mass proposals (accepted iff
+// u <= p'(token), p' without the siblings rejected before), decided in fp64 from the
+// gathered logits; after the last rejection the block draws the final token from p' by
+// inverse CDF: the part where the remaining mass crosses u x total, from the stored part
+// sums minus the rejected tokens' weights, then one pass over that part.
 //
 // tree_compact_kernel: one block per (cache, KV head, sequence) moves the accepted
 // path's key or value rows into consecutive positions after the context.
@@ -21,12 +27,15 @@
 
 namespace specv {
 
+// Row blocks of the tree acceptance kernel resident per SM (80 registers a thread).
+constexpr int kTreeBlocksPerSm = 6;
+
 TreeLayout tree_layout(int batch, int nodes, int vocab, size_t base, int sms, bool vec) {
   TreeLayout L;
   const int lane = vec ? 64 : 32;
   const int nlanes = (vocab + lane - 1) / lane;
   const int64_t rows = static_cast<int64_t>(batch) * nodes;
-  int64_t splits = (static_cast<int64_t>(kFiltBlocksPerSm) * sms + rows - 1) / rows;
+  int64_t splits = (static_cast<int64_t>(kTreeBlocksPerSm) * sms + rows - 1) / rows;
   splits = splits < 1 ? 1 : (splits > kFiltMaxSplits ? kFiltMaxSplits : splits);
   if (splits > nlanes) splits = nlanes;
   L.elems_per_split = static_cast<int>((nlanes + splits - 1) / splits) * lane;
@@ -35,7 +44,8 @@ TreeLayout tree_layout(int batch, int nodes, int vocab, size_t base, int sms, bo
   L.row_tickets = ws_round(L.tickets + sizeof(uint32_t) * batch);
   L.parts = ws_round(L.row_tickets + sizeof(uint32_t) * rows);
   L.argmax = ws_round(L.parts + 16 * rows * L.splits);
-  L.end = ws_round(L.argmax + sizeof(int32_t) * rows);
+  L.rowstat = ws_round(L.argmax + sizeof(int32_t) * rows);
+  L.end = ws_round(L.rowstat + sizeof(float) * 2 * rows);
   return L;
 }
 
@@ -57,7 +67,10 @@ struct TreeParams {
   uint32_t* tickets;
   uint32_t* row_tickets;
   uint4* parts;
-  int32_t* argmax;         // [batch][nodes]; -1 marks a row with NaN
+  int32_t* argmax;         // [batch][nodes]; -1 marks an unusable row
+  float2* rowstat;         // [batch][nodes]: (max logit, sum of 2^((l - max) log2e / T))
+  const float* temperature;  // [batch] or NULL (greedy)
+  const float* uniforms;     // [batch][nodes]
 };
 
 template <bool BF16>
@@ -71,22 +84,40 @@ __device__ __forceinline__ uint32_t order_key(float x) {
   if (f == 0x80000000u) f = 0u;
   return (f & 0x80000000u) ? ~f : (f | 0x80000000u);
 }
+// The float whose order_key is k.
+__device__ __forceinline__ float key_to_float(uint32_t k) {
+  return __uint_as_float((k & 0x80000000u) ? (k & 0x7fffffffu) : ~k);
+}
+// 2^((x - m) * c) for a running reference m (an all -inf prefix has m = -inf and weight 0).
+__device__ __forceinline__ float rel_weight(float x, float m, float c) {
+  return m == -INFINITY ? 0.f : ex2((x - m) * c);
+}
 
 template <bool BF16, bool VEC>
-__global__ void __launch_bounds__(kThreads, 8) tree_greedy_kernel(TreeParams p) {
+__global__ void __launch_bounds__(kThreads, kTreeBlocksPerSm) tree_greedy_kernel(TreeParams p) {
   __shared__ unsigned long long s_red[kThreads / 32];
+  __shared__ float s_fsum[kThreads / 32];
   __shared__ int s_bad, s_last;
   __shared__ int s_arg[64];
+  // hand-off from the walking warp to the sampled final draw
+  __shared__ int s_final, s_len, s_nrm, s_kcross, s_tok;
+  __shared__ int s_rm[64];                 // tokens rejected at the final node, ascending
+  __shared__ float s_rmw[64];              // their weights 2^((l - M) log2e / T)
+  __shared__ double s_target, s_dsum[kThreads / 32], s_mass[kFiltMaxSplits];
   const int split = blockIdx.x, j = blockIdx.y, b = blockIdx.z, tid = threadIdx.x;
   const int N = p.nodes, V = p.vocab;
   const int64_t rid = static_cast<int64_t>(b) * N + j;
   const char* rowp = static_cast<const char*>(p.target) + rid * V * (BF16 ? 2 : 4);
   const int e_begin = split * p.elems_per_split, e_end = min(V, e_begin + p.elems_per_split);
+  const float T = p.temperature ? p.temperature[b] : 0.f;
+  const bool tempered = T > 0.f;
+  const float cs = tempered ? kLog2e / T : 0.f;
   if (tid == 0) s_bad = 0;
   __syncthreads();
 
-  // the lowest-index maximum of this part of the row
-  float m = -INFINITY;
+  // the lowest-index maximum of this part of the row and, for a tempered sequence, the
+  // sum of 2^((l - max) log2e / T) over it (rescaled whenever the running maximum grows)
+  float m = -INFINITY, sum = 0.f;
   int a = INT_MAX;
   bool bad = false;
   if (VEC) {
@@ -102,17 +133,28 @@ __global__ void __launch_bounds__(kThreads, 8) tree_greedy_kernel(TreeParams p) 
         const int vi = v0 + k * kThreads + tid;
         dv[k] = vi < vend ? __ldg(rv + vi) : make_uint4(ninf, ninf, ninf, ninf);
       }
+      auto val = [&](int k, int q) {
+        const uint32_t wv[4] = {dv[k].x, dv[k].y, dv[k].z, dv[k].w};
+        return BF16 ? __uint_as_float((q & 1) ? (wv[q >> 1] & 0xffff0000u) : (wv[q >> 1] << 16))
+                    : __uint_as_float(wv[q]);
+      };
+      const float m_old = m;
 #pragma unroll
       for (int k = 0; k < kUnroll; ++k) {
         const int vi = v0 + k * kThreads + tid;
-        const uint32_t wv[4] = {dv[k].x, dv[k].y, dv[k].z, dv[k].w};
 #pragma unroll
         for (int q = 0; q < kEpv; ++q) {
-          const float x = BF16 ? __uint_as_float((q & 1) ? (wv[q >> 1] & 0xffff0000u) : (wv[q >> 1] << 16))
-                               : __uint_as_float(wv[q]);
-          bad |= x != x;
+          const float x = val(k, q);
+          bad |= x != x || (tempered && x == INFINITY);
           if (x > m) { m = x; a = vi * kEpv + q; }
         }
+      }
+      if (tempered) {
+        sum = m_old == -INFINITY ? 0.f : sum * ex2((m_old - m) * cs);
+#pragma unroll
+        for (int k = 0; k < kUnroll; ++k)
+#pragma unroll
+          for (int q = 0; q < kEpv; ++q) sum += rel_weight(val(k, q), m, cs);
       }
     }
   } else {
@@ -124,10 +166,16 @@ __global__ void __launch_bounds__(kThreads, 8) tree_greedy_kernel(TreeParams p) 
         const int ei = e0 + k * kThreads + tid;
         x[k] = ei < e_end ? load_elem<BF16>(rowp, ei) : -INFINITY;
       }
+      const float m_old = m;
 #pragma unroll
       for (int k = 0; k < kUnroll; ++k) {
-        bad |= x[k] != x[k];
+        bad |= x[k] != x[k] || (tempered && x[k] == INFINITY);
         if (x[k] > m) { m = x[k]; a = e0 + k * kThreads + tid; }
+      }
+      if (tempered) {
+        sum = m_old == -INFINITY ? 0.f : sum * ex2((m_old - m) * cs);
+#pragma unroll
+        for (int k = 0; k < kUnroll; ++k) sum += rel_weight(x[k], m, cs);
       }
     }
   }
@@ -144,11 +192,26 @@ __global__ void __launch_bounds__(kThreads, 8) tree_greedy_kernel(TreeParams p) 
   best = s_red[0];
 #pragma unroll
   for (int k = 1; k < kThreads / 32; ++k) best = s_red[k] > best ? s_red[k] : best;
+  float part_sum = 0.f;
+  if (tempered) {
+    // the part's sum relative to its maximum
+    const float pm = key_to_float(static_cast<uint32_t>(best >> 32));
+    float v = (pm == -INFINITY || !(pm < INFINITY)) ? 0.f : sum * rel_weight(m, pm, cs) * (m == -INFINITY ? 0.f : 1.f);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    __syncthreads();  // s_red is read above by every thread
+    if ((tid & 31) == 0) s_fsum[tid >> 5] = v;
+    __syncthreads();
+    for (int k = 0; k < kThreads / 32; ++k) part_sum += s_fsum[k];
+  }
 
-  if (p.splits > 1) {
+  float2 stat = make_float2(key_to_float(static_cast<uint32_t>(best >> 32)), part_sum);
+  if (p.splits > 1 || tempered) {
     if (tid == 0)
       p.parts[rid * p.splits + split] = make_uint4(static_cast<uint32_t>(best), static_cast<uint32_t>(best >> 32),
-                                                   static_cast<uint32_t>(s_bad), 0u);
+                                                   static_cast<uint32_t>(s_bad), __float_as_uint(part_sum));
+  }
+  if (p.splits > 1) {
     __threadfence();
     __syncthreads();
     if (tid == 0) {
@@ -174,15 +237,33 @@ __global__ void __launch_bounds__(kThreads, 8) tree_greedy_kernel(TreeParams p) 
         bb = y > bb ? y : bb;
       }
       anybad = __reduce_or_sync(0xffffffffu, anybad);
+      // the row's sum relative to its maximum
+      const float M = key_to_float(static_cast<uint32_t>(bb >> 32));
+      float z = 0.f;
+      if (tempered && M > -INFINITY && M < INFINITY) {
+        for (int k = tid; k < p.splits; k += 32) {
+          const uint4 q = __ldcg(p.parts + rid * p.splits + k);
+          z += __uint_as_float(q.w) * rel_weight(key_to_float(q.y), M, cs);
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) z += __shfl_xor_sync(0xffffffffu, z, o);
+      }
       if (tid == 0) {
         s_red[0] = bb;
         s_bad = anybad ? 1 : 0;
+        s_fsum[0] = z;
       }
     }
     __syncthreads();
     best = s_red[0];
+    stat = make_float2(key_to_float(static_cast<uint32_t>(best >> 32)), s_fsum[0]);
   }
-  if (tid == 0) p.argmax[rid] = s_bad ? -1 : static_cast<int>(0xffffffffu - static_cast<uint32_t>(best));
+  if (tid == 0) {
+    // a tempered row needs a finite maximum (NaN and +inf are flagged above)
+    const bool unusable = s_bad || (tempered && !(stat.x > -INFINITY));
+    p.argmax[rid] = unusable ? -1 : static_cast<int>(0xffffffffu - static_cast<uint32_t>(best));
+    if (tempered) p.rowstat[rid] = stat;
+  }
 
   // the sequence's last row block walks the tree
   __threadfence();
@@ -196,65 +277,270 @@ __global__ void __launch_bounds__(kThreads, 8) tree_greedy_kernel(TreeParams p) 
   if (!s_last) return;
   __threadfence();
   if (tid < N) s_arg[tid] = __ldcg(p.argmax + static_cast<int64_t>(b) * N + tid);
+  if (tid == 0) s_final = -1;
   __syncthreads();
-  if (tid >= 32) return;
-  // one warp: lane c holds node c (N <= 64: two nodes per lane)
-  const int lane = tid;
   const int64_t brow = static_cast<int64_t>(b) * N;
-  int tok[2], par[2];
-  uint32_t bad_in = 0;
-#pragma unroll
-  for (int h = 0; h < 2; ++h) {
-    const int c = lane + 32 * h;
-    tok[h] = c < N ? p.tokens[brow + c] : -1;
-    par[h] = c < N ? p.parents[brow + c] : -2;
-    if (c < N) {
-      if (tok[h] < 0 || tok[h] >= V) bad_in |= SPEC_FLAG_BAD_TOKEN;
-      if (c == 0 ? par[h] != -1 : (par[h] < 0 || par[h] >= c)) bad_in |= SPEC_FLAG_BAD_TREE;
-      if (s_arg[c] < 0) bad_in |= SPEC_FLAG_BAD_LOGITS;
-    }
-  }
-  bad_in = __reduce_or_sync(0xffffffffu, bad_in);
   int32_t* path = p.path + brow;
   int32_t* out = p.out_tokens + static_cast<int64_t>(b) * (N + 1);
-  if (bad_in) {
-    for (int c = lane; c < N; c += 32) path[c] = -1;
-    for (int c = lane; c <= N; c += 32) out[c] = -1;
-    if (lane == 0) {
-      p.num_accepted[b] = -1;
-      p.num_emitted[b] = 0;
-      set_status(p.status, bad_in);
+  if (tid < 32) {
+    // one warp: lane c holds node c (N <= 64: two nodes per lane)
+    const int lane = tid;
+    int tok[2], par[2];
+    uint32_t bad_in = 0;
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int c = lane + 32 * h;
+      tok[h] = c < N ? p.tokens[brow + c] : -1;
+      par[h] = c < N ? p.parents[brow + c] : -2;
+      if (c < N) {
+        if (tok[h] < 0 || tok[h] >= V) bad_in |= SPEC_FLAG_BAD_TOKEN;
+        if (c == 0 ? par[h] != -1 : (par[h] < 0 || par[h] >= c)) bad_in |= SPEC_FLAG_BAD_TREE;
+        if (s_arg[c] < 0) bad_in |= SPEC_FLAG_BAD_LOGITS;
+      }
     }
-    return;
-  }
-  int cur = 0, len = 1;
-  if (lane == 0) {
-    path[0] = 0;
-    out[0] = tok[0];  // the root: lane 0 holds node 0
-  }
-  for (int step = 1; step < N; ++step) {
-    const int want = s_arg[cur];
-    const unsigned m0 = __ballot_sync(0xffffffffu, par[0] == cur && tok[0] == want);
-    const unsigned m1 = __ballot_sync(0xffffffffu, par[1] == cur && tok[1] == want);
-    int nxt = -1;
-    if (m0) nxt = __ffs(m0) - 1;
-    else if (m1) nxt = 32 + __ffs(m1) - 1;
-    if (nxt < 0) break;
-    const int t = __shfl_sync(0xffffffffu, nxt < 32 ? tok[0] : tok[1], nxt & 31);
-    if (lane == 0) {
-      path[len] = nxt;
-      out[len] = t;
+    bad_in = __reduce_or_sync(0xffffffffu, bad_in);
+    if (bad_in) {
+      for (int c = lane; c < N; c += 32) path[c] = -1;
+      for (int c = lane; c <= N; c += 32) out[c] = -1;
+      if (lane == 0) {
+        p.num_accepted[b] = -1;
+        p.num_emitted[b] = 0;
+        set_status(p.status, bad_in);
+      }
+    } else {
+      int cur = 0, len = 1;
+      if (lane == 0) {
+        path[0] = 0;
+        out[0] = tok[0];  // the root: lane 0 holds node 0
+      }
+      if (!tempered) {
+        for (int step = 1; step < N; ++step) {
+          const int want = s_arg[cur];
+          const unsigned m0 = __ballot_sync(0xffffffffu, par[0] == cur && tok[0] == want);
+          const unsigned m1 = __ballot_sync(0xffffffffu, par[1] == cur && tok[1] == want);
+          int nxt = -1;
+          if (m0) nxt = __ffs(m0) - 1;
+          else if (m1) nxt = 32 + __ffs(m1) - 1;
+          if (nxt < 0) break;
+          const int t = __shfl_sync(0xffffffffu, nxt < 32 ? tok[0] : tok[1], nxt & 31);
+          if (lane == 0) {
+            path[len] = nxt;
+            out[len] = t;
+          }
+          cur = nxt;
+          ++len;
+        }
+        for (int c = len + lane; c < N; c += 32) path[c] = -1;
+        if (lane == 0) out[len] = s_arg[cur];
+        for (int c = len + 1 + lane; c <= N; c += 32) out[c] = -1;
+        if (lane == 0) {
+          p.num_accepted[b] = len - 1;
+          p.num_emitted[b] = len + 1;
+        }
+      } else {
+        // sampled walk: the children of the current node, in node order, are point-mass
+        // proposals; child c is accepted iff u[c] <= p'(token), p' the node's target
+        // distribution without the tokens of the siblings rejected before it
+        const float* u = p.uniforms + brow;
+        const char* tbase = static_cast<const char*>(p.target);
+        for (int step = 1; step <= N; ++step) {
+          const float2 rs = __ldcg(p.rowstat + brow + cur);
+          const char* crow = tbase + (brow + cur) * V * (BF16 ? 2 : 4);
+          double e[2];
+          bool ch[2];
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            ch[h] = par[h] == cur;
+            e[h] = ch[h] ? exp((static_cast<double>(load_elem<BF16>(crow, tok[h])) - rs.x) /
+                               static_cast<double>(T))
+                         : 0.0;
+          }
+          // a repeated sibling token was removed with its first occurrence: probability 0
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            bool dup = false;
+            for (int o = 0; o < 64; ++o) {
+              const int t_o = __shfl_sync(0xffffffffu, o < 32 ? tok[0] : tok[1], o & 31);
+              const int p_o = __shfl_sync(0xffffffffu, o < 32 ? par[0] : par[1], o & 31);
+              dup |= o < lane + 32 * h && p_o == cur && t_o == tok[h];
+            }
+            if (dup) e[h] = 0.0;
+          }
+          // mass removed before each child: exclusive prefix over node order
+          double inc0 = e[0], inc1 = e[1];
+#pragma unroll
+          for (int o = 1; o < 32; o <<= 1) {
+            const double y0 = __shfl_up_sync(0xffffffffu, inc0, o);
+            const double y1 = __shfl_up_sync(0xffffffffu, inc1, o);
+            if (lane >= o) { inc0 += y0; inc1 += y1; }
+          }
+          const double tot0 = __shfl_sync(0xffffffffu, inc0, 31);
+          const double ex0 = inc0 - e[0], ex1 = tot0 + inc1 - e[1];
+          bool acc[2];
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const double S = static_cast<double>(rs.y) - (h == 0 ? ex0 : ex1);
+            acc[h] = ch[h] && e[h] > 0.0 &&
+                     (S <= e[h] || static_cast<double>(u[lane + 32 * h]) <= e[h] / S);
+          }
+          const unsigned m0 = __ballot_sync(0xffffffffu, acc[0]);
+          const unsigned m1 = __ballot_sync(0xffffffffu, acc[1]);
+          int nxt = -1;
+          if (m0) nxt = __ffs(m0) - 1;
+          else if (m1) nxt = 32 + __ffs(m1) - 1;
+          if (nxt >= 0) {
+            const int t = __shfl_sync(0xffffffffu, nxt < 32 ? tok[0] : tok[1], nxt & 31);
+            if (lane == 0) {
+              path[len] = nxt;
+              out[len] = t;
+            }
+            cur = nxt;
+            ++len;
+            continue;
+          }
+          // every child rejected: hand the final node and its rejected tokens (ascending,
+          // with their weights relative to the row maximum) to the whole block
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const bool mine = ch[h] && e[h] > 0.0;
+            int rank = 0;
+            for (int o = 0; o < 64; ++o) {
+              const int t_o = __shfl_sync(0xffffffffu, o < 32 ? tok[0] : tok[1], o & 31);
+              const int p_o = __shfl_sync(0xffffffffu, o < 32 ? par[0] : par[1], o & 31);
+              const double e_o = __shfl_sync(0xffffffffu, o < 32 ? e[0] : e[1], o & 31);
+              const bool in = p_o == cur && e_o > 0.0;
+              rank += in && (t_o < tok[h] || (t_o == tok[h] && o < lane + 32 * h));
+            }
+            if (mine) {
+              s_rm[rank] = tok[h];
+              s_rmw[rank] = rel_weight(load_elem<BF16>(crow, tok[h]), rs.x, cs);
+            }
+          }
+          const int nrm = __popc(__ballot_sync(0xffffffffu, ch[0] && e[0] > 0.0)) +
+                          __popc(__ballot_sync(0xffffffffu, ch[1] && e[1] > 0.0));
+          if (lane == 0) {
+            s_final = cur;
+            s_len = len;
+            s_nrm = nrm;
+          }
+          break;
+        }
+        for (int c = len + lane; c < N; c += 32) path[c] = -1;
+      }
     }
-    cur = nxt;
-    ++len;
   }
-  for (int c = len + lane; c < N; c += 32) path[c] = -1;
-  if (lane == 0) out[len] = s_arg[cur];
-  for (int c = len + 1 + lane; c <= N; c += 32) out[c] = -1;
-  if (lane == 0) {
+  __syncthreads();
+  if (s_final < 0) return;  // greedy, bad input: done
+
+  // ---- the final draw from p' of node s_final: inverse CDF in ascending token order ----
+  const int fin = s_final, len = s_len, nrm = s_nrm;
+  const int64_t frid = brow + fin;
+  const float M = __ldcg(p.rowstat + frid).x;
+  const int eps = p.elems_per_split;
+  if (tid == 0) {
+    // remaining mass of each part (its sum minus its rejected tokens' weights), the total,
+    // and the part where the cumulative mass reaches u[0] x total
+    double* mass = s_mass;
+    double S = 0.0;
+    for (int pass = 0; pass < 2 && !(S > 0.0); ++pass) {
+      for (int k = 0; k < p.splits; ++k) {
+        const uint4 q = __ldcg(p.parts + frid * p.splits + k);
+        mass[k] = static_cast<double>(__uint_as_float(q.w)) * rel_weight(key_to_float(q.y), M, cs);
+      }
+      if (pass == 0) {
+        for (int r = 0; r < nrm; ++r) mass[s_rm[r] / eps] -= static_cast<double>(s_rmw[r]);
+      } else {
+        s_nrm = 0;  // nothing left after the removals (rounding only): draw from p itself
+      }
+      S = 0.0;
+      for (int k = 0; k < p.splits; ++k) {
+        if (mass[k] < 0.0) mass[k] = 0.0;
+        S += mass[k];
+      }
+    }
+    const double target = static_cast<double>(p.uniforms[brow]) * S;
+    int kc = -1;
+    double before = 0.0, C = 0.0;
+    for (int k = 0; k < p.splits; ++k) {
+      if (mass[k] > 0.0 && C + mass[k] >= target) { kc = k; before = C; break; }
+      C += mass[k];
+    }
+    if (kc < 0) {  // rounding left the target above the total: the last part with mass
+      C = 0.0;
+      for (int k = 0; k < p.splits; ++k) {
+        if (mass[k] > 0.0) { kc = k; before = C; }
+        C += mass[k];
+      }
+    }
+    s_kcross = kc < 0 ? 0 : kc;  // the part of the row maximum always has mass
+    s_target = target - before;
+  }
+  __syncthreads();
+  const int kc = s_kcross, nrm_scan = s_nrm;
+  const double tin = s_target;
+  // each thread a contiguous run of the crossing part (multiples of 8 elements)
+  const int pb = kc * eps, pe = min(V, pb + eps);
+  const int per = ((pe - pb + kThreads - 1) / kThreads + 7) / 8 * 8;
+  const int lo = min(pe, pb + tid * per), hi = min(pe, lo + per);
+  const char* frow = static_cast<const char*>(p.target) + frid * V * (BF16 ? 2 : 4);
+  int ptr = 0;
+  while (ptr < nrm_scan && s_rm[ptr] < lo) ++ptr;
+  auto weight_at = [&](int x, int& q) {
+    bool removed = false;
+    while (q < nrm_scan && s_rm[q] <= x) { removed |= s_rm[q] == x; ++q; }
+    return removed ? 0.f : rel_weight(load_elem<BF16>(frow, x), M, cs);
+  };
+  float run = 0.f;
+  {
+    int q = ptr;
+    for (int x = lo; x < hi; ++x) run += weight_at(x, q);
+  }
+  // block exclusive scan of the runs' sums; the run that holds the crossing is the last
+  // one with weight whose exclusive prefix is below the target
+  double incl = static_cast<double>(run);
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const double y = __shfl_up_sync(0xffffffffu, incl, o);
+    if ((tid & 31) >= o) incl += y;
+  }
+  double prev = __shfl_up_sync(0xffffffffu, incl, 1);
+  if ((tid & 31) == 0) prev = 0.0;
+  if ((tid & 31) == 31) s_dsum[tid >> 5] = incl;
+  __syncthreads();
+  double wbase = 0.0;
+  for (int k = 0; k < (tid >> 5); ++k) wbase += s_dsum[k];
+  const double excl = wbase + prev;
+  int owner = (run > 0.f && excl < tin) ? tid : -1;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) owner = max(owner, __shfl_xor_sync(0xffffffffu, owner, o));
+  __syncthreads();  // every thread has read s_dsum
+  if ((tid & 31) == 0) s_fsum[tid >> 5] = __int_as_float(owner);
+  __syncthreads();
+  owner = -1;
+  for (int k = 0; k < kThreads / 32; ++k) owner = max(owner, __float_as_int(s_fsum[k]));
+  if (tid == owner) {
+    // walk the run: the first token whose cumulative weight reaches the target, else (if
+    // rounding leaves the target above the run) its last positive-weight token
+    double C = excl;
+    int q = ptr, pick = -1;
+    for (int x = lo; x < hi; ++x) {
+      const float w = weight_at(x, q);
+      C += static_cast<double>(w);
+      if (w > 0.f) {
+        pick = x;
+        if (C >= tin) break;
+      }
+    }
+    s_tok = pick;
+  }
+  if (owner < 0 && tid == 0) s_tok = s_arg[fin];  // no weight left in fp32: the row maximum
+  __syncthreads();
+  if (tid == 0) {
+    out[len] = s_tok;
     p.num_accepted[b] = len - 1;
     p.num_emitted[b] = len + 1;
   }
+  for (int c = len + 1 + tid; c <= N; c += kThreads) out[c] = -1;
 }
 
 // Flags of sequence b's commit inputs (0 = valid), evaluated by one full warp: kv_len
@@ -1046,6 +1332,9 @@ cudaError_t launch_tree_greedy(const spec_tree_accept_args_t& a, const TreeLayou
   p.row_tickets = reinterpret_cast<uint32_t*>(ws + L.row_tickets);
   p.parts = reinterpret_cast<uint4*>(ws + L.parts);
   p.argmax = reinterpret_cast<int32_t*>(ws + L.argmax);
+  p.rowstat = reinterpret_cast<float2*>(ws + L.rowstat);
+  p.temperature = a.temperature;
+  p.uniforms = a.uniforms;
   (void)cudaGetLastError();
   if (a.logits_dtype == SPEC_BF16)
     return vec ? launch_tree_typed<true, true>(p, stream) : launch_tree_typed<true, false>(p, stream);

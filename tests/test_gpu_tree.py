@@ -372,3 +372,134 @@ def test_tree_step_end_to_end(oracle_mod):
     o_out, o_lse, _ = oracle_mod.verify_attention(inp.q, inp.k_cache, inp.v_cache, inp.page_table,
                                                   inp.kv_len, N, rows=rows, tree_mask=tree["mask"])
     compare_attention(out.float().cpu().numpy(), lse.cpu().numpy(), o_out, o_lse, rows)
+
+
+# ---------------------------------------------------------------------------------
+# sampled (T > 0) tree acceptance
+# ---------------------------------------------------------------------------------
+def random_tree(rng, tl, T, N, branch=3):
+    """A tree whose children are distinct tokens drawn from their parent's target row (so
+    that acceptance happens), parents chosen among the first nodes with room."""
+    V = tl.shape[1]
+    par = np.full(N, -1, np.int32)
+    tok = np.zeros(N, np.int32)
+    tok[0] = rng.integers(V)
+    kids = {0: set()}
+    for c in range(1, N):
+        cands = [u for u in range(c) if len(kids[u]) < branch]
+        u = int(cands[min(len(cands) - 1, int(rng.integers(0, min(4, len(cands)))))])
+        z = tl[u].astype(np.float64) / (T if T > 0 else 1.0)
+        pr = np.exp(z - z.max())
+        for t in kids[u]:
+            pr[t] = 0.0
+        pr /= pr.sum()
+        t = int(rng.choice(V, p=pr)) if rng.random() < 0.8 else int(rng.integers(V))
+        par[c], tok[c] = u, t
+        kids[u].add(t)
+        kids[c] = set()
+    return tok, par
+
+
+def compare_tree_sampled(g, o):
+    """Bit-exact but for ties: a sequence may differ only where one of the oracle's
+    decisions or its final draw lay within TIE_MARGIN of its threshold."""
+    from helpers import TIE_MARGIN
+    ties = []
+    for b in range(len(o["num_accepted"])):
+        if o["status"][b] != 0:
+            assert g["num_accepted"][b] == -1 and g["num_emitted"][b] == 0, b
+            assert np.all(g["out_tokens"][b] == -1) and np.all(g["path"][b] == -1), b
+            continue
+        same = all(np.array_equal(g[k][b], o[k][b])
+                   for k in ("path", "num_accepted", "out_tokens", "num_emitted"))
+        if not same:
+            fin = o["accept_margin"][b][np.isfinite(o["accept_margin"][b])]
+            m = min(fin.min() if fin.size else np.inf, o["sample_margin"][b])
+            assert m < TIE_MARGIN, (b, g["out_tokens"][b], o["out_tokens"][b], m)
+            ties.append((b, float(m)))
+    return ties
+
+
+def gpu_accept_tree_sampled(tl, tok, par, T=None, u=None):
+    r = binding.accept_tree(logits_dev(tl), dev(tok), dev(par),
+                            temperature=None if T is None else dev(np.asarray(T, np.float32)),
+                            uniforms=None if u is None else dev(np.asarray(u, np.float32)))
+    torch.cuda.synchronize()
+    return {k: v.cpu().numpy() for k, v in r.items()}
+
+
+@pytest.mark.parametrize("V,dtype,B,N", [(128256, "bf16", 4, 33), (32000, "f32", 6, 33),
+                                         (1000, "bf16", 16, 17), (65, "f32", 24, 9),
+                                         (8193, "bf16", 8, 64)])
+def test_sampled_tree_acceptance_matches_oracle(oracle_mod, V, dtype, B, N):
+    rng = np.random.default_rng(V + N)
+    T = np.resize(np.array([1.0, 0.7, 0.0, 1.3], np.float32), B)
+    tl32 = (rng.standard_normal((B, N, V)) * 3.0).astype(np.float32)
+    tl = W.f32_to_bf16_bits(tl32) if dtype == "bf16" else tl32
+    seen = W.bf16_bits_to_f32(tl) if dtype == "bf16" else tl32
+    tok = np.zeros((B, N), np.int32)
+    par = np.zeros((B, N), np.int32)
+    for b in range(B):
+        tok[b], par[b] = random_tree(rng, seen[b], float(T[b]), N)
+    if N >= 3:  # a repeated sibling token: the second occurrence has probability 0
+        kids = [c for c in range(1, N) if par[0, c] == par[0, 1]]
+        if len(kids) >= 2:
+            tok[0, kids[1]] = tok[0, kids[0]]
+    u = (1.0 - rng.random((B, N))).astype(np.float32)
+    g = gpu_accept_tree_sampled(tl, tok, par, T, u)
+    o = oracle_mod.accept_tree_sampled(tl, tok, par, T, u)
+    assert np.all(o["status"] == 0)
+    ties = compare_tree_sampled(g, o)
+    assert len(ties) <= max(1, B // 20), ties
+    assert np.all(g["num_emitted"] == g["num_accepted"] + 2)
+    print(f"V={V} N={N}: mean accepted {g['num_accepted'].mean():.2f}, ties {len(ties)}")
+
+
+def test_sampled_tree_output_law_chi_square():
+    """200,000 GPU verifications of one small tree (V = 4, rows in quarters) against the
+    target's own law of the emitted tokens."""
+    from scipy import stats
+    import test_oracle_tree as OT
+    p, tok, par = OT.TREE4_P, OT.TREE4_TOK, OT.TREE4_PAR
+    N, V = p.shape
+    want = OT.target_tree_law(p, tok, par)
+    keys = sorted(want)
+    with np.errstate(divide="ignore"):
+        logits = np.log(p).astype(np.float32)
+    chunk, total = 50_000, 200_000
+    counts = dict.fromkeys(keys, 0)
+    tl = torch.from_numpy(np.broadcast_to(logits, (chunk, N, V)).copy()).cuda()
+    tk = torch.from_numpy(np.broadcast_to(tok, (chunk, N)).copy()).cuda()
+    pr = torch.from_numpy(np.broadcast_to(par, (chunk, N)).copy()).cuda()
+    T = torch.ones(chunk, dtype=torch.float32, device="cuda")
+    for c in range(total // chunk):
+        u = binding.philox_uniforms(W.uniform_seed(7000 + c), chunk * N).view(chunk, N)
+        r = binding.accept_tree(tl, tk, pr, temperature=T, uniforms=u)
+        out, ne = r["out_tokens"].cpu().numpy(), r["num_emitted"].cpu().numpy()
+        for b in range(chunk):
+            counts[tuple(int(x) for x in out[b, 1:ne[b]])] += 1
+    obs = np.array([counts[k] for k in keys], np.float64)
+    exp = np.array([want[k] for k in keys]) * total
+    assert stats.chisquare(obs, exp).pvalue > 1e-3
+
+
+def test_sampled_tree_bad_inputs_are_flagged():
+    rng = np.random.default_rng(9)
+    B, N, V = 6, 5, 300
+    tl = rng.standard_normal((B, N, V)).astype(np.float32)
+    tok = rng.integers(0, V, (B, N)).astype(np.int32)
+    par = np.broadcast_to(np.array([-1, 0, 0, 1, 1], np.int32), (B, N)).copy()
+    T = np.ones(B, np.float32)
+    tl[1, 2, 7] = np.inf        # +inf in a tempered row
+    tl[2, 3, :] = -np.inf       # no finite logit in a tempered row
+    tok[3, 4] = V               # token outside the vocabulary
+    tl[4, 0, 3] = np.nan        # NaN
+    u = (1.0 - rng.random((B, N))).astype(np.float32)
+    r = binding.accept_tree(dev(tl), dev(tok), dev(par), temperature=dev(T), uniforms=dev(u))
+    torch.cuda.synchronize()
+    g = {k: v.cpu().numpy() for k, v in r.items()}
+    for b in (1, 2, 3, 4):
+        assert g["num_accepted"][b] == -1 and g["num_emitted"][b] == 0
+        assert np.all(g["out_tokens"][b] == -1)
+    for b in (0, 5):
+        assert g["num_emitted"][b] == g["num_accepted"][b] + 2
