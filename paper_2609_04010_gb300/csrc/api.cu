@@ -292,7 +292,7 @@ AttnPlan attn_plan(const spec_attn_args_t& a, size_t base, int num_sms, int path
     units = static_cast<int64_t>(a.batch) * a.num_kv_heads * P.row_tiles;
     P.nsplit = 1;
     P.tiles_per_split = 0;
-    P.grid = num_sms * tc_ctas_per_sm(a.head_dim, P.rows_per_cta, a.batch);
+    P.grid = num_sms * tc_ctas_per_sm(a.head_dim, P.rows_per_cta, P.rows, a.batch);
     P.slot_rows = P.rows < P.rows_per_cta ? P.rows : P.rows_per_cta;
     P.slots = units + P.grid;
   }

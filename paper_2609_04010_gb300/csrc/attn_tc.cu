@@ -41,8 +41,14 @@ namespace {
 constexpr int TK = kTcKeyTile;               // keys per tile
 
 
-template <int D, int MT>
+// QR: query rows one Q or P buffer of an M tile holds: 128, or 64 when a KV group has at
+// most 64 query rows. The MMAs still read M = 128 rows; with QR = 64 the buffers are laid
+// out Q, P, K/V stages, so that the 64 padding rows each read comes from the next
+// buffer (their scores and outputs are never used), and the freed 32 KB (D = 128) holds
+// one more K/V stage: more bytes in flight per SM.
+template <int D, int MT, int QR = 128>
 struct TcCfg {
+  static_assert(QR == 128 || (QR == 64 && MT == 1), "64-row buffers only with one M tile");
   static constexpr int DH = D / 64;                   // 128-byte column halves of a row
   // Softmax warps per 32-row quadrant. With one M tile, two warps share each quadrant,
   // one per half of the tile's keys, each with its own online-softmax state and its own
@@ -50,20 +56,22 @@ struct TcCfg {
   static constexpr int SPLIT = MT == 1 ? 2 : 1;
   static constexpr int KH = TK / SPLIT;               // keys of a tile per softmax warp
   static constexpr int PB = MT == 1 ? 2 : 1;          // P buffers (double with one M tile)
-  static constexpr int STAGES = (D == 128 && MT == 2) || (D == 64 && MT == 1) ? 3 : 4;
+  static constexpr int STAGES = QR == 64 ? 5 : ((D == 128 && MT == 2) || (D == 64 && MT == 1) ? 3 : 4);
   static constexpr int THREADS = 128 + 256;           // 4 producer / MMA warps + 8 softmax
   // Starting a unit inside a block's range costs about this many tiles of time (its Q
   // tile, the pipeline refill and the previous unit's epilogue). When blocks hold
   // several unit starts the work list charges it, so that blocks stay balanced.
   static constexpr int UNIT_OVERHEAD = MT == 1 ? 3 : 2;
-  static constexpr uint32_t Q_BYTES = MT * DH * 16384;  // [MT][DH][128 rows x 128 B]
+  static constexpr uint32_t QHALF = QR * 128u;          // one column half of an M tile's Q
+  static constexpr uint32_t PBUF = QR * 128u;           // one P buffer of an M tile
+  static constexpr uint32_t Q_BYTES = MT * DH * QHALF;  // [MT][DH][QR rows x 128 B]
   static constexpr uint32_t KV_BYTES = DH * 8192;       // one stage of K (or V): [DH][64 x 128 B]
-  static constexpr uint32_t P_BYTES = PB * MT * 16384;  // [PB][MT][128 rows x 128 B]
+  static constexpr uint32_t P_BYTES = PB * MT * PBUF;   // [PB][MT][QR rows x 128 B]
   static constexpr uint32_t OFF_Q = 0;
-  static constexpr uint32_t OFF_K = OFF_Q + Q_BYTES;
+  static constexpr uint32_t OFF_P = QR == 64 ? OFF_Q + Q_BYTES : OFF_Q + Q_BYTES + 2 * STAGES * KV_BYTES;
+  static constexpr uint32_t OFF_K = QR == 64 ? OFF_P + P_BYTES : OFF_Q + Q_BYTES;
   static constexpr uint32_t OFF_V = OFF_K + STAGES * KV_BYTES;
-  static constexpr uint32_t OFF_P = OFF_V + STAGES * KV_BYTES;
-  static constexpr uint32_t OFF_BAR = OFF_P + P_BYTES;
+  static constexpr uint32_t OFF_BAR = QR == 64 ? OFF_V + STAGES * KV_BYTES : OFF_P + P_BYTES;
   // barriers: kv_full[S], kv_empty[S], s_full[MT][2], s_free[MT][2], p_full[MT][PB],
   // pv_done[MT][PB], seg_ready, drain[2], xch[4], q_full, seg_flag_ready[8]
   static constexpr int NBAR = 2 * STAGES + 4 * MT + 2 * MT * PB + 3 + 4 + 1 + 8;
@@ -114,12 +122,12 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
 // The kernel
 // ---------------------------------------------------------------------------------
 // TREE: tree attention (a per-row mask over the block keys) instead of the causal block.
-template <int D, int MT, bool TREE>
-__global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
+template <int D, int MT, bool TREE, int QR>
+__global__ void __launch_bounds__(TcCfg<D, MT, QR>::THREADS, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
                    const __grid_constant__ CUtensorMap tmap_v,
                    const __grid_constant__ CUtensorMap tmap_q, AttnParams p) {
-  using C = TcCfg<D, MT>;
+  using C = TcCfg<D, MT, QR>;
   constexpr int SPLIT = C::SPLIT, KH = C::KH, PB = C::PB;
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>(
@@ -324,10 +332,10 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
     // Q tiles of a segment (all M tiles, both column halves) by TMA, on q_full
     auto issue_q = [&](const Seg& sg) {
       if (lane == 0) {
-        mbar_arrive_tx(q_full, MT * C::DH * 16384u);
+        mbar_arrive_tx(q_full, C::Q_BYTES);
         for (int mt = 0; mt < MT; ++mt)
           for (int half = 0; half < C::DH; ++half)
-            tma_load_q(sbase + C::OFF_Q + (mt * C::DH + half) * 16384u, &tmap_q, half,
+            tma_load_q(sbase + C::OFF_Q + (mt * C::DH + half) * C::QHALF, &tmap_q, half,
                        sg.g * p.group,
                        sg.b * p.gamma + (sg.rt * p.rows_per_cta + mt * 128) / p.group, q_full);
       }
@@ -374,7 +382,7 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
               const uint32_t d_tmem = tmem + C::S_COL + (mt * 2 + (x & 1)) * TK;
 #pragma unroll
               for (int kk = 0; kk < D / 16; ++kk) {
-                const uint32_t qa = sbase + C::OFF_Q + (mt * C::DH + kk / 4) * 16384u + (kk % 4) * 32u;
+                const uint32_t qa = sbase + C::OFF_Q + (mt * C::DH + kk / 4) * C::QHALF + (kk % 4) * 32u;
                 const uint32_t kb = sbase + C::OFF_K + st * C::KV_BYTES + (kk / 4) * 1024u + (kk % 4) * 32u;
                 mma_bf16(d_tmem, desc_sw128(qa, 16, 1024), desc_sw128(kb, 16, kGroup), kIdescQK, kk > 0);
               }
@@ -406,7 +414,7 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
 #pragma unroll
                 for (int kk = 0; kk < KH / 16; ++kk) {
                   const int kg = hf * (KH / 16) + kk;  // 16-key step within the tile
-                  const uint32_t pa = sbase + C::OFF_P + (pbuf * MT + mt) * 16384u + kg * 32u;
+                  const uint32_t pa = sbase + C::OFF_P + (pbuf * MT + mt) * C::PBUF + kg * 32u;
                   const uint32_t vb = sbase + C::OFF_V + st * C::KV_BYTES + kg * 2u * kGroup;
                   mma_bf16(d_tmem, desc_sw128(pa, 16, 1024), desc_sw128(vb, 1024, kGroup), kIdescPV,
                            (k > 0 || kk > 0) ? 1u : 0u);
@@ -472,7 +480,7 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
 #pragma unroll
       for (int c2 = 0; c2 < kChunks; ++c2) {
         const int c = hf * kChunks + c2, half = c >> 3, ch = c & 7;
-        *reinterpret_cast<uint4*>(smem + C::OFF_Q + (mt * C::DH + half) * 16384u + row * 128u +
+        *reinterpret_cast<uint4*>(smem + C::OFF_Q + (mt * C::DH + half) * C::QHALF + row * 128u +
                                   ((ch ^ (row & 7)) << 4)) = qr[c2];
       }
       fence_async_smem();
@@ -577,7 +585,7 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
           }
           tmem_wait_st();
         }
-        unsigned char* prow = smem + C::OFF_P + (pbuf * MT + mt) * 16384u + row * 128u;
+        unsigned char* prow = smem + C::OFF_P + (pbuf * MT + mt) * C::PBUF + row * 128u;
 #pragma unroll
         for (int c2 = 0; c2 < KH / 8; ++c2) {
           const int c = hf * (KH / 8) + c2;
@@ -722,15 +730,15 @@ __global__ void __launch_bounds__(TcCfg<D, MT>::THREADS, 1)
 // ---------------------------------------------------------------------------------
 // Host side
 // ---------------------------------------------------------------------------------
-template <int D, int MT>
+template <int D, int MT, int QR>
 cudaError_t launch_typed(const spec_attn_args_t& a, const AttnPlan& P, char* ws,
                          cudaStream_t stream) {
-  using Cf = TcCfg<D, MT>;
+  using Cf = TcCfg<D, MT, QR>;
   CUtensorMap mk, mv, mq;
   if (!encode_cache_map(&mk, a.k_cache, a) || !encode_cache_map(&mv, a.v_cache, a))
     return cudaErrorInvalidValue;
   AttnParams p = make_attn_params(a, P, ws);
-  p.q_tma = encode_q_map(&mq, a, 128) ? 1 : 0;
+  p.q_tma = encode_q_map(&mq, a, QR) ? 1 : 0;
   // Charge unit starts only when blocks hold several of them; when every unit is spread
   // over several blocks, a block holds at most one start and the charge would mostly
   // move real tiles away from blocks that pay no boundary.
@@ -738,7 +746,7 @@ cudaError_t launch_typed(const spec_attn_args_t& a, const AttnPlan& P, char* ws,
   p.unit_overhead = units > P.grid ? Cf::UNIT_OVERHEAD : 0;
   if (!p.q_tma) mq = mk;  // unused
   const size_t smem = Cf::smem_bytes(a.batch);
-  auto kernel = a.tree_mask ? attn_tc_kernel<D, MT, true> : attn_tc_kernel<D, MT, false>;
+  auto kernel = a.tree_mask ? attn_tc_kernel<D, MT, true, QR> : attn_tc_kernel<D, MT, false, QR>;
   cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
@@ -791,15 +799,25 @@ bool encode_q_map(CUtensorMap* map, const spec_attn_args_t& a, int tile_rows) {
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-size_t tc_smem_bytes(int head_dim, int rows_per_cta, int batch) {
-  const bool two = rows_per_cta > 128;
-  if (head_dim == 128) return two ? TcCfg<128, 2>::smem_bytes(batch) : TcCfg<128, 1>::smem_bytes(batch);
-  return two ? TcCfg<64, 2>::smem_bytes(batch) : TcCfg<64, 1>::smem_bytes(batch);
+// The buffer configuration of the row-tile kernel: two M tiles, one M tile with 128-row
+// buffers, or one M tile with 64-row buffers (at most 64 query rows per KV group).
+enum TcVariant { kTwoTiles, kOneTile, kOneTileHalf };
+TcVariant tc_variant(int rows_per_cta, int rows) {
+  return rows_per_cta > 128 ? kTwoTiles : (rows <= 64 ? kOneTileHalf : kOneTile);
 }
 
-int tc_ctas_per_sm(int head_dim, int rows_per_cta, int batch) {
+size_t tc_smem_bytes(int head_dim, int rows_per_cta, int rows, int batch) {
+  const TcVariant v = tc_variant(rows_per_cta, rows);
+  if (head_dim == 128)
+    return v == kTwoTiles ? TcCfg<128, 2>::smem_bytes(batch)
+           : v == kOneTile ? TcCfg<128, 1>::smem_bytes(batch) : TcCfg<128, 1, 64>::smem_bytes(batch);
+  return v == kTwoTiles ? TcCfg<64, 2>::smem_bytes(batch)
+         : v == kOneTile ? TcCfg<64, 1>::smem_bytes(batch) : TcCfg<64, 1, 64>::smem_bytes(batch);
+}
+
+int tc_ctas_per_sm(int head_dim, int rows_per_cta, int rows, int batch) {
   // Shared memory bounds residency (227 KB usable per SM); TMEM (512 columns) too.
-  const size_t smem = tc_smem_bytes(head_dim, rows_per_cta, batch);
+  const size_t smem = tc_smem_bytes(head_dim, rows_per_cta, rows, batch);
   int by_smem = static_cast<int>((227u * 1024u) / (smem + 1024));
   const bool two = rows_per_cta > 128;
   const int cols = static_cast<int>(
@@ -812,10 +830,14 @@ int tc_ctas_per_sm(int head_dim, int rows_per_cta, int batch) {
 
 cudaError_t launch_attn_tc(const spec_attn_args_t& a, const AttnPlan& P, char* ws,
                            cudaStream_t stream) {
-  const bool two = P.rows_per_cta > 128;
+  const TcVariant v = tc_variant(P.rows_per_cta, P.rows);
   if (a.head_dim == 128)
-    return two ? launch_typed<128, 2>(a, P, ws, stream) : launch_typed<128, 1>(a, P, ws, stream);
-  return two ? launch_typed<64, 2>(a, P, ws, stream) : launch_typed<64, 1>(a, P, ws, stream);
+    return v == kTwoTiles ? launch_typed<128, 2, 128>(a, P, ws, stream)
+           : v == kOneTile ? launch_typed<128, 1, 128>(a, P, ws, stream)
+                           : launch_typed<128, 1, 64>(a, P, ws, stream);
+  return v == kTwoTiles ? launch_typed<64, 2, 128>(a, P, ws, stream)
+         : v == kOneTile ? launch_typed<64, 1, 128>(a, P, ws, stream)
+                         : launch_typed<64, 1, 64>(a, P, ws, stream);
 }
 
 }  // namespace specv

@@ -228,8 +228,8 @@ struct DeviceScope {
   DeviceScope& operator=(const DeviceScope&) = delete;
 };
 
-int tc_ctas_per_sm(int head_dim, int rows_per_cta, int batch);
-size_t tc_smem_bytes(int head_dim, int rows_per_cta, int batch);
+int tc_ctas_per_sm(int head_dim, int rows_per_cta, int rows, int batch);
+size_t tc_smem_bytes(int head_dim, int rows_per_cta, int rows, int batch);
 constexpr int kTcMaxBatch = 4096;  // batch prefix sums live in shared memory
 
 }  // namespace specv
