@@ -42,19 +42,21 @@ L2_FLUSH_BYTES = 256 << 20
 # DRAM traffic of the dominant kernel from one ncu capture (dram__bytes_read.sum +
 # dram__bytes_write.sum per launch), keyed by (workload, kernel). It is reported only
 # while the kernel's sources still hash to what they were when the capture was taken.
+_ATTN_TC_SOURCES = {
+    "paper_2609_04010_gb300/csrc/attn_tc.cu":
+        "5eb43e061b102d671d64228bf3527ee2127c0cab52f91cc977f1dc7d38a9f622",
+    "paper_2609_04010_gb300/csrc/attn_common.cuh":
+        "f40099bd8694937bd15eea6be4daf2acfb32c854796d36687c536d36125785c5",
+    "paper_2609_04010_gb300/csrc/tc_ptx.cuh":
+        "454e6292796962dc5d99ba7b8ef616bc35d19cba2cd41ccd327ecc20bf78a970",
+}
 MEASURED_TRAFFIC = {
-    ("llama8b", "attention"): {
-        "bytes": 138_931_200,
-        "profile": "profiles/attn_tc_kernel_llama8b.md",
-        "sources": {
-            "paper_2609_04010_gb300/csrc/attn_tc.cu":
-                "6020780dbb93c56d1b611d8120783c54b7ebdba4990de33ec3256db3aa5ff4f6",
-            "paper_2609_04010_gb300/csrc/attn_common.cuh":
-                "fcccb38e95b02d314a545f1bc6bab2f21d76dea3e287ecd0ac3833d50a3798cc",
-            "paper_2609_04010_gb300/csrc/common.cuh":
-                "fb34291b5c1d1b7986c17ea7c68c55fcec41cefae83e63c137374784cb8cac46",
-        },
-    },
+    ("serve64", "attention"): {"bytes": 626_900_000,
+                               "profile": "profiles/attn_tc_kernel_serve64.md",
+                               "sources": _ATTN_TC_SOURCES},
+    ("long70b", "attention"): {"bytes": 548_180_000,
+                               "profile": "profiles/attn_tc_kernel_long70b.md",
+                               "sources": _ATTN_TC_SOURCES},
 }
 
 
@@ -531,7 +533,7 @@ def run_ours(args, wl, ai, ci, rank, world, local_rank):
     # the one filtered acceptance kernel
     launches_per_step = 2 if filtered else 4
     traffic, traffic_src = (None, None)
-    if dominant == "attention" and attn_path_name(args.attn_path, binding, ai).startswith("tensor"):
+    if dominant == "attention" and attn_path_name(args.attn_path, binding, ai) == "tensor cores, row tiles":
         traffic, traffic_src = measured_traffic(args.workload, "attention")
     result = {
         "metric": METRIC, "value": whole_job_tokens_per_s(world, B, G, ms), "unit": UNIT,
@@ -606,6 +608,9 @@ def time_other_workload(name, args, binding, dev, rank, graph_of, timed_loop, lo
     peak, peak_src = measured_peaks()
     step_gbs = tm["baseline"] / (ms["step"] / 1000.0) / 1e9
     attn_gbs = tm["kv"] / (ms["attention"] / 1000.0) / 1e9
+    traffic, traffic_src = (None, None)
+    if attn_path_name(args.attn_path, binding, ai) == "tensor cores, row tiles":
+        traffic, traffic_src = measured_traffic(name, "attention")
     emitted = int(S.ne.sum().item())
     res = {"ms_per_step": ms["step"],
            "value": whole_job_tokens_per_s(1, ci.batch, ci.gamma, ms["step"]), "unit": UNIT,
@@ -614,6 +619,7 @@ def time_other_workload(name, args, binding, dev, rank, graph_of, timed_loop, lo
            "attention_roofline": {"bound": "hbm", "achieved": round(attn_gbs, 1), "peak": peak,
                                   "unit": "GB/s", "frac": round(attn_gbs / peak, 4),
                                   "peak_source": peak_src,
+                                  "traffic": traffic, "traffic_source": traffic_src,
                                   "algorithmic_bytes_per_launch": int(tm["kv"]),
                                   "launch_ms": ms["attention"]},
            "step_roofline": {"bytes": int(tm["baseline"]), "strict_bytes": int(tm["strict"]),
