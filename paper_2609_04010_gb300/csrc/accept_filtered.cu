@@ -659,7 +659,54 @@ __global__ void __launch_bounds__(kRowThreads, 8) filter_row_kernel(FiltParams p
     const uint4* rv = reinterpret_cast<const uint4*>(rowp);
     uint32_t nacc = 0;
     if (vbeg + tid < vend) a = (vbeg + tid) * kEpv;  // a thread's first element starts its argmax
-    for (int v0 = vbeg; v0 < vend; v0 += kRowThreads * kRowUnroll) {
+    bool packed = false;
+    if constexpr (BF16) {
+      if (!greedy) {
+        // Sampled bf16 rows need only the lane maxima. Each thread folds each of its
+        // vectors to a bf16 pair by packed maxima, then the 8 threads of a lane trade
+        // halves in three shuffle rounds (bits 2, 1, 0 of the thread's index in its
+        // group), after which thread i of the group holds the maximum of the lane the
+        // group read in unroll step i: one conversion, key and shared atomic per lane
+        // instead of per vector. The maxima propagate NaNs, so one test per lane finds
+        // them.
+        static_assert(kRowUnroll == 8 && kGroup == 8, "one lane per thread of a group");
+        packed = true;
+        const int gi = tid & 7;
+        auto hmax = [](uint32_t x, uint32_t y) {
+          const __nv_bfloat162 r = __hmax2_nan(*reinterpret_cast<const __nv_bfloat162*>(&x),
+                                               *reinterpret_cast<const __nv_bfloat162*>(&y));
+          return *reinterpret_cast<const uint32_t*>(&r);
+        };
+        for (int v0 = vbeg; v0 < vend; v0 += kRowThreads * kRowUnroll) {
+          uint4 dv[kRowUnroll];
+#pragma unroll
+          for (int u = 0; u < kRowUnroll; ++u) {
+            const int vi = v0 + u * kRowThreads + tid;
+            dv[u] = vi < vend ? __ldg(rv + vi) : make_uint4(ninf, ninf, ninf, ninf);
+          }
+          uint32_t h[kRowUnroll];
+#pragma unroll
+          for (int u = 0; u < kRowUnroll; ++u) h[u] = hmax(hmax(dv[u].x, dv[u].y), hmax(dv[u].z, dv[u].w));
+#pragma unroll
+          for (int half = 4; half >= 1; half >>= 1) {
+            const bool up = (gi & half) != 0;
+#pragma unroll
+            for (int i = 0; i < half; ++i) {
+              const uint32_t send = up ? h[i] : h[i + half], keep = up ? h[i + half] : h[i];
+              h[i] = hmax(keep, __shfl_xor_sync(0xffffffffu, send, half));
+            }
+          }
+          const int vl = v0 + gi * kRowThreads + (tid & ~7);  // the owned lane's first vector here
+          if (vl < vend) {
+            nacc |= (h[0] & nan_mask) + nan_add;
+            const float lm = fmaxf(__uint_as_float(h[0] << 16), __uint_as_float(h[0] & 0xffff0000u));
+            m = fmaxf(m, lm);
+            atomicMax(&lanes[vl / vpl - l0], order_key(lm));
+          }
+        }
+      }
+    }
+    for (int v0 = packed ? vend : vbeg; v0 < vend; v0 += kRowThreads * kRowUnroll) {
       uint4 dv[kRowUnroll];
 #pragma unroll
       for (int u = 0; u < kRowUnroll; ++u) {

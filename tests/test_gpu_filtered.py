@@ -145,6 +145,32 @@ def test_bad_filter_parameters_flagged(oracle_mod):
     compare_accept(g, o, inp.gamma, skip={1, 2, 4, 5})
 
 
+def test_bad_logits_flagged(oracle_mod):
+    # NaN and +inf in bf16 rows read by the vectorised scan (vocabulary 30,000: a ragged
+    # last lane of 48 logits): a NaN in a sampled target row (inside a lane, and the very
+    # last logit), +inf in a tempered drafter row, a NaN in a greedy sequence's drafter
+    # row (never read) and in its target row (read).
+    B, gamma, V = 7, 4, 30000
+    T = [1.0, 1.0, 1.0, 1.0, 0.0, 1.0, 0.0]
+    inp = W.make_accept_inputs(B, gamma, V, "bf16", 3.0, 1.0, T, seed=16)
+    nan, inf = np.uint16(0x7FC0), np.uint16(0x7F80)
+    inp.target_logits[1, 3, 17] = nan
+    inp.target_logits[2, 0, V - 1] = nan
+    inp.drafter_logits[3, 1, 63] = inf
+    inp.drafter_logits[4, 2, 5] = nan   # greedy: the drafter row is not read
+    inp.target_logits[6, 1, 12345] = nan  # greedy: every target row is read
+    ws = binding.new_workspace(1 << 24)
+    g = gpu_filtered(inp, 50, 0.95, max_top_k=64, ws=ws)
+    code, flags = binding.read_device_status(ws)
+    assert flags & binding.FLAG_BAD_LOGITS
+    o = oracle_filtered(oracle_mod, inp, np.full(B, 50, np.int32), np.full(B, 0.95, np.float32))
+    assert [int(x != 0) for x in o["status"]] == [0, 1, 1, 1, 0, 0, 1]
+    for b in (1, 2, 3, 6):
+        assert g["num_accepted"][b] == -1 and g["num_emitted"][b] == 0
+        assert np.all(g["out_tokens"][b] == -1)
+    compare_accept(g, o, inp.gamma, skip={1, 2, 3, 6})
+
+
 def test_filter_off_matches_unfiltered_entry_point(oracle_mod):
     # k = vocab, top_p = 1: the filtered call must reproduce spec_accept_block
     inp = W.make_accept_inputs(16, 6, 1000, "bf16", 3.0, 1.0, [1.0, 0.0, 0.6], seed=15)
