@@ -352,13 +352,18 @@ class StepSetup:
         self.host_in, self.d, self.out, self.lse = host_in, d, out, lse
         self.na, self.ot, self.ne = na, ot, ne
         self.a, self.c, self.f, self.ws, self.filtered = a, c, (f if filtered else None), ws, filtered
+        # one workspace per call configuration: each lays its counters out differently
+        ws_attn = binding.new_workspace(binding.workspace_size(a, None), dev)
         if filtered:
+            ws_acc = binding.new_workspace(binding.filtered_workspace_size(c, f, None), dev)
             self.step = lambda: binding.verify_step_filtered_args(a, c, f, ws)
-            self.acc_only = lambda: binding.verify_step_filtered_args(None, c, f, ws)
+            self.acc_only = lambda: binding.verify_step_filtered_args(None, c, f, ws_acc)
         else:
+            ws_acc = binding.new_workspace(binding.workspace_size(None, c), dev)
             self.step = lambda: binding.verify_step_args(a, c, ws)
-            self.acc_only = lambda: binding.verify_step_args(None, c, ws)
-        self.attn_only = lambda: binding.verify_step_args(a, None, ws)
+            self.acc_only = lambda: binding.verify_step_args(None, c, ws_acc)
+        self.attn_only = lambda: binding.verify_step_args(a, None, ws_attn)
+        self.ws_attn, self.ws_acc = ws_attn, ws_acc
 
 
 def run_ours(args, wl, ai, ci, rank, world, local_rank):

@@ -31,7 +31,12 @@
  *   - `ws` is a caller-owned device workspace of at least spec_workspace_size()
  *     bytes, 256-byte aligned. A new workspace must be zero-filled once (e.g.
  *     spec_workspace_init); every call leaves its internal counters at zero again.
- *     Concurrent calls need distinct workspaces.
+ *     Concurrent calls need distinct workspaces. A workspace holds the counters of
+ *     one call configuration (the entry point, which of its parts are given, and
+ *     their sizes): calls of another configuration lay their scratch data out
+ *     differently and may leave non-zero words where this one keeps counters, so
+ *     give each configuration its own workspace, or zero-fill it again when
+ *     switching (CUDA graphs captured for different configurations included).
  *   - Host-side argument checks happen before any launch and return
  *     SPEC_ERR_INVALID_ARGUMENT / SPEC_ERR_UNSUPPORTED / SPEC_ERR_WORKSPACE_TOO_SMALL
  *     without touching the device. Launch failures return SPEC_ERR_CUDA.
