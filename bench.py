@@ -36,6 +36,7 @@ METRIC = "verify-step tokens/s on 1 GB300; achieved HBM GB/s as fraction of ~8 T
 UNIT = "tokens/s"
 NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
+FALLBACK_BF16_TFLOPS = 1900.0  # burst bf16 dense, the same earlier measurement
 L2_FLUSH_BYTES = 256 << 20
 
 
@@ -115,6 +116,17 @@ def measured_peaks():
         return float(d["hbm_gbs"]), "measured"
     except Exception:
         return FALLBACK_HBM_GBS, "fallback"
+
+
+def measured_bf16_tflops():
+    """The burst bf16 tensor peak (TFLOP/s) and its source."""
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["bf16_tflops"]), "measured"
+    except Exception:
+        return FALLBACK_BF16_TFLOPS, "fallback"
 
 
 # ----------------------------------------------------------------------------------
@@ -669,14 +681,25 @@ def time_lm_head(ai, ci, binding, dev, graph_of, timed_loop, n):
     if code != 0:
         raise RuntimeError(f"lm head: device status {code} flags {flags}")
     nbytes = (V + R) * H * 2
-    peak = measured_peaks()[0]
+    flops = 2.0 * R * H * V
+    peak, psrc = measured_peaks()
+    tpeak, tsrc = measured_bf16_tflops()
     gbs = nbytes / (ms / 1000.0) / 1e9
+    tflops = flops / (ms / 1000.0) / 1e12
+    # the roofline that binds: the weight stream (few rows) or the tensor pipe (many)
+    tensor_bound = flops / (tpeak * 1e12) > nbytes / (peak * 1e9)
     del weight
     torch.cuda.empty_cache()
     return {"shape": {"rows": R, "hidden": H, "vocab": V},
             "lm_head_ms": ms, "algorithmic_bytes": int(nbytes), "achieved_gbs": round(gbs, 1),
             "frac_of_measured": round(gbs / peak, 4),
-            "useful_tflops": round(2.0 * R * H * V / (ms / 1000.0) / 1e12, 1),
+            "useful_tflops": round(tflops, 1),
+            "roofline": {"bound": "tensor" if tensor_bound else "hbm",
+                         "achieved": round(tflops if tensor_bound else gbs, 1),
+                         "peak": tpeak if tensor_bound else peak,
+                         "unit": "TFLOP/s" if tensor_bound else "GB/s",
+                         "frac": round((tflops / tpeak) if tensor_bound else (gbs / peak), 4),
+                         "peak_source": tsrc if tensor_bound else psrc},
             "timing": "CUDA-graph replays of spec_lm_head_stats, L2 flushed before each"}
 
 

@@ -10,7 +10,9 @@
 // from the root. Greedy: to the child whose token is the current node's argmax.
 // Sampled: the children are tried in node order as point-mass proposals (accepted iff
 // u <= p'(token), p' without the siblings rejected before), decided in fp64 from the
-// gathered logits; after the last rejection the block draws the final token from p' by
+// gathered logits (every node's weight under its parent's row and its earlier siblings'
+// weight are taken once, before the walk, so a step is a shuffle, a division and two
+// ballots); after the last rejection the block draws the final token from p' by
 // inverse CDF: the part where the remaining mass crosses u x total, from the stored part
 // sums minus the rejected tokens' weights, then one pass over that part.
 //
@@ -103,7 +105,8 @@ __global__ void __launch_bounds__(kThreads, kTreeBlocksPerSm) tree_greedy_kernel
   __shared__ int s_final, s_len, s_nrm, s_kcross, s_tok;
   __shared__ int s_rm[64];                 // tokens rejected at the final node, ascending
   __shared__ float s_rmw[64];              // their weights 2^((l - M) log2e / T)
-  __shared__ double s_target, s_dsum[kThreads / 32], s_mass[kFiltMaxSplits];
+  __shared__ int s_rmk[64];                // their parts of the row
+  __shared__ double s_target, s_dsum[kThreads / 32];
   const int split = blockIdx.x, j = blockIdx.y, b = blockIdx.z, tid = threadIdx.x;
   const int N = p.nodes, V = p.vocab;
   const int64_t rid = static_cast<int64_t>(b) * N + j;
@@ -340,34 +343,57 @@ __global__ void __launch_bounds__(kThreads, kTreeBlocksPerSm) tree_greedy_kernel
       } else {
         // sampled walk: the children of the current node, in node order, are point-mass
         // proposals; child c is accepted iff u[c] <= p'(token), p' the node's target
-        // distribution without the tokens of the siblings rejected before it
-        const float* u = p.uniforms + brow;
+        // distribution without the tokens of the siblings rejected before it.
+        // Everything a step reads is fixed by the tree, so it is gathered once, for all
+        // nodes at the same time: each node's weight e_c = exp((l(t_c) - M) / T) in fp64
+        // under its parent's row (M that row's maximum; 0 for a repeated sibling token,
+        // removed with its first occurrence), the weight of its earlier siblings in node
+        // order, its own row's (maximum, sum) and its uniform.
         const char* tbase = static_cast<const char*>(p.target);
+        const size_t rbytes = static_cast<size_t>(V) * (BF16 ? 2 : 4);
+        double e[2];
+        float2 own[2];
+        float uu[2];
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const int c = lane + 32 * h;
+          own[h] = c < N ? __ldcg(p.rowstat + brow + c) : make_float2(0.f, 0.f);
+          uu[h] = c < N ? p.uniforms[brow + c] : 1.f;
+          e[h] = 0.0;
+        }
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const int c = lane + 32 * h;
+          if (c >= 1 && c < N) {
+            const float2 prs = __ldcg(p.rowstat + brow + par[h]);
+            const float x = load_elem<BF16>(tbase + (brow + par[h]) * rbytes, tok[h]);
+            e[h] = exp((static_cast<double>(x) - prs.x) / static_cast<double>(T));
+          }
+        }
+        bool dup[2] = {false, false};
+        for (int o = 0; o < 64; ++o) {
+          const int t_o = __shfl_sync(0xffffffffu, o < 32 ? tok[0] : tok[1], o & 31);
+          const int p_o = __shfl_sync(0xffffffffu, o < 32 ? par[0] : par[1], o & 31);
+#pragma unroll
+          for (int h = 0; h < 2; ++h) dup[h] |= o < lane + 32 * h && p_o == par[h] && t_o == tok[h];
+        }
+        int live[2];  // a proposal with weight (not a repeat)
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          if (dup[h]) e[h] = 0.0;
+          live[h] = e[h] > 0.0 ? 1 : 0;
+        }
         for (int step = 1; step <= N; ++step) {
-          const float2 rs = __ldcg(p.rowstat + brow + cur);
-          const char* crow = tbase + (brow + cur) * V * (BF16 ? 2 : 4);
-          double e[2];
-          bool ch[2];
+          const float s_cur = __shfl_sync(0xffffffffu, cur < 32 ? own[0].y : own[1].y, cur & 31);
+          bool ch[2], acc[2];
+          double w[2];
 #pragma unroll
           for (int h = 0; h < 2; ++h) {
             ch[h] = par[h] == cur;
-            e[h] = ch[h] ? exp((static_cast<double>(load_elem<BF16>(crow, tok[h])) - rs.x) /
-                               static_cast<double>(T))
-                         : 0.0;
-          }
-          // a repeated sibling token was removed with its first occurrence: probability 0
-#pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            bool dup = false;
-            for (int o = 0; o < 64; ++o) {
-              const int t_o = __shfl_sync(0xffffffffu, o < 32 ? tok[0] : tok[1], o & 31);
-              const int p_o = __shfl_sync(0xffffffffu, o < 32 ? par[0] : par[1], o & 31);
-              dup |= o < lane + 32 * h && p_o == cur && t_o == tok[h];
-            }
-            if (dup) e[h] = 0.0;
+            w[h] = ch[h] ? e[h] : 0.0;
           }
           // mass removed before each child: exclusive prefix over node order
-          double inc0 = e[0], inc1 = e[1];
+          double inc0 = w[0], inc1 = w[1];
 #pragma unroll
           for (int o = 1; o < 32; o <<= 1) {
             const double y0 = __shfl_up_sync(0xffffffffu, inc0, o);
@@ -375,13 +401,12 @@ __global__ void __launch_bounds__(kThreads, kTreeBlocksPerSm) tree_greedy_kernel
             if (lane >= o) { inc0 += y0; inc1 += y1; }
           }
           const double tot0 = __shfl_sync(0xffffffffu, inc0, 31);
-          const double ex0 = inc0 - e[0], ex1 = tot0 + inc1 - e[1];
-          bool acc[2];
+          const double ex0 = inc0 - w[0], ex1 = tot0 + inc1 - w[1];
 #pragma unroll
           for (int h = 0; h < 2; ++h) {
-            const double S = static_cast<double>(rs.y) - (h == 0 ? ex0 : ex1);
-            acc[h] = ch[h] && e[h] > 0.0 &&
-                     (S <= e[h] || static_cast<double>(u[lane + 32 * h]) <= e[h] / S);
+            const double S = static_cast<double>(s_cur) - (h == 0 ? ex0 : ex1);
+            acc[h] = ch[h] && live[h] &&
+                     (S <= w[h] || static_cast<double>(uu[h]) <= w[h] / S);
           }
           const unsigned m0 = __ballot_sync(0xffffffffu, acc[0]);
           const unsigned m1 = __ballot_sync(0xffffffffu, acc[1]);
@@ -398,26 +423,33 @@ __global__ void __launch_bounds__(kThreads, kTreeBlocksPerSm) tree_greedy_kernel
             ++len;
             continue;
           }
+          const float m_cur = __shfl_sync(0xffffffffu, cur < 32 ? own[0].x : own[1].x, cur & 31);
+          const char* crow = tbase + (brow + cur) * rbytes;
           // every child rejected: hand the final node and its rejected tokens (ascending,
           // with their weights relative to the row maximum) to the whole block
+          float wrm[2];
 #pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            const bool mine = ch[h] && e[h] > 0.0;
-            int rank = 0;
-            for (int o = 0; o < 64; ++o) {
-              const int t_o = __shfl_sync(0xffffffffu, o < 32 ? tok[0] : tok[1], o & 31);
-              const int p_o = __shfl_sync(0xffffffffu, o < 32 ? par[0] : par[1], o & 31);
-              const double e_o = __shfl_sync(0xffffffffu, o < 32 ? e[0] : e[1], o & 31);
-              const bool in = p_o == cur && e_o > 0.0;
-              rank += in && (t_o < tok[h] || (t_o == tok[h] && o < lane + 32 * h));
-            }
-            if (mine) {
-              s_rm[rank] = tok[h];
-              s_rmw[rank] = rel_weight(load_elem<BF16>(crow, tok[h]), rs.x, cs);
-            }
+          for (int h = 0; h < 2; ++h)
+            wrm[h] = ch[h] && live[h] ? rel_weight(load_elem<BF16>(crow, tok[h]), m_cur, cs) : 0.f;
+          int rank[2] = {0, 0};
+          for (int o = 0; o < 64; ++o) {
+            const int t_o = __shfl_sync(0xffffffffu, o < 32 ? tok[0] : tok[1], o & 31);
+            const int p_o = __shfl_sync(0xffffffffu, o < 32 ? par[0] : par[1], o & 31);
+            const int l_o = __shfl_sync(0xffffffffu, o < 32 ? live[0] : live[1], o & 31);
+            const bool in = p_o == cur && l_o;
+#pragma unroll
+            for (int h = 0; h < 2; ++h)
+              rank[h] += in && (t_o < tok[h] || (t_o == tok[h] && o < lane + 32 * h));
           }
-          const int nrm = __popc(__ballot_sync(0xffffffffu, ch[0] && e[0] > 0.0)) +
-                          __popc(__ballot_sync(0xffffffffu, ch[1] && e[1] > 0.0));
+#pragma unroll
+          for (int h = 0; h < 2; ++h)
+            if (ch[h] && live[h]) {
+              s_rm[rank[h]] = tok[h];
+              s_rmw[rank[h]] = wrm[h];
+              s_rmk[rank[h]] = tok[h] / p.elems_per_split;
+            }
+          const int nrm = __popc(__ballot_sync(0xffffffffu, ch[0] && live[0])) +
+                          __popc(__ballot_sync(0xffffffffu, ch[1] && live[1]));
           if (lane == 0) {
             s_final = cur;
             s_len = len;
@@ -437,43 +469,49 @@ __global__ void __launch_bounds__(kThreads, kTreeBlocksPerSm) tree_greedy_kernel
   const int64_t frid = brow + fin;
   const float M = __ldcg(p.rowstat + frid).x;
   const int eps = p.elems_per_split;
-  if (tid == 0) {
+  if (tid < 32) {
     // remaining mass of each part (its sum minus its rejected tokens' weights), the total,
-    // and the part where the cumulative mass reaches u[0] x total
-    double* mass = s_mass;
-    double S = 0.0;
-    for (int pass = 0; pass < 2 && !(S > 0.0); ++pass) {
-      for (int k = 0; k < p.splits; ++k) {
-        const uint4 q = __ldcg(p.parts + frid * p.splits + k);
-        mass[k] = static_cast<double>(__uint_as_float(q.w)) * rel_weight(key_to_float(q.y), M, cs);
-      }
-      if (pass == 0) {
-        for (int r = 0; r < nrm; ++r) mass[s_rm[r] / eps] -= static_cast<double>(s_rmw[r]);
-      } else {
-        s_nrm = 0;  // nothing left after the removals (rounding only): draw from p itself
-      }
-      S = 0.0;
-      for (int k = 0; k < p.splits; ++k) {
-        if (mass[k] < 0.0) mass[k] = 0.0;
-        S += mass[k];
-      }
+    // and the part where the cumulative mass reaches u[0] x total: one part per lane
+    // (at most kFiltMaxSplits parts)
+    const int k = tid;
+    double base = 0.0;
+    if (k < p.splits) {
+      const uint4 q = __ldcg(p.parts + frid * p.splits + k);
+      base = static_cast<double>(__uint_as_float(q.w)) * rel_weight(key_to_float(q.y), M, cs);
+    }
+    double removed = 0.0;
+    for (int r = 0; r < nrm; ++r)
+      if (s_rmk[r] == k) removed += static_cast<double>(s_rmw[r]);
+    double mass = base - removed;
+    if (mass < 0.0) mass = 0.0;
+    double S = mass;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) S += __shfl_xor_sync(0xffffffffu, S, o);
+    if (!(S > 0.0)) {
+      // nothing left after the removals (rounding only): draw from p itself
+      mass = base;
+      S = mass;
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) S += __shfl_xor_sync(0xffffffffu, S, o);
+      if (k == 0) s_nrm = 0;
     }
     const double target = static_cast<double>(p.uniforms[brow]) * S;
-    int kc = -1;
-    double before = 0.0, C = 0.0;
-    for (int k = 0; k < p.splits; ++k) {
-      if (mass[k] > 0.0 && C + mass[k] >= target) { kc = k; before = C; break; }
-      C += mass[k];
+    double incl = mass;  // inclusive prefix over parts
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const double y = __shfl_up_sync(0xffffffffu, incl, o);
+      if (k >= o) incl += y;
     }
-    if (kc < 0) {  // rounding left the target above the total: the last part with mass
-      C = 0.0;
-      for (int k = 0; k < p.splits; ++k) {
-        if (mass[k] > 0.0) { kc = k; before = C; }
-        C += mass[k];
-      }
+    const double excl = incl - mass;
+    const unsigned hit = __ballot_sync(0xffffffffu, mass > 0.0 && incl >= target);
+    // rounding may leave the target above the total: then the last part with mass
+    const unsigned pos = __ballot_sync(0xffffffffu, mass > 0.0);
+    const int kc = hit ? __ffs(hit) - 1 : (pos ? 31 - __clz(pos) : -1);
+    const double before = __shfl_sync(0xffffffffu, excl, kc < 0 ? 0 : kc);
+    if (k == 0) {
+      s_kcross = kc < 0 ? 0 : kc;  // the part of the row maximum always has mass
+      s_target = target - before;
     }
-    s_kcross = kc < 0 ? 0 : kc;  // the part of the row maximum always has mass
-    s_target = target - before;
   }
   __syncthreads();
   const int kc = s_kcross, nrm_scan = s_nrm;
@@ -485,15 +523,50 @@ __global__ void __launch_bounds__(kThreads, kTreeBlocksPerSm) tree_greedy_kernel
   const char* frow = static_cast<const char*>(p.target) + frid * V * (BF16 ? 2 : 4);
   int ptr = 0;
   while (ptr < nrm_scan && s_rm[ptr] < lo) ++ptr;
-  auto weight_at = [&](int x, int& q) {
-    bool removed = false;
-    while (q < nrm_scan && s_rm[q] <= x) { removed |= s_rm[q] == x; ++q; }
-    return removed ? 0.f : rel_weight(load_elem<BF16>(frow, x), M, cs);
+  // The run is read kChunk elements at a time, all of a chunk's loads issued before any
+  // is used (16-byte vectors when the rows allow: a run starts on a multiple of 8
+  // elements, and hi is a multiple of the vector's elements).
+  constexpr int kChunk = 16;
+  auto load_chunk = [&](int x0, float* lv) {
+    if (VEC) {
+      constexpr int kEpv = BF16 ? 8 : 4;
+#pragma unroll
+      for (int v = 0; v < kChunk / kEpv; ++v) {
+        const int x = x0 + v * kEpv;
+        uint4 raw = make_uint4(0u, 0u, 0u, 0u);
+        if (x < hi) raw = __ldg(reinterpret_cast<const uint4*>(frow + static_cast<int64_t>(x) * (BF16 ? 2 : 4)));
+        const uint32_t wv[4] = {raw.x, raw.y, raw.z, raw.w};
+#pragma unroll
+        for (int q = 0; q < kEpv; ++q)
+          lv[v * kEpv + q] = BF16 ? __uint_as_float((q & 1) ? (wv[q >> 1] & 0xffff0000u) : (wv[q >> 1] << 16))
+                                  : __uint_as_float(wv[q]);
+      }
+    } else {
+#pragma unroll
+      for (int i = 0; i < kChunk; ++i) lv[i] = x0 + i < hi ? load_elem<BF16>(frow, x0 + i) : 0.f;
+    }
+  };
+  // The weight of element x from its logit l, 0 for a removed token. Elements come in
+  // ascending order and the removed tokens are distinct and ascending, so the next one is
+  // kept in a register.
+  auto weight_of = [&](int x, float l, int& q, int& next_rm) {
+    if (x == next_rm) {
+      ++q;
+      next_rm = q < nrm_scan ? s_rm[q] : INT_MAX;
+      return 0.f;
+    }
+    return rel_weight(l, M, cs);
   };
   float run = 0.f;
   {
-    int q = ptr;
-    for (int x = lo; x < hi; ++x) run += weight_at(x, q);
+    int q = ptr, next_rm = ptr < nrm_scan ? s_rm[ptr] : INT_MAX;
+    for (int x0 = lo; x0 < hi; x0 += kChunk) {
+      float lv[kChunk];
+      load_chunk(x0, lv);
+#pragma unroll
+      for (int i = 0; i < kChunk; ++i)
+        if (x0 + i < hi) run += weight_of(x0 + i, lv[i], q, next_rm);
+    }
   }
   // block exclusive scan of the runs' sums; the run that holds the crossing is the last
   // one with weight whose exclusive prefix is below the target
@@ -522,13 +595,18 @@ __global__ void __launch_bounds__(kThreads, kTreeBlocksPerSm) tree_greedy_kernel
     // walk the run: the first token whose cumulative weight reaches the target, else (if
     // rounding leaves the target above the run) its last positive-weight token
     double C = excl;
-    int q = ptr, pick = -1;
-    for (int x = lo; x < hi; ++x) {
-      const float w = weight_at(x, q);
-      C += static_cast<double>(w);
-      if (w > 0.f) {
-        pick = x;
-        if (C >= tin) break;
+    int q = ptr, next_rm = ptr < nrm_scan ? s_rm[ptr] : INT_MAX, pick = -1;
+    bool done = false;
+    for (int x0 = lo; x0 < hi && !done; x0 += kChunk) {
+      float lv[kChunk];
+      load_chunk(x0, lv);
+      for (int i = 0; i < kChunk && !done && x0 + i < hi; ++i) {
+        const float w = weight_of(x0 + i, lv[i], q, next_rm);
+        C += static_cast<double>(w);
+        if (w > 0.f) {
+          pick = x0 + i;
+          done = C >= tin;
+        }
       }
     }
     s_tok = pick;
