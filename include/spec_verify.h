@@ -527,6 +527,27 @@ spec_status_t spec_lm_head_stats(const spec_lm_head_args_t* lm, void* ws, size_t
 #define SPEC_NOALLOC_SCRATCH_BYTES (4u << 20)
 spec_status_t spec_accept_block_noalloc(const spec_accept_args_t* accept, spec_stream_t stream);
 
+/* ---------------------------------------------------------------------------------------
+ * Test hooks for the timeout path (not part of the verify step)
+ *
+ * The kernels' internal waits on asynchronous copies and tensor-core operations are
+ * bounded (about 1 s of SM clock); one that runs out sets SPEC_FLAG_TIMEOUT, the block
+ * releases its resources and returns, and the context stays usable. These two calls make
+ * that happen on purpose, so that it can be tested: each is the launch of its product
+ * call (spec_verify_attention on the tensor-core row-tile path, spec_lm_head_stats), with
+ * the same arguments, workspace rules and errors, except that the kernel's copy producer
+ * issues nothing, so every consumer's wait runs out (about 1 s). Afterwards the workspace
+ * status word holds SPEC_FLAG_TIMEOUT (spec_read_device_status returns
+ * SPEC_ERR_TIMEOUT and clears it), the outputs are undefined, and the workspace's
+ * counters are still zero, so the same workspace serves the next product call.
+ * spec_test_attention_wait_timeout returns SPEC_ERR_UNSUPPORTED for shapes the
+ * tensor-core row-tile kernel does not take. Nothing traps, faults or waits without bound.
+ * ------------------------------------------------------------------------------------- */
+spec_status_t spec_test_attention_wait_timeout(const spec_attn_args_t* attn, void* ws,
+                                               size_t ws_bytes, spec_stream_t stream);
+spec_status_t spec_test_lm_head_wait_timeout(const spec_lm_head_args_t* lm, void* ws,
+                                             size_t ws_bytes, spec_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -181,6 +181,9 @@ def lib(build_if_missing: bool = True):
             L.spec_tree_build_workspace_size.restype = ctypes.c_size_t
             L.spec_build_tree.argtypes = [P, P, ctypes.c_size_t, P]
             L.spec_build_tree.restype = ctypes.c_int
+            for f in ("spec_test_attention_wait_timeout", "spec_test_lm_head_wait_timeout"):
+                getattr(L, f).argtypes = [P, P, ctypes.c_size_t, P]
+                getattr(L, f).restype = ctypes.c_int
             for f in ("spec_workspace_init", "spec_verify_attention", "spec_accept_block",
                       "spec_verify_step", "spec_philox_uniforms", "spec_read_device_status"):
                 getattr(L, f).restype = ctypes.c_int
@@ -277,6 +280,14 @@ def new_workspace(nbytes: int, device=None) -> torch.Tensor:
 def verify_attention_args(attn: AttnArgs, ws: torch.Tensor, stream=None):
     _raise(lib().spec_verify_attention(ctypes.byref(attn), _ptr(ws), ws.numel(), _stream(stream)),
            "spec_verify_attention")
+
+
+def test_attention_wait_timeout_args(attn: AttnArgs, ws: torch.Tensor, stream=None):
+    """Test hook: spec_verify_attention on the tensor-core row-tile path with its copy
+    producers idle, so that the kernel's bounded waits run out (about 1 s) and it returns
+    with SPEC_FLAG_TIMEOUT set."""
+    _raise(lib().spec_test_attention_wait_timeout(ctypes.byref(attn), _ptr(ws), ws.numel(),
+                                                  _stream(stream)), "spec_test_attention_wait_timeout")
 
 
 def accept_block_args(acc: AcceptArgs, ws: torch.Tensor, stream=None):
@@ -626,6 +637,13 @@ def lm_head_workspace_size(a: LmHeadArgs) -> int:
 def lm_head_stats_args(a: LmHeadArgs, ws: torch.Tensor, stream=None):
     _raise(lib().spec_lm_head_stats(ctypes.byref(a), _ptr(ws), ws.numel(), _stream(stream)),
            "spec_lm_head_stats")
+
+
+def test_lm_head_wait_timeout_args(a: LmHeadArgs, ws: torch.Tensor, stream=None):
+    """Test hook: spec_lm_head_stats with its copy producer idle, so that the kernel's
+    bounded waits run out (about 1 s) and it returns with SPEC_FLAG_TIMEOUT set."""
+    _raise(lib().spec_test_lm_head_wait_timeout(ctypes.byref(a), _ptr(ws), ws.numel(),
+                                                _stream(stream)), "spec_test_lm_head_wait_timeout")
 
 
 def lm_head_stats(hidden_states, weight, temperature, rows_per_seq: int, tokens=None,

@@ -472,6 +472,26 @@ spec_status_t spec_accept_block(const spec_accept_args_t* accept, void* ws, size
   return run(nullptr, accept, nullptr, ws, ws_bytes, stream);
 }
 
+spec_status_t spec_test_attention_wait_timeout(const spec_attn_args_t* attn, void* ws,
+                                               size_t ws_bytes, spec_stream_t stream_) {
+  if (!attn) return SPEC_ERR_INVALID_ARGUMENT;
+  const spec_status_t st = check_attn(attn);
+  if (st != SPEC_OK) return st;
+  if (!ws || (reinterpret_cast<uintptr_t>(ws) % kWsAlign) != 0) return SPEC_ERR_INVALID_ARGUMENT;
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  DeviceScope scope(stream);
+  if (!scope.ok) return SPEC_ERR_CUDA;
+  (void)cudaGetLastError();
+  size_t attn_base = 0;
+  if (required_bytes(attn, nullptr, nullptr, scope.sms, &attn_base) > ws_bytes)
+    return SPEC_ERR_WORKSPACE_TOO_SMALL;
+  const AttnPlan P = attn_plan(*attn, attn_base, scope.sms, SPEC_ATTN_TENSOR_CORES);
+  if (P.path != SPEC_ATTN_TENSOR_CORES || P.keys_on_lanes) return SPEC_ERR_UNSUPPORTED;
+  return launch_attn_tc(*attn, P, static_cast<char*>(ws), stream, /*starve=*/true) == cudaSuccess
+             ? SPEC_OK
+             : SPEC_ERR_CUDA;
+}
+
 spec_status_t spec_verify_step(const spec_attn_args_t* attn, const spec_accept_args_t* accept,
                                void* ws, size_t ws_bytes, spec_stream_t stream) {
   return run(attn, accept, nullptr, ws, ws_bytes, stream);
@@ -641,6 +661,21 @@ spec_status_t spec_lm_head_stats(const spec_lm_head_args_t* a, void* ws, size_t 
   DeviceScope scope(stream);
   if (!scope.ok) return SPEC_ERR_CUDA;
   return launch_lm_head(*a, L, static_cast<char*>(ws), stream) == cudaSuccess ? SPEC_OK : SPEC_ERR_CUDA;
+}
+
+spec_status_t spec_test_lm_head_wait_timeout(const spec_lm_head_args_t* a, void* ws,
+                                             size_t ws_bytes, spec_stream_t stream_) {
+  const spec_status_t st = check_lm_head(a);
+  if (st != SPEC_OK) return st;
+  if (!ws || (reinterpret_cast<uintptr_t>(ws) % kWsAlign) != 0) return SPEC_ERR_INVALID_ARGUMENT;
+  const LmLayout L = lm_layout(*a, kWsHeader);
+  if (L.end > ws_bytes) return SPEC_ERR_WORKSPACE_TOO_SMALL;
+  cudaStream_t stream = reinterpret_cast<cudaStream_t>(stream_);
+  DeviceScope scope(stream);
+  if (!scope.ok) return SPEC_ERR_CUDA;
+  return launch_lm_head(*a, L, static_cast<char*>(ws), stream, /*starve=*/true) == cudaSuccess
+             ? SPEC_OK
+             : SPEC_ERR_CUDA;
 }
 
 spec_status_t spec_commit_tree_kv(const spec_tree_commit_args_t* c, spec_stream_t stream) {

@@ -34,6 +34,7 @@ struct AttnParams {
   int q_tma;           // tensor-core kernel: Q tiles arrive by TMA (else softmax warps load them)
   int unit_overhead;   // tensor-core kernel: tiles charged per unit start in the work list
   const uint64_t* tree_mask;  // [batch][gamma] block keys each query sees, or NULL (causal)
+  int starve;  // test hook: the producers issue no copies, so the consumers' waits run out
 };
 
 inline AttnParams make_attn_params(const spec_attn_args_t& a, const AttnPlan& P, char* ws) {
@@ -69,6 +70,7 @@ inline AttnParams make_attn_params(const spec_attn_args_t& a, const AttnPlan& P,
   p.q_tma = 0;
   p.unit_overhead = 0;
   p.tree_mask = a.tree_mask;
+  p.starve = 0;
   return p;
 }
 

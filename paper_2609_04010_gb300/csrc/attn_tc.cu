@@ -263,7 +263,7 @@ __global__ void __launch_bounds__(TcCfg<D, MT, QR>::THREADS, 1)
     };
     const uint32_t box_bytes = static_cast<uint32_t>(p.page_size) * D * 2;  // one page of one head
     uint32_t seg_no = 0;
-    for (Seg s = locate<TK>(t0, t1, p, pb, OVH); s.ntile > 0 && ok; ++seg_no) {
+    for (Seg s = locate<TK>(t0, t1, p, pb, OVH); s.ntile > 0 && ok && !p.starve; ++seg_no) {
       const bool bad = !s.len_ok;  // nothing to read
       bool flag = bad;             // ... or a page id out of range (read as page 0)
       for (int k = 0; k < s.ntile && ok; ++k, ++it) {
@@ -732,12 +732,13 @@ __global__ void __launch_bounds__(TcCfg<D, MT, QR>::THREADS, 1)
 // ---------------------------------------------------------------------------------
 template <int D, int MT, int QR>
 cudaError_t launch_typed(const spec_attn_args_t& a, const AttnPlan& P, char* ws,
-                         cudaStream_t stream) {
+                         cudaStream_t stream, bool starve) {
   using Cf = TcCfg<D, MT, QR>;
   CUtensorMap mk, mv, mq;
   if (!encode_cache_map(&mk, a.k_cache, a) || !encode_cache_map(&mv, a.v_cache, a))
     return cudaErrorInvalidValue;
   AttnParams p = make_attn_params(a, P, ws);
+  p.starve = starve ? 1 : 0;
   p.q_tma = encode_q_map(&mq, a, QR) ? 1 : 0;
   // Charge unit starts only when blocks hold several of them; when every unit is spread
   // over several blocks, a block holds at most one start and the charge would mostly
@@ -829,15 +830,15 @@ int tc_ctas_per_sm(int head_dim, int rows_per_cta, int rows, int batch) {
 }
 
 cudaError_t launch_attn_tc(const spec_attn_args_t& a, const AttnPlan& P, char* ws,
-                           cudaStream_t stream) {
+                           cudaStream_t stream, bool starve) {
   const TcVariant v = tc_variant(P.rows_per_cta, P.rows);
   if (a.head_dim == 128)
-    return v == kTwoTiles ? launch_typed<128, 2, 128>(a, P, ws, stream)
-           : v == kOneTile ? launch_typed<128, 1, 128>(a, P, ws, stream)
-                           : launch_typed<128, 1, 64>(a, P, ws, stream);
-  return v == kTwoTiles ? launch_typed<64, 2, 128>(a, P, ws, stream)
-         : v == kOneTile ? launch_typed<64, 1, 128>(a, P, ws, stream)
-                         : launch_typed<64, 1, 64>(a, P, ws, stream);
+    return v == kTwoTiles ? launch_typed<128, 2, 128>(a, P, ws, stream, starve)
+           : v == kOneTile ? launch_typed<128, 1, 128>(a, P, ws, stream, starve)
+                           : launch_typed<128, 1, 64>(a, P, ws, stream, starve);
+  return v == kTwoTiles ? launch_typed<64, 2, 128>(a, P, ws, stream, starve)
+         : v == kOneTile ? launch_typed<64, 1, 128>(a, P, ws, stream, starve)
+                         : launch_typed<64, 1, 64>(a, P, ws, stream, starve);
 }
 
 }  // namespace specv

@@ -169,8 +169,10 @@ cudaError_t launch_accept_filtered(const spec_accept_args_t& a, const spec_filte
                                    float* draw_q = nullptr);
 cudaError_t launch_attn_simt(const spec_attn_args_t& a, const AttnPlan& P, char* ws,
                              cudaStream_t stream);
+// starve (test hook only): the kernel's producers issue no copies, so its bounded waits
+// run out and it returns with SPEC_FLAG_TIMEOUT set.
 cudaError_t launch_attn_tc(const spec_attn_args_t& a, const AttnPlan& P, char* ws,
-                           cudaStream_t stream);
+                           cudaStream_t stream, bool starve = false);
 cudaError_t launch_attn_kl(const spec_attn_args_t& a, const AttnPlan& P, char* ws,
                            cudaStream_t stream);
 cudaError_t launch_philox(uint64_t seed, uint64_t offset, int64_t n, float* out, cudaStream_t s);

@@ -66,6 +66,7 @@ struct LmParams {
   float* row_sum;
   int32_t* row_argmax;
   float* token_logit;
+  int starve;  // test hook: the producer issues no copies, so the MMA warp's waits run out
 };
 
 __device__ __forceinline__ float row_c2(const LmParams& p, int row) {
@@ -126,7 +127,7 @@ __global__ void __launch_bounds__(kThreads)
     if (lane == 0) {
       int k = 0;
       bool ok = true;
-      for (; k < p.nk; ++k) {
+      for (; k < p.nk && !p.starve; ++k) {
         const int s = k % kStages;
         if (k >= kStages) ok = mbar_wait(empty(s), ((k / kStages) - 1) & 1, abort_flag, p.status);
         if (!ok) break;
@@ -281,7 +282,7 @@ __global__ void __launch_bounds__(128) lm_merge_kernel(LmParams p) {
 }  // namespace
 
 cudaError_t launch_lm_head(const spec_lm_head_args_t& a, const LmLayout& L, char* ws,
-                           cudaStream_t stream) {
+                           cudaStream_t stream, bool starve) {
   CUtensorMap mh, mw;
   if (!encode_rows_map(&mh, a.hidden_states, a.rows, a.hidden, kLmTileM) ||
       !encode_rows_map(&mw, a.weight, a.vocab, a.hidden, kLmTileN))
@@ -302,6 +303,7 @@ cudaError_t launch_lm_head(const spec_lm_head_args_t& a, const LmLayout& L, char
   p.row_sum = a.row_sum;
   p.row_argmax = a.row_argmax;
   p.token_logit = a.token_logit;
+  p.starve = starve ? 1 : 0;
   (void)cudaGetLastError();
   cudaError_t e = cudaFuncSetAttribute(lm_head_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(kSmem));

@@ -13,7 +13,9 @@ struct LmLayout {
   int ntiles_n, ntiles_m;
 };
 LmLayout lm_layout(const spec_lm_head_args_t& a, size_t base);
+// starve (test hook only): the producer issues no copies, so the kernel's bounded waits
+// run out and it returns with SPEC_FLAG_TIMEOUT set (outputs undefined).
 cudaError_t launch_lm_head(const spec_lm_head_args_t& a, const LmLayout& L, char* ws,
-                           cudaStream_t stream);
+                           cudaStream_t stream, bool starve = false);
 
 }  // namespace specv
