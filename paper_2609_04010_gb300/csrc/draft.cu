@@ -176,9 +176,9 @@ __global__ void __launch_bounds__(kThreads, 8) draft_sample_kernel(DraftParams p
         for (int q = 0; q < kEpv; ++q)
           x[q] = BF16 ? __uint_as_float((q & 1) ? (wv[q >> 1] & 0xffff0000u) : (wv[q >> 1] << 16))
                       : __uint_as_float(wv[q]);
-#pragma unroll
-        for (int q = 0; q < 4; ++q) nacc |= (wv[q] & nan_mask) + nan_add;
         if (greedy) {
+#pragma unroll
+          for (int q = 0; q < 4; ++q) nacc |= (wv[q] & nan_mask) + nan_add;
 #pragma unroll
           for (int q = 0; q < kEpv; ++q)
             if (x[q] > m) { m = x[q]; a = vi * kEpv + q; }
@@ -190,18 +190,28 @@ __global__ void __launch_bounds__(kThreads, 8) draft_sample_kernel(DraftParams p
           float lm = vm;
 #pragma unroll
           for (int o = 1; o < kGroup; o <<= 1) lm = fmaxf(lm, __shfl_xor_sync(0xffffffffu, lm, o));
+          // The lane's weights 2^((x - lm) c), each argument one fused multiply-add. A NaN
+          // logit makes its lane's sum NaN (tested once per lane below), except in a lane
+          // with no finite maximum, whose words are tested here.
           float ls = 0.f;
           if (lm != -INFINITY) {
+            const float nlc = -lm * c;
 #pragma unroll
-            for (int q = 0; q < kEpv; ++q) ls += exp2f((x[q] - lm) * c);
+            for (int q = 0; q < kEpv; ++q) ls += ex2(fmaf(x[q], c, nlc));
+          } else {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) nacc |= (wv[q] & nan_mask) + nan_add;
           }
 #pragma unroll
           for (int o = 1; o < kGroup; o <<= 1) ls += __shfl_xor_sync(0xffffffffu, ls, o);
-          if ((tid & (kGroup - 1)) == 0 && vi < vend) lanes[vi / kGroup - l0] = make_float2(lm, ls);
+          if ((tid & (kGroup - 1)) == 0 && vi < vend) {
+            lanes[vi / kGroup - l0] = make_float2(lm, ls);
+            bad |= ls != ls;
+          }
         }
       }
     }
-    bad = (nacc & nan_top) != 0;
+    bad |= (nacc & nan_top) != 0;
   } else {
     if (e_begin + tid < e_end) a = e_begin + tid;
     for (int e0 = e_begin; e0 < e_end; e0 += kThreads * kUnroll) {
