@@ -30,7 +30,7 @@ DraftLayout draft_layout(const spec_draft_args_t& a, size_t base, int sms, bool 
   L.lane_elems = vec ? 64 : 32;
   L.nlanes = static_cast<int>((static_cast<int64_t>(a.vocab) + L.lane_elems - 1) / L.lane_elems);
   const int64_t rows = static_cast<int64_t>(a.batch) * a.gamma;
-  int64_t splits = (static_cast<int64_t>(kFiltBlocksPerSm) * sms + rows - 1) / rows;
+  int64_t splits = static_cast<int64_t>(kFiltBlocksPerSm) * sms / rows;  // within one wave
   splits = splits < 1 ? 1 : (splits > kFiltMaxSplits ? kFiltMaxSplits : splits);
   if (splits > L.nlanes) splits = L.nlanes;
   L.lanes_per_split = static_cast<int>((L.nlanes + splits - 1) / splits);
