@@ -64,6 +64,33 @@ def test_small_shapes_full(oracle_mod, case, path):
     compare_attention(g_out, g_lse, o_out, o_lse)
 
 
+def random_shape(seed):
+    """A seeded random attention problem: GQA group, KV heads, head dim, page size,
+    block size and ragged contexts drawn over the ranges the kernels take (up to 512
+    query rows per KV head), with spare pages in the pool."""
+    rng = np.random.default_rng(1000 + seed)
+    group = int(rng.choice([1, 2, 3, 4, 6, 8, 16]))
+    hkv = int(rng.choice([1, 2, 4, 8]))
+    gamma = int(rng.integers(1, max(2, min(64, 512 // group)) + 1))
+    lo = int(rng.integers(0, 900))
+    hi = lo + int(rng.integers(0, 700))
+    return dict(batch=int(rng.integers(1, 5)), gamma=gamma, num_q_heads=group * hkv,
+                num_kv_heads=hkv, head_dim=int(rng.choice([64, 128])),
+                page_size=int(rng.choice([16, 32, 64])), ctx=(lo, hi),
+                extra_pages=int(rng.integers(0, 8)))
+
+
+@pytest.mark.parametrize("path", PATHS)
+@pytest.mark.parametrize("seed", range(20))
+def test_random_shapes(oracle_mod, seed, path):
+    shape = random_shape(seed)
+    inp = W.make_attn_inputs(seed=seed, **shape)
+    g_out, g_lse = gpu_attention(inp, path)
+    o_out, o_lse, st = oracle_attn(oracle_mod, inp)
+    assert np.all(st == 0)
+    compare_attention(g_out, g_lse, o_out, o_lse)
+
+
 @pytest.mark.parametrize("name", ["tiny", "llama8b", "serve64", "long70b"])
 def test_named_workloads_sampled(oracle_mod, name):
     """Full-size workloads, in the launch configuration the benchmark times (automatic
