@@ -212,7 +212,7 @@ spec_status_t check_lm_head(const spec_lm_head_args_t* a) {
     return SPEC_ERR_INVALID_ARGUMENT;
   if ((reinterpret_cast<uintptr_t>(a->hidden_states) | reinterpret_cast<uintptr_t>(a->weight)) & 15u)
     return SPEC_ERR_INVALID_ARGUMENT;
-  if ((a->rows + kLmTileM - 1) / kLmTileM > 65535) return SPEC_ERR_UNSUPPORTED;
+  if ((a->vocab + kLmTileN - 1) / kLmTileN > 65535) return SPEC_ERR_UNSUPPORTED;  // grid y
   return SPEC_OK;
 }
 

@@ -105,7 +105,10 @@ __global__ void __launch_bounds__(kThreads)
   uint32_t* misc = reinterpret_cast<uint32_t*>(smem + kOffMisc);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 1);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int n0 = blockIdx.x * kLmTileN, m0 = blockIdx.y * kLmTileM;
+  // blockIdx.x is the row tile, so the row tiles that share a weight tile run together
+  // and read it from DRAM once (the others hit L2)
+  const int tn = blockIdx.y;  // vocab tile
+  const int n0 = tn * kLmTileN, m0 = blockIdx.x * kLmTileM;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
@@ -234,7 +237,7 @@ __global__ void __launch_bounds__(kThreads)
         out.s = s;
         out.arg = bad ? -2 : a;
         out.tok = tl;
-        p.parts[static_cast<int64_t>(row) * p.ntn + blockIdx.x] = out;
+        p.parts[static_cast<int64_t>(row) * p.ntn + tn] = out;
       }
     }
   }
@@ -308,7 +311,7 @@ cudaError_t launch_lm_head(const spec_lm_head_args_t& a, const LmLayout& L, char
   cudaError_t e = cudaFuncSetAttribute(lm_head_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(kSmem));
   if (e != cudaSuccess) return e;
-  lm_head_kernel<<<dim3(L.ntiles_n, L.ntiles_m), kThreads, kSmem, stream>>>(mh, mw, p);
+  lm_head_kernel<<<dim3(L.ntiles_m, L.ntiles_n), kThreads, kSmem, stream>>>(mh, mw, p);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   lm_merge_kernel<<<(a.rows + 3) / 4, 128, 0, stream>>>(p);
