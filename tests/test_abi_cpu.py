@@ -229,7 +229,7 @@ def _lm(**kw):
 @pytest.mark.parametrize("kw,code", [
     (dict(rows=0), 1), (dict(hidden=12), 1), (dict(hidden=4), 1), (dict(vocab=0), 1),
     (dict(rows_per_seq=0), 1), (dict(weight=None), 1), (dict(row_argmax=None), 1),
-    (dict(hidden_states=4104), 1), (dict(weight=4100), 1), (dict(rows=128 * 65536), 2),
+    (dict(hidden_states=4104), 1), (dict(weight=4100), 1), (dict(vocab=224 * 65536), 2),
 ])
 def test_lm_head_host_checks(lib, kw, code):
     a = _lm(**kw)

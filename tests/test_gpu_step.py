@@ -30,6 +30,55 @@ def test_philox_matches_generator(offset, n):
     np.testing.assert_array_equal(dev.view(np.uint32), host.view(np.uint32))
 
 
+@pytest.mark.parametrize("temps", [(1.0,), (1.0, 0.0, 0.7)])
+def test_large_step(oracle_mod, temps):
+    """A step with 381 MB of logits (48 sequences x 31 rows x 128,256 bf16) and 64 query
+    rows per KV head, some sequences greedy: the step equals its two parts called
+    separately, repeats bit-identically on one workspace (every counter left at zero),
+    and agrees with the oracle."""
+    B, G, V = 48, 16, 128256
+    ai = W.make_attn_inputs(B, G, 32, 8, 128, 16, (100, 600), True, seed=5)
+    ci = W.make_accept_inputs(B, G, V, "bf16", 3.0, 1.0, list(temps), seed=6)
+    at, ct = attn_tensors(ai), accept_tensors(ci)
+
+    def outputs():
+        return (torch.empty_like(at[0]), torch.empty(at[0].shape[:3], dtype=torch.float32, device="cuda"),
+                dict(num_accepted=torch.empty(B, dtype=torch.int32, device="cuda"),
+                     out_tokens=torch.empty(B, G + 1, dtype=torch.int32, device="cuda"),
+                     num_emitted=torch.empty(B, dtype=torch.int32, device="cuda"),
+                     diag=torch.empty(B, G, 2, dtype=torch.float32, device="cuda")))
+
+    out, lse, res = outputs()
+    a = binding.attn_args(*at, out, lse)
+    c = binding.accept_args(*ct, res["num_accepted"], res["out_tokens"], res["num_emitted"],
+                            res["diag"])
+    ws = binding.new_workspace(binding.workspace_size(a, c))
+    binding.verify_step_args(a, c, ws)
+    torch.cuda.synchronize()
+    assert binding.read_device_status(ws) == (0, 0)
+    first = [out.clone(), lse.clone()] + [res[k].clone() for k in res]
+    binding.verify_step_args(a, c, ws)
+    torch.cuda.synchronize()
+    assert binding.read_device_status(ws) == (0, 0)
+    again = [out, lse] + [res[k] for k in res]
+    for x, y in zip(first, again):
+        assert torch.equal(x.nan_to_num(-7), y.nan_to_num(-7))
+    part_out, part_lse = binding.verify_attention(*at)
+    part_acc = binding.accept_block(*ct)
+    assert torch.equal(out, part_out) and torch.equal(lse, part_lse)
+    for k in res:
+        assert torch.equal(res[k].nan_to_num(-7), part_acc[k].nan_to_num(-7)), k
+    n = 8
+    o = oracle_mod.accept_block(ci.target_logits[:n], ci.drafter_logits[:n], ci.block_tokens[:n],
+                                ci.temperature[:n], ci.uniforms[:n])
+    compare_accept({k: v[:n].cpu().numpy() for k, v in res.items()}, o, G)
+    rows = sample_rows(ai, 24)
+    o_out, o_lse, st = oracle_mod.verify_attention(ai.q, ai.k_cache, ai.v_cache, ai.page_table,
+                                                   ai.kv_len, G, rows=rows)
+    assert np.all(st == 0)
+    compare_attention(out.float().cpu().numpy(), lse.cpu().numpy(), o_out, o_lse, rows)
+
+
 @pytest.mark.parametrize("name", ["tiny", "llama8b"])
 def test_step_equals_parts(oracle_mod, name):
     wl = W.workload(name)
