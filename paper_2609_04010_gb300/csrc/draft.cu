@@ -87,14 +87,6 @@ __device__ __forceinline__ int cand_idx(unsigned long long c) {
   return static_cast<int>(0xffffffffu - static_cast<uint32_t>(c));
 }
 
-// Merge of two (max, sum of exp2((l - max) c)) pairs.
-__device__ __forceinline__ float2 merge_ms(float2 a, float2 b, float c) {
-  const float m = fmaxf(a.x, b.x);
-  if (m == -INFINITY) return make_float2(-INFINITY, 0.f);
-  return make_float2(m, (a.x == -INFINITY ? 0.f : a.y * exp2f((a.x - m) * c)) +
-                            (b.x == -INFINITY ? 0.f : b.y * exp2f((b.x - m) * c)));
-}
-
 // Block-wide exclusive scan of one float per thread, in thread order; *total gets the sum.
 __device__ __forceinline__ float block_excl_scan(float x, float* sh, float* total) {
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
