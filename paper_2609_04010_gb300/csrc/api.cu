@@ -244,6 +244,7 @@ spec_status_t check_accept(const spec_accept_args_t* a) {
 
 AttnPlan attn_plan(const spec_attn_args_t& a, size_t base, int num_sms, int path_override) {
   AttnPlan P;
+  P.head_pair = 0;
   P.rows = (a.num_q_heads / a.num_kv_heads) * a.gamma;
   int path = path_override;
   if (path == SPEC_ATTN_AUTO)
@@ -289,11 +290,13 @@ AttnPlan attn_plan(const spec_attn_args_t& a, size_t base, int num_sms, int path
     P.rows_per_cta = P.rows <= 128 ? 128 : kTcMaxRows;
     P.key_tile = kTcKeyTile;
     P.row_tiles = (P.rows + P.rows_per_cta - 1) / P.rows_per_cta;
-    units = static_cast<int64_t>(a.batch) * a.num_kv_heads * P.row_tiles;
+    P.head_pair = tc_head_pair(a.head_dim, P.rows, a.num_kv_heads, a.batch) ? 1 : 0;
+    units = static_cast<int64_t>(a.batch) * (a.num_kv_heads / (1 + P.head_pair)) * P.row_tiles;
     P.nsplit = 1;
     P.tiles_per_split = 0;
-    P.grid = num_sms * tc_ctas_per_sm(a.head_dim, P.rows_per_cta, P.rows, a.batch);
-    P.slot_rows = P.rows < P.rows_per_cta ? P.rows : P.rows_per_cta;
+    P.grid = num_sms * tc_ctas_per_sm(a.head_dim, P.rows_per_cta, P.rows, a.batch, P.head_pair != 0);
+    // a slot keeps a unit's rows (a head pair's second head after its first)
+    P.slot_rows = (P.rows < P.rows_per_cta ? P.rows : P.rows_per_cta) * (1 + P.head_pair);
     P.slots = units + P.grid;
   }
   P.tickets = base;

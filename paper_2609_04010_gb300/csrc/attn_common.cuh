@@ -15,6 +15,8 @@ namespace specv {
 
 struct AttnParams {
   int batch, gamma, hq, hkv, group, rows, row_tiles, rows_per_cta;
+  int hunits;        // KV-head units per sequence: Hkv, or Hkv / 2 when a block serves
+                     // two adjacent KV heads together (tensor-core head-pair variant)
   int page_size, max_pages, num_pages;
   int nsplit, tiles_per_split;
   int slot_rows;     // rows stored per partial slot
@@ -43,6 +45,7 @@ inline AttnParams make_attn_params(const spec_attn_args_t& a, const AttnPlan& P,
   p.gamma = a.gamma;
   p.hq = a.num_q_heads;
   p.hkv = a.num_kv_heads;
+  p.hunits = P.head_pair ? a.num_kv_heads / 2 : a.num_kv_heads;
   p.group = a.num_q_heads / a.num_kv_heads;
   p.rows = P.rows;
   p.row_tiles = P.row_tiles;
@@ -75,9 +78,11 @@ inline AttnParams make_attn_params(const spec_attn_args_t& a, const AttnPlan& P,
 }
 
 // Tensor maps of the tensor-core kernels (attn_tc.cu): the K or V cache with one page of
-// one KV head per box, and Q with one tile of tile_rows query rows of one KV group per
-// box (false if group does not divide tile_rows or the encoder is missing).
-bool encode_cache_map(CUtensorMap* map, const void* base, const spec_attn_args_t& a);
+// one KV head (or of two adjacent KV heads, heads_per_box = 2) per box, and Q with one
+// tile of tile_rows query rows of one KV group per box (false if group does not divide
+// tile_rows or the encoder is missing).
+bool encode_cache_map(CUtensorMap* map, const void* base, const spec_attn_args_t& a,
+                      int heads_per_box = 1);
 bool encode_q_map(CUtensorMap* map, const spec_attn_args_t& a, int tile_rows);
 
 #ifdef __CUDACC__
@@ -96,8 +101,8 @@ __device__ __forceinline__ int unit_tiles(int kv_len, const AttnParams& p) {
 // with no real tile, and then it is the range's last (a first segment without real
 // tiles means the block has no work).
 struct Seg {
-  int b, g, rt;      // sequence, KV head, row tile
-  int64_t u;         // unit index (b * Hkv + g) * row_tiles + rt
+  int b, g, rt;      // sequence, KV head (or head pair), row tile
+  int64_t u;         // unit index (b * hunits + g) * row_tiles + rt
   int tile0, ntile;  // first real tile within the unit and real tile count of this segment
   int unit_tiles;    // real tiles of the whole unit
   int kv_len;
@@ -125,7 +130,7 @@ __device__ __forceinline__ Seg locate(int64_t v, int64_t v1, const AttnParams& p
   const int64_t vstart = v - rem % vlen;  // the unit's first (overhead) virtual tile
   s.g = ub / p.row_tiles;
   s.rt = ub % p.row_tiles;
-  s.u = static_cast<int64_t>(lo) * p.hkv * p.row_tiles + ub;
+  s.u = static_cast<int64_t>(lo) * p.hunits * p.row_tiles + ub;
   s.unit_start = vstart + ovh;
   const int64_t vend = vstart + vlen;
   s.vnext = vend < v1 ? vend : v1;
@@ -174,13 +179,14 @@ __device__ __forceinline__ void write_lse(const AttnParams& p, int b, int g, int
 
 // Combines the split-KV partials of one unit, held in slots [slot0, slot0 + nslots), for
 // rows [row0, row0 + nrows) and writes the final outputs (nthreads threads from tid
-// cooperate; no block synchronization). Each (row, 8-column) item walks the slots in
+// cooperate; no block synchronization). Row r of the range sits at row prow0 + r of a
+// slot (a head-pair unit keeps its second head's rows after the first's). Each (row, 8-column) item walks the slots in
 // batches of four, loading a batch's (m, l) pairs and output pieces together and
 // folding them into a running base-2 max, so a unit with up to four slots costs one
 // round trip to L2.
 template <int D>
 __device__ void merge_unit(const AttnParams& p, int b, int g, int row0, int nrows, int64_t slot0,
-                           int nslots, int tid, int nthreads) {
+                           int nslots, int tid, int nthreads, int prow0 = 0) {
   constexpr int C8 = D / 8;
   for (int idx = tid; idx < nrows * C8; idx += nthreads) {
     const int r = idx / C8, c8 = idx % C8;
@@ -194,7 +200,7 @@ __device__ void merge_unit(const AttnParams& p, int b, int g, int row0, int nrow
 #pragma unroll
       for (int e = 0; e < 4; ++e) {
         if (s0 + e < nslots) {
-          const int64_t slot = (slot0 + s0 + e) * p.slot_rows + r;
+          const int64_t slot = (slot0 + s0 + e) * p.slot_rows + prow0 + r;
           ml[e] = __ldcg(&p.partial_ml[slot]);
           const float4* src = reinterpret_cast<const float4*>(p.partial_o + slot * D) + 2 * c8;
           lo[e] = __ldcg(src);

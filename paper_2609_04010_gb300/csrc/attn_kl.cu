@@ -176,7 +176,7 @@ __global__ void __launch_bounds__(384, 1)
     int carry = 0;
     for (int b0 = 0; b0 < p.batch; b0 += 32) {
       const int b = b0 + lane;
-      int v = b < p.batch ? (unit_tiles<KT>(p.kv_len[b], p) + p.unit_overhead) * p.hkv : 0;
+      int v = b < p.batch ? (unit_tiles<KT>(p.kv_len[b], p) + p.unit_overhead) * p.hunits : 0;
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
         const int y = __shfl_up_sync(0xffffffffu, v, o);
@@ -197,7 +197,7 @@ __global__ void __launch_bounds__(384, 1)
   // then split into equal parts with no unit boundary inside any block's range).
   int ctas = static_cast<int>(total < gridDim.x ? total : gridDim.x);
   {
-    const int units = p.batch * p.hkv;
+    const int units = p.batch * p.hunits;
     if (units <= static_cast<int>(gridDim.x)) {
       const int aligned = units * (static_cast<int>(gridDim.x) / units);
       if (aligned < ctas) ctas = aligned;

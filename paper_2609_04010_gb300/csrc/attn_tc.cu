@@ -5,7 +5,16 @@
 //
 // One block holds every query row of one KV head (row r = block position j * group +
 // head-in-group), padded to M = 128 rows per tensor-core tile (two tiles when the
-// group has up to 256 rows), so each KV page is read from HBM once.
+// group has up to 256 rows), so each KV page is read from HBM once. When a group has at
+// most 64 rows and Hkv is even, the head-pair variant serves two adjacent KV heads in
+// one M tile (the first head's rows in TMEM lanes 0..63, the second's in 64..127): the
+// cache stores the heads of a page next to each other, so one copy brings a page of both
+// (8 KB instead of 4 KB with 16-token pages; the copy engine's rate grows with the size
+// of its copies). Each head has its own Q K^T and P V MMAs over the whole tile (the rows
+// of the other head are computed and ignored, as the padding rows of a 64-row group are
+// otherwise). P stays in tensor memory, written as bf16 over the first head's S columns
+// of its tile and read by the P V MMAs from there, so the shared memory of the P buffers
+// holds one more V stage; K and V stages have separate rings.
 //
 // Warp roles (one block per SM, persistent):
 //   warps 0,2   KV producers: gather each 64-key tile of K and V page by page through
@@ -46,44 +55,60 @@ constexpr int TK = kTcKeyTile;               // keys per tile
 // out Q, P, K/V stages, so that the 64 padding rows each read comes from the next
 // buffer (their scores and outputs are never used), and the freed 32 KB (D = 128) holds
 // one more K/V stage: more bytes in flight per SM.
-template <int D, int MT, int QR = 128>
+// HP: KV heads per block (2: the head-pair variant; QR = 64, one M tile of 2 x 64 rows).
+template <int D, int MT, int QR = 128, int HP = 1>
 struct TcCfg {
   static_assert(QR == 128 || (QR == 64 && MT == 1), "64-row buffers only with one M tile");
+  static_assert(HP == 1 || (HP == 2 && QR == 64), "head pairs only with groups of <= 64 rows");
   static constexpr int DH = D / 64;                   // 128-byte column halves of a row
-  // Softmax warps per 32-row quadrant. With one M tile, two warps share each quadrant,
-  // one per half of the tile's keys, each with its own online-softmax state and its own
-  // O accumulator (merged once per unit); with two M tiles one warp per quadrant.
-  static constexpr int SPLIT = MT == 1 ? 2 : 1;
+  // Softmax warps per 32-row quadrant. With one M tile of one head, two warps share each
+  // quadrant, one per half of the tile's keys, each with its own online-softmax state
+  // and its own O accumulator (merged once per unit); otherwise one warp per quadrant
+  // (with two heads the second O pair would not fit in TMEM).
+  static constexpr int SPLIT = (MT == 1 && HP == 1) ? 2 : 1;
   static constexpr int KH = TK / SPLIT;               // keys of a tile per softmax warp
   static constexpr int PB = MT == 1 ? 2 : 1;          // P buffers (double with one M tile)
+  static constexpr int MR = QR * HP;                  // rows of a Q or P buffer
+  // P in tensor memory (head pairs): P[buf] over the first 32 columns of S[0][buf], which
+  // then stays busy until the tile's P V MMAs complete
+  static constexpr bool PTMEM = HP == 2;
+  // one ring of K+V stages (HP = 1), or KST stages of K and VST of V (HP = 2)
   static constexpr int STAGES = QR == 64 ? 5 : ((D == 128 && MT == 2) || (D == 64 && MT == 1) ? 3 : 4);
+  static constexpr int KST = HP == 2 ? (D == 128 ? 3 : 4) : STAGES;
+  static constexpr int VST = HP == 2 ? (D == 128 ? 3 : 4) : STAGES;
+  static constexpr int RINGBARS = HP == 2 ? 2 * (KST + VST) : 2 * STAGES;
   static constexpr int THREADS = 128 + 256;           // 4 producer / MMA warps + 8 softmax
   // Starting a unit inside a block's range costs about this many tiles of time (its Q
   // tile, the pipeline refill and the previous unit's epilogue). When blocks hold
   // several unit starts the work list charges it, so that blocks stay balanced.
   static constexpr int UNIT_OVERHEAD = MT == 1 ? 3 : 2;
-  static constexpr uint32_t QHALF = QR * 128u;          // one column half of an M tile's Q
-  static constexpr uint32_t PBUF = QR * 128u;           // one P buffer of an M tile
-  static constexpr uint32_t Q_BYTES = MT * DH * QHALF;  // [MT][DH][QR rows x 128 B]
-  static constexpr uint32_t KV_BYTES = DH * 8192;       // one stage of K (or V): [DH][64 x 128 B]
-  static constexpr uint32_t P_BYTES = PB * MT * PBUF;   // [PB][MT][QR rows x 128 B]
+  static constexpr uint32_t QHALF = MR * 128u;          // one column half of an M tile's Q
+  static constexpr uint32_t PBUF = MR * 128u;           // one P buffer of an M tile
+  static constexpr uint32_t Q_BYTES = MT * DH * QHALF;  // [MT][DH][MR rows x 128 B]
+  // one stage of K (or V): [8-key group][head][DH][8 keys x 128 B]
+  static constexpr uint32_t KV_BYTES = HP * DH * 8192;
+  static constexpr uint32_t P_BYTES = PTMEM ? 0 : PB * MT * PBUF;  // [PB][MT][MR rows x 128 B]
   static constexpr uint32_t OFF_Q = 0;
   static constexpr uint32_t OFF_P = QR == 64 ? OFF_Q + Q_BYTES : OFF_Q + Q_BYTES + 2 * STAGES * KV_BYTES;
   static constexpr uint32_t OFF_K = QR == 64 ? OFF_P + P_BYTES : OFF_Q + Q_BYTES;
-  static constexpr uint32_t OFF_V = OFF_K + STAGES * KV_BYTES;
-  static constexpr uint32_t OFF_BAR = QR == 64 ? OFF_V + STAGES * KV_BYTES : OFF_P + P_BYTES;
-  // barriers: kv_full[S], kv_empty[S], s_full[MT][2], s_free[MT][2], p_full[MT][PB],
-  // pv_done[MT][PB], seg_ready, drain[2], xch[4], q_full, seg_flag_ready[8]
-  static constexpr int NBAR = 2 * STAGES + 4 * MT + 2 * MT * PB + 3 + 4 + 1 + 8;
+  static constexpr uint32_t OFF_V = OFF_K + KST * KV_BYTES;
+  static constexpr uint32_t OFF_BAR = QR == 64 ? OFF_V + VST * KV_BYTES : OFF_P + P_BYTES;
+  // barriers: ring (kv_full[S], kv_empty[S], or k_full[KST], v_full[VST], k_empty[KST],
+  // v_empty[VST]), s_full[MT][2], s_free[MT][2], p_full[MT][PB], pv_done[MT][PB],
+  // seg_ready, drain[2], xch[4], q_full, seg_flag_ready[8]
+  static constexpr int NBAR = RINGBARS + 4 * MT + 2 * MT * PB + 3 + 4 + 1 + 8;
   static constexpr uint32_t OFF_MISC = OFF_BAR + NBAR * 8;  // tmem base, abort, pending count
   static constexpr uint32_t OFF_XCH = OFF_MISC + 16;        // [4][2][32] float2 (m, l) per half
   static constexpr uint32_t OFF_PEND = OFF_XCH + (SPLIT == 2 ? 4 * 2 * 32 * 8 : 0);  // [2][8]
   static constexpr uint32_t OFF_FLAG = OFF_PEND + 64;  // [8] bad flags of segments
   static constexpr uint32_t OFF_PB = (OFF_FLAG + 32 + 15) / 16 * 16;
-  static constexpr uint32_t TMEM_NEED = MT * 128 + MT * SPLIT * D;
+  // accumulators a = mt * HP + head: S[a][buf] at (a * 2 + buf) * 64, O[a][half] at
+  // O_COL + (a * SPLIT + half) * D
+  static constexpr uint32_t TMEM_NEED = MT * HP * 128 + MT * HP * SPLIT * D;
   static constexpr uint32_t TMEM_COLS = TMEM_NEED <= 256 ? 256 : 512;
-  static constexpr uint32_t S_COL = 0;           // S[mt][buf] at (mt * 2 + buf) * 64
-  static constexpr uint32_t O_COL = MT * 128;    // O[mt][half] at O_COL + (mt * SPLIT + half) * D
+  static_assert(TMEM_NEED <= 512, "TMEM holds 512 columns");
+  static constexpr uint32_t S_COL = 0;
+  static constexpr uint32_t O_COL = MT * HP * 128;
   static size_t smem_bytes(int batch) { return OFF_PB + 4u * (batch + 1) + 1024; }
 };
 
@@ -92,15 +117,19 @@ struct TcCfg {
 // ---------------------------------------------------------------------------------
 using namespace tcx;
 constexpr long long kWaitLimitCycles = kWaitCycles;
-// One page of one KV head (box of the 5-D view of the cache, see encode_cache_map),
-// landing as [8-row group][128-byte column half][8 rows][128 B], 128-byte swizzle.
+// One page of one KV head, or of two adjacent ones (box of the 5-D view of the cache, see
+// encode_cache_map), landing as [8-row group][head][128-byte column half][8 rows][128 B],
+// 128-byte swizzle.
+// The page-and-head coordinate is the map's last dimension with one head per box and
+// its fourth with two (see encode_cache_map).
+template <int HP>
 __device__ __forceinline__ void tma_load_page(uint32_t dst, const CUtensorMap* map, int page_head,
                                               uint32_t bar) {
   asm volatile(
       "cp.async.bulk.tensor.5d.shared::cluster.global.mbarrier::complete_tx::bytes"
       " [%0], [%1, {%2, %3, %4, %5, %6}], [%7];" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(map)), "r"(0), "r"(0), "r"(0), "r"(0), "r"(page_head),
-      "r"(bar)
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(0), "r"(0), "r"(0), "r"(HP == 2 ? page_head : 0),
+      "r"(HP == 2 ? 0 : page_head), "r"(bar)
       : "memory");
 }
 // Rows of one M tile of Q: 128 / group block positions of `group` heads, one
@@ -122,28 +151,35 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
 // The kernel
 // ---------------------------------------------------------------------------------
 // TREE: tree attention (a per-row mask over the block keys) instead of the causal block.
-template <int D, int MT, bool TREE, int QR>
-__global__ void __launch_bounds__(TcCfg<D, MT, QR>::THREADS, 1)
+template <int D, int MT, bool TREE, int QR, int HP>
+__global__ void __launch_bounds__(TcCfg<D, MT, QR, HP>::THREADS, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmap_k,
                    const __grid_constant__ CUtensorMap tmap_v,
                    const __grid_constant__ CUtensorMap tmap_q, AttnParams p) {
-  using C = TcCfg<D, MT, QR>;
+  using C = TcCfg<D, MT, QR, HP>;
   constexpr int SPLIT = C::SPLIT, KH = C::KH, PB = C::PB;
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   const uint32_t sbase = smem_u32(smem);
   const uint32_t bar0 = sbase + C::OFF_BAR;
+  // HP = 1: one ring of K+V stages
   auto kv_full = [&](int s) { return bar0 + 8u * s; };
   auto kv_empty = [&](int s) { return bar0 + 8u * (C::STAGES + s); };
-  auto s_full = [&](int mt, int bf) { return bar0 + 8u * (2 * C::STAGES + mt * 2 + bf); };
-  auto s_free = [&](int mt, int bf) { return bar0 + 8u * (2 * C::STAGES + 2 * MT + mt * 2 + bf); };
+  // HP = 2: a ring of K stages (freed by the Q K^T MMAs) and a ring of V stages
+  auto k_full = [&](int s) { return bar0 + 8u * s; };
+  auto v_full = [&](int s) { return bar0 + 8u * (C::KST + s); };
+  auto k_empty = [&](int s) { return bar0 + 8u * (C::KST + C::VST + s); };
+  auto v_empty = [&](int s) { return bar0 + 8u * (2 * C::KST + C::VST + s); };
+  constexpr uint32_t RB = C::RINGBARS;
+  auto s_full = [&](int mt, int bf) { return bar0 + 8u * (RB + mt * 2 + bf); };
+  auto s_free = [&](int mt, int bf) { return bar0 + 8u * (RB + 2 * MT + mt * 2 + bf); };
   // P buffer pb of M tile mt: written by the softmax warps, read by the P V MMAs
-  auto p_full = [&](int mt, int pb) { return bar0 + 8u * (2 * C::STAGES + 4 * MT + mt * PB + pb); };
+  auto p_full = [&](int mt, int pb) { return bar0 + 8u * (RB + 4 * MT + mt * PB + pb); };
   auto pv_done = [&](int mt, int pb) {
-    return bar0 + 8u * (2 * C::STAGES + 4 * MT + MT * PB + mt * PB + pb);
+    return bar0 + 8u * (RB + 4 * MT + MT * PB + mt * PB + pb);
   };
-  const uint32_t seg_ready = bar0 + 8u * (2 * C::STAGES + 4 * MT + 2 * MT * PB);
+  const uint32_t seg_ready = bar0 + 8u * (RB + 4 * MT + 2 * MT * PB);
   auto drain_bar = [&](int i) { return seg_ready + 8 + 8u * i; };  // per MMA issuer
   auto xch_bar = [&](int q) { return seg_ready + 24 + 8u * q; };   // the two halves of quadrant q
   const uint32_t q_full = seg_ready + 56;  // Q tile of the next segment landed (TMA)
@@ -164,23 +200,39 @@ __global__ void __launch_bounds__(TcCfg<D, MT, QR>::THREADS, 1)
 
   // ---- roles ----
   // Softmax warps take part only as far as the row tile has real rows (32 per warp).
+  // With a head pair, quadrants 0-1 hold the first head's rows and 2-3 the second's.
   const int rows_cta = min(p.rows_per_cta, p.rows);
-  int nact[MT];
+  int nact[MT];  // active quadrants of each M tile
   int nact_total = 0;
 #pragma unroll
   for (int mt = 0; mt < MT; ++mt) {
-    nact[mt] = min(4, max(0, (rows_cta - 128 * mt + 31) / 32));
+    nact[mt] = HP == 2 ? 2 * min(2, (rows_cta + 31) / 32) : min(4, max(0, (rows_cta - 128 * mt + 31) / 32));
     nact_total += nact[mt];
   }
   const int nsoft = nact_total * SPLIT;  // active softmax warps
+  auto soft_active = [&](int sw) {  // softmax warp sw = warp - 4 has real rows
+    if (HP == 2) return sw < 4 && (sw & 1) * 32 < rows_cta;
+    return (sw & 3) < nact[(sw >> 2) / SPLIT];
+  };
   constexpr int nprod = 2;  // KV producer warps 0 and 2
   const int pw = warp == 0 ? 0 : (warp == 2 ? 1 : -1);
 
   // ---- prologue: barriers, TMEM, per-sequence tile prefix sums ----
   if (threadIdx.x == 0) {
-    for (int s = 0; s < C::STAGES; ++s) {
-      mbar_init(kv_full(s), nprod);
-      mbar_init(kv_empty(s), 1);
+    if (HP == 2) {
+      for (int s = 0; s < C::KST; ++s) {
+        mbar_init(k_full(s), 1);
+        mbar_init(k_empty(s), 1);
+      }
+      for (int s = 0; s < C::VST; ++s) {
+        mbar_init(v_full(s), 1);
+        mbar_init(v_empty(s), 1);
+      }
+    } else {
+      for (int s = 0; s < C::STAGES; ++s) {
+        mbar_init(kv_full(s), nprod);
+        mbar_init(kv_empty(s), 1);
+      }
     }
     for (int mt = 0; mt < MT; ++mt) {
       const uint32_t nw = nact[mt] > 0 ? nact[mt] * SPLIT : 1;
@@ -205,7 +257,7 @@ __global__ void __launch_bounds__(TcCfg<D, MT, QR>::THREADS, 1)
   }
   if (warp == 1) tmem_alloc(smem_u32(misc), C::TMEM_COLS);
   if (warp == 0) {
-    const int per_b = p.hkv * p.row_tiles;
+    const int per_b = p.hunits * p.row_tiles;
     int carry = 0;
     for (int b0 = 0; b0 < p.batch; b0 += 32) {
       const int b = b0 + lane;
@@ -232,7 +284,7 @@ __global__ void __launch_bounds__(TcCfg<D, MT, QR>::THREADS, 1)
   // every SM). Ranges stay equal in tiles, so ragged lengths stay balanced.
   int ctas = static_cast<int>(total < gridDim.x ? total : gridDim.x);
   {
-    const int units = p.batch * p.hkv * p.row_tiles;
+    const int units = p.batch * p.hunits * p.row_tiles;
     if (units <= static_cast<int>(gridDim.x)) {
       const int aligned = units * (static_cast<int>(gridDim.x) / units);
       if (aligned < ctas) ctas = aligned;
@@ -245,8 +297,9 @@ __global__ void __launch_bounds__(TcCfg<D, MT, QR>::THREADS, 1)
 
   if (pw >= 0) {
     // ============================ KV producers ============================
-    // A tile needs one box per (page, K or V); producer pw issues boxes pw, pw + nprod,
-    // ... (one issuer cannot keep the copy engine busy with page-sized boxes).
+    // A tile needs one box per (page, K or V): producer 0 issues the K boxes, producer 1
+    // the V boxes (one issuer cannot keep the copy engine busy with page-sized boxes).
+    // With one head both fill the same K+V stage; with a head pair each has its own ring.
     uint32_t it = 0;
     bool ok = true;
     // Page ids are read 32 at a time (lane i holds page cache_base + i of sequence
@@ -261,39 +314,41 @@ __global__ void __launch_bounds__(TcCfg<D, MT, QR>::THREADS, 1)
       }
       return __shfl_sync(0xffffffffu, cache_val, pi - cache_base);
     };
-    const uint32_t box_bytes = static_cast<uint32_t>(p.page_size) * D * 2;  // one page of one head
+    // one page of HP heads
+    const uint32_t box_bytes = static_cast<uint32_t>(p.page_size) * D * 2 * HP;
+    const uint32_t RS = HP == 2 ? (pw == 0 ? C::KST : C::VST) : C::STAGES;  // ring stages
+    auto ring_full = [&](uint32_t st) {
+      return HP == 2 ? (pw == 0 ? k_full(st) : v_full(st)) : kv_full(st);
+    };
+    auto ring_empty = [&](uint32_t st) {
+      return HP == 2 ? (pw == 0 ? k_empty(st) : v_empty(st)) : kv_empty(st);
+    };
+    const uint32_t ring_base = sbase + (pw == 0 ? C::OFF_K : C::OFF_V);
+    const CUtensorMap* map = pw == 0 ? &tmap_k : &tmap_v;
     uint32_t seg_no = 0;
     for (Seg s = locate<TK>(t0, t1, p, pb, OVH); s.ntile > 0 && ok && !p.starve; ++seg_no) {
       const bool bad = !s.len_ok;  // nothing to read
       bool flag = bad;             // ... or a page id out of range (read as page 0)
       for (int k = 0; k < s.ntile && ok; ++k, ++it) {
-        const int st = it % C::STAGES;
-        if (it >= static_cast<uint32_t>(C::STAGES))
-          ok = mbar_wait(kv_empty(st), ((it / C::STAGES) - 1) & 1, abort_flag, p.status);
+        const uint32_t st = it % RS;
+        if (it >= RS) ok = mbar_wait(ring_empty(st), ((it / RS) - 1) & 1, abort_flag, p.status);
         if (!ok) break;
         if (bad) {
-          if (lane == 0) mbar_arrive(kv_full(st));
+          if (lane == 0) mbar_arrive(ring_full(st));
         } else {
           const int key0 = (s.tile0 + k) * TK;
           const int npg = TK / p.page_size;
           int nvalid = 0;
           for (int q = 0; q < npg; ++q) nvalid += (key0 + q * p.page_size) < s.kv_len;
-          // box bx: page q = bx >> 1, K (even) or V (odd)
-          const int nbox = 2 * nvalid;
-          uint32_t mine = 0;
-          for (int bx = pw; bx < nbox; bx += nprod) mine += box_bytes;
-          if (lane == 0) mbar_arrive_tx(kv_full(st), mine);
-          for (int bx = pw; bx < nbox; bx += nprod) {
-            const int q = bx >> 1, isv = bx & 1;
+          if (lane == 0) mbar_arrive_tx(ring_full(st), static_cast<uint32_t>(nvalid) * box_bytes);
+          for (int q = 0; q < nvalid; ++q) {
             const int raw = page_of(s.b, key0 / p.page_size + q);
             const bool in_range = raw >= 0 && raw < p.num_pages;
             flag |= !in_range;
             const int page = in_range ? raw : 0;
-            if (lane == 0) {
-              const uint32_t dst = sbase + (isv ? C::OFF_V : C::OFF_K) + st * C::KV_BYTES +
-                                   static_cast<uint32_t>(q) * box_bytes;
-              tma_load_page(dst, isv ? &tmap_v : &tmap_k, page * p.hkv + s.g, kv_full(st));
-            }
+            if (lane == 0)
+              tma_load_page<HP>(ring_base + st * C::KV_BYTES + static_cast<uint32_t>(q) * box_bytes, map,
+                                page * p.hkv + s.g * HP, ring_full(st));
           }
         }
         __syncwarp();
@@ -305,11 +360,10 @@ __global__ void __launch_bounds__(TcCfg<D, MT, QR>::THREADS, 1)
       if (!has_more(s, t1, OVH)) break;
       s = locate<TK>(s.vnext, t1, p, pb, OVH);
     }
-    if (!ok) {  // drain this block's copies still in flight (bounded)
-      for (uint32_t x = it > static_cast<uint32_t>(C::STAGES) ? it - C::STAGES : 0; x < it; ++x) {
+    if (!ok) {  // drain this producer's copies still in flight (bounded)
+      for (uint32_t x = it > RS ? it - RS : 0; x < it; ++x) {
         const long long t_0 = clock64();
-        while (!mbar_try(kv_full(x % C::STAGES), (x / C::STAGES) & 1) &&
-               clock64() - t_0 < kWaitLimitCycles) {
+        while (!mbar_try(ring_full(x % RS), (x / RS) & 1) && clock64() - t_0 < kWaitLimitCycles) {
         }
       }
     }
@@ -319,25 +373,45 @@ __global__ void __launch_bounds__(TcCfg<D, MT, QR>::THREADS, 1)
     // tile's K has landed and its S buffer is free (so it runs up to two tiles ahead),
     // warp 3 issues O += P V as soon as a tile's P is written. A blocked issue of one
     // kind never delays the other.
-    // K and V stages hold a tile as [8-key group][128-byte column half][8 keys][128 B]:
-    // 8-key groups sit at a uniform stride of DH KB across pages, so Q K^T runs with
-    // N = 64 keys and P V reads V MN-major with the column halves 1 KB apart.
-    constexpr uint32_t kGroup = C::DH * 1024u;
+    // K and V stages hold a tile as [8-key group][head][128-byte column half][8 keys]
+    // [128 B]: 8-key groups sit at a uniform stride of HP * DH KB across pages, so Q K^T
+    // runs with N = 64 keys and P V reads V MN-major with the column halves 1 KB apart.
+    constexpr uint32_t kGroup = HP * C::DH * 1024u;
+    constexpr uint32_t kHead = C::DH * 1024u;  // the second head of a pair in a key group
     constexpr uint32_t kIdescQK = idesc_bf16(128, TK, false);
     constexpr uint32_t kIdescPV = idesc_bf16(128, D, true);
     const bool qk_role = warp == 1;
     uint32_t it = 0, seg_no = 0;
     bool ok = true;
     bool issued = false;
-    // Q tiles of a segment (all M tiles, both column halves) by TMA, on q_full
+    // Q tiles of a segment (all M tiles, both column halves, each head of a pair) by TMA,
+    // on q_full
     auto issue_q = [&](const Seg& sg) {
       if (lane == 0) {
         mbar_arrive_tx(q_full, C::Q_BYTES);
         for (int mt = 0; mt < MT; ++mt)
           for (int half = 0; half < C::DH; ++half)
-            tma_load_q(sbase + C::OFF_Q + (mt * C::DH + half) * C::QHALF, &tmap_q, half,
-                       sg.g * p.group,
-                       sg.b * p.gamma + (sg.rt * p.rows_per_cta + mt * 128) / p.group, q_full);
+            for (int h = 0; h < HP; ++h)
+              tma_load_q(sbase + C::OFF_Q + (mt * C::DH + half) * C::QHALF + h * (QR * 128u), &tmap_q,
+                         half, (sg.g * HP + h) * p.group,
+                         sg.b * p.gamma + (sg.rt * p.rows_per_cta + mt * 128) / p.group, q_full);
+      }
+      __syncwarp();
+    };
+    // keys past the end of the sequence: zero their V rows so that P = 0 meets finite V
+    auto zero_v_tail = [&](uint32_t vstage, const Seg& sg, int k) {
+      const int key0 = (sg.tile0 + k) * TK;
+      const int nvalid = sg.len_ok ? min(TK, max(0, sg.kv_len - key0)) : TK;
+      if (nvalid < TK) {
+        unsigned char* vst = smem + C::OFF_V + vstage * C::KV_BYTES;
+        constexpr int kPieces = HP * C::DH * 8;  // 16-byte pieces of one key's rows
+        for (int i = lane; i < (TK - nvalid) * kPieces; i += 32) {
+          const int key = nvalid + i / kPieces, r = i % kPieces;
+          const int h = r / (C::DH * 8), hh = (r / 8) % C::DH, c = r % 8;
+          *reinterpret_cast<uint4*>(vst + (key >> 3) * kGroup + h * kHead + hh * 1024u +
+                                    (key & 7) * 128u + c * 16u) = make_uint4(0, 0, 0, 0);
+        }
+        fence_async_smem();
       }
       __syncwarp();
     };
@@ -353,41 +427,37 @@ __global__ void __launch_bounds__(TcCfg<D, MT, QR>::THREADS, 1)
       }
       for (int k = 0; k < s.ntile && ok; ++k) {
         const uint32_t x = it + k;
-        const int st = x % C::STAGES;
         if (qk_role) {
-          // S = Q K^T for tile x into S[mt][x & 1]
-          ok = mbar_wait(kv_full(st), (x / C::STAGES) & 1, abort_flag, p.status);
+          // S = Q K^T for tile x into S[mt * HP + h][x & 1]
+          const uint32_t st = x % C::KST;
+          ok = HP == 2 ? mbar_wait(k_full(st), (x / C::KST) & 1, abort_flag, p.status)
+                       : mbar_wait(kv_full(st), (x / C::STAGES) & 1, abort_flag, p.status);
           if (!ok) break;
-          // keys past the end of the sequence: zero their V rows so that P = 0 meets
-          // finite V
-          const int key0 = (s.tile0 + k) * TK;
-          const int nvalid = s.len_ok ? min(TK, max(0, s.kv_len - key0)) : TK;
-          if (nvalid < TK) {
-            unsigned char* vst = smem + C::OFF_V + st * C::KV_BYTES;
-            for (int i = lane; i < (TK - nvalid) * C::DH * 8; i += 32) {
-              const int key = nvalid + i / (C::DH * 8), h = (i / 8) % C::DH, c = i % 8;
-              *reinterpret_cast<uint4*>(vst + (key >> 3) * kGroup + h * 1024u + (key & 7) * 128u +
-                                        c * 16u) = make_uint4(0, 0, 0, 0);
-            }
-            fence_async_smem();
-          }
-          __syncwarp();
+          if (HP == 1) zero_v_tail(st, s, k);  // the stage's V has landed with its K
+          // S[x & 1] is free once tile x - 2's softmax has read it (and, with P in TMEM,
+          // once that tile's P V MMAs have read its P)
           if (x >= 2)
             for (int mt = 0; mt < MT && ok; ++mt)
-              ok = mbar_wait(s_free(mt, x & 1), ((x >> 1) - 1) & 1, abort_flag, p.status);
+              ok = mbar_wait(C::PTMEM ? pv_done(mt, x & 1) : s_free(mt, x & 1), ((x >> 1) - 1) & 1,
+                             abort_flag, p.status);
           if (!ok) break;
           tc_fence_after();
           if (lane == 0) {
             for (int mt = 0; mt < MT; ++mt) {
-              const uint32_t d_tmem = tmem + C::S_COL + (mt * 2 + (x & 1)) * TK;
 #pragma unroll
-              for (int kk = 0; kk < D / 16; ++kk) {
-                const uint32_t qa = sbase + C::OFF_Q + (mt * C::DH + kk / 4) * C::QHALF + (kk % 4) * 32u;
-                const uint32_t kb = sbase + C::OFF_K + st * C::KV_BYTES + (kk / 4) * 1024u + (kk % 4) * 32u;
-                mma_bf16(d_tmem, desc_sw128(qa, 16, 1024), desc_sw128(kb, 16, kGroup), kIdescQK, kk > 0);
+              for (int h = 0; h < HP; ++h) {
+                const uint32_t d_tmem = tmem + C::S_COL + ((mt * HP + h) * 2 + (x & 1)) * TK;
+#pragma unroll
+                for (int kk = 0; kk < D / 16; ++kk) {
+                  const uint32_t qa = sbase + C::OFF_Q + (mt * C::DH + kk / 4) * C::QHALF + (kk % 4) * 32u;
+                  const uint32_t kb = sbase + C::OFF_K + st * C::KV_BYTES + h * kHead + (kk / 4) * 1024u +
+                                      (kk % 4) * 32u;
+                  mma_bf16(d_tmem, desc_sw128(qa, 16, 1024), desc_sw128(kb, 16, kGroup), kIdescQK, kk > 0);
+                }
               }
               mma_commit(s_full(mt, x & 1));
             }
+            if (HP == 2) mma_commit(k_empty(st));
             issued = true;
           }
           __syncwarp();
@@ -399,7 +469,14 @@ __global__ void __launch_bounds__(TcCfg<D, MT, QR>::THREADS, 1)
             issue_q(locate<TK>(s.vnext, t1, p, pb, OVH));
           }
         } else {
-          // O += P V for tile x (its P implies its S, hence its landed stage)
+          // O += P V for tile x (its P implies its S, hence its landed K stage; with a
+          // head pair the V stage has its own barrier)
+          const uint32_t st = x % C::VST;
+          if (HP == 2) {
+            ok = mbar_wait(v_full(st), (x / C::VST) & 1, abort_flag, p.status);
+            if (!ok) break;
+            zero_v_tail(st, s, k);
+          }
           const int pbuf = static_cast<int>(x % PB);
           for (int mt = 0; mt < MT && ok; ++mt)
             ok = mbar_wait(p_full(mt, pbuf), (x / PB) & 1, abort_flag, p.status);
@@ -408,21 +485,29 @@ __global__ void __launch_bounds__(TcCfg<D, MT, QR>::THREADS, 1)
           if (lane == 0) {
             for (int mt = 0; mt < MT; ++mt) {
 #pragma unroll
-              for (int hf = 0; hf < SPLIT; ++hf) {
-                // each key half accumulates into its own O
-                const uint32_t d_tmem = tmem + C::O_COL + (mt * SPLIT + hf) * D;
+              for (int h = 0; h < HP; ++h) {
 #pragma unroll
-                for (int kk = 0; kk < KH / 16; ++kk) {
-                  const int kg = hf * (KH / 16) + kk;  // 16-key step within the tile
-                  const uint32_t pa = sbase + C::OFF_P + (pbuf * MT + mt) * C::PBUF + kg * 32u;
-                  const uint32_t vb = sbase + C::OFF_V + st * C::KV_BYTES + kg * 2u * kGroup;
-                  mma_bf16(d_tmem, desc_sw128(pa, 16, 1024), desc_sw128(vb, 1024, kGroup), kIdescPV,
-                           (k > 0 || kk > 0) ? 1u : 0u);
+                for (int hf = 0; hf < SPLIT; ++hf) {
+                  // each key half accumulates into its own O
+                  const uint32_t d_tmem = tmem + C::O_COL + ((mt * HP + h) * SPLIT + hf) * D;
+#pragma unroll
+                  for (int kk = 0; kk < KH / 16; ++kk) {
+                    const int kg = hf * (KH / 16) + kk;  // 16-key step within the tile
+                    const uint32_t vb = sbase + C::OFF_V + st * C::KV_BYTES + h * kHead + kg * 2u * kGroup;
+                    if constexpr (C::PTMEM) {  // P from TMEM: 8 columns per 16 keys
+                      mma_bf16_ta(d_tmem, tmem + C::S_COL + pbuf * TK + kg * 8u, desc_sw128(vb, 1024, kGroup),
+                                  kIdescPV, (k > 0 || kk > 0) ? 1u : 0u);
+                    } else {
+                      const uint32_t pa = sbase + C::OFF_P + (pbuf * MT + mt) * C::PBUF + kg * 32u;
+                      mma_bf16(d_tmem, desc_sw128(pa, 16, 1024), desc_sw128(vb, 1024, kGroup), kIdescPV,
+                               (k > 0 || kk > 0) ? 1u : 0u);
+                    }
+                  }
                 }
               }
               mma_commit(pv_done(mt, pbuf));
             }
-            mma_commit(kv_empty(st));
+            mma_commit(HP == 2 ? v_empty(st) : kv_empty(st));
             issued = true;
           }
           __syncwarp();
@@ -441,20 +526,25 @@ __global__ void __launch_bounds__(TcCfg<D, MT, QR>::THREADS, 1)
       while (!mbar_try(db, 0) && clock64() - t_0 < kWaitLimitCycles) {
       }
     }
-  } else if (warp >= 4 && ((warp - 4) & 3) < nact[((warp - 4) >> 2) / SPLIT]) {
+  } else if (warp >= 4 && soft_active(warp - 4)) {
     // ====================== softmax (warps with real rows) ======================
-    const int sw = warp - 4, q4 = sw & 3, mt = (sw >> 2) / SPLIT, hf = (sw >> 2) % SPLIT;
-    const int row = q4 * 32 + lane;  // TMEM lane = row of this M tile
-    const int lrow = mt * 128 + row;  // row within the block's row tile
+    const int sw = warp - 4, q4 = sw & 3;
+    const int mt = HP == 2 ? 0 : (sw >> 2) / SPLIT, hf = HP == 2 ? 0 : (sw >> 2) % SPLIT;
+    const int hp = HP == 2 ? q4 >> 1 : 0;  // head of the pair
+    const int row = q4 * 32 + lane;        // TMEM lane = row of this M tile
+    // row within the unit's row tile (of its head)
+    const int lrow = HP == 2 ? (q4 & 1) * 32 + lane : mt * 128 + row;
+    const int acc = mt * HP + hp;          // this row's S and O accumulators
     const uint32_t lane_base = tmem + (static_cast<uint32_t>(q4 * 32) << 16);
-    const uint32_t ocol = lane_base + C::O_COL + (mt * SPLIT + hf) * D;  // this half's O
-    const uint32_t o0col = lane_base + C::O_COL + mt * SPLIT * D;        // first half's O
+    const uint32_t ocol = lane_base + C::O_COL + (acc * SPLIT + hf) * D;  // this half's O
+    const uint32_t o0col = lane_base + C::O_COL + acc * SPLIT * D;        // first half's O
+    const int prow = hp * p.rows + lrow;  // row within a partial slot
     constexpr int kChunks = D / 8 / SPLIT;  // 16-byte pieces of a query row per warp
     uint32_t it = 0, xphase = 0;
     bool ok = true;
     // A row of a segment: the unit row it holds and whether it is a real query row.
     struct RowOf {
-      int urow, j, h;
+      int urow, j, h, kvh;
       bool real;
     };
     auto row_of = [&](const Seg& sg) {
@@ -462,7 +552,8 @@ __global__ void __launch_bounds__(TcCfg<D, MT, QR>::THREADS, 1)
       r.urow = sg.rt * p.rows_per_cta + lrow;
       r.real = r.urow < p.rows && lrow < p.rows_per_cta;
       r.j = r.urow / p.group;
-      r.h = sg.g * p.group + r.urow % p.group;
+      r.kvh = sg.g * HP + hp;
+      r.h = r.kvh * p.group + r.urow % p.group;
       return r;
     };
     // this warp's share of a query row (zeros for padding rows)
@@ -510,7 +601,7 @@ __global__ void __launch_bounds__(TcCfg<D, MT, QR>::THREADS, 1)
         float v[KH];
         {
           uint32_t r[32];
-          const uint32_t col = C::S_COL + (mt * 2 + (x & 1)) * TK + hf * KH;
+          const uint32_t col = C::S_COL + (acc * 2 + (x & 1)) * TK + hf * KH;
 #pragma unroll
           for (int q = 0; q < KH / 32; ++q) {
             tmem_ld32(lane_base + col + q * 32, r);
@@ -521,7 +612,7 @@ __global__ void __launch_bounds__(TcCfg<D, MT, QR>::THREADS, 1)
         }
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(s_free(mt, x & 1));
+        if (lane == 0 && !C::PTMEM) mbar_arrive(s_free(mt, x & 1));
         // scale to base 2 and mask keys past ctx + j
         const int key0 = (s.tile0 + k) * TK + hf * KH;
         const int lim = ctx + ro.j - key0;  // keys c <= lim are visible
@@ -585,14 +676,20 @@ __global__ void __launch_bounds__(TcCfg<D, MT, QR>::THREADS, 1)
           }
           tmem_wait_st();
         }
-        unsigned char* prow = smem + C::OFF_P + (pbuf * MT + mt) * C::PBUF + row * 128u;
+        if constexpr (C::PTMEM) {
+          // P as bf16 pairs over the first 32 columns of S[0][x & 1] (this row's lane)
+          tmem_st32(lane_base + C::S_COL + (x & 1) * TK, pk);
+          tmem_wait_st();
+        } else {
+          unsigned char* prow = smem + C::OFF_P + (pbuf * MT + mt) * C::PBUF + row * 128u;
 #pragma unroll
-        for (int c2 = 0; c2 < KH / 8; ++c2) {
-          const int c = hf * (KH / 8) + c2;
-          *reinterpret_cast<uint4*>(prow + ((c ^ (row & 7)) << 4)) =
-              make_uint4(pk[4 * c2], pk[4 * c2 + 1], pk[4 * c2 + 2], pk[4 * c2 + 3]);
+          for (int c2 = 0; c2 < KH / 8; ++c2) {
+            const int c = hf * (KH / 8) + c2;
+            *reinterpret_cast<uint4*>(prow + ((c ^ (row & 7)) << 4)) =
+                make_uint4(pk[4 * c2], pk[4 * c2 + 1], pk[4 * c2 + 2], pk[4 * c2 + 3]);
+          }
+          fence_async_smem();
         }
-        fence_async_smem();
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(p_full(mt, pbuf));
@@ -667,9 +764,9 @@ __global__ void __launch_bounds__(TcCfg<D, MT, QR>::THREADS, 1)
             for (int e = 0; e < 32; ++e) o[e] = 0.f;
           }
 #pragma unroll
-          for (int e = 0; e < 32; e += 8) write_out_row<D>(p, s.b, s.g, ro.urow, cc * 32 + e, o + e, inv);
+          for (int e = 0; e < 32; e += 8) write_out_row<D>(p, s.b, ro.kvh, ro.urow, cc * 32 + e, o + e, inv);
         } else {
-          float4* dst = reinterpret_cast<float4*>(p.partial_o + (slot * p.slot_rows + lrow) * D + cc * 32);
+          float4* dst = reinterpret_cast<float4*>(p.partial_o + (slot * p.slot_rows + prow) * D + cc * 32);
 #pragma unroll
           for (int e = 0; e < 8; ++e)
             dst[e] = make_float4(o[4 * e], o[4 * e + 1], o[4 * e + 2], o[4 * e + 3]);
@@ -677,8 +774,8 @@ __global__ void __launch_bounds__(TcCfg<D, MT, QR>::THREADS, 1)
       }
       tc_fence_before();
       if (ro.real && hf == 0) {
-        if (whole) write_lse(p, s.b, s.g, ro.urow, M, L, bad);
-        else p.partial_ml[slot * p.slot_rows + lrow] = make_float2(M, bad ? -1.f : L);
+        if (whole) write_lse(p, s.b, ro.kvh, ro.urow, M, L, bad);
+        else p.partial_ml[slot * p.slot_rows + prow] = make_float2(M, bad ? -1.f : L);
       }
       if (!whole && sw == 0 && lane == 0) {
         // the ticket of a split unit is taken at the end of the block, after a fence
@@ -721,7 +818,13 @@ __global__ void __launch_bounds__(TcCfg<D, MT, QR>::THREADS, 1)
       if (any) __threadfence();
       for (int i = 0; i < np; ++i) {
         const int* e = pend + 8 * i;
-        if (e[7]) merge_unit<D>(p, e[0], e[1], e[2], e[3], e[4], e[5], threadIdx.x, C::THREADS);
+        if (!e[7]) continue;
+        if (HP == 2) {  // the pair's heads, the second's rows after the first's in a slot
+          merge_unit<D>(p, e[0], 2 * e[1], e[2], e[3], e[4], e[5], threadIdx.x, C::THREADS, 0);
+          merge_unit<D>(p, e[0], 2 * e[1] + 1, e[2], e[3], e[4], e[5], threadIdx.x, C::THREADS, p.rows);
+        } else {
+          merge_unit<D>(p, e[0], e[1], e[2], e[3], e[4], e[5], threadIdx.x, C::THREADS);
+        }
       }
     }
   }
@@ -730,12 +833,12 @@ __global__ void __launch_bounds__(TcCfg<D, MT, QR>::THREADS, 1)
 // ---------------------------------------------------------------------------------
 // Host side
 // ---------------------------------------------------------------------------------
-template <int D, int MT, int QR>
+template <int D, int MT, int QR, int HP>
 cudaError_t launch_typed(const spec_attn_args_t& a, const AttnPlan& P, char* ws,
                          cudaStream_t stream, bool starve) {
-  using Cf = TcCfg<D, MT, QR>;
+  using Cf = TcCfg<D, MT, QR, HP>;
   CUtensorMap mk, mv, mq;
-  if (!encode_cache_map(&mk, a.k_cache, a) || !encode_cache_map(&mv, a.v_cache, a))
+  if (!encode_cache_map(&mk, a.k_cache, a, HP) || !encode_cache_map(&mv, a.v_cache, a, HP))
     return cudaErrorInvalidValue;
   AttnParams p = make_attn_params(a, P, ws);
   p.starve = starve ? 1 : 0;
@@ -743,11 +846,11 @@ cudaError_t launch_typed(const spec_attn_args_t& a, const AttnPlan& P, char* ws,
   // Charge unit starts only when blocks hold several of them; when every unit is spread
   // over several blocks, a block holds at most one start and the charge would mostly
   // move real tiles away from blocks that pay no boundary.
-  const int64_t units = static_cast<int64_t>(a.batch) * a.num_kv_heads * P.row_tiles;
+  const int64_t units = static_cast<int64_t>(a.batch) * p.hunits * P.row_tiles;
   p.unit_overhead = units > P.grid ? Cf::UNIT_OVERHEAD : 0;
   if (!p.q_tma) mq = mk;  // unused
   const size_t smem = Cf::smem_bytes(a.batch);
-  auto kernel = a.tree_mask ? attn_tc_kernel<D, MT, true, QR> : attn_tc_kernel<D, MT, false, QR>;
+  auto kernel = a.tree_mask ? attn_tc_kernel<D, MT, true, QR, HP> : attn_tc_kernel<D, MT, false, QR, HP>;
   cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
@@ -762,15 +865,24 @@ cudaError_t launch_typed(const spec_attn_args_t& a, const AttnPlan& P, char* ws,
 // page/8 groups of 8 rows at stride 8*D*2 bytes; page * Hkv + head at stride page*D*2).
 // The box lands in shared memory as [row group][column half][8 rows][128 B], so the
 // 8-row groups of a 64-key tile sit at a uniform stride whatever the page size.
-bool encode_cache_map(CUtensorMap* map, const void* base, const spec_attn_args_t& a) {
+// With heads_per_box = 2 the last two dimensions swap places and the box takes two
+// adjacent heads (8 KB contiguous in the cache with 16-token pages, D = 128), landing as
+// [row group][head][column half][8 rows][128 B]: the groups of one head keep a uniform
+// stride, and the heads sit DH KB apart within a group.
+bool encode_cache_map(CUtensorMap* map, const void* base, const spec_attn_args_t& a,
+                      int heads_per_box) {
   tcx::EncodeTiledFn enc = tcx::encoder();
   if (!enc) return false;
   const cuuint64_t D = static_cast<cuuint64_t>(a.head_dim);
-  const cuuint64_t dims[5] = {64, 8, D / 64, static_cast<cuuint64_t>(a.page_size / 8),
-                              static_cast<cuuint64_t>(a.num_pages) * a.num_kv_heads};
-  const cuuint64_t strides[4] = {D * 2, 128, 8 * D * 2, static_cast<cuuint64_t>(a.page_size) * D * 2};
+  const cuuint64_t groups = static_cast<cuuint64_t>(a.page_size / 8);
+  const cuuint64_t page_heads = static_cast<cuuint64_t>(a.num_pages) * a.num_kv_heads;
+  const cuuint64_t page_stride = static_cast<cuuint64_t>(a.page_size) * D * 2;
+  const bool pair = heads_per_box == 2;
+  const cuuint64_t dims[5] = {64, 8, D / 64, pair ? page_heads : groups, pair ? groups : page_heads};
+  const cuuint64_t strides[4] = {D * 2, 128, pair ? page_stride : 8 * D * 2, pair ? 8 * D * 2 : page_stride};
   const cuuint32_t box[5] = {64, 8, static_cast<cuuint32_t>(D / 64),
-                             static_cast<cuuint32_t>(a.page_size / 8), 1};
+                             pair ? 2u : static_cast<cuuint32_t>(groups),
+                             pair ? static_cast<cuuint32_t>(groups) : 1u};
   const cuuint32_t estr[5] = {1, 1, 1, 1, 1};
   return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void*>(base), dims, strides, box,
              estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -801,44 +913,64 @@ bool encode_q_map(CUtensorMap* map, const spec_attn_args_t& a, int tile_rows) {
 }
 
 // The buffer configuration of the row-tile kernel: two M tiles, one M tile with 128-row
-// buffers, or one M tile with 64-row buffers (at most 64 query rows per KV group).
-enum TcVariant { kTwoTiles, kOneTile, kOneTileHalf };
-TcVariant tc_variant(int rows_per_cta, int rows) {
-  return rows_per_cta > 128 ? kTwoTiles : (rows <= 64 ? kOneTileHalf : kOneTile);
+// buffers, one M tile with 64-row buffers (at most 64 query rows per KV group), or one M
+// tile of two KV heads' 64-row groups.
+enum TcVariant { kTwoTiles, kOneTile, kOneTileHalf, kHeadPair };
+TcVariant tc_variant(int rows_per_cta, int rows, bool head_pair) {
+  return head_pair ? kHeadPair : rows_per_cta > 128 ? kTwoTiles : (rows <= 64 ? kOneTileHalf : kOneTile);
 }
 
-size_t tc_smem_bytes(int head_dim, int rows_per_cta, int rows, int batch) {
-  const TcVariant v = tc_variant(rows_per_cta, rows);
-  if (head_dim == 128)
-    return v == kTwoTiles ? TcCfg<128, 2>::smem_bytes(batch)
-           : v == kOneTile ? TcCfg<128, 1>::smem_bytes(batch) : TcCfg<128, 1, 64>::smem_bytes(batch);
-  return v == kTwoTiles ? TcCfg<64, 2>::smem_bytes(batch)
-         : v == kOneTile ? TcCfg<64, 1>::smem_bytes(batch) : TcCfg<64, 1, 64>::smem_bytes(batch);
+template <int D>
+size_t smem_of(TcVariant v, int batch) {
+  return v == kTwoTiles     ? TcCfg<D, 2>::smem_bytes(batch)
+         : v == kOneTile    ? TcCfg<D, 1>::smem_bytes(batch)
+         : v == kOneTileHalf ? TcCfg<D, 1, 64>::smem_bytes(batch)
+                             : TcCfg<D, 1, 64, 2>::smem_bytes(batch);
 }
 
-int tc_ctas_per_sm(int head_dim, int rows_per_cta, int rows, int batch) {
+size_t tc_smem_bytes(int head_dim, int rows_per_cta, int rows, int batch, bool head_pair) {
+  const TcVariant v = tc_variant(rows_per_cta, rows, head_pair);
+  return head_dim == 128 ? smem_of<128>(v, batch) : smem_of<64>(v, batch);
+}
+
+// With at most 32 rows per group a pair would leave two lane quadrants idle and give each
+// softmax warp a whole tile's keys where the one-head kernel splits them over two warps
+// (measured slower at 32 rows: llama8b attention 50.7 against 48.1 us).
+bool tc_head_pair(int head_dim, int rows, int num_kv_heads, int batch) {
+  return rows > 32 && rows <= 64 && num_kv_heads % 2 == 0 &&
+         tc_smem_bytes(head_dim, 128, rows, batch, true) <= kTcMaxSmem;
+}
+
+int tc_ctas_per_sm(int head_dim, int rows_per_cta, int rows, int batch, bool head_pair) {
   // Shared memory bounds residency (227 KB usable per SM); TMEM (512 columns) too.
-  const size_t smem = tc_smem_bytes(head_dim, rows_per_cta, rows, batch);
-  int by_smem = static_cast<int>((227u * 1024u) / (smem + 1024));
-  const bool two = rows_per_cta > 128;
-  const int cols = static_cast<int>(
-      head_dim == 128 ? (two ? TcCfg<128, 2>::TMEM_COLS : TcCfg<128, 1>::TMEM_COLS)
-                      : (two ? TcCfg<64, 2>::TMEM_COLS : TcCfg<64, 1>::TMEM_COLS));
-  const int by_tmem = 512 / cols;
+  const size_t smem = tc_smem_bytes(head_dim, rows_per_cta, rows, batch, head_pair);
+  int by_smem = static_cast<int>(kTcMaxSmem / (smem + 1024));
+  const TcVariant v = tc_variant(rows_per_cta, rows, head_pair);
+  const uint32_t cols =
+      head_dim == 128
+          ? (v == kTwoTiles ? TcCfg<128, 2>::TMEM_COLS
+             : v == kHeadPair ? TcCfg<128, 1, 64, 2>::TMEM_COLS : TcCfg<128, 1>::TMEM_COLS)
+          : (v == kTwoTiles ? TcCfg<64, 2>::TMEM_COLS
+             : v == kHeadPair ? TcCfg<64, 1, 64, 2>::TMEM_COLS : TcCfg<64, 1>::TMEM_COLS);
+  const int by_tmem = static_cast<int>(512 / cols);
   int n = by_smem < by_tmem ? by_smem : by_tmem;
   return n < 1 ? 1 : n;
 }
 
+template <int D>
+cudaError_t launch_d(TcVariant v, const spec_attn_args_t& a, const AttnPlan& P, char* ws,
+                     cudaStream_t stream, bool starve) {
+  return v == kTwoTiles     ? launch_typed<D, 2, 128, 1>(a, P, ws, stream, starve)
+         : v == kOneTile    ? launch_typed<D, 1, 128, 1>(a, P, ws, stream, starve)
+         : v == kOneTileHalf ? launch_typed<D, 1, 64, 1>(a, P, ws, stream, starve)
+                             : launch_typed<D, 1, 64, 2>(a, P, ws, stream, starve);
+}
+
 cudaError_t launch_attn_tc(const spec_attn_args_t& a, const AttnPlan& P, char* ws,
                            cudaStream_t stream, bool starve) {
-  const TcVariant v = tc_variant(P.rows_per_cta, P.rows);
-  if (a.head_dim == 128)
-    return v == kTwoTiles ? launch_typed<128, 2, 128>(a, P, ws, stream, starve)
-           : v == kOneTile ? launch_typed<128, 1, 128>(a, P, ws, stream, starve)
-                           : launch_typed<128, 1, 64>(a, P, ws, stream, starve);
-  return v == kTwoTiles ? launch_typed<64, 2, 128>(a, P, ws, stream, starve)
-         : v == kOneTile ? launch_typed<64, 1, 128>(a, P, ws, stream, starve)
-                         : launch_typed<64, 1, 64>(a, P, ws, stream, starve);
+  const TcVariant v = tc_variant(P.rows_per_cta, P.rows, P.head_pair != 0);
+  return a.head_dim == 128 ? launch_d<128>(v, a, P, ws, stream, starve)
+                           : launch_d<64>(v, a, P, ws, stream, starve);
 }
 
 }  // namespace specv

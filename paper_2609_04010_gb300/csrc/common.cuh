@@ -138,6 +138,7 @@ cudaError_t launch_tree_build(const spec_tree_build_args_t& t, const TreeBuildLa
 struct AttnPlan {
   int path;          // SPEC_ATTN_CUDA_CORES or SPEC_ATTN_TENSOR_CORES
   int keys_on_lanes; // tensor cores: the keys-on-lanes kernel (attn_kl.cu), else row tiles
+  int head_pair;     // row tiles: one block serves two adjacent KV heads (8 KB page boxes)
   int rows;          // (Hq/Hkv) * gamma
   int rows_per_cta;  // rows one block handles (a row tile)
   int row_tiles;     // ceil(rows / rows_per_cta)
@@ -230,9 +231,13 @@ struct DeviceScope {
   DeviceScope& operator=(const DeviceScope&) = delete;
 };
 
-int tc_ctas_per_sm(int head_dim, int rows_per_cta, int rows, int batch);
-size_t tc_smem_bytes(int head_dim, int rows_per_cta, int rows, int batch);
+int tc_ctas_per_sm(int head_dim, int rows_per_cta, int rows, int batch, bool head_pair);
+size_t tc_smem_bytes(int head_dim, int rows_per_cta, int rows, int batch, bool head_pair);
+// Whether the row-tile kernel serves two adjacent KV heads per block: KV groups of 33 to
+// 64 rows, an even Hkv, and the batch's prefix sums fit beside its stages.
+bool tc_head_pair(int head_dim, int rows, int num_kv_heads, int batch);
 constexpr int kTcMaxBatch = 4096;  // batch prefix sums live in shared memory
+constexpr size_t kTcMaxSmem = 227u * 1024u;  // dynamic shared memory of one block
 
 }  // namespace specv
 

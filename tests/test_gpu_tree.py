@@ -180,9 +180,11 @@ def attn_tree_inputs(seed, batch, N, hq, hkv, D, P, ctx):
 
 
 @pytest.mark.parametrize("path", [binding.ATTN_TENSOR_CORES, binding.ATTN_CUDA_CORES])
+# 132 rows per KV group (one M tile), 244 (two), 17, and 48 (two KV heads per block)
 @pytest.mark.parametrize("N,hq,hkv,D,P,ctx,batch", [(33, 32, 8, 128, 16, 4096, 1),
                                                     (61, 32, 8, 128, 16, 2000, 2),
-                                                    (17, 8, 8, 64, 64, (100, 900), 4)])
+                                                    (17, 8, 8, 64, 64, (100, 900), 4),
+                                                    (12, 32, 8, 128, 16, (300, 1500), 3)])
 def test_tree_attention(oracle_mod, path, N, hq, hkv, D, P, ctx, batch):
     rng = np.random.default_rng(N * 7 + batch)
     inp = attn_tree_inputs(N + batch, batch, N, hq, hkv, D, P, ctx)
