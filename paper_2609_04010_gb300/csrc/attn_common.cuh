@@ -180,59 +180,88 @@ __device__ __forceinline__ void write_lse(const AttnParams& p, int b, int g, int
 // Combines the split-KV partials of one unit, held in slots [slot0, slot0 + nslots), for
 // rows [row0, row0 + nrows) and writes the final outputs (nthreads threads from tid
 // cooperate; no block synchronization). Row r of the range sits at row prow0 + r of a
-// slot (a head-pair unit keeps its second head's rows after the first's). Each (row, 8-column) item walks the slots in
-// batches of four, loading a batch's (m, l) pairs and output pieces together and
-// folding them into a running base-2 max, so a unit with up to four slots costs one
-// round trip to L2.
-template <int D>
+// slot (a head-pair unit keeps its second head's rows after the first's). A thread takes
+// its (row, 8-column) items IT at a time and walks their slots in batches of SB: the
+// (m, l) pairs and output pieces of those items and slots are loaded together, then
+// folded into each item's running base-2 max. The merges run at the end of a block
+// while the others still stream KV, when an L2 round trip takes about a microsecond:
+// units of 128 or more rows (2,048+ items for D = 128) take four items per thread
+// (IT = 4, SB = 2) to cut their dependent round trips; smaller ones keep one item per
+// thread with up to four slots per batch (IT = 1, SB = 4), which measured faster in the
+// fused step for 32-row units.
+template <int D, int IT = 1>
 __device__ void merge_unit(const AttnParams& p, int b, int g, int row0, int nrows, int64_t slot0,
                            int nslots, int tid, int nthreads, int prow0 = 0) {
   constexpr int C8 = D / 8;
-  for (int idx = tid; idx < nrows * C8; idx += nthreads) {
-    const int r = idx / C8, c8 = idx % C8;
-    float M = -INFINITY, L = 0.f, acc[8];
+  constexpr int SB = IT == 1 ? 4 : 2;  // slots per batch
+  const int nitems = nrows * C8;
+  for (int i0 = tid; i0 < nitems; i0 += IT * nthreads) {
+    float M[IT], L[IT], acc[IT][8];
+    bool bad[IT];
 #pragma unroll
-    for (int e = 0; e < 8; ++e) acc[e] = 0.f;
-    bool bad = false;
-    for (int s0 = 0; s0 < nslots; s0 += 4) {
-      float2 ml[4];
-      float4 lo[4], hi[4];
+    for (int i = 0; i < IT; ++i) {
+      M[i] = -INFINITY;
+      L[i] = 0.f;
+      bad[i] = false;
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        if (s0 + e < nslots) {
-          const int64_t slot = (slot0 + s0 + e) * p.slot_rows + prow0 + r;
-          ml[e] = __ldcg(&p.partial_ml[slot]);
-          const float4* src = reinterpret_cast<const float4*>(p.partial_o + slot * D) + 2 * c8;
-          lo[e] = __ldcg(src);
-          hi[e] = __ldcg(src + 1);
-        } else {
-          ml[e] = make_float2(-INFINITY, 0.f);
+      for (int e = 0; e < 8; ++e) acc[i][e] = 0.f;
+    }
+    for (int s0 = 0; s0 < nslots; s0 += SB) {
+      float2 ml[IT][SB];
+      float4 lo[IT][SB], hi[IT][SB];
+#pragma unroll
+      for (int i = 0; i < IT; ++i) {
+        const int idx = i0 + i * nthreads;
+        const int r = idx / C8, c8 = idx % C8;
+#pragma unroll
+        for (int e = 0; e < SB; ++e) {
+          if (idx < nitems && s0 + e < nslots) {
+            const int64_t slot = (slot0 + s0 + e) * p.slot_rows + prow0 + r;
+            ml[i][e] = __ldcg(&p.partial_ml[slot]);
+            const float4* src = reinterpret_cast<const float4*>(p.partial_o + slot * D) + 2 * c8;
+            lo[i][e] = __ldcg(src);
+            hi[i][e] = __ldcg(src + 1);
+          } else {
+            ml[i][e] = make_float2(-INFINITY, 0.f);
+            lo[i][e] = make_float4(0.f, 0.f, 0.f, 0.f);
+            hi[i][e] = lo[i][e];
+          }
         }
       }
-      float mb = M;
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        bad |= ml[e].y < 0.f;
-        if (ml[e].y > 0.f) mb = fmaxf(mb, ml[e].x);
+      for (int i = 0; i < IT; ++i) {
+        float mb = M[i];
+#pragma unroll
+        for (int e = 0; e < SB; ++e) {
+          bad[i] |= ml[i][e].y < 0.f;
+          if (ml[i][e].y > 0.f) mb = fmaxf(mb, ml[i][e].x);
+        }
+        if (mb == -INFINITY) continue;
+        const float scale = M[i] == -INFINITY ? 0.f : ex2(M[i] - mb);
+        L[i] *= scale;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc[i][e] *= scale;
+#pragma unroll
+        for (int e = 0; e < SB; ++e) {
+          if (!(ml[i][e].y > 0.f)) continue;
+          const float w = ex2(ml[i][e].x - mb);
+          const float4 a = lo[i][e], c = hi[i][e];
+          L[i] += ml[i][e].y * w;
+          acc[i][0] += a.x * w; acc[i][1] += a.y * w; acc[i][2] += a.z * w; acc[i][3] += a.w * w;
+          acc[i][4] += c.x * w; acc[i][5] += c.y * w; acc[i][6] += c.z * w; acc[i][7] += c.w * w;
+        }
+        M[i] = mb;
       }
-      if (mb == -INFINITY) continue;
-      const float scale = M == -INFINITY ? 0.f : ex2(M - mb);
-      L *= scale;
-#pragma unroll
-      for (int e = 0; e < 8; ++e) acc[e] *= scale;
-#pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        if (!(ml[e].y > 0.f)) continue;
-        const float w = ex2(ml[e].x - mb);
-        L += ml[e].y * w;
-        acc[0] += lo[e].x * w; acc[1] += lo[e].y * w; acc[2] += lo[e].z * w; acc[3] += lo[e].w * w;
-        acc[4] += hi[e].x * w; acc[5] += hi[e].y * w; acc[6] += hi[e].z * w; acc[7] += hi[e].w * w;
-      }
-      M = mb;
     }
-    const bool dead = bad || !(L > 0.f);
-    write_out_row<D>(p, b, g, row0 + r, c8 * 8, acc, dead ? 0.f : 1.f / L);
-    if (c8 == 0) write_lse(p, b, g, row0 + r, M, L, dead);
+#pragma unroll
+    for (int i = 0; i < IT; ++i) {
+      const int idx = i0 + i * nthreads;
+      if (idx >= nitems) break;
+      const int r = idx / C8, c8 = idx % C8;
+      const bool dead = bad[i] || !(L[i] > 0.f);
+      write_out_row<D>(p, b, g, row0 + r, c8 * 8, acc[i], dead ? 0.f : 1.f / L[i]);
+      if (c8 == 0) write_lse(p, b, g, row0 + r, M[i], L[i], dead);
+    }
   }
 }
 #endif

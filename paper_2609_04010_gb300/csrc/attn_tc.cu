@@ -819,11 +819,14 @@ __global__ void __launch_bounds__(TcCfg<D, MT, QR, HP>::THREADS, 1)
       for (int i = 0; i < np; ++i) {
         const int* e = pend + 8 * i;
         if (!e[7]) continue;
+        // units of 128+ rows (a head pair, two M tiles) keep four items per thread in flight
+        constexpr int kItems = (HP == 2 || MT == 2) ? 4 : 1;
         if (HP == 2) {  // the pair's heads, the second's rows after the first's in a slot
-          merge_unit<D>(p, e[0], 2 * e[1], e[2], e[3], e[4], e[5], threadIdx.x, C::THREADS, 0);
-          merge_unit<D>(p, e[0], 2 * e[1] + 1, e[2], e[3], e[4], e[5], threadIdx.x, C::THREADS, p.rows);
+          merge_unit<D, kItems>(p, e[0], 2 * e[1], e[2], e[3], e[4], e[5], threadIdx.x, C::THREADS, 0);
+          merge_unit<D, kItems>(p, e[0], 2 * e[1] + 1, e[2], e[3], e[4], e[5], threadIdx.x, C::THREADS,
+                                p.rows);
         } else {
-          merge_unit<D>(p, e[0], e[1], e[2], e[3], e[4], e[5], threadIdx.x, C::THREADS);
+          merge_unit<D, kItems>(p, e[0], e[1], e[2], e[3], e[4], e[5], threadIdx.x, C::THREADS);
         }
       }
     }
