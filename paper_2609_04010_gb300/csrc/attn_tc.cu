@@ -93,10 +93,13 @@ struct TcCfg {
   static constexpr uint32_t OFF_K = QR == 64 ? OFF_P + P_BYTES : OFF_Q + Q_BYTES;
   static constexpr uint32_t OFF_V = OFF_K + KST * KV_BYTES;
   static constexpr uint32_t OFF_BAR = QR == 64 ? OFF_V + VST * KV_BYTES : OFF_P + P_BYTES;
+  // the K and V stages, contiguous from OFF_K; at a block's end they stage the partials
+  // of the units it merges
+  static constexpr uint32_t RING_BYTES = (KST + VST) * KV_BYTES;
   // barriers: ring (kv_full[S], kv_empty[S], or k_full[KST], v_full[VST], k_empty[KST],
   // v_empty[VST]), s_full[MT][2], s_free[MT][2], p_full[MT][PB], pv_done[MT][PB],
-  // seg_ready, drain[2], xch[4], q_full, seg_flag_ready[8]
-  static constexpr int NBAR = RINGBARS + 4 * MT + 2 * MT * PB + 3 + 4 + 1 + 8;
+  // seg_ready, drain[2], xch[4], q_full, seg_flag_ready[8], merge_staged (HP = 2)
+  static constexpr int NBAR = RINGBARS + 4 * MT + 2 * MT * PB + 3 + 4 + 1 + 8 + (HP == 2 ? 1 : 0);
   static constexpr uint32_t OFF_MISC = OFF_BAR + NBAR * 8;  // tmem base, abort, pending count
   static constexpr uint32_t OFF_XCH = OFF_MISC + 16;        // [4][2][32] float2 (m, l) per half
   static constexpr uint32_t OFF_PEND = OFF_XCH + (SPLIT == 2 ? 4 * 2 * 32 * 8 : 0);  // [2][8]
@@ -142,9 +145,58 @@ __device__ __forceinline__ void tma_load_q(uint32_t dst, const CUtensorMap* map,
       "l"(reinterpret_cast<uint64_t>(map)), "r"(0), "r"(half), "r"(head0), "r"(pos0), "r"(bar)
       : "memory");
 }
+// Contiguous global -> shared copy by the copy engine, completing on bar (16-byte aligned
+// addresses, size a multiple of 16).
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+               "l"(src), "r"(bytes), "r"(bar)
+               : "memory");
+}
+// Orders this thread's view of global memory (generic proxy) before its later copies
+// by the copy engine (async proxy).
+__device__ __forceinline__ void fence_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
 __device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
   const __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
   return *reinterpret_cast<const uint32_t*>(&v);
+}
+
+// Merge of one unit from its partial slots staged in shared memory: so[nsl][slot_rows][D]
+// and sml[nsl][slot_rows] = (m, l), row r of [row0, row0 + nrows) at slot row prow0 + r.
+// The same combination as merge_unit, with every load from shared memory.
+template <int D>
+__device__ void merge_staged(const AttnParams& p, int b, int g, int row0, int nrows, const float* so,
+                             const float2* sml, int nsl, int prow0, int tid, int nthreads) {
+  constexpr int C8 = D / 8;
+  for (int idx = tid; idx < nrows * C8; idx += nthreads) {
+    const int r = idx / C8, c8 = idx % C8, pr = prow0 + r;
+    float mx = -INFINITY;
+    bool bad = false;
+    for (int i = 0; i < nsl; ++i) {
+      const float2 ml = sml[i * p.slot_rows + pr];
+      bad |= ml.y < 0.f;
+      if (ml.y > 0.f) mx = fmaxf(mx, ml.x);
+    }
+    float L = 0.f, acc[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) acc[e] = 0.f;
+    if (mx != -INFINITY) {
+      for (int i = 0; i < nsl; ++i) {
+        const float2 ml = sml[i * p.slot_rows + pr];
+        if (!(ml.y > 0.f)) continue;
+        const float w = ex2(ml.x - mx);
+        const float4* src = reinterpret_cast<const float4*>(so + (static_cast<size_t>(i) * p.slot_rows + pr) * D) + 2 * c8;
+        const float4 a = src[0], c = src[1];
+        L += ml.y * w;
+        acc[0] += a.x * w; acc[1] += a.y * w; acc[2] += a.z * w; acc[3] += a.w * w;
+        acc[4] += c.x * w; acc[5] += c.y * w; acc[6] += c.z * w; acc[7] += c.w * w;
+      }
+    }
+    const bool dead = bad || !(L > 0.f);
+    write_out_row<D>(p, b, g, row0 + r, c8 * 8, acc, dead ? 0.f : 1.f / L);
+    if (c8 == 0) write_lse(p, b, g, row0 + r, mx, L, dead);
+  }
 }
 
 // ---------------------------------------------------------------------------------
@@ -186,6 +238,7 @@ __global__ void __launch_bounds__(TcCfg<D, MT, QR, HP>::THREADS, 1)
   // segment flags: the producer publishes whether a segment reads a bad page or has a
   // malformed length (ring of 8, far more than the producer can run ahead)
   auto flag_bar = [&](int i) { return seg_ready + 64 + 8u * i; };
+  const uint32_t merge_bar = seg_ready + 128;  // a unit's partials staged in the ring
   volatile int* seg_flag = reinterpret_cast<volatile int*>(smem + C::OFF_FLAG);
   uint32_t* misc = reinterpret_cast<uint32_t*>(smem + C::OFF_MISC);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(misc + 1);
@@ -251,6 +304,7 @@ __global__ void __launch_bounds__(TcCfg<D, MT, QR, HP>::THREADS, 1)
     for (int q = 0; q < 4; ++q) mbar_init(xch_bar(q), 2);
     mbar_init(q_full, 1);
     for (int i = 0; i < 8; ++i) mbar_init(flag_bar(i), 1);
+    if (HP == 2) mbar_init(merge_bar, 1);
     *abort_flag = 0;
     *pend_count = 0;
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -816,9 +870,41 @@ __global__ void __launch_bounds__(TcCfg<D, MT, QR, HP>::THREADS, 1)
       bool any = false;
       for (int i = 0; i < np; ++i) any |= pend[8 * i + 7] != 0;
       if (any) __threadfence();
+      uint32_t mphase = 0;
       for (int i = 0; i < np; ++i) {
         const int* e = pend + 8 * i;
         if (!e[7]) continue;
+        // Head pairs: the unit's slots are consecutive, and when they fit in the idle K/V
+        // stages thread 0 brings them in with two bulk copies (one round trip instead of
+        // one per item batch) and every thread merges from shared memory. The (m, l) rows
+        // of a slot are 16-byte multiples only for an even slot_rows. (Measured slower in
+        // the fused llama8b step for 32-row units, so the one-head kernels keep the
+        // global merge.)
+        if constexpr (HP == 2) {
+          const uint32_t slot_bytes = static_cast<uint32_t>(p.slot_rows) * D * 4;
+          const uint32_t ml_bytes = static_cast<uint32_t>(p.slot_rows) * 8;
+          const int nsl = e[5];
+          if (p.slot_rows % 2 == 0 && static_cast<uint64_t>(nsl) * (slot_bytes + ml_bytes) <= C::RING_BYTES) {
+            float* so = reinterpret_cast<float*>(smem + C::OFF_K);
+            float2* sml = reinterpret_cast<float2*>(smem + C::OFF_K + nsl * slot_bytes);
+            if (threadIdx.x == 0) {
+              fence_async_global();  // the partials (generic stores) before the copy engine reads them
+              mbar_arrive_tx(merge_bar, nsl * (slot_bytes + ml_bytes));
+              bulk_load(smem_u32(so), p.partial_o + static_cast<int64_t>(e[4]) * p.slot_rows * D, nsl * slot_bytes,
+                        merge_bar);
+              bulk_load(smem_u32(sml), p.partial_ml + static_cast<int64_t>(e[4]) * p.slot_rows, nsl * ml_bytes,
+                        merge_bar);
+            }
+            const bool landed = mbar_wait(merge_bar, mphase & 1, abort_flag, p.status);
+            ++mphase;
+            if (landed) {
+              merge_staged<D>(p, e[0], 2 * e[1], e[2], e[3], so, sml, nsl, 0, threadIdx.x, C::THREADS);
+              merge_staged<D>(p, e[0], 2 * e[1] + 1, e[2], e[3], so, sml, nsl, p.rows, threadIdx.x, C::THREADS);
+            }
+            __syncthreads();  // the staging area is free for the next unit
+            continue;
+          }
+        }
         // units of 128+ rows (a head pair, two M tiles) keep four items per thread in flight
         constexpr int kItems = (HP == 2 || MT == 2) ? 4 : 1;
         if (HP == 2) {  // the pair's heads, the second's rows after the first's in a slot

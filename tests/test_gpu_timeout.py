@@ -30,9 +30,10 @@ def read_status(ws):
     return int(code), int(flags)
 
 
-@pytest.mark.parametrize("group,gamma", [(4, 8), (8, 32)])
+@pytest.mark.parametrize("group,gamma", [(4, 8), (4, 16), (8, 32)])
 def test_attention_wait_runs_out(oracle_mod, group, gamma):
-    # 32 rows per KV group (one M tile, 64-row buffers) and 256 (two M tiles)
+    # 32 rows per KV group (one M tile, 64-row buffers), 64 (two KV heads per block) and
+    # 256 (two M tiles)
     hkv = 2
     inp = W.make_attn_inputs(3, gamma, group * hkv, hkv, 128, 16, (100, 700), True, seed=91 + gamma)
     q, k, v, pt, kl = attn_tensors(inp)
