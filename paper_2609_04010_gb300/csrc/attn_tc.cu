@@ -67,13 +67,15 @@ struct TcCfg {
   // (with two heads the second O pair would not fit in TMEM).
   static constexpr int SPLIT = (MT == 1 && HP == 1) ? 2 : 1;
   static constexpr int KH = TK / SPLIT;               // keys of a tile per softmax warp
-  static constexpr int PB = MT == 1 ? 2 : 1;          // P buffers (double with one M tile)
+  // P in tensor memory (head pairs, two M tiles): P of M tile mt over the first 32
+  // columns of its (first head's) S buffer of the tile, which then stays busy until the
+  // tile's P V MMAs complete; double-buffered with S
+  static constexpr bool PTMEM = HP == 2 || MT == 2;
+  static constexpr int PB = (MT == 1 || PTMEM) ? 2 : 1;  // P buffers
   static constexpr int MR = QR * HP;                  // rows of a Q or P buffer
-  // P in tensor memory (head pairs): P[buf] over the first 32 columns of S[0][buf], which
-  // then stays busy until the tile's P V MMAs complete
-  static constexpr bool PTMEM = HP == 2;
-  // one ring of K+V stages (HP = 1), or KST stages of K and VST of V (HP = 2)
-  static constexpr int STAGES = QR == 64 ? 5 : ((D == 128 && MT == 2) || (D == 64 && MT == 1) ? 3 : 4);
+  // one ring of K+V stages (HP = 1), or KST stages of K and VST of V (HP = 2); two M tiles
+  // with P in TMEM have the P buffer's 32 KB as a fourth stage
+  static constexpr int STAGES = QR == 64 ? 5 : ((D == 64 && MT == 1) ? 3 : 4);
   static constexpr int KST = HP == 2 ? (D == 128 ? 3 : 4) : STAGES;
   static constexpr int VST = HP == 2 ? (D == 128 ? 3 : 4) : STAGES;
   static constexpr int RINGBARS = HP == 2 ? 2 * (KST + VST) : 2 * STAGES;
@@ -549,8 +551,8 @@ __global__ void __launch_bounds__(TcCfg<D, MT, QR, HP>::THREADS, 1)
                     const int kg = hf * (KH / 16) + kk;  // 16-key step within the tile
                     const uint32_t vb = sbase + C::OFF_V + st * C::KV_BYTES + h * kHead + kg * 2u * kGroup;
                     if constexpr (C::PTMEM) {  // P from TMEM: 8 columns per 16 keys
-                      mma_bf16_ta(d_tmem, tmem + C::S_COL + pbuf * TK + kg * 8u, desc_sw128(vb, 1024, kGroup),
-                                  kIdescPV, (k > 0 || kk > 0) ? 1u : 0u);
+                      mma_bf16_ta(d_tmem, tmem + C::S_COL + (mt * HP * 2 + pbuf) * TK + kg * 8u,
+                                  desc_sw128(vb, 1024, kGroup), kIdescPV, (k > 0 || kk > 0) ? 1u : 0u);
                     } else {
                       const uint32_t pa = sbase + C::OFF_P + (pbuf * MT + mt) * C::PBUF + kg * 32u;
                       mma_bf16(d_tmem, desc_sw128(pa, 16, 1024), desc_sw128(vb, 1024, kGroup), kIdescPV,
@@ -731,8 +733,9 @@ __global__ void __launch_bounds__(TcCfg<D, MT, QR, HP>::THREADS, 1)
           tmem_wait_st();
         }
         if constexpr (C::PTMEM) {
-          // P as bf16 pairs over the first 32 columns of S[0][x & 1] (this row's lane)
-          tmem_st32(lane_base + C::S_COL + (x & 1) * TK, pk);
+          // P as bf16 pairs over the first 32 columns of the M tile's (first head's) S
+          // buffer of this tile (this row's lane)
+          tmem_st32(lane_base + C::S_COL + (mt * HP * 2 + (x & 1)) * TK, pk);
           tmem_wait_st();
         } else {
           unsigned char* prow = smem + C::OFF_P + (pbuf * MT + mt) * C::PBUF + row * 128u;
