@@ -5,8 +5,8 @@
 //
 // One block holds every query row of one KV head (row r = block position j * group +
 // head-in-group), padded to M = 128 rows per tensor-core tile (two tiles when the
-// group has up to 256 rows), so each KV page is read from HBM once. When a group has at
-// most 64 rows and Hkv is even, the head-pair variant serves two adjacent KV heads in
+// group has up to 256 rows), so each KV page is read from HBM once. When a group has 33
+// to 64 rows and Hkv is even, the head-pair variant serves two adjacent KV heads in
 // one M tile (the first head's rows in TMEM lanes 0..63, the second's in 64..127): the
 // cache stores the heads of a page next to each other, so one copy brings a page of both
 // (8 KB instead of 4 KB with 16-token pages; the copy engine's rate grows with the size
@@ -25,19 +25,23 @@
 //               8-key groups so that the MMAs below can span pages.
 //   warp 1      Q K^T issuer: S = Q K^T (tcgen05.mma kind::f16, M = 128, N = 64, K = 16
 //               steps over D) into a double-buffered fp32 TMEM accumulator.
-//   warp 3      P V issuer: O += P V (N = D) with P from shared memory, V read MN-major.
+//   warp 3      P V issuer: O += P V (N = D) with V read MN-major and P from shared
+//               memory, or, with two M tiles or a head pair, from tensor memory.
 //   warps 4..11 softmax, one thread per query row; with one M tile two warps share a
 //               32-row quadrant, one per half of each tile's keys, each with its own
 //               online softmax and O (merged at the end of a unit); with two M tiles
 //               one warp per quadrant. Load S from TMEM, scale and mask, online
 //               softmax in base 2 with lazy rescale of O (only when the running max
-//               grows by more than 2^8), write P as bf16 in the swizzled layout the MMA
-//               reads (double-buffered with one M tile), and at the end of a unit read
-//               O from TMEM and write the output. Warps without real rows idle.
+//               grows by more than 2^8), write P as bf16 (in the swizzled shared-memory
+//               layout the MMA reads, double-buffered, with one M tile of one head;
+//               otherwise over the first 32 columns of the tile's S buffer in TMEM,
+//               double-buffered with S), and at the end of a unit read O from TMEM and
+//               write the output. Warps without real rows idle.
 // Work is balanced across blocks "stream-K" style: all 64-key tiles of all (sequence,
 // KV head, row tile) units form one list that is cut into equal contiguous ranges; a
 // unit split between blocks is merged from fp32 partials by the last block to finish
-// it (atomic ticket, no waiting). Every mbarrier wait is bounded: a wait that runs out
+// it (atomic ticket, no waiting; a head pair's slots are first brought into the idle
+// K/V stages by bulk copies). Every mbarrier wait is bounded: a wait that runs out
 // sets SPEC_FLAG_TIMEOUT, drains the block's own copies and MMAs, frees TMEM and exits.
 #include <cuda.h>  // CUtensorMap and its encoder's signature (resolved at run time)
 
