@@ -45,7 +45,7 @@ L2_FLUSH_BYTES = 256 << 20
 # while the kernel's sources still hash to what they were when the capture was taken.
 _ATTN_TC_SOURCES = {
     "paper_2609_04010_gb300/csrc/attn_tc.cu":
-        "9eada2fa4a04ac158cb40acd13ccb0d66cad65f63702921e42e2a4382d1679e5",
+        "e555e3a344557cf1bb6db379b0d33a34ffc488dc808a29893a54a6c6180959a5",
     "paper_2609_04010_gb300/csrc/attn_common.cuh":
         "f598688828a4f71ceae6be8600fa576646644fda3e2e6b4c87c0b1b8fea65f0c",
     "paper_2609_04010_gb300/csrc/tc_ptx.cuh":
