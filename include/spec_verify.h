@@ -79,7 +79,10 @@ typedef enum {
   SPEC_ATTN_AUTO = 0,          /* tensor cores when (Hq/Hkv)*gamma >= the crossover, else CUDA cores */
   SPEC_ATTN_CUDA_CORES = 1,    /* fp32 CUDA-core kernel                                  */
   SPEC_ATTN_TENSOR_CORES = 2,  /* tcgen05 (TMEM accumulators, TMA-staged KV pages), the
-                                  row-tile kernel (M = 128 query rows per tile)           */
+                                  row-tile kernel (M = 128 query rows per tile); with 33
+                                  to 64 query rows per KV head and an even Hkv (batch <=
+                                  407 for head_dim 128) one block serves two adjacent KV
+                                  heads, reading 8 KB page boxes                          */
   SPEC_ATTN_TENSOR_CORES_KEYS_ON_LANES = 3  /* tcgen05 with the keys of a tile on the MMA's
                                   M dimension (S^T = K Q^T, O^T = V^T P^T), where it applies
                                   (head_dim 128, at most 64 query rows per KV head, 64 %
