@@ -46,6 +46,11 @@ SMALL = [
          ctx=(1, 260)),
     dict(batch=4, gamma=16, num_q_heads=32, num_kv_heads=8, head_dim=128, page_size=16,
          ctx=(0, 100)),
+    # two KV heads per block with 64-token pages (32 KB page boxes), head dim 128 and 64
+    dict(batch=3, gamma=16, num_q_heads=16, num_kv_heads=4, head_dim=128, page_size=64,
+         ctx=(50, 900)),
+    dict(batch=2, gamma=10, num_q_heads=32, num_kv_heads=8, head_dim=64, page_size=64,
+         ctx=(300, 700)),
 ]
 
 
